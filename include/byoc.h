@@ -1,0 +1,199 @@
+/*
+ * byoc.h -- C ABI of the GB300 (sm_103a) execution engine for partitioned,
+ * offloaded regions ("Bring Your Own Codegen", arXiv 2105.03215).
+ *
+ * The paper's flow (Section 3) partitions a model graph, encapsulates every
+ * offloadable region as a function with a target attribute (Section 3.1.3),
+ * hands that function to the accelerator's code generator (Section 3.3), and
+ * at run time calls it as an external function that reads its inputs from,
+ * and writes its outputs to, pre-allocated data entries (Section 3.4,
+ * "Execute the graph nodes on the accelerator").  Constants live in the
+ * metadata module and are loaded once at initialisation; the accelerator's
+ * execution engine is built once and cached (Section 3.4).
+ *
+ * This header is that boundary:
+ *   byoc_compile  -- the per-region code generation + engine initialisation:
+ *                    validates the op list, folds batch norm into the weights
+ *                    and bias, rounds and packs the weights, uploads them, and
+ *                    picks a kernel plan.  Run once; the handle is the cache.
+ *   byoc_run      -- the external call F1(...): enqueues the region's kernels
+ *                    on a CUDA stream; reads inputs / writes outputs in
+ *                    caller-owned device memory (the data entries).
+ *   byoc_release  -- frees what byoc_compile allocated.
+ *
+ * Conventions shared by every entry point:
+ *   - Activations are bf16, NHWC for 4-D tensors and row-major [rows, features]
+ *     for 2-D tensors (Section 3.2: the accelerator fixes its layout; the
+ *     caller transforms at the region boundary).  Constants are fp32, host
+ *     memory, copied during byoc_compile (the caller may free them after it
+ *     returns).
+ *   - Device pointers passed to byoc_run must be 16-byte aligned and point to
+ *     contiguous tensors of the shapes given at compile time.
+ *   - Every call that can fail returns a byoc_status; on failure a thread-local
+ *     message is available from byoc_last_error().  Nothing falls back to the
+ *     CPU: an op chain the kernels cannot run is rejected at compile time with
+ *     BYOC_ERR_UNSUPPORTED (the paper's cost/annotation rules keep such ops on
+ *     the host, Section 3.1.2-3.1.3).
+ *   - Device-side waits are bounded; a kernel whose wait expires records
+ *     BYOC_ERR_TIMEOUT in a per-handle error word that byoc_check() reports.
+ */
+#ifndef BYOC_H_
+#define BYOC_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BYOC_ABI_VERSION 1u
+
+typedef struct byoc_handle byoc_handle; /* opaque: packed constants, workspace, plans */
+
+typedef enum {
+    BYOC_OK = 0,
+    BYOC_ERR_INVALID_ARG = 1, /* malformed descriptor, null/misaligned pointer, bad shape */
+    BYOC_ERR_UNSUPPORTED = 2, /* valid op chain that no kernel here implements */
+    BYOC_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed */
+    BYOC_ERR_OOM = 4,         /* device or host allocation failed */
+    BYOC_ERR_TIMEOUT = 5      /* a kernel's bounded wait expired (reported by byoc_check) */
+} byoc_status;
+
+typedef enum { BYOC_BF16 = 0, BYOC_FP32 = 1 } byoc_dtype;
+
+typedef enum {
+    BYOC_LAYOUT_NHWC = 0, /* 4-D activation [N, H, W, C] */
+    BYOC_LAYOUT_NC = 1    /* 2-D activation [rows, features] */
+} byoc_layout;
+
+/* Operators of the composite patterns (Section 3.1.1: Conv2D, Add/bias, ReLU;
+ * Section 4 models add batch norm, ReLU6, GELU and residual add). */
+typedef enum {
+    BYOC_OP_CONV2D = 0,     /* in[0]=data; consts[0]=weight OIHW [K, C/groups, kh, kw] */
+    BYOC_OP_DENSE = 1,      /* in[0]=data [M, I]; consts[0]=weight [units, I] */
+    BYOC_OP_BIAS_ADD = 2,   /* in[0]; consts[0]=bias [C] (channel = innermost axis) */
+    BYOC_OP_BATCH_NORM = 3, /* in[0]; consts = gamma, beta, moving_mean, moving_var [C]; eps */
+    BYOC_OP_RELU = 4,
+    BYOC_OP_RELU6 = 5,      /* clip(x, 0, 6) */
+    BYOC_OP_GELU = 6,       /* 0.5 x (1 + erf(x / sqrt 2)) */
+    BYOC_OP_ADD = 7         /* in[0] + in[1], same shape */
+} byoc_op_kind;
+
+typedef struct {
+    int32_t ndim;     /* 4 (NHWC) or 2 (NC) */
+    int64_t shape[4]; /* unused trailing entries ignored */
+    int32_t dtype;    /* byoc_dtype; activations must be BYOC_BF16 */
+    int32_t layout;   /* byoc_layout */
+} byoc_tensor;
+
+typedef struct {
+    int32_t kind;        /* byoc_op_kind */
+    int32_t n_in;        /* 1, or 2 for BYOC_OP_ADD */
+    int32_t in[3];       /* tensor ids (indices into byoc_region_desc.tensors) */
+    int32_t out;         /* tensor id of the result */
+    int32_t kernel[2];   /* conv2d: kh, kw */
+    int32_t stride[2];   /* conv2d: sh, sw */
+    int32_t pad[4];      /* conv2d: top, left, bottom, right */
+    int32_t dilation[2]; /* conv2d: dh, dw */
+    int32_t groups;      /* conv2d: 1, or C for depthwise */
+    float eps;           /* batch_norm epsilon */
+    const float *consts[4]; /* host fp32 constants, see byoc_op_kind */
+} byoc_op;
+
+/* One partitioned region: the function the partitioner encapsulates
+ * (Section 3.1.3) in the JSON-like graph form of codegen Option 1
+ * (Section 3.3): tensors, ops in topological order, boundary tensor ids. */
+typedef struct {
+    uint32_t abi_version;         /* must equal BYOC_ABI_VERSION */
+    const char *name;             /* region / composite name, informational */
+    int32_t n_tensors;
+    const byoc_tensor *tensors;
+    int32_t n_ops;
+    const byoc_op *ops;           /* topological order */
+    int32_t n_inputs;
+    const int32_t *input_ids;     /* order of byoc_run's inputs[] */
+    int32_t n_outputs;
+    const int32_t *output_ids;    /* order of byoc_run's outputs[] */
+} byoc_region_desc;
+
+/* Figures describing a compiled region. */
+typedef struct {
+    double flops;           /* algorithmic 2 x MACs per byoc_run (conv2d + dense only) */
+    double bytes;           /* algorithmic HBM bytes per byoc_run: every launch reads its
+                               inputs and weights once and writes its output once */
+    size_t workspace_bytes; /* device workspace owned by the handle (region intermediates) */
+    size_t const_bytes;     /* device bytes of packed constants */
+    int32_t n_launches;     /* kernel launches one byoc_run enqueues */
+    int32_t n_inputs;
+    int32_t n_outputs;
+} byoc_info;
+
+/* Compile one region (Section 3.3 code generation + Section 3.4 engine
+ * initialisation).  Validates the descriptor, folds batch norm and bias into
+ * per-channel weight scales and biases in fp64, rounds the folded weights to
+ * bf16 (round to nearest even), packs them K-major for the tensor cores,
+ * copies all constants to the current CUDA device, and allocates the
+ * region's workspace.  Launches no kernel.
+ *   desc : read only during the call.
+ *   out  : receives the new handle (NULL on failure).
+ * Errors: INVALID_ARG (malformed), UNSUPPORTED (chain not implemented),
+ *         OOM, CUDA. */
+byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out);
+
+/* Run a compiled region: the external function call of Section 3.4.
+ *   inputs[i]  : device pointer of the tensor desc->input_ids[i]
+ *   outputs[i] : device pointer of the tensor desc->output_ids[i]
+ *   cuda_stream: a cudaStream_t (NULL = legacy default stream)
+ * Asynchronous: enqueues the kernels and returns.  Pointers must be non-null,
+ * 16-byte aligned, and stay valid until the stream reaches the end of the
+ * region.  A handle's workspace is shared by its runs, so two runs of one
+ * handle must not overlap on the GPU.
+ * Errors: INVALID_ARG (null handle / pointer, misalignment), CUDA (launch). */
+byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *outputs,
+                     void *cuda_stream);
+
+/* Read and clear the handle's device error word.  Call after the stream that
+ * ran the handle has been synchronised; returns BYOC_ERR_TIMEOUT if a kernel
+ * gave up on a bounded wait since the previous check, else BYOC_OK.
+ * Synchronous (one 4-byte device-to-host copy). */
+byoc_status byoc_check(byoc_handle *h);
+
+/* Free everything byoc_compile allocated.  NULL-safe.  The caller must make
+ * sure no run of this handle is still in flight. */
+void byoc_release(byoc_handle *h);
+
+/* Thread-local message describing the last non-OK status of this thread. */
+const char *byoc_last_error(void);
+
+/* Describe a compiled region (see byoc_info). */
+byoc_status byoc_query(const byoc_handle *h, byoc_info *info);
+
+/* ---------------------------------------------------------------------------
+ * Host-side operators.  In the paper, operators that stay outside every
+ * region run on the host through the compiler's own code generation, and CUDA
+ * may serve as the host (Section 3.4, footnote on the metadata module;
+ * Section 4.1).  These are the ones the ResNet-50 host graph needs, written
+ * here as CUDA kernels so that no step of the graph leaves this library.
+ * All are asynchronous on cuda_stream; bf16 NHWC; C must be a multiple of 8;
+ * pointers 16-byte aligned.  Errors: INVALID_ARG, CUDA.
+ * ------------------------------------------------------------------------- */
+
+/* max_pool2d, window k x k, stride s, symmetric zero-cost padding p (padded
+ * positions never win).  x [N,H,W,C] -> y [N,Ho,Wo,C], Ho = (H+2p-k)/s+1. */
+byoc_status byoc_max_pool2d_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W,
+                                 int32_t C, int32_t k, int32_t s, int32_t p, void *cuda_stream);
+
+/* global_avg_pool2d: x [N,H,W,C] -> y [N,C] (fp32 sum, bf16 result). */
+byoc_status byoc_global_avg_pool_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W,
+                                      int32_t C, void *cuda_stream);
+
+/* Number of SMs and the device's compute capability, for host-side planning
+ * (current device).  Errors: CUDA. */
+byoc_status byoc_device_info(int32_t *num_sms, int32_t *cc_major, int32_t *cc_minor);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BYOC_H_ */

@@ -1,0 +1,272 @@
+// aux_kernels.cu -- the bandwidth-bound kernels of the offloaded path:
+//   * depthwise 3x3 conv + folded BN + activation (MobileNetV2 composite),
+//   * the space-to-depth boundary transform that turns a stride-2 stem over
+//     3 channels into a stride-1 convolution over 16 channels (a layout
+//     transformation node inserted at a region boundary, Section 3.2),
+//   * the host-graph operators of ResNet-50 (max pool, global average pool),
+//     which the paper leaves on the host (Section 3.4, CUDA as the host).
+// All tensors are bf16 NHWC; every thread moves 8 channels (16 bytes) at a
+// time so that a warp's accesses are contiguous along C.
+#include "internal.h"
+#include "ptx.cuh"
+
+namespace byoc {
+
+__device__ __forceinline__ void unpack8(const uint4 &v, float (&f)[8]) {
+    f[0] = bf16lo(v.x); f[1] = bf16hi(v.x);
+    f[2] = bf16lo(v.y); f[3] = bf16hi(v.y);
+    f[4] = bf16lo(v.z); f[5] = bf16hi(v.z);
+    f[6] = bf16lo(v.w); f[7] = bf16hi(v.w);
+}
+
+__device__ __forceinline__ uint4 pack8(const float (&f)[8]) {
+    uint4 o;
+    o.x = pack_bf16x2(f[0], f[1]);
+    o.y = pack_bf16x2(f[2], f[3]);
+    o.z = pack_bf16x2(f[4], f[5]);
+    o.w = pack_bf16x2(f[6], f[7]);
+    return o;
+}
+
+__device__ __forceinline__ uint4 ldg_v4(const void *p) {
+    return __ldg(reinterpret_cast<const uint4 *>(p));
+}
+
+// ------------------------------------------------------------ depthwise 3x3
+//
+// Thread <-> (image n, output column q, 8-channel vector cv, ROWS consecutive
+// output rows).  cv varies fastest across threads, so a warp reads and writes
+// contiguous 16-byte vectors of one image row.  The three input rows under
+// the filter live in registers and slide down the column (stride 1: one new
+// row per output row; stride 2: two), so each input vector is loaded about
+// (ROWS+2)/ROWS times per filter column instead of three; the three filter
+// columns of neighbouring q are served by L1.
+template <int STRIDE, int ROWS>
+__global__ void __launch_bounds__(256) dwconv3x3_kernel(const DwArgs a) {
+    const int CV = a.C >> 3;
+    const int PB = (a.Ho + ROWS - 1) / ROWS;
+    const long long total = (long long)a.N * PB * a.Wo * CV;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int cv = (int)(idx % CV);
+    long long t = idx / CV;
+    const int q = (int)(t % a.Wo);
+    t /= a.Wo;
+    const int pb = (int)(t % PB);
+    const int n = (int)(t / PB);
+    const int c0 = cv * 8;
+
+    float w[9][8];
+#pragma unroll
+    for (int tap = 0; tap < 9; ++tap) {
+        const float4 lo = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0));
+        const float4 hi = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0 + 4));
+        w[tap][0] = lo.x; w[tap][1] = lo.y; w[tap][2] = lo.z; w[tap][3] = lo.w;
+        w[tap][4] = hi.x; w[tap][5] = hi.y; w[tap][6] = hi.z; w[tap][7] = hi.w;
+    }
+    float bias[8];
+    {
+        const float4 lo = __ldg(reinterpret_cast<const float4 *>(a.bias + c0));
+        const float4 hi = __ldg(reinterpret_cast<const float4 *>(a.bias + c0 + 4));
+        bias[0] = lo.x; bias[1] = lo.y; bias[2] = lo.z; bias[3] = lo.w;
+        bias[4] = hi.x; bias[5] = hi.y; bias[6] = hi.z; bias[7] = hi.w;
+    }
+
+    const int wc0 = q * STRIDE - a.pad;
+    const __nv_bfloat16 *xn = a.x + (size_t)n * a.H * a.W * a.C + c0;
+    auto load_row = [&](int h, uint4 (&r)[3]) {
+        const bool hv = h >= 0 && h < a.H;
+#pragma unroll
+        for (int s = 0; s < 3; ++s) {
+            const int wc = wc0 + s;
+            if (hv && wc >= 0 && wc < a.W)
+                r[s] = ldg_v4(xn + ((size_t)h * a.W + wc) * a.C);
+            else
+                r[s] = make_uint4(0u, 0u, 0u, 0u);
+        }
+    };
+
+    const int p0 = pb * ROWS;
+    uint4 win[3][3];
+    load_row(p0 * STRIDE - a.pad, win[0]);
+    load_row(p0 * STRIDE - a.pad + 1, win[1]);
+#pragma unroll
+    for (int i = 0; i < ROWS; ++i) {
+        const int p = p0 + i;
+        const int hb = p * STRIDE - a.pad;
+        if (i > 0) {
+            if (STRIDE == 1) {
+#pragma unroll
+                for (int s = 0; s < 3; ++s) {
+                    win[0][s] = win[1][s];
+                    win[1][s] = win[2][s];
+                }
+            } else {
+#pragma unroll
+                for (int s = 0; s < 3; ++s) win[0][s] = win[2][s];
+                load_row(hb + 1, win[1]);
+            }
+        }
+        load_row(hb + 2, win[2]);
+        if (p < a.Ho) {
+            float acc[8];
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] = bias[j];
+#pragma unroll
+            for (int r = 0; r < 3; ++r) {
+#pragma unroll
+                for (int s = 0; s < 3; ++s) {
+                    float f[8];
+                    unpack8(win[r][s], f);
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) acc[j] = fmaf(f[j], w[r * 3 + s][j], acc[j]);
+                }
+            }
+#pragma unroll
+            for (int j = 0; j < 8; ++j) {
+                float v = acc[j];
+                if (a.act == kActRelu) v = fmaxf(v, 0.0f);
+                else if (a.act == kActRelu6) v = fminf(fmaxf(v, 0.0f), 6.0f);
+                else if (a.act == kActGelu) v = 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
+                acc[j] = v;
+            }
+            *reinterpret_cast<uint4 *>(a.y + (((size_t)n * a.Ho + p) * a.Wo + q) * a.C + c0) =
+                pack8(acc);
+        }
+    }
+}
+
+cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st) {
+    (void)num_sms;
+    const int CV = a.C / 8;
+    const int threads = 256;
+    if (a.stride == 1) {
+        constexpr int R = 8;
+        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CV;
+        dwconv3x3_kernel<1, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
+    } else {
+        constexpr int R = 4;
+        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CV;
+        dwconv3x3_kernel<2, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
+    }
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ space-to-depth
+// z[n, i, j, (dy*2+dx)*C + c] = x[n, 2i+dy-pad, 2j+dx-pad, c]; other channels 0.
+__global__ void s2d_kernel(const S2dArgs a) {
+    const long long total = (long long)a.N * a.Hz * a.Wz;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int j = (int)(idx % a.Wz);
+    const long long t = idx / a.Wz;
+    const int i = (int)(t % a.Hz);
+    const int n = (int)(t / a.Hz);
+    float v[16];
+#pragma unroll
+    for (int k = 0; k < 16; ++k) v[k] = 0.0f;
+    const unsigned short *xs = reinterpret_cast<const unsigned short *>(a.x);
+#pragma unroll
+    for (int dy = 0; dy < 2; ++dy) {
+#pragma unroll
+        for (int dx = 0; dx < 2; ++dx) {
+            const int h = 2 * i + dy - a.pad;
+            const int w = 2 * j + dx - a.pad;
+            if (h < 0 || h >= a.H || w < 0 || w >= a.W) continue;
+            const size_t off = (((size_t)n * a.H + h) * a.W + w) * a.C;
+            for (int c = 0; c < a.C; ++c) {
+                const int k = (dy * 2 + dx) * a.C + c;
+                if (k < 16) v[k] = __uint_as_float((uint32_t)__ldg(xs + off + c) << 16);
+            }
+        }
+    }
+    uint4 *zp = reinterpret_cast<uint4 *>(a.z + (size_t)idx * a.Cz);
+    float lo[8], hi[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        lo[k] = v[k];
+        hi[k] = v[8 + k];
+    }
+    zp[0] = pack8(lo);
+    zp[1] = pack8(hi);
+}
+
+cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
+    const long long total = (long long)a.N * a.Hz * a.Wz;
+    s2d_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(a);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ max pool
+__global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                               int k, int s, int p, int Ho, int Wo) {
+    const int CV = C >> 3;
+    const long long total = (long long)N * Ho * Wo * CV;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int cv = (int)(idx % CV);
+    long long t = idx / CV;
+    const int q = (int)(t % Wo);
+    t /= Wo;
+    const int pp = (int)(t % Ho);
+    const int n = (int)(t / Ho);
+    float m[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) m[j] = -INFINITY;
+    for (int r = 0; r < k; ++r) {
+        const int h = pp * s - p + r;
+        if (h < 0 || h >= H) continue;
+        for (int c = 0; c < k; ++c) {
+            const int w = q * s - p + c;
+            if (w < 0 || w >= W) continue;
+            float f[8];
+            unpack8(ldg_v4(x + (((size_t)n * H + h) * W + w) * C + cv * 8), f);
+#pragma unroll
+            for (int j = 0; j < 8; ++j) m[j] = fmaxf(m[j], f[j]);
+        }
+    }
+    *reinterpret_cast<uint4 *>(y + (((size_t)n * Ho + pp) * Wo + q) * C + cv * 8) = pack8(m);
+}
+
+cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                           int k, int s, int p, cudaStream_t st) {
+    const int Ho = (H + 2 * p - k) / s + 1;
+    const int Wo = (W + 2 * p - k) / s + 1;
+    const long long total = (long long)N * Ho * Wo * (C / 8);
+    maxpool_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C, k, s, p, Ho, Wo);
+    return cudaGetLastError();
+}
+
+// ------------------------------------------------------------ global average pool
+__global__ void avgpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W,
+                               int C) {
+    const int CV = C >> 3;
+    const long long total = (long long)N * CV;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int cv = (int)(idx % CV);
+    const int n = (int)(idx / CV);
+    float acc[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] = 0.0f;
+    const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
+    for (int i = 0; i < H * W; ++i) {
+        float f[8];
+        unpack8(ldg_v4(xn + (size_t)i * C), f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] += f[j];
+    }
+    const float inv = 1.0f / (float)(H * W);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) acc[j] *= inv;
+    *reinterpret_cast<uint4 *>(y + (size_t)n * C + cv * 8) = pack8(acc);
+}
+
+cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                           cudaStream_t st) {
+    const long long total = (long long)N * (C / 8);
+    avgpool_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C);
+    return cudaGetLastError();
+}
+
+}  // namespace byoc

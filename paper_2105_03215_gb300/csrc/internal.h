@@ -1,0 +1,85 @@
+// internal.h -- declarations shared by the translation units of libbyoc.so.
+// Not part of the public ABI (include/byoc.h is).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+namespace byoc {
+
+enum Act : int { kActNone = 0, kActRelu = 1, kActRelu6 = 2, kActGelu = 3 };
+
+// Implicit-GEMM problem: out[M, N] = act(A[M, K] . B[N, K]^T + bias [+ residual]).
+//  A is either a row-major [M, K] matrix (dense, 1x1 stride-1 conv) read with a
+//  2-D tiled tensor map, or the implicit im2col matrix of an NHWC activation
+//  read with an im2col tensor map: row m = output pixel (n, p, q), column
+//  k = (tap r*kw+s, channel chunk, channel).  B is the packed weight matrix.
+struct GemmArgs {
+    int M;          // output rows
+    int N;          // output channels = row stride of out / residual (elements)
+    int num_kb;     // k-blocks per tile (taps * chunks)
+    int chunks;     // channel chunks (of BK channels) per filter tap
+    int kw;         // filter width
+    int dil_h, dil_w;
+    int Ho, Wo;     // output spatial size (im2col)
+    int stride_h, stride_w;
+    int pad_t, pad_l;
+    int tiles_n;    // number of BN-wide column tiles
+    int num_tiles;  // tiles_m * tiles_n
+    int act;        // Act
+    const float *bias;                // [tiles_n * BN], zero padded; may be null
+    const __nv_bfloat16 *residual;    // [M, N] or null
+    __nv_bfloat16 *out;               // [M, N]
+    int *err;                         // device error word
+};
+
+struct GemmConfig {
+    int bn;       // tile width in output channels: 32, 64, 128, 256
+    int bk;       // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
+    bool im2col;  // A operand through an im2col tensor map
+};
+
+constexpr int kGemmBM = 128;
+constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+
+bool gemm_config_supported(const GemmConfig &cfg);
+size_t gemm_smem_bytes(const GemmConfig &cfg);
+int gemm_stages(const GemmConfig &cfg);
+cudaError_t gemm_prepare(const GemmConfig &cfg);  // raises the dynamic smem limit
+cudaError_t launch_gemm(const GemmConfig &cfg, const CUtensorMap &tmA, const CUtensorMap &tmB,
+                        const GemmArgs &a, int grid, cudaStream_t st);
+
+// Depthwise conv (groups = C), square kernel k in {3}, NHWC bf16, folded
+// weights fp32 [k*k][C] (tap-major), bias fp32 [C], fused activation.
+struct DwArgs {
+    const __nv_bfloat16 *x;
+    const float *w;
+    const float *bias;
+    __nv_bfloat16 *y;
+    int N, H, W, C, Ho, Wo;
+    int stride, pad;
+    int act;
+};
+cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st);
+
+// Boundary layout transform for a stride-2 stem with few input channels
+// (space-to-depth with zero padding): z[n, i, j, (dy*2+dx)*C + c] =
+// x[n, 2i+dy-pad, 2j+dx-pad, c] (zero outside), channels >= 4C zero.
+struct S2dArgs {
+    const __nv_bfloat16 *x;
+    __nv_bfloat16 *z;
+    int N, H, W, C;   // input
+    int Hz, Wz, Cz;   // output (Cz = 16)
+    int pad;
+};
+cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st);
+
+cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                           int k, int s, int p, cudaStream_t st);
+cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                           cudaStream_t st);
+
+}  // namespace byoc

@@ -1,0 +1,946 @@
+// runtime.cu -- the C ABI of include/byoc.h and include/byoc_plan.h.
+//
+// byoc_compile = plan (host only) + materialise (device):
+//   plan        validate the region descriptor; group its ops into launches
+//               (a conv2d / dense absorbs the bias_add, batch_norm, add and
+//               activation that follow it: the composite of Section 3.1.1
+//               runs as one kernel); fold batch norm and bias into a
+//               per-channel scale and shift in fp64; scale the weights,
+//               round them to bf16 (RNE) and pack them K-major; pick tiles;
+//               lay out the workspace for the region's intermediates, which
+//               are not data entries (Section 3.4).
+//   materialise cudaMalloc + copy of the constants (the metadata module's
+//               one-time load, Section 3.4), TMA descriptors of the weights,
+//               kernel attributes.  The handle is the cached engine.
+// byoc_run = the external call: patch activation pointers into cached TMA
+// descriptors and launch the region's kernels on the caller's stream.
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <cudaTypedefs.h>
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <mutex>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "byoc.h"
+#include "byoc_plan.h"
+#include "internal.h"
+
+using byoc::GemmArgs;
+using byoc::GemmConfig;
+
+namespace {
+
+thread_local std::string g_err;
+
+byoc_status fail(byoc_status st, const char *fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof buf, fmt, ap);
+    va_end(ap);
+    g_err = buf;
+    return st;
+}
+
+byoc_status cuda_fail(cudaError_t e, const char *what) {
+    return fail(e == cudaErrorMemoryAllocation ? BYOC_ERR_OOM : BYOC_ERR_CUDA, "%s: %s (%s)", what,
+                cudaGetErrorName(e), cudaGetErrorString(e));
+}
+
+// ------------------------------------------------------------ driver entry points
+
+PFN_cuTensorMapEncodeTiled_v12000 p_encode_tiled = nullptr;
+PFN_cuTensorMapEncodeIm2col_v12000 p_encode_im2col = nullptr;
+std::once_flag g_driver_once;
+cudaError_t g_driver_err = cudaSuccess;
+
+cudaError_t load_driver() {
+    std::call_once(g_driver_once, [] {
+        cudaDriverEntryPointQueryResult q1, q2;
+        cudaError_t e = cudaGetDriverEntryPointByVersion(
+            "cuTensorMapEncodeTiled", reinterpret_cast<void **>(&p_encode_tiled), 12000,
+            cudaEnableDefault, &q1);
+        if (e == cudaSuccess)
+            e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeIm2col",
+                                                 reinterpret_cast<void **>(&p_encode_im2col),
+                                                 12000, cudaEnableDefault, &q2);
+        if (e == cudaSuccess && (q1 != cudaDriverEntryPointSuccess ||
+                                 q2 != cudaDriverEntryPointSuccess || !p_encode_tiled ||
+                                 !p_encode_im2col))
+            e = cudaErrorSymbolNotFound;
+        g_driver_err = e;
+    });
+    return g_driver_err;
+}
+
+CUtensorMapSwizzle swizzle_for(int bk) {
+    return bk == 64 ? CU_TENSOR_MAP_SWIZZLE_128B
+                    : (bk == 32 ? CU_TENSOR_MAP_SWIZZLE_64B : CU_TENSOR_MAP_SWIZZLE_32B);
+}
+
+// 2-D row-major bf16 matrix [rows, cols]; box = [box_cols, box_rows].
+CUresult encode_2d(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                   uint32_t box_cols, int bk) {
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {box_cols, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// im2col map over an NHWC bf16 tensor for a k x k filter, stride s, padding
+// (lo before, hi after), dilation d; 128 pixels x bk channels per load.
+CUresult encode_im2col(CUtensorMap *m, const void *ptr, int N, int H, int W, int C, int k, int s,
+                       int pad_lo, int pad_hi, int d, int bk) {
+    cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+    // Bounding box of filter origins: from -pad_lo to (dim-1) + pad_hi - (k-1)*d.
+    int lower[2] = {-pad_lo, -pad_lo};
+    int upper[2] = {pad_hi - (k - 1) * d, pad_hi - (k - 1) * d};
+    cuuint32_t es[4] = {1, (cuuint32_t)s, (cuuint32_t)s, 1};
+    return p_encode_im2col(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
+                           strides, lower, upper, (cuuint32_t)bk, (cuuint32_t)byoc::kGemmBM, es,
+                           CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
+                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+// ------------------------------------------------------------ bf16 rounding (host)
+
+uint16_t f32_to_bf16_rne(float f) {
+    uint32_t u;
+    std::memcpy(&u, &f, 4);
+    if ((u & 0x7F800000u) == 0x7F800000u) return (uint16_t)((u >> 16) | ((u & 0xFFFFu) ? 0x40u : 0u));
+    u += 0x7FFFu + ((u >> 16) & 1u);
+    return (uint16_t)(u >> 16);
+}
+
+size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
+
+// ------------------------------------------------------------ plan structures
+
+struct TensorInfo {
+    int ndim = 0;
+    int64_t shape[4] = {0, 0, 0, 0};
+    size_t elems() const {
+        size_t e = 1;
+        for (int i = 0; i < ndim; ++i) e *= (size_t)shape[i];
+        return e;
+    }
+    size_t bytes() const { return elems() * 2; }
+    int64_t channels() const { return shape[ndim - 1]; }
+};
+
+struct LaunchPlan {
+    int kind = BYOC_LAUNCH_GEMM;
+    int first_op = -1, n_ops = 0;
+    int x = -1, y = -1, res = -1;  // tensor ids (may index internal scratch tensors)
+    int act = byoc::kActNone;
+    // GEMM
+    GemmConfig cfg{64, 64, false};
+    GemmArgs args{};
+    int grid = 0;
+    int n_pad = 0, k_pack = 0;
+    // A operand geometry
+    int aN = 0, aH = 0, aW = 0, aC = 0, ksz = 1, kstride = 1, pad_lo = 0, pad_hi = 0, dil = 1;
+    int64_t aM = 0, aK = 0;
+    // constants: byte offsets into the constant blob
+    size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
+    // depthwise / space-to-depth
+    byoc::DwArgs dw{};
+    byoc::S2dArgs s2d{};
+    double flops = 0, bytes = 0;
+};
+
+struct Plan {
+    std::vector<TensorInfo> tensors;  // region tensors, then internal scratch tensors
+    int n_region_tensors = 0;
+    std::vector<int> inputs, outputs;
+    std::vector<LaunchPlan> launches;
+    std::vector<uint8_t> blob;  // packed constants (device image)
+    std::vector<size_t> ws_off;  // per tensor: workspace offset, or SIZE_MAX for boundary
+    size_t ws_bytes = 0;
+    double flops = 0, bytes = 0;
+    int num_sms = 148;
+};
+
+size_t blob_append(std::vector<uint8_t> &blob, const void *src, size_t bytes) {
+    size_t off = align_up(blob.size(), 256);
+    blob.resize(off + bytes);
+    std::memcpy(blob.data() + off, src, bytes);
+    return off;
+}
+
+// ------------------------------------------------------------ validation
+
+byoc_status validate(const byoc_region_desc *d, Plan &P) {
+    if (!d) return fail(BYOC_ERR_INVALID_ARG, "null region descriptor");
+    if (d->abi_version != BYOC_ABI_VERSION)
+        return fail(BYOC_ERR_INVALID_ARG, "abi_version %u, expected %u", d->abi_version,
+                    BYOC_ABI_VERSION);
+    if (d->n_tensors <= 0 || !d->tensors) return fail(BYOC_ERR_INVALID_ARG, "no tensors");
+    if (d->n_ops <= 0 || !d->ops) return fail(BYOC_ERR_INVALID_ARG, "no ops");
+    if (d->n_inputs <= 0 || !d->input_ids || d->n_outputs <= 0 || !d->output_ids)
+        return fail(BYOC_ERR_INVALID_ARG, "region needs at least one input and one output");
+    const int nt = d->n_tensors;
+    P.tensors.resize(nt);
+    P.n_region_tensors = nt;
+    for (int i = 0; i < nt; ++i) {
+        const byoc_tensor &t = d->tensors[i];
+        if (t.ndim != 2 && t.ndim != 4)
+            return fail(BYOC_ERR_INVALID_ARG, "tensor %d: ndim %d (2 or 4 expected)", i, t.ndim);
+        if ((t.ndim == 4) != (t.layout == BYOC_LAYOUT_NHWC))
+            return fail(BYOC_ERR_INVALID_ARG, "tensor %d: layout %d does not match ndim %d", i,
+                        t.layout, t.ndim);
+        if (t.dtype != BYOC_BF16)
+            return fail(BYOC_ERR_UNSUPPORTED, "tensor %d: activations must be bf16", i);
+        P.tensors[i].ndim = t.ndim;
+        for (int k = 0; k < t.ndim; ++k) {
+            if (t.shape[k] <= 0 || t.shape[k] > (int64_t)1 << 31)
+                return fail(BYOC_ERR_INVALID_ARG, "tensor %d: bad extent %lld", i,
+                            (long long)t.shape[k]);
+            P.tensors[i].shape[k] = t.shape[k];
+        }
+        if (P.tensors[i].elems() >= ((size_t)1 << 40))
+            return fail(BYOC_ERR_INVALID_ARG, "tensor %d too large", i);
+    }
+    std::vector<int> producer(nt, -1), is_input(nt, 0), is_output(nt, 0);
+    for (int i = 0; i < d->n_inputs; ++i) {
+        int id = d->input_ids[i];
+        if (id < 0 || id >= nt) return fail(BYOC_ERR_INVALID_ARG, "input id %d out of range", id);
+        if (is_input[id]) return fail(BYOC_ERR_INVALID_ARG, "input id %d repeated", id);
+        is_input[id] = 1;
+        P.inputs.push_back(id);
+    }
+    for (int i = 0; i < d->n_outputs; ++i) {
+        int id = d->output_ids[i];
+        if (id < 0 || id >= nt) return fail(BYOC_ERR_INVALID_ARG, "output id %d out of range", id);
+        if (is_output[id]) return fail(BYOC_ERR_INVALID_ARG, "output id %d repeated", id);
+        if (is_input[id]) return fail(BYOC_ERR_INVALID_ARG, "tensor %d is both input and output", id);
+        is_output[id] = 1;
+        P.outputs.push_back(id);
+    }
+    for (int o = 0; o < d->n_ops; ++o) {
+        const byoc_op &op = d->ops[o];
+        if (op.kind < BYOC_OP_CONV2D || op.kind > BYOC_OP_ADD)
+            return fail(BYOC_ERR_INVALID_ARG, "op %d: unknown kind %d", o, op.kind);
+        const int want_in = op.kind == BYOC_OP_ADD ? 2 : 1;
+        if (op.n_in != want_in)
+            return fail(BYOC_ERR_INVALID_ARG, "op %d: %d inputs, expected %d", o, op.n_in, want_in);
+        for (int k = 0; k < op.n_in; ++k) {
+            int id = op.in[k];
+            if (id < 0 || id >= nt) return fail(BYOC_ERR_INVALID_ARG, "op %d: input id %d", o, id);
+            if (!is_input[id] && producer[id] < 0)
+                return fail(BYOC_ERR_INVALID_ARG,
+                            "op %d reads tensor %d before any op produces it (ops must be in "
+                            "topological order)",
+                            o, id);
+        }
+        if (op.out < 0 || op.out >= nt) return fail(BYOC_ERR_INVALID_ARG, "op %d: output id", o);
+        if (is_input[op.out] || producer[op.out] >= 0)
+            return fail(BYOC_ERR_INVALID_ARG, "op %d: tensor %d produced twice", o, op.out);
+        producer[op.out] = o;
+        const TensorInfo &X = P.tensors[op.in[0]];
+        const TensorInfo &Y = P.tensors[op.out];
+        auto same_shape = [](const TensorInfo &a, const TensorInfo &b) {
+            if (a.ndim != b.ndim) return false;
+            for (int k = 0; k < a.ndim; ++k)
+                if (a.shape[k] != b.shape[k]) return false;
+            return true;
+        };
+        switch (op.kind) {
+            case BYOC_OP_CONV2D: {
+                if (X.ndim != 4 || Y.ndim != 4)
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: conv2d needs NHWC tensors", o);
+                if (!op.consts[0]) return fail(BYOC_ERR_INVALID_ARG, "op %d: conv2d weight is null", o);
+                if (op.kernel[0] < 1 || op.kernel[1] < 1 || op.stride[0] < 1 || op.stride[1] < 1 ||
+                    op.dilation[0] < 1 || op.dilation[1] < 1 || op.groups < 1 || op.pad[0] < 0 ||
+                    op.pad[1] < 0 || op.pad[2] < 0 || op.pad[3] < 0)
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: bad conv2d attributes", o);
+                const int64_t C = X.shape[3], K = Y.shape[3];
+                if (C % op.groups || K % op.groups)
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: channels not divisible by groups", o);
+                const int64_t Ho = (X.shape[1] + op.pad[0] + op.pad[2] -
+                                    (int64_t)op.dilation[0] * (op.kernel[0] - 1) - 1) /
+                                       op.stride[0] + 1;
+                const int64_t Wo = (X.shape[2] + op.pad[1] + op.pad[3] -
+                                    (int64_t)op.dilation[1] * (op.kernel[1] - 1) - 1) /
+                                       op.stride[1] + 1;
+                if (Y.shape[0] != X.shape[0] || Y.shape[1] != Ho || Y.shape[2] != Wo || Ho < 1 ||
+                    Wo < 1)
+                    return fail(BYOC_ERR_INVALID_ARG,
+                                "op %d: conv2d output shape [%lld,%lld,%lld,%lld] does not match "
+                                "[%lld,%lld,%lld,%lld]",
+                                o, (long long)Y.shape[0], (long long)Y.shape[1],
+                                (long long)Y.shape[2], (long long)Y.shape[3], (long long)X.shape[0],
+                                (long long)Ho, (long long)Wo, (long long)K);
+                break;
+            }
+            case BYOC_OP_DENSE:
+                if (X.ndim != 2 || Y.ndim != 2 || X.shape[0] != Y.shape[0])
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: dense needs [M,I] -> [M,U]", o);
+                if (!op.consts[0]) return fail(BYOC_ERR_INVALID_ARG, "op %d: dense weight is null", o);
+                break;
+            case BYOC_OP_BIAS_ADD:
+                if (!op.consts[0]) return fail(BYOC_ERR_INVALID_ARG, "op %d: bias is null", o);
+                if (!same_shape(X, Y)) return fail(BYOC_ERR_INVALID_ARG, "op %d: shape mismatch", o);
+                break;
+            case BYOC_OP_BATCH_NORM:
+                for (int k = 0; k < 4; ++k)
+                    if (!op.consts[k])
+                        return fail(BYOC_ERR_INVALID_ARG, "op %d: batch_norm constant %d is null", o, k);
+                if (!(op.eps >= 0.0f)) return fail(BYOC_ERR_INVALID_ARG, "op %d: eps < 0", o);
+                if (!same_shape(X, Y)) return fail(BYOC_ERR_INVALID_ARG, "op %d: shape mismatch", o);
+                for (int64_t c = 0; c < X.channels(); ++c)
+                    if (!((double)op.consts[3][c] + op.eps > 0.0))
+                        return fail(BYOC_ERR_INVALID_ARG, "op %d: var + eps <= 0 at channel %lld", o,
+                                    (long long)c);
+                break;
+            case BYOC_OP_ADD:
+                if (!same_shape(X, Y) || !same_shape(P.tensors[op.in[1]], Y))
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: add operands differ in shape", o);
+                break;
+            default:
+                if (!same_shape(X, Y)) return fail(BYOC_ERR_INVALID_ARG, "op %d: shape mismatch", o);
+        }
+    }
+    for (int id : P.outputs)
+        if (producer[id] < 0)
+            return fail(BYOC_ERR_INVALID_ARG, "output tensor %d is produced by no op", id);
+    return BYOC_OK;
+}
+
+// ------------------------------------------------------------ planning
+
+int pick_bk(int64_t C) {
+    if (C <= 16) return 16;
+    if (C <= 32) return 32;
+    return 64;
+}
+
+// Choose the output-channel tile among the compiled configurations: fewest
+// rounds of the persistent grid, weighted by the tile's width (its MMA time)
+// plus a fixed per-tile cost.
+int pick_bn(int64_t M, int64_t N, int64_t ksteps, int bk, bool im2col, int num_sms) {
+    int best = -1;
+    double best_cost = 1e300;
+    for (int bn : {256, 128, 64, 32}) {
+        GemmConfig c{bn, bk, im2col};
+        if (!byoc::gemm_config_supported(c)) continue;
+        const int64_t tiles = ((M + 127) / 128) * ((N + bn - 1) / bn);
+        const int64_t grid = std::min<int64_t>(tiles, num_sms);
+        const int64_t rounds = (tiles + grid - 1) / grid;
+        // Per 16-deep k-step a 128 x bn MMA needs bn/2 tensor-core cycles and
+        // streams (128 + bn) x 32 B of operands through shared memory at
+        // ~128 B/cycle; a tile also pays a fixed fill / epilogue cost.
+        const double step = std::max(bn / 2.0, 32.0 + bn / 4.0);
+        const double cost = (double)rounds * (step * (double)ksteps + 400.0);
+        if (cost < best_cost - 1e-9) {
+            best_cost = cost;
+            best = bn;
+        }
+    }
+    return best;
+}
+
+struct Affine {
+    std::vector<double> scale, shift;
+};
+
+// Builds the launch list (no device work).
+byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
+    P = Plan();
+    P.num_sms = num_sms > 0 ? num_sms : 148;
+    byoc_status st = validate(d, P);
+    if (st != BYOC_OK) return st;
+    const int nt = d->n_tensors;
+    std::vector<int> consumers(nt, 0), is_output(nt, 0), is_input(nt, 0);
+    for (int o = 0; o < d->n_ops; ++o)
+        for (int k = 0; k < d->ops[o].n_in; ++k) consumers[d->ops[o].in[k]]++;
+    for (int id : P.outputs) is_output[id] = 1;
+    for (int id : P.inputs) is_input[id] = 1;
+
+    int o = 0;
+    while (o < d->n_ops) {
+        const byoc_op &op = d->ops[o];
+        if (op.kind != BYOC_OP_CONV2D && op.kind != BYOC_OP_DENSE)
+            return fail(BYOC_ERR_UNSUPPORTED,
+                        "op %d (kind %d) is not preceded by a conv2d/dense it can fuse into; "
+                        "standalone elementwise ops stay on the host",
+                        o, op.kind);
+        if ((int)P.launches.size() >= BYOC_PLAN_MAX_LAUNCHES - 1)
+            return fail(BYOC_ERR_UNSUPPORTED, "region needs more than %d launches",
+                        BYOC_PLAN_MAX_LAUNCHES - 1);
+        const TensorInfo X = P.tensors[op.in[0]];
+        const TensorInfo Yp = P.tensors[op.out];
+        const int64_t Cout = Yp.channels();
+        // ---------------- epilogue chain
+        Affine af;
+        af.scale.assign(Cout, 1.0);
+        af.shift.assign(Cout, 0.0);
+        int cur = op.out, res = -1, act = byoc::kActNone, stage = 0, j = o + 1;
+        for (; j < d->n_ops; ++j) {
+            const byoc_op &nx = d->ops[j];
+            const bool reads_cur = nx.in[0] == cur || (nx.kind == BYOC_OP_ADD && nx.in[1] == cur);
+            if (!reads_cur || consumers[cur] != 1 || is_output[cur]) break;
+            if (nx.kind == BYOC_OP_BIAS_ADD && stage == 0) {
+                for (int64_t c = 0; c < Cout; ++c) af.shift[c] += (double)nx.consts[0][c];
+            } else if (nx.kind == BYOC_OP_BATCH_NORM && stage == 0) {
+                for (int64_t c = 0; c < Cout; ++c) {
+                    const double s = (double)nx.consts[0][c] /
+                                     std::sqrt((double)nx.consts[3][c] + (double)nx.eps);
+                    af.scale[c] *= s;
+                    af.shift[c] = af.shift[c] * s + ((double)nx.consts[1][c] - s * (double)nx.consts[2][c]);
+                }
+            } else if (nx.kind == BYOC_OP_ADD && stage == 0) {
+                res = nx.in[0] == cur ? nx.in[1] : nx.in[0];
+                if (res == cur) break;  // x + x: not a residual pattern
+                stage = 1;
+            } else if ((nx.kind == BYOC_OP_RELU || nx.kind == BYOC_OP_RELU6 ||
+                        nx.kind == BYOC_OP_GELU) && stage <= 1) {
+                act = nx.kind == BYOC_OP_RELU ? byoc::kActRelu
+                                              : (nx.kind == BYOC_OP_RELU6 ? byoc::kActRelu6
+                                                                          : byoc::kActGelu);
+                stage = 2;
+            } else {
+                break;
+            }
+            cur = nx.out;
+        }
+        const TensorInfo Y = P.tensors[cur];
+        LaunchPlan L;
+        L.first_op = o;
+        L.n_ops = j - o;
+        L.x = op.in[0];
+        L.y = cur;
+        L.res = res;
+        L.act = act;
+        if (Cout % 8)
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: %lld output channels (multiple of 8 needed)",
+                        o, (long long)Cout);
+
+        if (op.kind == BYOC_OP_CONV2D && op.groups > 1) {
+            // ---------------- depthwise
+            const int64_t C = X.channels();
+            if (op.groups != C || Cout != C)
+                return fail(BYOC_ERR_UNSUPPORTED, "op %d: grouped conv other than depthwise", o);
+            if (op.kernel[0] != 3 || op.kernel[1] != 3 || op.dilation[0] != 1 ||
+                op.dilation[1] != 1 || op.stride[0] != op.stride[1] ||
+                (op.stride[0] != 1 && op.stride[0] != 2) || op.pad[0] != op.pad[1] ||
+                op.pad[0] != op.pad[2] || op.pad[1] != op.pad[3])
+                return fail(BYOC_ERR_UNSUPPORTED,
+                            "op %d: depthwise supports 3x3, stride 1|2, symmetric padding", o);
+            if (res >= 0) return fail(BYOC_ERR_UNSUPPORTED, "op %d: residual add after depthwise", o);
+            L.kind = BYOC_LAUNCH_DEPTHWISE;
+            std::vector<float> w(9 * C), b(C);
+            for (int64_t c = 0; c < C; ++c) {
+                for (int t = 0; t < 9; ++t)
+                    w[t * C + c] = (float)((double)op.consts[0][c * 9 + t] * af.scale[c]);
+                b[c] = (float)af.shift[c];
+            }
+            L.w_off = blob_append(P.blob, w.data(), w.size() * 4);
+            L.w_bytes = w.size() * 4;
+            L.b_off = blob_append(P.blob, b.data(), b.size() * 4);
+            L.b_bytes = b.size() * 4;
+            L.dw.N = (int)X.shape[0];
+            L.dw.H = (int)X.shape[1];
+            L.dw.W = (int)X.shape[2];
+            L.dw.C = (int)C;
+            L.dw.Ho = (int)Y.shape[1];
+            L.dw.Wo = (int)Y.shape[2];
+            L.dw.stride = op.stride[0];
+            L.dw.pad = op.pad[0];
+            L.dw.act = act;
+            L.flops = 2.0 * (double)Y.elems() * 9.0;
+            L.bytes = (double)X.bytes() + (double)Y.bytes() + (double)(w.size() + b.size()) * 4;
+            P.launches.push_back(L);
+            o = j;
+            continue;
+        }
+
+        // ---------------- GEMM (conv2d groups=1, or dense)
+        int64_t M, Kreal;
+        int kh = 1, kw = 1, taps = 1, chunks, bk;
+        int64_t C;
+        std::vector<double> wsrc;  // weights as [Cout][kh][kw][C] (channel innermost)
+        bool im2col = false;
+        if (op.kind == BYOC_OP_DENSE) {
+            C = X.shape[1];
+            M = X.shape[0];
+            if (C % 8)
+                return fail(BYOC_ERR_UNSUPPORTED, "op %d: dense input width %lld (multiple of 8)", o,
+                            (long long)C);
+            wsrc.assign(op.consts[0], op.consts[0] + Cout * C);
+            L.aM = M;
+            L.aK = C;
+        } else {
+            C = X.channels();
+            kh = op.kernel[0];
+            kw = op.kernel[1];
+            M = Y.shape[0] * Y.shape[1] * Y.shape[2];
+            const bool square = kh == kw && op.stride[0] == op.stride[1] &&
+                                op.dilation[0] == op.dilation[1] && op.pad[0] == op.pad[1] &&
+                                op.pad[2] == op.pad[3];
+            if (C % 8) {
+                // Few-channel stride-2 stem: space-to-depth boundary transform, then a
+                // stride-1 (kh+1)/2 square conv over 16 channels.
+                if (!(square && op.stride[0] == 2 && op.dilation[0] == 1 && C <= 4 && (kh % 2) == 1))
+                    return fail(BYOC_ERR_UNSUPPORTED,
+                                "op %d: %lld input channels: only a stride-2 odd square stem with "
+                                "<= 4 channels is supported",
+                                o, (long long)C);
+                const int k2 = (kh + 1) / 2;
+                TensorInfo Z;
+                Z.ndim = 4;
+                Z.shape[0] = X.shape[0];
+                Z.shape[1] = Y.shape[1] + k2 - 1;
+                Z.shape[2] = Y.shape[2] + k2 - 1;
+                Z.shape[3] = 16;
+                const int zid = (int)P.tensors.size();
+                P.tensors.push_back(Z);
+                LaunchPlan S;
+                S.kind = BYOC_LAUNCH_S2D;
+                S.x = op.in[0];
+                S.y = zid;
+                S.s2d.N = (int)X.shape[0];
+                S.s2d.H = (int)X.shape[1];
+                S.s2d.W = (int)X.shape[2];
+                S.s2d.C = (int)C;
+                S.s2d.Hz = (int)Z.shape[1];
+                S.s2d.Wz = (int)Z.shape[2];
+                S.s2d.Cz = 16;
+                S.s2d.pad = op.pad[0];
+                S.bytes = (double)X.bytes() + (double)Z.bytes();
+                P.launches.push_back(S);
+                // Remapped weights w'[k][a][b][(dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx].
+                wsrc.assign((size_t)Cout * k2 * k2 * 16, 0.0);
+                for (int64_t k = 0; k < Cout; ++k)
+                    for (int a = 0; a < k2; ++a)
+                        for (int b = 0; b < k2; ++b)
+                            for (int dy = 0; dy < 2; ++dy)
+                                for (int dx = 0; dx < 2; ++dx)
+                                    for (int64_t c = 0; c < C; ++c) {
+                                        const int r = 2 * a + dy, s = 2 * b + dx;
+                                        if (r >= kh || s >= kw) continue;
+                                        wsrc[((k * k2 + a) * k2 + b) * 16 + (dy * 2 + dx) * C + c] =
+                                            op.consts[0][((k * C + c) * kh + r) * kw + s];
+                                    }
+                L.x = zid;
+                C = 16;
+                kh = kw = k2;
+                im2col = true;
+                L.aN = (int)Z.shape[0];
+                L.aH = (int)Z.shape[1];
+                L.aW = (int)Z.shape[2];
+                L.aC = 16;
+                L.ksz = k2;
+                L.kstride = 1;
+                L.pad_lo = 0;
+                L.pad_hi = 0;
+                L.dil = 1;
+                L.args.stride_h = L.args.stride_w = 1;
+                L.args.pad_t = L.args.pad_l = 0;
+                L.args.dil_h = L.args.dil_w = 1;
+            } else {
+                wsrc.assign((size_t)Cout * kh * kw * C, 0.0);
+                for (int64_t k = 0; k < Cout; ++k)
+                    for (int r = 0; r < kh; ++r)
+                        for (int s = 0; s < kw; ++s)
+                            for (int64_t c = 0; c < C; ++c)
+                                wsrc[((k * kh + r) * kw + s) * C + c] =
+                                    op.consts[0][((k * C + c) * kh + r) * kw + s];
+                const bool plain = kh == 1 && kw == 1 && op.stride[0] == 1 && op.stride[1] == 1 &&
+                                   op.pad[0] == 0 && op.pad[1] == 0 && op.pad[2] == 0 &&
+                                   op.pad[3] == 0;
+                if (plain) {
+                    L.aM = M;
+                    L.aK = C;
+                } else {
+                    if (!square)
+                        return fail(BYOC_ERR_UNSUPPORTED,
+                                    "op %d: implicit GEMM needs a square kernel with equal "
+                                    "strides, dilations and symmetric padding",
+                                    o);
+                    const int lo = op.pad[0], hi = op.pad[2];
+                    const int up = hi - (kh - 1) * op.dilation[0];
+                    if (lo > 128 || up < -128 || up > 127)
+                        return fail(BYOC_ERR_UNSUPPORTED, "op %d: padding outside TMA im2col range", o);
+                    im2col = true;
+                    L.aN = (int)X.shape[0];
+                    L.aH = (int)X.shape[1];
+                    L.aW = (int)X.shape[2];
+                    L.aC = (int)C;
+                    L.ksz = kh;
+                    L.kstride = op.stride[0];
+                    L.pad_lo = lo;
+                    L.pad_hi = hi;
+                    L.dil = op.dilation[0];
+                    L.args.stride_h = L.args.stride_w = op.stride[0];
+                    L.args.pad_t = L.args.pad_l = lo;
+                    L.args.dil_h = L.args.dil_w = op.dilation[0];
+                }
+            }
+        }
+        taps = kh * kw;
+        bk = op.kind == BYOC_OP_DENSE ? 64 : pick_bk(C);
+        chunks = (int)((C + bk - 1) / bk);
+        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks * bk / 16, bk, im2col, P.num_sms);
+        if (bn < 0)
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d im2col=%d", o, bk,
+                        (int)im2col);
+        L.cfg = GemmConfig{bn, bk, im2col};
+        L.n_pad = (int)((Cout + bn - 1) / bn * bn);
+        L.k_pack = taps * chunks * bk;
+        Kreal = (int64_t)taps * C;
+        // Folded, bf16-rounded, K-major packed weights [n_pad][k_pack].
+        std::vector<uint16_t> wp((size_t)L.n_pad * L.k_pack, 0);
+        for (int64_t k = 0; k < Cout; ++k)
+            for (int t = 0; t < taps; ++t)
+                for (int64_t c = 0; c < C; ++c) {
+                    const double v = wsrc[((size_t)k * taps + t) * C + c] * af.scale[k];
+                    const size_t col = ((size_t)t * chunks + c / bk) * bk + c % bk;
+                    wp[(size_t)k * L.k_pack + col] = f32_to_bf16_rne((float)v);
+                }
+        std::vector<float> bias((size_t)L.n_pad, 0.0f);
+        for (int64_t k = 0; k < Cout; ++k) bias[k] = (float)af.shift[k];
+        L.w_off = blob_append(P.blob, wp.data(), wp.size() * 2);
+        L.w_bytes = wp.size() * 2;
+        L.b_off = blob_append(P.blob, bias.data(), bias.size() * 4);
+        L.b_bytes = bias.size() * 4;
+
+        GemmArgs &A = L.args;
+        A.M = (int)M;
+        A.N = (int)Cout;
+        A.num_kb = taps * chunks;
+        A.chunks = chunks;
+        A.kw = kw;
+        if (!im2col) {
+            A.dil_h = A.dil_w = 1;
+            A.stride_h = A.stride_w = 1;
+        }
+        A.Ho = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[1];
+        A.Wo = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[2];
+        A.tiles_n = L.n_pad / bn;
+        A.num_tiles = (int)(((M + 127) / 128) * A.tiles_n);
+        A.act = act;
+        L.grid = std::min(A.num_tiles, P.num_sms);
+        L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
+        const double in_bytes = L.x < P.n_region_tensors ? (double)X.bytes()
+                                                         : (double)P.tensors[L.x].bytes();
+        L.bytes = in_bytes + (double)Y.bytes() + (double)Cout * Kreal * 2 + (double)Cout * 4 +
+                  (res >= 0 ? (double)P.tensors[res].bytes() : 0.0);
+        P.launches.push_back(L);
+        o = j;
+    }
+    // Workspace: every tensor that is neither a region input nor output.
+    P.ws_off.assign(P.tensors.size(), SIZE_MAX);
+    size_t ws = 256;  // [0, 256): device error word
+    for (size_t t = 0; t < P.tensors.size(); ++t) {
+        const bool boundary = (int)t < nt && (is_input[t] || is_output[t]);
+        if (boundary) continue;
+        bool used = false;
+        for (const LaunchPlan &L : P.launches) used |= (L.x == (int)t || L.y == (int)t || L.res == (int)t);
+        if (!used) continue;
+        P.ws_off[t] = ws;
+        ws = align_up(ws + P.tensors[t].bytes(), 256);
+    }
+    P.ws_bytes = ws;
+    for (const LaunchPlan &L : P.launches) {
+        P.flops += L.flops;
+        P.bytes += L.bytes;
+    }
+    return BYOC_OK;
+}
+
+void fill_report(const Plan &P, byoc_plan_report *r) {
+    std::memset(r, 0, sizeof *r);
+    r->n_launches = (int32_t)P.launches.size();
+    for (size_t i = 0; i < P.launches.size(); ++i) {
+        const LaunchPlan &L = P.launches[i];
+        r->kind[i] = L.kind;
+        r->first_op[i] = L.first_op;
+        r->n_ops[i] = L.n_ops;
+        r->act[i] = L.act;
+        r->residual[i] = L.res;
+        r->gemm_m[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.M : 0;
+        r->gemm_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.N : 0;
+        r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : 0;
+        r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : 0;
+        r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : 0;
+        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? (int)L.cfg.im2col : 0;
+        r->grid[i] = L.grid;
+    }
+    r->flops = P.flops;
+    r->bytes = P.bytes;
+    r->const_bytes = P.blob.size();
+    r->workspace_bytes = P.ws_bytes;
+}
+
+}  // namespace
+
+// ------------------------------------------------------------ the handle
+
+struct byoc_handle {
+    Plan P;
+    uint8_t *d_const = nullptr;
+    uint8_t *d_ws = nullptr;
+    int *d_err = nullptr;
+    int device = 0;
+    std::vector<CUtensorMap> tmB;         // per launch (GEMM only)
+    std::vector<CUtensorMap> tmA;         // per launch, cached
+    std::vector<const void *> tmA_ptr;    // pointer each cached A map encodes
+    std::vector<void *> ptrs;             // scratch: resolved tensor pointers
+};
+
+extern "C" {
+
+const char *byoc_last_error(void) { return g_err.c_str(); }
+
+byoc_status byoc_plan(const byoc_region_desc *desc, int32_t num_sms, byoc_plan_report *rep) {
+    if (!rep) return fail(BYOC_ERR_INVALID_ARG, "null report");
+    Plan P;
+    byoc_status st = plan_region(desc, num_sms, P);
+    if (st != BYOC_OK) return st;
+    fill_report(P, rep);
+    return BYOC_OK;
+}
+
+byoc_status byoc_plan_constants(const byoc_region_desc *desc, int32_t num_sms, int32_t launch,
+                                int32_t what, void *dst, size_t dst_bytes, size_t *needed) {
+    Plan P;
+    byoc_status st = plan_region(desc, num_sms, P);
+    if (st != BYOC_OK) return st;
+    if (launch < 0 || launch >= (int)P.launches.size())
+        return fail(BYOC_ERR_INVALID_ARG, "launch %d out of range", launch);
+    const LaunchPlan &L = P.launches[launch];
+    if (L.kind == BYOC_LAUNCH_S2D) return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants", launch);
+    const size_t off = what == 0 ? L.w_off : L.b_off;
+    const size_t n = what == 0 ? L.w_bytes : L.b_bytes;
+    if (needed) *needed = n;
+    if (!dst) return BYOC_OK;
+    if (dst_bytes < n) return fail(BYOC_ERR_INVALID_ARG, "destination too small (%zu < %zu)", dst_bytes, n);
+    std::memcpy(dst, P.blob.data() + off, n);
+    return BYOC_OK;
+}
+
+byoc_status byoc_device_info(int32_t *num_sms, int32_t *cc_major, int32_t *cc_minor) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "cudaGetDevice");
+    int v = 0;
+    if (num_sms) {
+        if ((e = cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess)
+            return cuda_fail(e, "cudaDeviceGetAttribute");
+        *num_sms = v;
+    }
+    if (cc_major) {
+        if ((e = cudaDeviceGetAttribute(&v, cudaDevAttrComputeCapabilityMajor, dev)) != cudaSuccess)
+            return cuda_fail(e, "cudaDeviceGetAttribute");
+        *cc_major = v;
+    }
+    if (cc_minor) {
+        if ((e = cudaDeviceGetAttribute(&v, cudaDevAttrComputeCapabilityMinor, dev)) != cudaSuccess)
+            return cuda_fail(e, "cudaDeviceGetAttribute");
+        *cc_minor = v;
+    }
+    return BYOC_OK;
+}
+
+void byoc_release(byoc_handle *h) {
+    if (!h) return;
+    int cur = -1;
+    cudaGetDevice(&cur);
+    if (cur != h->device) cudaSetDevice(h->device);
+    if (h->d_const) cudaFree(h->d_const);
+    if (h->d_ws) cudaFree(h->d_ws);
+    if (cur >= 0 && cur != h->device) cudaSetDevice(cur);
+    delete h;
+}
+
+byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
+    if (!out) return fail(BYOC_ERR_INVALID_ARG, "null output handle pointer");
+    *out = nullptr;
+    int32_t sms = 0, ccM = 0, ccm = 0;
+    byoc_status st = byoc_device_info(&sms, &ccM, &ccm);
+    if (st != BYOC_OK) return st;
+    if (ccM != 10 || ccm != 3)
+        return fail(BYOC_ERR_UNSUPPORTED, "device is sm_%d%d; this library is built for sm_103a", ccM, ccm);
+    cudaError_t e = load_driver();
+    if (e != cudaSuccess) return cuda_fail(e, "driver entry points for TMA descriptors");
+    byoc_handle *h = new (std::nothrow) byoc_handle();
+    if (!h) return fail(BYOC_ERR_OOM, "host allocation");
+    st = plan_region(desc, sms, h->P);
+    if (st != BYOC_OK) {
+        delete h;
+        return st;
+    }
+    cudaGetDevice(&h->device);
+    Plan &P = h->P;
+    if (!P.blob.empty()) {
+        if ((e = cudaMalloc(&h->d_const, P.blob.size())) != cudaSuccess) {
+            byoc_release(h);
+            return cuda_fail(e, "cudaMalloc(constants)");
+        }
+        if ((e = cudaMemcpy(h->d_const, P.blob.data(), P.blob.size(), cudaMemcpyHostToDevice)) !=
+            cudaSuccess) {
+            byoc_release(h);
+            return cuda_fail(e, "cudaMemcpy(constants)");
+        }
+    }
+    if ((e = cudaMalloc(&h->d_ws, P.ws_bytes)) != cudaSuccess) {
+        byoc_release(h);
+        return cuda_fail(e, "cudaMalloc(workspace)");
+    }
+    if ((e = cudaMemset(h->d_ws, 0, 256)) != cudaSuccess) {
+        byoc_release(h);
+        return cuda_fail(e, "cudaMemset(error word)");
+    }
+    h->d_err = reinterpret_cast<int *>(h->d_ws);
+    const size_t nl = P.launches.size();
+    h->tmB.resize(nl);
+    h->tmA.resize(nl);
+    h->tmA_ptr.assign(nl, nullptr);
+    h->ptrs.assign(P.tensors.size(), nullptr);
+    for (size_t i = 0; i < nl; ++i) {
+        LaunchPlan &L = P.launches[i];
+        if (L.kind == BYOC_LAUNCH_GEMM) {
+            L.args.bias = reinterpret_cast<const float *>(h->d_const + L.b_off);
+            L.args.err = h->d_err;
+            CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
+                                   (uint64_t)L.k_pack, (uint32_t)L.cfg.bn, (uint32_t)L.cfg.bk,
+                                   L.cfg.bk);
+            if (r != CUDA_SUCCESS) {
+                byoc_release(h);
+                return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(weights) = %d", i, (int)r);
+            }
+            if ((e = byoc::gemm_prepare(L.cfg)) != cudaSuccess) {
+                byoc_release(h);
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            }
+        } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
+            L.dw.w = reinterpret_cast<const float *>(h->d_const + L.w_off);
+            L.dw.bias = reinterpret_cast<const float *>(h->d_const + L.b_off);
+        }
+    }
+    *out = h;
+    return BYOC_OK;
+}
+
+byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *outputs,
+                     void *cuda_stream) {
+    if (!h) return fail(BYOC_ERR_INVALID_ARG, "null handle");
+    Plan &P = h->P;
+    if (!inputs || !outputs) return fail(BYOC_ERR_INVALID_ARG, "null input/output array");
+    cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+    for (size_t i = 0; i < P.inputs.size(); ++i) {
+        const void *p = inputs[i];
+        if (!p || (reinterpret_cast<uintptr_t>(p) & 15u))
+            return fail(BYOC_ERR_INVALID_ARG, "input %zu: null or not 16-byte aligned", i);
+        h->ptrs[P.inputs[i]] = const_cast<void *>(p);
+    }
+    for (size_t i = 0; i < P.outputs.size(); ++i) {
+        void *p = outputs[i];
+        if (!p || (reinterpret_cast<uintptr_t>(p) & 15u))
+            return fail(BYOC_ERR_INVALID_ARG, "output %zu: null or not 16-byte aligned", i);
+        h->ptrs[P.outputs[i]] = p;
+    }
+    for (size_t t = 0; t < P.tensors.size(); ++t)
+        if (P.ws_off[t] != SIZE_MAX) h->ptrs[t] = h->d_ws + P.ws_off[t];
+
+    for (size_t i = 0; i < P.launches.size(); ++i) {
+        LaunchPlan &L = P.launches[i];
+        cudaError_t e = cudaSuccess;
+        if (L.kind == BYOC_LAUNCH_GEMM) {
+            const void *xa = h->ptrs[L.x];
+            if (h->tmA_ptr[i] != xa) {
+                CUresult r;
+                if (L.cfg.im2col)
+                    r = encode_im2col(&h->tmA[i], xa, L.aN, L.aH, L.aW, L.aC, L.ksz, L.kstride,
+                                      L.pad_lo, L.pad_hi, L.dil, L.cfg.bk);
+                else
+                    r = encode_2d(&h->tmA[i], xa, (uint64_t)L.aM, (uint64_t)L.aK, byoc::kGemmBM,
+                                  (uint32_t)L.cfg.bk, L.cfg.bk);
+                if (r != CUDA_SUCCESS)
+                    return fail(BYOC_ERR_CUDA, "launch %zu: encoding the activation TMA map failed (%d)",
+                                i, (int)r);
+                h->tmA_ptr[i] = xa;
+            }
+            GemmArgs a = L.args;
+            a.out = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
+            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a, L.grid, st);
+        } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
+            byoc::DwArgs a = L.dw;
+            a.x = static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]);
+            a.y = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            e = byoc::launch_dwconv(a, P.num_sms, st);
+        } else {
+            byoc::S2dArgs a = L.s2d;
+            a.x = static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]);
+            a.z = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            e = byoc::launch_s2d(a, st);
+        }
+        if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
+    }
+    return BYOC_OK;
+}
+
+byoc_status byoc_check(byoc_handle *h) {
+    if (!h) return fail(BYOC_ERR_INVALID_ARG, "null handle");
+    int v = 0;
+    cudaError_t e = cudaMemcpy(&v, h->d_err, sizeof v, cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(e, "reading the error word");
+    if (v != 0) {
+        cudaMemset(h->d_err, 0, sizeof v);
+        return fail(BYOC_ERR_TIMEOUT, "a kernel's bounded wait expired (code %d)", v);
+    }
+    return BYOC_OK;
+}
+
+byoc_status byoc_query(const byoc_handle *h, byoc_info *info) {
+    if (!h || !info) return fail(BYOC_ERR_INVALID_ARG, "null handle or info");
+    const Plan &P = h->P;
+    info->flops = P.flops;
+    info->bytes = P.bytes;
+    info->workspace_bytes = P.ws_bytes;
+    info->const_bytes = P.blob.size();
+    info->n_launches = (int32_t)P.launches.size();
+    info->n_inputs = (int32_t)P.inputs.size();
+    info->n_outputs = (int32_t)P.outputs.size();
+    return BYOC_OK;
+}
+
+byoc_status byoc_max_pool2d_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W, int32_t C,
+                                 int32_t k, int32_t s, int32_t p, void *cuda_stream) {
+    if (!x || !y || ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u))
+        return fail(BYOC_ERR_INVALID_ARG, "max_pool2d: null or misaligned pointer");
+    if (N < 1 || H < 1 || W < 1 || C < 8 || C % 8 || k < 1 || s < 1 || p < 0 || p >= k ||
+        H + 2 * p < k || W + 2 * p < k)
+        return fail(BYOC_ERR_INVALID_ARG, "max_pool2d: bad shape");
+    cudaError_t e = byoc::launch_maxpool(static_cast<const __nv_bfloat16 *>(x),
+                                         static_cast<__nv_bfloat16 *>(y), N, H, W, C, k, s, p,
+                                         static_cast<cudaStream_t>(cuda_stream));
+    return e == cudaSuccess ? BYOC_OK : cuda_fail(e, "max_pool2d launch");
+}
+
+byoc_status byoc_global_avg_pool_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W,
+                                      int32_t C, void *cuda_stream) {
+    if (!x || !y || ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u))
+        return fail(BYOC_ERR_INVALID_ARG, "global_avg_pool: null or misaligned pointer");
+    if (N < 1 || H < 1 || W < 1 || C < 8 || C % 8)
+        return fail(BYOC_ERR_INVALID_ARG, "global_avg_pool: bad shape");
+    cudaError_t e = byoc::launch_avgpool(static_cast<const __nv_bfloat16 *>(x),
+                                         static_cast<__nv_bfloat16 *>(y), N, H, W, C,
+                                         static_cast<cudaStream_t>(cuda_stream));
+    return e == cudaSuccess ? BYOC_OK : cuda_fail(e, "global_avg_pool launch");
+}
+
+}  // extern "C"

@@ -169,6 +169,10 @@ class _Builder:
         N, H, W, C = self.g.shape_of(x)
         return self._add("nn.global_avg_pool2d", [x], (N, C))
 
+    def batch_flatten(self, x):
+        shp = self.g.shape_of(x)
+        return self._add("nn.batch_flatten", [x], (shp[0], int(np.prod(shp[1:]))))
+
 
 def _draw_constants(g: Graph, rng: np.random.Generator) -> None:
     """Weights in node order, then biases / BN statistics in node order."""
@@ -204,8 +208,10 @@ def _draw_inputs(g: Graph, rng: np.random.Generator) -> Dict[str, np.ndarray]:
     return out
 
 
-def _finish(b: _Builder, outputs: List[str], seed: int):
+def _finish(b: _Builder, outputs: List[str], seed: int, draw: bool = True):
     b.g.outputs = list(outputs)
+    if not draw:
+        return b.g, {}
     rng = np.random.Generator(np.random.PCG64(seed))
     inputs = _draw_inputs(b.g, rng)
     _draw_constants(b.g, rng)
@@ -276,7 +282,7 @@ def resnet_bottleneck(N=32, H=14, W=14, C=1024, width=256, stride=1, seed=3):
 RESNET50_STAGES = ((3, 64, 1), (4, 128, 2), (6, 256, 2), (3, 512, 2))
 
 
-def resnet50(N=64, H=224, W=224, num_classes=1000, seed=4, stages=RESNET50_STAGES):
+def resnet50(N=64, H=224, W=224, num_classes=1000, seed=4, stages=RESNET50_STAGES, draw=True):
     """ResNet-50 v1b backbone + classifier: 53 convolutions, 1 dense."""
     b = _Builder("resnet50_v1b")
     x = b.input("data", (N, H, W, 3))
@@ -290,7 +296,66 @@ def resnet50(N=64, H=224, W=224, num_classes=1000, seed=4, stages=RESNET50_STAGE
             cin = 4 * width
     p = b.global_avg_pool2d(t)
     y = b.bias_add(b.dense(p, num_classes, init="kaiming"))
-    return _finish(b, [y], seed)
+    return _finish(b, [y], seed, draw)
+
+
+def resnet18(N=1, H=224, W=224, num_classes=1000, seed=5, draw=False):
+    """ResNet-18: basic blocks (3x3 conv-BN-ReLU, 3x3 conv-BN, add, ReLU)."""
+    b = _Builder("resnet18")
+    x = b.input("data", (N, H, W, 3))
+    t = b.max_pool2d(b.relu(b.batch_norm(b.conv2d(x, 64, 7, stride=2, pad=3))), 3, 2, 1)
+    cin = 64
+    for i, width in enumerate((64, 128, 256, 512)):
+        for j in range(2):
+            s = 2 if (i > 0 and j == 0) else 1
+            u = b.relu(b.batch_norm(b.conv2d(t, width, 3, stride=s)))
+            u = b.batch_norm(b.conv2d(u, width, 3))
+            sc = b.batch_norm(b.conv2d(t, width, 1, stride=s, pad=0)) if (s != 1 or cin != width) else t
+            t = b.relu(b.add(u, sc))
+            cin = width
+    y = b.bias_add(b.dense(b.global_avg_pool2d(t), num_classes))
+    return _finish(b, [y], seed, draw)
+
+
+def vgg19(N=1, H=224, W=224, num_classes=1000, seed=6, draw=False):
+    """VGG19: 16 conv3x3 + bias + ReLU in five stages, then three dense layers."""
+    b = _Builder("vgg19")
+    t = b.input("data", (N, H, W, 3))
+    for nconv, width in ((2, 64), (2, 128), (4, 256), (4, 512), (4, 512)):
+        for _ in range(nconv):
+            t = b.relu(b.bias_add(b.conv2d(t, width, 3)))
+        t = b.max_pool2d(t, 2, 2, 0)
+    t = b.batch_flatten(t)
+    t = b.relu(b.bias_add(b.dense(t, 4096)))
+    t = b.relu(b.bias_add(b.dense(t, 4096)))
+    y = b.bias_add(b.dense(t, num_classes))
+    return _finish(b, [y], seed, draw)
+
+
+MOBILENET_V2_BLOCKS = ((1, 16, 1, 1), (6, 24, 2, 2), (6, 32, 3, 2), (6, 64, 4, 2), (6, 96, 3, 1),
+                       (6, 160, 3, 2), (6, 320, 1, 1))
+
+
+def mobilenet_v2(N=1, H=224, W=224, num_classes=1000, seed=7, draw=False):
+    """MobileNetV2 1.0: inverted residual blocks (expand 1x1, depthwise 3x3,
+    project 1x1, residual add when shapes allow), ReLU6 activations."""
+    b = _Builder("mobilenet_v2")
+    x = b.input("data", (N, H, W, 3))
+    t = b.relu6(b.batch_norm(b.conv2d(x, 32, 3, stride=2)))
+    cin = 32
+    for tt, c, n, s in MOBILENET_V2_BLOCKS:
+        for i in range(n):
+            stride = s if i == 0 else 1
+            u = t
+            if tt != 1:
+                u = b.relu6(b.batch_norm(b.conv2d(u, cin * tt, 1)))
+            u = b.relu6(b.batch_norm(b.conv2d(u, cin * tt, 3, stride=stride, groups=cin * tt)))
+            u = b.batch_norm(b.conv2d(u, c, 1))
+            t = b.add(u, t) if (stride == 1 and cin == c) else u
+            cin = c
+    t = b.relu6(b.batch_norm(b.conv2d(t, 1280, 1)))
+    y = b.bias_add(b.dense(b.global_avg_pool2d(t), num_classes))
+    return _finish(b, [y], seed, draw)
 
 
 def small_int_conv(N=2, H=9, W=11, C=64, K=64, k=3, stride=1, pad=1, seed=7, act="relu"):

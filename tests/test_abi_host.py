@@ -1,0 +1,136 @@
+"""CPU tests of the C ABI: the library builds and loads without a GPU,
+exports every function the headers declare, and its host-side planning
+(validation, epilogue fusion, batch-norm folding, weight packing) behaves as
+specified.  No test here calls a CUDA function."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+from paper_2105_03215_gb300 import abi
+from paper_2105_03215_gb300 import inputs as I
+from paper_2105_03215_gb300 import region as R
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _declared_functions():
+    names = set()
+    for h in os.listdir(os.path.join(ROOT, "include")):
+        src = open(os.path.join(ROOT, "include", h)).read()
+        src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+        names.update(re.findall(r"\b(byoc_[a-z0-9_]+)\s*\(", src))
+    return names
+
+
+def test_library_exports_every_declared_function():
+    path = abi.lib().__getattribute__("_name")
+    out = subprocess.run(["nm", "-D", "--defined-only", path], capture_output=True, text=True).stdout
+    exported = set(re.findall(r" T (byoc_\w+)", out))
+    declared = _declared_functions()
+    assert declared, "no declarations parsed"
+    assert declared <= exported, f"declared but not exported: {sorted(declared - exported)}"
+    assert set(abi.declared_symbols()) == declared
+
+
+def _plan(g, **kw):
+    return R.whole_graph_region(g).plan(**kw)
+
+
+def test_plan_fuses_composites_into_launches():
+    rep = _plan(I.resnet_bottleneck(N=2, H=14, W=14, C=256, width=64)[0])
+    assert rep.n_launches == 3
+    assert [rep.n_ops[i] for i in range(3)] == [3, 3, 4]      # conv+bn+relu x2, conv+bn+add+relu
+    assert [rep.act[i] for i in range(3)] == [1, 1, 1]
+    assert rep.residual[2] == 0 and rep.residual[0] == -1     # residual = region input 0
+    assert [rep.im2col[i] for i in range(3)] == [0, 1, 0]     # 1x1 as GEMM, 3x3 as im2col
+    rep = _plan(I.bert_ffn(M=64, D=128, F=256)[0])
+    assert rep.n_launches == 2 and rep.act[0] == 3 and rep.act[1] == 0
+    rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0])
+    assert [rep.kind[i] for i in range(2)] == [abi.LAUNCH_DEPTHWISE, abi.LAUNCH_GEMM]
+    assert rep.act[0] == 2
+
+
+def test_plan_stem_inserts_space_to_depth():
+    g, _ = I.resnet50(N=1, H=32, W=32)
+    rep = R.Region(g, [n.name for n in g.nodes[:3]], "stem").plan()
+    assert rep.n_launches == 2
+    assert rep.kind[0] == abi.LAUNCH_S2D and rep.kind[1] == abi.LAUNCH_GEMM
+    assert rep.gemm_k[1] == 4 * 4 * 16 and rep.tile_k[1] == 16
+
+
+def test_plan_flops_match_mac_count():
+    for g, _ in [I.bert_ffn(), I.resnet_bottleneck(), I.conv_bias_relu()]:
+        assert _plan(g).flops == pytest.approx(I.region_flops(g), rel=1e-12)
+
+
+def test_packed_weights_are_folded_rounded_and_k_major():
+    g, _ = I.conv_bias_relu(N=1, H=8, W=8, C=64, K=32, seed=3)
+    g2, _ = I.mbv2_dw_pw(N=1, H=8, W=8, C=64, Cout=32)
+    # conv -> bn (from the pointwise part of g2) : fold checked on the GEMM launch
+    reg = R.whole_graph_region(g2)
+    rep = reg.plan()
+    pw = g2.nodes[3]
+    bn = g2.nodes[4]
+    s = bn.consts["gamma"].astype(np.float64) / np.sqrt(bn.consts["moving_var"].astype(np.float64) + 1e-5)
+    shift = bn.consts["beta"] - s * bn.consts["moving_mean"]
+    w = pw.consts["weight"][:, :, 0, 0].astype(np.float64) * s[:, None]
+    raw = np.frombuffer(reg.plan_constants(1, 0), dtype=np.uint16)
+    Kp = rep.gemm_k[1]
+    packed = raw.reshape(-1, Kp)
+    assert np.array_equal(packed[:32, :64], I.bf16_bits(w.astype(np.float32)))
+    assert not packed[:32, 64:].any() and not packed[32:].any()
+    bias = np.frombuffer(reg.plan_constants(1, 1), dtype=np.float32)
+    np.testing.assert_allclose(bias[:32], shift, rtol=1e-6, atol=1e-7)
+    # 3x3 conv: column index = (tap r*3+s) * Cin_pad + c
+    reg = R.whole_graph_region(g)
+    rep = reg.plan()
+    packed = np.frombuffer(reg.plan_constants(0, 0), dtype=np.uint16).reshape(-1, rep.gemm_k[0])
+    wc = g.nodes[0].consts["weight"]
+    for (k, c, r, t) in [(0, 0, 0, 0), (5, 17, 2, 1), (31, 63, 1, 2)]:
+        assert packed[k, (r * 3 + t) * 64 + c] == I.bf16_bits(wc[k, c, r, t:t + 1])[0]
+
+
+def _bad(mutate):
+    g, _ = I.conv_bias_relu(N=1, H=8, W=8, C=64, K=64)
+    reg = R.whole_graph_region(g)
+    desc, keep = reg.to_desc()
+    mutate(desc)
+    rep = abi.PlanReport()
+    return abi.lib().byoc_plan(ctypes.byref(desc), 148, ctypes.byref(rep))
+
+
+def test_validation_rejects_malformed_descriptors():
+    assert _bad(lambda d: None) == abi.OK
+    assert _bad(lambda d: setattr(d, "abi_version", 99)) == abi.ERR_INVALID_ARG
+    assert _bad(lambda d: setattr(d, "n_ops", 0)) == abi.ERR_INVALID_ARG
+    def bad_shape(d):
+        d.tensors[1].shape[1] = 7
+    assert _bad(bad_shape) == abi.ERR_INVALID_ARG
+    def null_weight(d):
+        d.ops[0].consts[0] = None
+    assert _bad(null_weight) == abi.ERR_INVALID_ARG
+    def bad_order(d):
+        d.ops[1].in_[0] = 3   # reads the output of a later op
+    assert _bad(bad_order) == abi.ERR_INVALID_ARG
+    def fp32_act(d):
+        d.tensors[0].dtype = abi.FP32
+    assert _bad(fp32_act) == abi.ERR_UNSUPPORTED
+    assert b"" != abi.lib().byoc_last_error()
+
+
+def test_unsupported_chains_are_rejected_not_run_elsewhere():
+    b = I._Builder("lone_relu")
+    x = b.input("x", (1, 4, 4, 8))
+    y = b.relu(x)
+    g, _ = I._finish(b, [y], 0)
+    with pytest.raises(abi.ByocError) as e:
+        R.whole_graph_region(g).plan()
+    assert e.value.status == abi.ERR_UNSUPPORTED
+    g, _ = I.conv_bias_relu(N=1, H=8, W=8, C=64, K=20)   # Cout not a multiple of 8
+    with pytest.raises(abi.ByocError) as e:
+        R.whole_graph_region(g).plan()
+    assert e.value.status == abi.ERR_UNSUPPORTED

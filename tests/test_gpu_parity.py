@@ -1,0 +1,131 @@
+"""GPU parity: every offloaded composite, run through the C ABI on cuda:0,
+against the fp64 oracle on the same seeded inputs.
+
+Small-integer cases must match bit for bit (every fp32 partial sum is an
+exact integer, so the GPU's bf16 output equals the bf16 rounding of the exact
+result); float cases must satisfy |gpu - ref| <= 1e-2 + 2e-2 |ref|.
+"""
+import numpy as np
+import pytest
+
+from oracle import graph as ograph
+from paper_2105_03215_gb300 import inputs as I
+from paper_2105_03215_gb300 import region as R
+
+from .parity import assert_bit_exact, assert_close, run_region
+
+pytestmark = pytest.mark.gpu
+
+
+def _check_graph(g, inp, bit_exact=False, what=""):
+    reg = R.whole_graph_region(g)
+    got, cr = run_region(reg, inp)
+    ref = ograph.evaluate(g, inp)
+    for name in g.outputs:
+        if bit_exact:
+            assert_bit_exact(got[name], ref[name], what or g.name)
+        else:
+            assert_close(got[name], ref[name], what or g.name)
+    cr.release()
+    return got, ref
+
+
+# ------------------------------------------------------------ exact (small integers)
+
+@pytest.mark.parametrize("M,Iw,U", [(200, 192, 320), (128, 64, 64), (37, 136, 24), (300, 768, 1000)])
+def test_dense_small_int_bit_exact(M, Iw, U):
+    g, inp = I.small_int_dense(M=M, I=Iw, U=U)
+    _check_graph(g, inp, bit_exact=True)
+
+
+@pytest.mark.parametrize("N,H,W,C,K,k,stride,pad", [
+    (2, 9, 11, 64, 64, 3, 1, 1),      # im2col, ragged M = 198
+    (1, 7, 7, 64, 128, 1, 1, 0),      # 1x1 as plain GEMM, M < 128
+    (2, 13, 10, 128, 96, 3, 2, 1),    # stride-2 3x3
+    (2, 14, 14, 64, 256, 1, 2, 0),    # stride-2 1x1 (downsample)
+    (1, 12, 12, 144, 32, 3, 1, 1),    # 144 channels: zero-filled tail chunk in im2col
+    (1, 8, 9, 32, 64, 3, 1, 1),       # 32 channels: 64-byte swizzle
+])
+def test_conv_small_int_bit_exact(N, H, W, C, K, k, stride, pad):
+    g, inp = I.small_int_conv(N=N, H=H, W=W, C=C, K=K, k=k, stride=stride, pad=pad)
+    _check_graph(g, inp, bit_exact=True)
+
+
+# ------------------------------------------------------------ float parity
+
+def test_conv3x3_bias_relu_56x56():
+    g, inp = I.conv_bias_relu(N=1, H=56, W=56, C=64, K=64, seed=0)
+    _check_graph(g, inp)
+
+
+@pytest.mark.parametrize("act", ["relu6", "gelu", "none"])
+def test_conv_epilogue_activations(act):
+    g, inp = I.conv_bias_relu(N=2, H=10, W=10, C=64, K=64, seed=5, act=act)
+    _check_graph(g, inp)
+
+
+def test_bert_ffn_small():
+    g, inp = I.bert_ffn(M=256, D=256, F=512, seed=1)
+    _check_graph(g, inp)
+
+
+def test_bert_ffn_full():
+    g, inp = I.bert_ffn(seed=1)
+    _check_graph(g, inp)
+
+
+def test_mbv2_dw_pw_small():
+    g, inp = I.mbv2_dw_pw(N=2, H=20, W=17, C=144, Cout=24, seed=2)
+    _check_graph(g, inp)
+
+
+def test_mbv2_dw_pw_full():
+    g, inp = I.mbv2_dw_pw(seed=2)
+    _check_graph(g, inp)
+
+
+def test_depthwise_stride2():
+    g, inp = I.mbv2_dw_pw(N=2, H=21, W=20, C=96, Cout=32, seed=9, stride=2)
+    _check_graph(g, inp)
+
+
+def test_bottleneck_small():
+    g, inp = I.resnet_bottleneck(N=2, H=14, W=14, C=256, width=64, seed=3)
+    _check_graph(g, inp)
+
+
+def test_bottleneck_downsample_stride2():
+    g, inp = I.resnet_bottleneck(N=2, H=14, W=14, C=256, width=128, stride=2, seed=3)
+    _check_graph(g, inp)
+
+
+def test_bottleneck_full():
+    g, inp = I.resnet_bottleneck(seed=3)
+    _check_graph(g, inp)
+
+
+def test_stem_space_to_depth():
+    g, inp = I.resnet50(N=2, H=64, W=48, seed=4)
+    stem = [n.name for n in g.nodes[:3]]  # conv 7x7/2 + bn + relu
+    reg = R.Region(g, stem, "stem")
+    got, cr = run_region(reg, inp)
+    ref = ograph.evaluate(g, inp, nodes=stem, keep=reg.outputs)
+    assert_close(got[reg.outputs[0]], ref[reg.outputs[0]], "stem")
+    cr.release()
+
+
+def test_region_can_run_twice_with_new_pointers():
+    import torch
+    from .parity import to_dev
+    g, inp = I.conv_bias_relu(N=1, H=16, W=16, C=64, K=64, seed=11)
+    reg = R.whole_graph_region(g)
+    cr = reg.compile()
+    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    for _ in range(2):
+        x = to_dev(inp["x"])
+        y = torch.full(g.shape_of(g.outputs[0]), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cr.run([x], [y])
+        torch.cuda.synchronize()
+        cr.check()
+        assert_close(y.float().cpu().numpy(), ref, "rerun")
+    cr.release()
