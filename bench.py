@@ -1,0 +1,423 @@
+"""Benchmark: ResNet-50 v1b (N=64, 224x224, bf16 NHWC, synthetic inputs and
+random-init weights) partitioned into 54 offloaded regions -- 53 conv2d
+composites and 1 dense -- with max pool and global average pool on the host,
+run through this library's C ABI.  A step is one forward pass over one batch.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line.  ``value`` is images/s over all ranks with inputs
+resident in HBM, timed with CUDA events around CUDA-graph replays of the
+forward pass, L2 flushed (a 256 MB write) before every timed step.  ``e2e``
+is the same metric through pinned host buffers (input upload and logits
+download inside the timed region).  ``roofline`` describes the dominant
+kernel (the tcgen05 implicit-GEMM kernel) from per-launch CUDA events.
+``cpu_baseline`` times the fp64 oracle on a one-image sample on the host
+cores.  ``--impl reference`` times that oracle alone (the reference arm).
+Multi-GPU: replicas only (one independent batch per rank, weak scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "offloaded-region TFLOP/s (% BF16 peak) / GB/s (% HBM); ResNet-50-shape imgs/s"
+BATCH, IMG = 64, 224
+L2_FLUSH_BYTES = 256 << 20
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+# ---------------------------------------------------------------- distributed plumbing
+
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def reduce_max(value: float, world: int):
+    """Max over ranks (identity at world size 1)."""
+    if world == 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([value], dtype=torch.float64, device=dev)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 50 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        try:
+            fd, self.path = tempfile.mkstemp(suffix=".csv")
+            os.close(fd)
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-i", str(self.gpu), "-lms", "50"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9 and parts[1].replace(".", "").isdigit():
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        sm = [float(r[1]) for r in rows]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[5 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": float(rows[0][2]),
+                "samples": len(rows), "power_w_max": max(float(r[3]) for r in rows
+                                                         if r[3].replace(".", "").isdigit()),
+                "reasons": reasons}
+
+
+# ---------------------------------------------------------------- CPU baseline (oracle)
+
+def oracle_sample(graph, data, images: int = 1):
+    """Seconds the fp64 oracle takes for a forward pass over `images` images."""
+    from oracle import graph as ograph
+    from oracle import ops as oops
+    t0 = time.perf_counter()
+    ograph.evaluate(graph, {"data": data[:images]})
+    return time.perf_counter() - t0, oops.num_threads()
+
+
+def run_reference(args, world, rank):
+    """The reference arm: the fp64 oracle on the host cores, one image per step."""
+    if rank != 0:
+        return
+    from paper_2105_03215_gb300 import inputs as I
+    g, inp = I.resnet50(N=BATCH, H=IMG, W=IMG, seed=4)
+    for _ in range(args.warmup):
+        oracle_sample(g, inp["data"], 1)
+    times = []
+    cores = 1
+    for _ in range(args.steps):
+        t, cores = oracle_sample(g, inp["data"], 1)
+        times.append(t)
+    total = sum(times)
+    value = args.steps / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "images/s",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "resnet50_v1b_N64_224", "global_batch": BATCH, "image": IMG,
+                   "sample": "1 image of the batch per step"},
+        "cpu_baseline": {"value": value, "unit": "images/s", "cores": cores, "kind": "oracle",
+                         "sample": "1 of 64 images per step, fp64 direct loops"},
+        "e2e": {"value": value, "unit": "images/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------- region micro-benchmarks
+
+def time_region(cr, ins, outs, flush, reps=20):
+    import torch
+    st = torch.cuda.current_stream()
+    for _ in range(3):
+        cr.run(ins, outs, st)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for a, b in evs:
+        flush.zero_()
+        a.record(st)
+        cr.run(ins, outs, st)
+        b.record(st)
+    torch.cuda.synchronize()
+    cr.check()
+    return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3  # seconds
+
+
+def region_figures(flush, peaks):
+    """Configs 1-4 of the workload list, each as one region (cold L2)."""
+    import torch
+    from paper_2105_03215_gb300 import inputs as I
+    from paper_2105_03215_gb300 import region as R
+    out = {}
+    cases = {
+        "conv3x3_bias_relu_1x56x56x64": I.conv_bias_relu(seed=0),
+        "bert_ffn_1024x768x3072": I.bert_ffn(seed=1),
+        "mbv2_dw_pw_32x56x56x144": I.mbv2_dw_pw(seed=2),
+        "resnet50_bottleneck_32x14x14x1024": I.resnet_bottleneck(seed=3),
+    }
+    for name, (g, inp) in cases.items():
+        reg = R.whole_graph_region(g)
+        cr = reg.compile()
+        ins = [torch.from_numpy(inp[n]).to(torch.bfloat16).cuda() for n in reg.inputs]
+        outs = [torch.empty(g.shape_of(n), dtype=torch.bfloat16, device="cuda") for n in reg.outputs]
+        t = time_region(cr, ins, outs, flush)
+        tf = cr.flops / t / 1e12
+        gb = cr.bytes / t / 1e9
+        out[name] = {"us": t * 1e6, "tflops": tf, "gbps": gb, "launches": cr.n_launches,
+                     "tensor_frac_of_measured": tf / peaks["bf16_tflops"],
+                     "hbm_frac_of_measured": gb / peaks["hbm_gbs"]}
+        if name.startswith("mbv2"):
+            # the depthwise launch alone (the bandwidth-bound composite)
+            dwg, dwi = I.mbv2_dw_pw(seed=2)
+            dreg = R.Region(dwg, [n.name for n in dwg.nodes[:3]], "dw")
+            dcr = dreg.compile()
+            din = [torch.from_numpy(dwi["x"]).to(torch.bfloat16).cuda()]
+            dout = [torch.empty(dwg.shape_of(dreg.outputs[0]), dtype=torch.bfloat16, device="cuda")]
+            td = time_region(dcr, din, dout, flush)
+            out["depthwise3x3_bn_relu6_32x56x56x144"] = {
+                "us": td * 1e6, "gbps": dcr.bytes / td / 1e9,
+                "hbm_frac_of_measured": dcr.bytes / td / 1e9 / peaks["hbm_gbs"]}
+            dcr.release()
+        cr.release()
+    return out
+
+
+# ---------------------------------------------------------------- main (ours)
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-regions", action="store_true", help="skip the per-config region figures")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--dump", default=None, help="write the per-region timing breakdown (JSON) here")
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl" if args.impl == "ours" else "gloo")
+    if args.impl == "reference":
+        run_reference(args, world, rank)
+        barrier(world)
+        return
+
+    import torch
+    from paper_2105_03215_gb300 import abi
+    from paper_2105_03215_gb300 import executor as E
+
+    torch.cuda.set_device(local)
+    peaks, peak_src = load_peaks()
+    res, inp = E.build_resnet50(N=BATCH, H=IMG, W=IMG)
+    ex = E.Executor(res)
+    host_in = torch.from_numpy(inp["data"]).to(torch.bfloat16).pin_memory()
+    host_out = torch.empty(ex.output().shape, dtype=torch.bfloat16).pin_memory()
+    ex.set_input("data", host_in)
+    ex.capture()
+    flush = torch.empty(L2_FLUSH_BYTES, dtype=torch.uint8, device="cuda")
+    st = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        ex.replay()
+    torch.cuda.synchronize()
+    ex.check()
+
+    # ------------------------------------------------ timed: device-resident inputs
+    clocks = ClockSampler(local)
+    clocks.start()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    w0 = time.perf_counter()
+    for a, b in evs:
+        flush.zero_()
+        a.record(st)
+        ex.replay()
+        b.record(st)
+    torch.cuda.synchronize()
+    barrier(world)
+    wall = time.perf_counter() - w0
+    clk = clocks.stop()
+    ex.check()
+    step_s = [a.elapsed_time(b) * 1e-3 for a, b in evs]
+    total = reduce_max(sum(step_s), world)
+    images = BATCH * args.steps * world
+    value = images / total
+
+    # ------------------------------------------------ per-launch events (roofline)
+    n_steps = len(ex.steps)
+    rec = []
+
+    def hook(kind, i, when):
+        e = torch.cuda.Event(enable_timing=True)
+        e.record(st)
+        rec.append((i, when, e))
+
+    inst_steps = max(3, args.steps // 4)
+    per_step = {i: [] for i in range(n_steps)}
+    for _ in range(inst_steps):
+        rec.clear()
+        flush.zero_()
+        ex.run_steps(st, hooks=hook)
+        torch.cuda.synchronize()
+        pre = {}
+        for i, when, e in rec:
+            if when == "pre":
+                pre[i] = e
+            else:
+                per_step[i].append(pre[i].elapsed_time(e) * 1e-3)
+    ex.check()
+    gemm_t = gemm_f = gemm_b = 0.0
+    hbm_roof = tensor_roof = 0.0
+    launches = []
+    pf = peaks["bf16_tflops_sustained"] * 1e12
+    pb = peaks["hbm_gbs"] * 1e9
+    for i, (kind, x) in enumerate(ex.steps):
+        t = statistics.median(per_step[i])
+        if kind != "region":
+            continue
+        c = ex.compiled[x]
+        if c.n_launches != 1:
+            continue  # the stem region also runs its space-to-depth transform
+        gemm_t += t
+        gemm_f += c.flops
+        gemm_b += c.bytes
+        tensor_roof += c.flops / pf
+        hbm_roof += max(c.flops / pf, c.bytes / pb)
+        launches.append((c.flops / t / 1e12, c.bytes / t / 1e9, t * 1e6, ex.regions[x].name))
+    achieved = gemm_f / gemm_t / 1e12
+    if args.dump and rank == 0:
+        rows = []
+        for i, (kind, x) in enumerate(ex.steps):
+            t = statistics.median(per_step[i])
+            if kind == "region":
+                c = ex.compiled[x]
+                r = ex.regions[x]
+                first = r.nodes[0]
+                rows.append({"step": i, "region": r.name, "us": t * 1e6, "gflop": c.flops / 1e9,
+                             "mb": c.bytes / 1e6, "tflops": c.flops / t / 1e12,
+                             "gbps": c.bytes / t / 1e9, "launches": c.n_launches,
+                             "in": list(ex.graph.shape_of(first.inputs[0])),
+                             "out": list(ex.graph.shape_of(r.outputs[0])),
+                             "kernel": first.attrs.get("kernel_size"),
+                             "roof_us": max(c.flops / pf, c.bytes / pb) * 1e6})
+            else:
+                rows.append({"step": i, "host": x, "us": t * 1e6})
+        with open(args.dump, "w") as f:
+            json.dump(rows, f, indent=1)
+    traffic = None
+    tpath = os.path.join(ROOT, "profiles", "gemm_traffic.json")
+    if os.path.exists(tpath):
+        try:
+            from paper_2105_03215_gb300 import build as B
+            with open(tpath) as f:
+                tj = json.load(f)
+            if tj.get("source_digest") == B._digest():
+                traffic = tj.get("bytes_per_launch")
+        except Exception:
+            traffic = None
+
+    # ------------------------------------------------ e2e through host buffers
+    e2e_t = []
+    for _ in range(max(3, args.steps // 2)):
+        torch.cuda.synchronize()
+        t0 = time.perf_counter()
+        ex.set_input("data", host_in, non_blocking=True)
+        ex.replay()
+        host_out.copy_(ex.output(), non_blocking=True)
+        torch.cuda.synchronize()
+        e2e_t.append(time.perf_counter() - t0)
+    e2e_total = reduce_max(sum(e2e_t), world)
+    e2e_value = BATCH * len(e2e_t) * world / e2e_total
+
+    regions = None
+    if not args.no_regions and rank == 0:
+        regions = region_figures(flush, peaks)
+
+    cpu = None
+    if not args.no_cpu_baseline and rank == 0 and world == 1:
+        t, cores = oracle_sample(res.graph, inp["data"], 2)
+        cpu = {"value": 2.0 / t, "unit": "images/s", "cores": cores, "kind": "oracle",
+               "sample": "2 of the 64 images, fp64 direct loops, same weights", "seconds": t}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "images/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "resnet50_v1b_N64_224 (54 offloaded regions, pools on host)",
+                       "global_batch": BATCH * world, "image": IMG, "regions": len(ex.regions),
+                       "parallelism": f"replicas{world}",
+                       "l2": "flushed by a 256 MB write before every timed step",
+                       "timing": "CUDA events around CUDA-graph replays"},
+            "tflops": value / BATCH * sum(c.flops for c in ex.compiled) / 1e12,
+            "wall_s": wall,
+            "clocks": clk,
+            "e2e": {"value": e2e_value, "unit": "images/s",
+                    "h2d_bytes_per_step": host_in.numel() * 2,
+                    "d2h_bytes_per_step": host_out.numel() * 2},
+            "gpu_launches": ex.n_launches * args.steps,
+            "roofline": {"bound": "tensor", "achieved": achieved,
+                         "peak": peaks["bf16_tflops_sustained"], "unit": "TFLOP/s",
+                         "frac": achieved / peaks["bf16_tflops_sustained"], "traffic": traffic,
+                         "peak_source": f"{peak_src} bf16 sustained",
+                         "kernel": "gemm_tcgen05_kernel (53 single-launch conv/dense regions)",
+                         "per_region_roofline_time_frac": hbm_roof / gemm_t,
+                         "gemm_gbps": gemm_b / gemm_t / 1e9},
+            "cpu_baseline": cpu,
+            "regions": regions,
+        }
+        print(json.dumps(line), flush=True)
+    ex.release()
+    barrier(world)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -34,133 +34,148 @@ __device__ __forceinline__ uint4 ldg_v4(const void *p) {
 
 // ------------------------------------------------------------ depthwise 3x3
 //
-// Thread <-> (image n, output column q, 8-channel vector cv, ROWS consecutive
-// output rows).  cv varies fastest across threads, so a warp reads and writes
-// contiguous 16-byte vectors of one image row.  The three input rows under
-// the filter live in registers and slide down the column (stride 1: one new
-// row per output row; stride 2: two), so each input vector is loaded about
-// (ROWS+2)/ROWS times per filter column instead of three; the three filter
-// columns of neighbouring q are served by L1.
+// Thread <-> (image n, output column q, 4-channel group, ROWS consecutive
+// output rows).  The channel group varies fastest across threads, so a warp
+// reads and writes one contiguous 256-byte run of an image row per access.
+// The 3 x 3 input window lives in registers as fp32 and slides down the
+// column: each output row loads one new input row (stride 1; two for stride
+// 2), and the next row is loaded before the current one is computed, so two
+// rows of loads are in flight per thread.  Registers stay under 80, so a
+// multiprocessor holds enough warps to keep HBM busy.
 template <int STRIDE, int ROWS>
-__global__ void __launch_bounds__(256) dwconv3x3_kernel(const DwArgs a) {
-    const int CV = a.C >> 3;
+__global__ void __launch_bounds__(256, 2) dwconv3x3_kernel(const DwArgs a) {
+    const int CG = a.C >> 2;  // 4-channel groups
     const int PB = (a.Ho + ROWS - 1) / ROWS;
-    const long long total = (long long)a.N * PB * a.Wo * CV;
+    const long long total = (long long)a.N * PB * a.Wo * CG;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= total) return;
-    const int cv = (int)(idx % CV);
-    long long t = idx / CV;
+    const int cg = (int)(idx % CG);
+    long long t = idx / CG;
     const int q = (int)(t % a.Wo);
     t /= a.Wo;
     const int pb = (int)(t % PB);
     const int n = (int)(t / PB);
-    const int c0 = cv * 8;
+    const int c0 = cg * 4;
 
-    float w[9][8];
+    float w[9][4];
 #pragma unroll
     for (int tap = 0; tap < 9; ++tap) {
-        const float4 lo = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0));
-        const float4 hi = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0 + 4));
-        w[tap][0] = lo.x; w[tap][1] = lo.y; w[tap][2] = lo.z; w[tap][3] = lo.w;
-        w[tap][4] = hi.x; w[tap][5] = hi.y; w[tap][6] = hi.z; w[tap][7] = hi.w;
+        const float4 v = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0));
+        w[tap][0] = v.x; w[tap][1] = v.y; w[tap][2] = v.z; w[tap][3] = v.w;
     }
-    float bias[8];
-    {
-        const float4 lo = __ldg(reinterpret_cast<const float4 *>(a.bias + c0));
-        const float4 hi = __ldg(reinterpret_cast<const float4 *>(a.bias + c0 + 4));
-        bias[0] = lo.x; bias[1] = lo.y; bias[2] = lo.z; bias[3] = lo.w;
-        bias[4] = hi.x; bias[5] = hi.y; bias[6] = hi.z; bias[7] = hi.w;
-    }
+    const float4 b4 = __ldg(reinterpret_cast<const float4 *>(a.bias + c0));
 
     const int wc0 = q * STRIDE - a.pad;
     const __nv_bfloat16 *xn = a.x + (size_t)n * a.H * a.W * a.C + c0;
-    auto load_row = [&](int h, uint4 (&r)[3]) {
+    // one input row under the filter: 3 columns x 4 channels, zero outside the image
+    auto load_row = [&](int h, uint2 (&r)[3]) {
         const bool hv = h >= 0 && h < a.H;
 #pragma unroll
         for (int s = 0; s < 3; ++s) {
             const int wc = wc0 + s;
-            if (hv && wc >= 0 && wc < a.W)
-                r[s] = ldg_v4(xn + ((size_t)h * a.W + wc) * a.C);
-            else
-                r[s] = make_uint4(0u, 0u, 0u, 0u);
+            r[s] = (hv && wc >= 0 && wc < a.W)
+                       ? __ldg(reinterpret_cast<const uint2 *>(xn + ((size_t)h * a.W + wc) * a.C))
+                       : make_uint2(0u, 0u);
+        }
+    };
+    auto unpack_row = [&](const uint2 (&r)[3], float (&f)[3][4]) {
+#pragma unroll
+        for (int s = 0; s < 3; ++s) {
+            f[s][0] = bf16lo(r[s].x); f[s][1] = bf16hi(r[s].x);
+            f[s][2] = bf16lo(r[s].y); f[s][3] = bf16hi(r[s].y);
         }
     };
 
     const int p0 = pb * ROWS;
-    uint4 win[3][3];
-    load_row(p0 * STRIDE - a.pad, win[0]);
-    load_row(p0 * STRIDE - a.pad + 1, win[1]);
+    float win[3][3][4];
+    uint2 raw[3], nxt[3];
+    load_row(p0 * STRIDE - a.pad, raw);
+    unpack_row(raw, win[0]);
+    load_row(p0 * STRIDE - a.pad + 1, raw);
+    unpack_row(raw, win[1]);
+    load_row(p0 * STRIDE - a.pad + 2, nxt);
 #pragma unroll
     for (int i = 0; i < ROWS; ++i) {
         const int p = p0 + i;
+        if (p >= a.Ho) break;
         const int hb = p * STRIDE - a.pad;
-        if (i > 0) {
+        unpack_row(nxt, win[2]);
+        // prefetch what the next output row needs beyond the rows kept
+        uint2 mid[3];
+        if (i + 1 < ROWS) {
             if (STRIDE == 1) {
-#pragma unroll
-                for (int s = 0; s < 3; ++s) {
-                    win[0][s] = win[1][s];
-                    win[1][s] = win[2][s];
-                }
+                load_row(hb + 3, nxt);
             } else {
-#pragma unroll
-                for (int s = 0; s < 3; ++s) win[0][s] = win[2][s];
-                load_row(hb + 1, win[1]);
+                load_row(hb + 3, mid);
+                load_row(hb + 4, nxt);
             }
         }
-        load_row(hb + 2, win[2]);
-        if (p < a.Ho) {
-            float acc[8];
+        float acc[4] = {b4.x, b4.y, b4.z, b4.w};
 #pragma unroll
-            for (int j = 0; j < 8; ++j) acc[j] = bias[j];
+        for (int r = 0; r < 3; ++r)
 #pragma unroll
-            for (int r = 0; r < 3; ++r) {
+            for (int s = 0; s < 3; ++s)
 #pragma unroll
-                for (int s = 0; s < 3; ++s) {
-                    float f[8];
-                    unpack8(win[r][s], f);
+                for (int j = 0; j < 4; ++j) acc[j] = fmaf(win[r][s][j], w[r * 3 + s][j], acc[j]);
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) acc[j] = fmaf(f[j], w[r * 3 + s][j], acc[j]);
+        for (int j = 0; j < 4; ++j) {
+            float v = acc[j];
+            if (a.act == kActRelu) v = fmaxf(v, 0.0f);
+            else if (a.act == kActRelu6) v = fminf(fmaxf(v, 0.0f), 6.0f);
+            else if (a.act == kActGelu) v = 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
+            acc[j] = v;
+        }
+        uint2 o;
+        o.x = pack_bf16x2(acc[0], acc[1]);
+        o.y = pack_bf16x2(acc[2], acc[3]);
+        *reinterpret_cast<uint2 *>(a.y + (((size_t)n * a.Ho + p) * a.Wo + q) * a.C + c0) = o;
+        // slide the window
+        if (STRIDE == 1) {
+#pragma unroll
+            for (int s = 0; s < 3; ++s)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) {
+                    win[0][s][j] = win[1][s][j];
+                    win[1][s][j] = win[2][s][j];
                 }
-            }
+        } else {
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
-                float v = acc[j];
-                if (a.act == kActRelu) v = fmaxf(v, 0.0f);
-                else if (a.act == kActRelu6) v = fminf(fmaxf(v, 0.0f), 6.0f);
-                else if (a.act == kActGelu) v = 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
-                acc[j] = v;
-            }
-            *reinterpret_cast<uint4 *>(a.y + (((size_t)n * a.Ho + p) * a.Wo + q) * a.C + c0) =
-                pack8(acc);
+            for (int s = 0; s < 3; ++s)
+#pragma unroll
+                for (int j = 0; j < 4; ++j) win[0][s][j] = win[2][s][j];
+            if (i + 1 < ROWS) unpack_row(mid, win[1]);
         }
     }
 }
 
 cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st) {
     (void)num_sms;
-    const int CV = a.C / 8;
+    const int CG = a.C / 4;
     const int threads = 256;
     if (a.stride == 1) {
         constexpr int R = 8;
-        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CV;
+        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CG;
         dwconv3x3_kernel<1, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
     } else {
         constexpr int R = 4;
-        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CV;
+        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CG;
         dwconv3x3_kernel<2, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
     }
     return cudaGetLastError();
 }
 
 // ------------------------------------------------------------ space-to-depth
-// z[n, i, j, (dy*2+dx)*C + c] = x[n, 2i+dy-pad, 2j+dx-pad, c]; other channels 0.
+// z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]; one
+// thread per 16-channel group (a) of one output pixel, writing 32 bytes.
 __global__ void s2d_kernel(const S2dArgs a) {
-    const long long total = (long long)a.N * a.Hz * a.Wz;
+    const long long total = (long long)a.N * a.Hz * a.Wz * a.taps;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= total) return;
-    const int j = (int)(idx % a.Wz);
-    const long long t = idx / a.Wz;
-    const int i = (int)(t % a.Hz);
+    const int tap = (int)(idx % a.taps);
+    long long t = idx / a.taps;
+    const int j = (int)(t % a.Wz);
+    t /= a.Wz;
+    const int p = (int)(t % a.Hz);
     const int n = (int)(t / a.Hz);
     float v[16];
 #pragma unroll
@@ -170,17 +185,16 @@ __global__ void s2d_kernel(const S2dArgs a) {
     for (int dy = 0; dy < 2; ++dy) {
 #pragma unroll
         for (int dx = 0; dx < 2; ++dx) {
-            const int h = 2 * i + dy - a.pad;
+            const int h = 2 * (p + tap) + dy - a.pad;
             const int w = 2 * j + dx - a.pad;
             if (h < 0 || h >= a.H || w < 0 || w >= a.W) continue;
             const size_t off = (((size_t)n * a.H + h) * a.W + w) * a.C;
-            for (int c = 0; c < a.C; ++c) {
-                const int k = (dy * 2 + dx) * a.C + c;
-                if (k < 16) v[k] = __uint_as_float((uint32_t)__ldg(xs + off + c) << 16);
-            }
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+                if (c < a.C) v[(dy * 2 + dx) * a.C + c] = __uint_as_float((uint32_t)__ldg(xs + off + c) << 16);
         }
     }
-    uint4 *zp = reinterpret_cast<uint4 *>(a.z + (size_t)idx * a.Cz);
+    uint4 *zp = reinterpret_cast<uint4 *>(a.z + (((size_t)n * a.Hz + p) * a.Wz + j) * a.Cz + tap * 16);
     float lo[8], hi[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
@@ -192,7 +206,7 @@ __global__ void s2d_kernel(const S2dArgs a) {
 }
 
 cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
-    const long long total = (long long)a.N * a.Hz * a.Wz;
+    const long long total = (long long)a.N * a.Hz * a.Wz * a.taps;
     s2d_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(a);
     return cudaGetLastError();
 }

@@ -43,7 +43,8 @@ struct GemmConfig {
 };
 
 constexpr int kGemmBM = 128;
-constexpr int kGemmThreads = 192;  // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kGemmEpiWarps = 8;
+constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
 
 bool gemm_config_supported(const GemmConfig &cfg);
 size_t gemm_smem_bytes(const GemmConfig &cfg);
@@ -66,13 +67,15 @@ struct DwArgs {
 cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st);
 
 // Boundary layout transform for a stride-2 stem with few input channels
-// (space-to-depth with zero padding): z[n, i, j, (dy*2+dx)*C + c] =
-// x[n, 2i+dy-pad, 2j+dx-pad, c] (zero outside), channels >= 4C zero.
+// (space-to-depth with zero padding, vertical filter taps stacked):
+//   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
+// for a < taps, zero outside the image and in channels a*16 + [4C, 16).
 struct S2dArgs {
     const __nv_bfloat16 *x;
     __nv_bfloat16 *z;
     int N, H, W, C;   // input
-    int Hz, Wz, Cz;   // output (Cz = 16)
+    int Hz, Wz, Cz;   // output: Hz = output rows, Cz = 16 * taps
+    int taps;
     int pad;
 };
 cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st);

@@ -97,16 +97,23 @@ CUresult encode_2d(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
-// im2col map over an NHWC bf16 tensor for a k x k filter, stride s, padding
-// (lo before, hi after), dilation d; 128 pixels x bk channels per load.
-CUresult encode_im2col(CUtensorMap *m, const void *ptr, int N, int H, int W, int C, int k, int s,
-                       int pad_lo, int pad_hi, int d, int bk) {
-    cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
-    cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
-    // Bounding box of filter origins: from -pad_lo to (dim-1) + pad_hi - (k-1)*d.
-    int lower[2] = {-pad_lo, -pad_lo};
-    int upper[2] = {pad_hi - (k - 1) * d, pad_hi - (k - 1) * d};
-    cuuint32_t es[4] = {1, (cuuint32_t)s, (cuuint32_t)s, 1};
+// Geometry of an im2col-read convolution input.
+struct Im2colGeom {
+    int N, H, W, C;
+    int kh, kw, sh, sw, pt, pl, pb, pr, dh, dw;
+};
+
+// im2col map over an NHWC bf16 tensor; 128 pixels x bk channels per load.
+// The bounding box of filter origins runs, per spatial dimension, from -pad_before
+// to (dim - 1) + pad_after - (k - 1) * dilation; corner and offset arrays list
+// the spatial dimensions innermost first (W, then H), like the tensor's dims.
+CUresult encode_im2col(CUtensorMap *m, const void *ptr, const Im2colGeom &g, int bk) {
+    cuuint64_t dims[4] = {(cuuint64_t)g.C, (cuuint64_t)g.W, (cuuint64_t)g.H, (cuuint64_t)g.N};
+    cuuint64_t strides[3] = {(cuuint64_t)g.C * 2, (cuuint64_t)g.W * g.C * 2,
+                             (cuuint64_t)g.H * g.W * g.C * 2};
+    int lower[2] = {-g.pl, -g.pt};
+    int upper[2] = {g.pr - (g.kw - 1) * g.dw, g.pb - (g.kh - 1) * g.dh};
+    cuuint32_t es[4] = {1, (cuuint32_t)g.sw, (cuuint32_t)g.sh, 1};
     return p_encode_im2col(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
                            strides, lower, upper, (cuuint32_t)bk, (cuuint32_t)byoc::kGemmBM, es,
                            CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
@@ -150,7 +157,7 @@ struct LaunchPlan {
     int grid = 0;
     int n_pad = 0, k_pack = 0;
     // A operand geometry
-    int aN = 0, aH = 0, aW = 0, aC = 0, ksz = 1, kstride = 1, pad_lo = 0, pad_hi = 0, dil = 1;
+    Im2colGeom geo{};
     int64_t aM = 0, aK = 0;
     // constants: byte offsets into the constant blob
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
@@ -326,10 +333,17 @@ int pick_bk(int64_t C) {
     return 64;
 }
 
-// Choose the output-channel tile among the compiled configurations: fewest
-// rounds of the persistent grid, weighted by the tile's width (its MMA time)
-// plus a fixed per-tile cost.
-int pick_bn(int64_t M, int64_t N, int64_t ksteps, int bk, bool im2col, int num_sms) {
+// Choose the output-channel tile among the compiled configurations by a
+// makespan estimate of the persistent grid, in SM cycles, calibrated on
+// GB300 traces of this kernel:
+//   mainloop per tile  = 300 + k-blocks x max(2.5 bn, 450): a 64-deep k-block
+//                        costs ~450 cycles of TMA delivery at small bn and is
+//                        tensor-core bound (~640 cycles) at bn = 256;
+//   epilogue per tile  = ~600 cycles per pair of 32-column chunks (two warps
+//                        per accumulator row block work in parallel).
+// A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
+// time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
+int pick_bn(int64_t M, int64_t N, int64_t kblocks, int bk, bool im2col, int num_sms) {
     int best = -1;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
@@ -338,11 +352,9 @@ int pick_bn(int64_t M, int64_t N, int64_t ksteps, int bk, bool im2col, int num_s
         const int64_t tiles = ((M + 127) / 128) * ((N + bn - 1) / bn);
         const int64_t grid = std::min<int64_t>(tiles, num_sms);
         const int64_t rounds = (tiles + grid - 1) / grid;
-        // Per 16-deep k-step a 128 x bn MMA needs bn/2 tensor-core cycles and
-        // streams (128 + bn) x 32 B of operands through shared memory at
-        // ~128 B/cycle; a tile also pays a fixed fill / epilogue cost.
-        const double step = std::max(bn / 2.0, 32.0 + bn / 4.0);
-        const double cost = (double)rounds * (step * (double)ksteps + 400.0);
+        const double mainloop = 300.0 + (double)kblocks * std::max(2.5 * bn, 450.0);
+        const double epilogue = 600.0 * std::max(1, bn / 64);
+        const double cost = (double)rounds * std::max(mainloop, epilogue) + std::min(mainloop, epilogue);
         if (cost < best_cost - 1e-9) {
             best_cost = cost;
             best = bn;
@@ -490,20 +502,26 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                                 op.dilation[0] == op.dilation[1] && op.pad[0] == op.pad[1] &&
                                 op.pad[2] == op.pad[3];
             if (C % 8) {
-                // Few-channel stride-2 stem: space-to-depth boundary transform, then a
-                // stride-1 (kh+1)/2 square conv over 16 channels.
+                // Few-channel stride-2 stem.  A space-to-depth boundary transform
+                // turns the k x k stride-2 conv over C channels into a k2 x k2
+                // stride-1 conv over 4C (<= 16) channels, k2 = (k+1)/2, and also
+                // stacks the k2 vertical taps into the channel dimension, so the
+                // GEMM is a 1 x k2 conv over 16*k2 channels:
+                //   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
+                //   w''[k][b][a*16 + (dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx]
                 if (!(square && op.stride[0] == 2 && op.dilation[0] == 1 && C <= 4 && (kh % 2) == 1))
                     return fail(BYOC_ERR_UNSUPPORTED,
                                 "op %d: %lld input channels: only a stride-2 odd square stem with "
                                 "<= 4 channels is supported",
                                 o, (long long)C);
                 const int k2 = (kh + 1) / 2;
+                const int Cz = 16 * k2;
                 TensorInfo Z;
                 Z.ndim = 4;
                 Z.shape[0] = X.shape[0];
-                Z.shape[1] = Y.shape[1] + k2 - 1;
+                Z.shape[1] = Y.shape[1];
                 Z.shape[2] = Y.shape[2] + k2 - 1;
-                Z.shape[3] = 16;
+                Z.shape[3] = Cz;
                 const int zid = (int)P.tensors.size();
                 P.tensors.push_back(Z);
                 LaunchPlan S;
@@ -516,12 +534,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                 S.s2d.C = (int)C;
                 S.s2d.Hz = (int)Z.shape[1];
                 S.s2d.Wz = (int)Z.shape[2];
-                S.s2d.Cz = 16;
+                S.s2d.Cz = Cz;
+                S.s2d.taps = k2;
                 S.s2d.pad = op.pad[0];
                 S.bytes = (double)X.bytes() + (double)Z.bytes();
                 P.launches.push_back(S);
-                // Remapped weights w'[k][a][b][(dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx].
-                wsrc.assign((size_t)Cout * k2 * k2 * 16, 0.0);
+                wsrc.assign((size_t)Cout * k2 * Cz, 0.0);
                 for (int64_t k = 0; k < Cout; ++k)
                     for (int a = 0; a < k2; ++a)
                         for (int b = 0; b < k2; ++b)
@@ -530,22 +548,16 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                                     for (int64_t c = 0; c < C; ++c) {
                                         const int r = 2 * a + dy, s = 2 * b + dx;
                                         if (r >= kh || s >= kw) continue;
-                                        wsrc[((k * k2 + a) * k2 + b) * 16 + (dy * 2 + dx) * C + c] =
+                                        wsrc[((size_t)k * k2 + b) * Cz + a * 16 + (dy * 2 + dx) * C + c] =
                                             op.consts[0][((k * C + c) * kh + r) * kw + s];
                                     }
                 L.x = zid;
-                C = 16;
-                kh = kw = k2;
+                C = Cz;
+                kh = 1;
+                kw = k2;
                 im2col = true;
-                L.aN = (int)Z.shape[0];
-                L.aH = (int)Z.shape[1];
-                L.aW = (int)Z.shape[2];
-                L.aC = 16;
-                L.ksz = k2;
-                L.kstride = 1;
-                L.pad_lo = 0;
-                L.pad_hi = 0;
-                L.dil = 1;
+                L.geo = Im2colGeom{(int)Z.shape[0], (int)Z.shape[1], (int)Z.shape[2], Cz,
+                                   1, k2, 1, 1, 0, 0, 0, 0, 1, 1};
                 L.args.stride_h = L.args.stride_w = 1;
                 L.args.pad_t = L.args.pad_l = 0;
                 L.args.dil_h = L.args.dil_w = 1;
@@ -564,35 +576,31 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                     L.aM = M;
                     L.aK = C;
                 } else {
-                    if (!square)
-                        return fail(BYOC_ERR_UNSUPPORTED,
-                                    "op %d: implicit GEMM needs a square kernel with equal "
-                                    "strides, dilations and symmetric padding",
-                                    o);
-                    const int lo = op.pad[0], hi = op.pad[2];
-                    const int up = hi - (kh - 1) * op.dilation[0];
-                    if (lo > 128 || up < -128 || up > 127)
+                    // im2col bounding-box corners must fit the 8-bit range of a
+                    // 4-D map; filter-tap offsets the 16-bit instruction field
+                    const int up_h = op.pad[2] - (kh - 1) * op.dilation[0];
+                    const int up_w = op.pad[3] - (kw - 1) * op.dilation[1];
+                    if (op.pad[0] > 128 || op.pad[1] > 128 || up_h < -128 || up_h > 127 ||
+                        up_w < -128 || up_w > 127 || (kh - 1) * op.dilation[0] > 65535 ||
+                        (kw - 1) * op.dilation[1] > 65535)
                         return fail(BYOC_ERR_UNSUPPORTED, "op %d: padding outside TMA im2col range", o);
                     im2col = true;
-                    L.aN = (int)X.shape[0];
-                    L.aH = (int)X.shape[1];
-                    L.aW = (int)X.shape[2];
-                    L.aC = (int)C;
-                    L.ksz = kh;
-                    L.kstride = op.stride[0];
-                    L.pad_lo = lo;
-                    L.pad_hi = hi;
-                    L.dil = op.dilation[0];
-                    L.args.stride_h = L.args.stride_w = op.stride[0];
-                    L.args.pad_t = L.args.pad_l = lo;
-                    L.args.dil_h = L.args.dil_w = op.dilation[0];
+                    L.geo = Im2colGeom{(int)X.shape[0], (int)X.shape[1], (int)X.shape[2], (int)C,
+                                       kh, kw, op.stride[0], op.stride[1], op.pad[0], op.pad[1],
+                                       op.pad[2], op.pad[3], op.dilation[0], op.dilation[1]};
+                    L.args.stride_h = op.stride[0];
+                    L.args.stride_w = op.stride[1];
+                    L.args.pad_t = op.pad[0];
+                    L.args.pad_l = op.pad[1];
+                    L.args.dil_h = op.dilation[0];
+                    L.args.dil_w = op.dilation[1];
                 }
             }
         }
         taps = kh * kw;
         bk = op.kind == BYOC_OP_DENSE ? 64 : pick_bk(C);
         chunks = (int)((C + bk - 1) / bk);
-        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks * bk / 16, bk, im2col, P.num_sms);
+        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks, bk, im2col, P.num_sms);
         if (bn < 0)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d im2col=%d", o, bk,
                         (int)im2col);
@@ -863,8 +871,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             if (h->tmA_ptr[i] != xa) {
                 CUresult r;
                 if (L.cfg.im2col)
-                    r = encode_im2col(&h->tmA[i], xa, L.aN, L.aH, L.aW, L.aC, L.ksz, L.kstride,
-                                      L.pad_lo, L.pad_hi, L.dil, L.cfg.bk);
+                    r = encode_im2col(&h->tmA[i], xa, L.geo, L.cfg.bk);
                 else
                     r = encode_2d(&h->tmA[i], xa, (uint64_t)L.aM, (uint64_t)L.aK, byoc::kGemmBM,
                                   (uint32_t)L.cfg.bk, L.cfg.bk);

@@ -1,0 +1,194 @@
+"""Graph executor for a partitioned model (Section 3.4, runtime).
+
+Initialisation compiles every region once (the cached execution engines) and
+pre-allocates the data entries: one device buffer for every tensor that
+crosses a step boundary (graph inputs and outputs, region inputs and
+outputs, host-operator inputs and outputs).  Region intermediates are not
+data entries; they live in each region's workspace.  ``run`` then visits the
+steps in a topological order of the partitioned graph: host operators run
+through this library's host kernels (CUDA serving as the host), regions
+through their external call ``byoc_run``.  All work is enqueued on one CUDA
+stream; ``capture()`` records the whole sequence as a CUDA graph so a forward
+pass costs one launch.
+"""
+from __future__ import annotations
+
+import heapq
+from typing import Dict, List, Optional, Sequence, Tuple
+
+from . import abi
+from .inputs import Graph, Node
+from .partition import PartitionResult
+
+HOST_OPS = ("nn.max_pool2d", "nn.global_avg_pool2d", "nn.batch_flatten")
+
+
+class Executor:
+    def __init__(self, result: PartitionResult):
+        import torch
+        self.torch = torch
+        self.result = result
+        self.graph: Graph = result.graph
+        g = self.graph
+        self.by_name = {n.name: n for n in g.nodes}
+        # steps: ("region", index) or ("host", node name), in a topological order
+        self.regions = result.region_objects()
+        self.compiled = [r.compile() for r in self.regions]
+        self.steps = self._order_steps()
+        # data entries
+        needed = set(g.outputs) | set(g.inputs)
+        for r in self.regions:
+            needed.update(r.inputs)
+            needed.update(r.outputs)
+        for kind, x in self.steps:
+            if kind == "host":
+                n = self.by_name[x]
+                needed.update(n.inputs)
+                needed.add(n.name)
+        self.entries: Dict[str, "torch.Tensor"] = {}
+        for name in sorted(needed, key=self._order_key):
+            node = self.by_name.get(name)
+            if node is not None and node.op == "nn.batch_flatten":
+                continue  # a view of its input, made below
+            self.entries[name] = torch.empty(g.shape_of(name), dtype=torch.bfloat16, device="cuda")
+        for name in needed:
+            node = self.by_name.get(name)
+            if node is not None and node.op == "nn.batch_flatten":
+                src = self.entries[node.inputs[0]]
+                self.entries[name] = src.view(node.shape)
+        self._graph = None
+        self.n_launches = sum(c.n_launches for c in self.compiled) + sum(
+            1 for k, x in self.steps if k == "host" and self.by_name[x].op != "nn.batch_flatten")
+
+    # ------------------------------------------------------------------ planning
+    def _order_key(self, name: str) -> int:
+        for i, n in enumerate(self.graph.nodes):
+            if n.name == name:
+                return i + 1
+        return 0
+
+    def _order_steps(self) -> List[Tuple[str, object]]:
+        """Kahn's algorithm over regions and host nodes (regions are convex,
+        so collapsing each into one step keeps the graph acyclic); ties are
+        broken by the position of the step's first node."""
+        g = self.graph
+        pos = {n.name: i for i, n in enumerate(g.nodes)}
+        step_of: Dict[str, int] = {}
+        steps: List[Tuple[str, object]] = []
+        first: List[int] = []
+        for ri, r in enumerate(self.regions):
+            for n in r.nodes:
+                step_of[n.name] = len(steps)
+            steps.append(("region", ri))
+            first.append(min(pos[n.name] for n in r.nodes))
+        for n in g.nodes:
+            if n.name not in step_of:
+                if n.op not in HOST_OPS:
+                    raise abi.ByocError(abi.ERR_UNSUPPORTED,
+                                        f"{n.name} ({n.op}) is neither offloaded nor a host operator")
+                step_of[n.name] = len(steps)
+                steps.append(("host", n.name))
+                first.append(pos[n.name])
+        preds = [set() for _ in steps]
+        for n in g.nodes:
+            s = step_of[n.name]
+            for i in n.inputs:
+                if i in step_of and step_of[i] != s:
+                    preds[s].add(step_of[i])
+        indeg = [len(p) for p in preds]
+        succ = [[] for _ in steps]
+        for s, ps in enumerate(preds):
+            for p in ps:
+                succ[p].append(s)
+        heap = [(first[s], s) for s in range(len(steps)) if indeg[s] == 0]
+        heapq.heapify(heap)
+        order = []
+        while heap:
+            _, s = heapq.heappop(heap)
+            order.append(steps[s])
+            for t in succ[s]:
+                indeg[t] -= 1
+                if indeg[t] == 0:
+                    heapq.heappush(heap, (first[t], t))
+        if len(order) != len(steps):
+            raise abi.ByocError(abi.ERR_INVALID_ARG, "partition is not convex: step graph has a cycle")
+        return order
+
+    # ------------------------------------------------------------------ running
+    def _host(self, node: Node, stream) -> None:
+        x = self.entries[node.inputs[0]]
+        y = self.entries[node.name]
+        if node.op == "nn.max_pool2d":
+            k = node.attrs["pool_size"][0]
+            s = node.attrs["strides"][0]
+            p = node.attrs["padding"][0]
+            abi.max_pool2d_nhwc(x, y, k, s, p, stream)
+        elif node.op == "nn.global_avg_pool2d":
+            abi.global_avg_pool_nhwc(x, y, stream)
+        # nn.batch_flatten: a view, nothing to run
+
+    def run_steps(self, stream=None, hooks=None) -> None:
+        """Enqueue one forward pass.  ``hooks(kind, index, 'pre'|'post')`` is
+        called around every step (used to record timing events)."""
+        st = abi._stream_ptr(stream)
+        for i, (kind, x) in enumerate(self.steps):
+            if hooks:
+                hooks(kind, i, "pre")
+            if kind == "region":
+                r = self.regions[x]
+                self.compiled[x].run([self.entries[n] for n in r.inputs],
+                                     [self.entries[n] for n in r.outputs], st)
+            else:
+                self._host(self.by_name[x], st)
+            if hooks:
+                hooks(kind, i, "post")
+
+    def set_input(self, name: str, src, non_blocking: bool = True) -> None:
+        self.entries[name].copy_(src, non_blocking=non_blocking)
+
+    def output(self, name: Optional[str] = None):
+        return self.entries[name or self.graph.outputs[0]]
+
+    def capture(self) -> None:
+        """Record one forward pass as a CUDA graph (after one eager warm-up)."""
+        torch = self.torch
+        s = torch.cuda.Stream()
+        s.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(s):
+            self.run_steps(s)
+        torch.cuda.current_stream().wait_stream(s)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run_steps()
+        self._graph = g
+
+    def replay(self) -> None:
+        if self._graph is None:
+            raise RuntimeError("capture() first")
+        self._graph.replay()
+
+    def check(self) -> None:
+        for c in self.compiled:
+            c.check()
+
+    def release(self) -> None:
+        for c in self.compiled:
+            c.release()
+        self.compiled = []
+        self._graph = None
+        self.entries = {}
+
+
+def build_resnet50(N: int = 64, H: int = 224, W: int = 224, seed: int = 4, max_ops: Optional[int] = 1,
+                   graph=None):
+    """ResNet-50 v1b partitioned for this library (pools on the host); with
+    ``max_ops=1`` every conv2d / dense composite is its own region (54)."""
+    from . import inputs as I
+    from . import partition as P
+    if graph is None:
+        graph, inp = I.resnet50(N=N, H=H, W=W, seed=seed)
+    else:
+        inp = None
+    res = P.partition(graph, P.PATTERN_TABLE, target=P.TARGET, max_ops=max_ops)
+    return res, inp

@@ -358,6 +358,39 @@ def mobilenet_v2(N=1, H=224, W=224, num_classes=1000, seed=7, draw=False):
     return _finish(b, [y], seed, draw)
 
 
+def conv_general(N=2, H=11, W=13, C=64, K=32, kernel=(1, 3), strides=(1, 1), padding=(0, 1, 0, 1),
+                 dilation=(1, 1), seed=12, small_int=False, act="relu"):
+    """conv2d + bias_add + activation with any kernel shape, per-dimension
+    strides / dilations and asymmetric padding (top, left, bottom, right)."""
+    b = _Builder("conv_general")
+    x = b.input("x", (N, H, W, C))
+    kh, kw = kernel
+    Ho = conv_out(H, kh, strides[0], padding[0], padding[2], dilation[0])
+    Wo = conv_out(W, kw, strides[1], padding[1], padding[3], dilation[1])
+    y = b._add("nn.conv2d", [x], (N, Ho, Wo, K),
+               dict(strides=tuple(strides), padding=tuple(padding), dilation=tuple(dilation),
+                    groups=1, kernel_size=(kh, kw), channels=K, init="kaiming",
+                    weight_shape=(K, C, kh, kw)))
+    y = b.bias_add(y)
+    if act == "relu":
+        y = b.relu(y)
+    g, inp = _finish(b, [y], seed)
+    if small_int:
+        rng = np.random.Generator(np.random.PCG64(seed + 1000))
+        inp = {"x": rng.integers(-4, 5, size=(N, H, W, C)).astype(np.float32)}
+        g.nodes[0].consts["weight"] = rng.integers(-2, 3, size=(K, C, kh, kw)).astype(np.float32)
+        g.nodes[1].consts["bias"] = rng.integers(-8, 9, size=K).astype(np.float32)
+    return g, inp
+
+
+def stem(N=2, H=32, W=30, k=7, cout=64, seed=13, C=3):
+    """A stride-2 k x k stem conv + BN + ReLU over an image with C (<= 4) channels."""
+    b = _Builder(f"stem{k}x{k}")
+    x = b.input("data", (N, H, W, C))
+    y = b.relu(b.batch_norm(b.conv2d(x, cout, k, stride=2, pad=k // 2)))
+    return _finish(b, [y], seed)
+
+
 def small_int_conv(N=2, H=9, W=11, C=64, K=64, k=3, stride=1, pad=1, seed=7, act="relu"):
     """Conv + bias + act with small-integer data (|v| <= 4), exact in bf16 and
     accumulated exactly in fp32: the GPU output must equal the bf16 rounding

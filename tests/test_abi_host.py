@@ -59,7 +59,8 @@ def test_plan_stem_inserts_space_to_depth():
     rep = R.Region(g, [n.name for n in g.nodes[:3]], "stem").plan()
     assert rep.n_launches == 2
     assert rep.kind[0] == abi.LAUNCH_S2D and rep.kind[1] == abi.LAUNCH_GEMM
-    assert rep.gemm_k[1] == 4 * 4 * 16 and rep.tile_k[1] == 16
+    # 7x7/2 over 3 channels -> 1x4 conv over 4 stacked taps x 16 channels
+    assert rep.gemm_k[1] == 4 * 64 and rep.tile_k[1] == 64 and rep.im2col[1] == 1
 
 
 def test_plan_flops_match_mac_count():

@@ -51,6 +51,19 @@ def test_conv_small_int_bit_exact(N, H, W, C, K, k, stride, pad):
     _check_graph(g, inp, bit_exact=True)
 
 
+@pytest.mark.parametrize("kernel,strides,padding,dilation", [
+    ((1, 3), (1, 1), (0, 1, 0, 1), (1, 1)),   # non-square: W taps only
+    ((3, 1), (1, 1), (1, 0, 1, 0), (1, 1)),   # non-square: H taps only
+    ((3, 3), (2, 1), (1, 0, 1, 2), (1, 1)),   # per-dimension stride, asymmetric padding
+    ((3, 3), (1, 1), (2, 2, 2, 2), (2, 2)),   # dilation 2
+    ((1, 4), (1, 1), (0, 0, 0, 0), (1, 1)),   # the shape the stem's GEMM uses
+])
+def test_conv_general_small_int_bit_exact(kernel, strides, padding, dilation):
+    g, inp = I.conv_general(kernel=kernel, strides=strides, padding=padding, dilation=dilation,
+                            small_int=True)
+    _check_graph(g, inp, bit_exact=True)
+
+
 # ------------------------------------------------------------ float parity
 
 def test_conv3x3_bias_relu_56x56():
@@ -112,6 +125,12 @@ def test_stem_space_to_depth():
     ref = ograph.evaluate(g, inp, nodes=stem, keep=reg.outputs)
     assert_close(got[reg.outputs[0]], ref[reg.outputs[0]], "stem")
     cr.release()
+
+
+@pytest.mark.parametrize("k,cout,C", [(7, 64, 3), (3, 32, 3), (5, 48, 4), (7, 64, 1)])
+def test_stem_variants(k, cout, C):
+    g, inp = I.stem(k=k, cout=cout, C=C)
+    _check_graph(g, inp, what=f"stem{k}x{k}")
 
 
 def test_region_can_run_twice_with_new_pointers():

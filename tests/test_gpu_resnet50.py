@@ -1,0 +1,155 @@
+"""ResNet-50 partitioned into 54 regions (53 conv2d composites + 1 dense) with
+max pool and global average pool left on the host, run by the executor.
+
+Parity is per region and teacher-forced: every region is checked against the
+oracle fed the GPU's own bf16 inputs for that region (a 54-deep bf16 chain
+compounds rounding, so an end-to-end comparison only gets reported).  At the
+full batch of 64 the oracle evaluates a random sample of each region's
+outputs one by one.
+"""
+import numpy as np
+import pytest
+
+from oracle import graph as ograph
+from oracle import ops
+from paper_2105_03215_gb300 import executor as E
+
+from .parity import assert_bit_exact, assert_close
+
+pytestmark = pytest.mark.gpu
+
+
+def _f64(t):
+    return t.float().cpu().numpy().astype(np.float64)
+
+
+def _check_host_steps(ex):
+    for kind, x in ex.steps:
+        if kind != "host":
+            continue
+        node = ex.by_name[x]
+        if node.op == "nn.batch_flatten":
+            continue
+        xin = _f64(ex.entries[node.inputs[0]])
+        got = _f64(ex.entries[node.name])
+        ref = ograph.eval_node(node, [xin])
+        if node.op == "nn.max_pool2d":
+            assert_bit_exact(got, ref, node.name)  # max of bf16 values is exact
+        else:
+            assert_close(got, ref, node.name)
+
+
+def test_resnet50_small_image_every_region_teacher_forced():
+    import torch
+    res, inp = E.build_resnet50(N=2, H=64, W=64)
+    assert len(res.regions) == 54
+    ex = E.Executor(res)
+    ex.set_input("data", torch.from_numpy(inp["data"]).to(torch.bfloat16).cuda())
+    ex.run_steps()
+    torch.cuda.synchronize()
+    ex.check()
+    g = ex.graph
+    for r in ex.regions:
+        feed = {n: _f64(ex.entries[n]) for n in r.inputs}
+        ref = ograph.evaluate(g, feed, nodes=[n.name for n in r.nodes], keep=r.outputs)
+        for o in r.outputs:
+            assert_close(_f64(ex.entries[o]), ref[o], f"{r.name}:{o}")
+    _check_host_steps(ex)
+    # end-to-end (not gated): fp64 oracle forward from the same input
+    full = ograph.evaluate(g, inp)[g.outputs[0]]
+    got = _f64(ex.output())
+    rel = np.linalg.norm(got - full) / np.linalg.norm(full)
+    print(f"resnet50 N=2 64x64 end-to-end logits relative L2 error {rel:.4f}")
+    assert rel < 0.2
+    ex.release()
+
+
+def test_resnet50_graph_replay_equals_eager():
+    import torch
+    res, inp = E.build_resnet50(N=2, H=64, W=64)
+    ex = E.Executor(res)
+    ex.set_input("data", torch.from_numpy(inp["data"]).to(torch.bfloat16).cuda())
+    ex.run_steps()
+    torch.cuda.synchronize()
+    eager = ex.output().clone()
+    ex.output().fill_(float("nan"))
+    ex.capture()
+    ex.replay()
+    torch.cuda.synchronize()
+    ex.check()
+    assert torch.equal(ex.output(), eager)
+    ex.release()
+
+
+def _sampled_region_ref(g, r, feed, out_name, rng, count):
+    """Oracle value of a single-composite region at `count` random outputs."""
+    nodes = r.nodes
+    conv = nodes[0]
+    assert conv.op in ("nn.conv2d", "nn.dense")
+    shp = g.shape_of(out_name)
+    C = shp[-1]
+    rows = int(np.prod(shp[:-1]))
+    pix = rng.integers(0, rows, size=count)
+    ks = rng.integers(0, C, size=count)
+    x = feed[conv.inputs[0]]
+    if conv.op == "nn.conv2d":
+        a = conv.attrs
+        v = ops.conv2d_nhwc_sampled(x, conv.consts["weight"], pix, ks, a["strides"], a["padding"],
+                                    a["dilation"], a["groups"])
+    else:
+        v = np.array([ops.dense(x[p:p + 1], conv.consts["weight"][k:k + 1])[0, 0]
+                      for p, k in zip(pix, ks)])
+    cur = conv.name
+    y = v.reshape(1, -1)
+    for n in nodes[1:]:
+        if n.op == "nn.bias_add":
+            y = ops.bias_add(y, n.consts["bias"][ks])
+        elif n.op == "nn.batch_norm":
+            y = ops.batch_norm(y, n.consts["gamma"][ks], n.consts["beta"][ks],
+                               n.consts["moving_mean"][ks], n.consts["moving_var"][ks],
+                               n.attrs.get("epsilon", 1e-5))
+        elif n.op == "add":
+            other = [i for i in n.inputs if i != cur][0]
+            y = ops.add(y, feed[other].reshape(-1, C)[pix, ks].reshape(1, -1))
+        elif n.op == "nn.relu":
+            y = ops.relu(y)
+        elif n.op == "clip":
+            y = ops.relu6(y)
+        else:
+            raise NotImplementedError(n.op)
+        cur = n.name
+    return pix, ks, y.ravel()
+
+
+def test_resnet50_full_batch64_sampled_teacher_forced():
+    """The benchmark's configuration: N=64, 224x224.  Every region checked on
+    512 sampled outputs against the oracle fed the GPU's region inputs."""
+    import torch
+    res, inp = E.build_resnet50(N=64)
+    ex = E.Executor(res)
+    ex.set_input("data", torch.from_numpy(inp["data"]).to(torch.bfloat16).cuda())
+    ex.capture()          # the benchmark's launch configuration: graph replay
+    ex.replay()
+    torch.cuda.synchronize()
+    ex.check()
+    g = ex.graph
+    rng = np.random.default_rng(123)
+    cache = {}
+    for r in ex.regions:
+        feed = {}
+        for n in r.inputs:
+            if n not in cache:
+                cache = {k: v for k, v in cache.items() if k in r.inputs}
+                cache[n] = _f64(ex.entries[n])
+            feed[n] = cache[n]
+        out = r.outputs[0]
+        pix, ks, ref = _sampled_region_ref(g, r, feed, out, rng, 512)
+        got = ex.entries[out].reshape(-1, g.shape_of(out)[-1])[torch.from_numpy(pix).cuda(),
+                                                              torch.from_numpy(ks).cuda()]
+        # element rule with the full output's dynamic range
+        scale = max(1.0, float(ex.entries[out].abs().max().float()))
+        d = np.abs(got.float().cpu().numpy() - ref)
+        bad = ~(d <= 1e-2 * scale + 2e-2 * np.abs(ref))
+        assert not bad.any(), f"{r.name}: {int(bad.sum())}/512 sampled outputs out of tolerance, max {d.max()}"
+    _check_host_steps(ex)
+    ex.release()
