@@ -188,6 +188,33 @@ byoc_status byoc_max_pool2d_nhwc(const void *x, void *y, int32_t N, int32_t H, i
 byoc_status byoc_global_avg_pool_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W,
                                       int32_t C, void *cuda_stream);
 
+/* ---------------------------------------------------------------------------
+ * Allocation-free entry point.  The paper has no counterpart: it exists for
+ * callers that cannot allocate device memory -- code running inside a memory
+ * pool or arena it does not own, or an inference path that must not take an
+ * allocator lock or trigger the implicit synchronisation of cudaMalloc.
+ * byoc_compile allocates; this call does not.
+ *
+ * Computes y = GELU(x . w1^T + b1) . w2^T + b2 (the dense + bias + GELU ->
+ * dense + bias chain) with the same tcgen05 kernel byoc_run uses:
+ *   x  [M, D] bf16, w1 [F, D] bf16, b1 [F] fp32, w2 [D, F] bf16, b2 [D] fp32,
+ *   y  [M, D] bf16; all device pointers, row-major, 16-byte aligned.
+ *   D and F must be multiples of 128; M * F must not exceed 8,388,608
+ *   (the hidden activation goes to a fixed 16 MiB device array that every GPU
+ *   loading the library reserves until exit); larger problems fail with
+ *   BYOC_ERR_INVALID_ARG -- split the rows over several calls.
+ * The first call on each device, with that device current, looks up the
+ * array's device address and raises the kernel's shared-memory limit; make
+ * that first call before any stream capture.  Every call shares the array,
+ * so calls that overlap on the GPU (for example on two streams) race; order
+ * them on one stream.  The call enqueues work on cuda_stream and returns; a
+ * bounded-wait timeout inside the kernels is recorded in the array but not
+ * reported.  It calls no cudaMalloc, cudaFree or other allocating routine.
+ * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
+byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int32_t F, const void *w1,
+                             const float *b1, const void *w2, const float *b2, void *y,
+                             void *cuda_stream);
+
 /* Number of SMs and the device's compute capability, for host-side planning
  * (current device).  Errors: CUDA. */
 byoc_status byoc_device_info(int32_t *num_sms, int32_t *cc_major, int32_t *cc_minor);

@@ -82,6 +82,9 @@ cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st);
 
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            int k, int s, int p, cudaStream_t st);
+// Sets the thread-local message byoc_last_error() returns.
+void set_last_error(const char *msg);
+
 cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            cudaStream_t st);
 

@@ -694,6 +694,10 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
 
 }  // namespace
 
+namespace byoc {
+void set_last_error(const char *msg) { g_err = msg ? msg : ""; }
+}  // namespace byoc
+
 // ------------------------------------------------------------ the handle
 
 struct byoc_handle {
