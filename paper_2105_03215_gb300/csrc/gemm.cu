@@ -4,49 +4,61 @@
 // (Section 3.1.1: a Conv2D-Add-ReLU style sequence mapped to one
 // "instruction") makes one pass over HBM.
 //
-// Structure (one persistent CTA per SM, 192 threads):
-//   warp 0     TMA producer: per k-block, one A tile (128 rows x BK) and one
-//              B tile (BN rows x BK) into a STAGES-deep shared-memory ring.
-//              A is a 2-D tile of a row-major matrix, or -- for convolutions --
-//              an im2col tile: 128 consecutive output pixels of one filter tap
-//              and channel chunk, with out-of-image taps zero-filled by TMA.
+// Structure (one persistent CTA per SM, 320 threads):
+//   warp 0 lane 0  TMA producer of the mainloop: per k-block, one A tile (128
+//              rows x BK) and one B tile (BN rows x BK) into a STAGES-deep
+//              shared-memory ring.  A is a 2-D tile of a row-major matrix, or
+//              -- for convolutions -- an im2col tile: 128 consecutive output
+//              pixels of one filter tap and channel chunk, with out-of-image
+//              taps zero-filled by TMA.
+//   warp 0 lane 1  producer of the epilogue operands: per tile, the tile's
+//              bias slice (bulk copy) and, when the region adds a residual,
+//              the 128 x BN residual tile (TMA) into one of two buffers, well
+//              before the epilogue needs them.
 //   warp 1     allocates TMEM; one lane issues tcgen05.mma (M=128, N=BN, K=16
 //              per instruction) into one of two fp32 accumulators in TMEM and
 //              tcgen05.commit's the ring slots and the finished accumulator.
 //   warps 2-9  epilogue: two warps per 32-row TMEM lane quarter, taking
 //              alternate 32-column chunks.  Per chunk: tcgen05.ld (one row per
-//              thread), + bias, + residual, activation, bf16 rounding, then a
-//              transpose through a 64-byte-swizzled shared-memory tile so that
-//              the global stores are coalesced 64-byte row segments.  The
-//              residual is read with the same coalesced pattern, two of the
-//              warp's chunks ahead, into registers.  The accumulator is
-//              released as soon as it has been read, so the next tile's MMAs
-//              overlap this tile's stores.
+//              thread), + bias and + residual from shared memory, activation,
+//              bf16 rounding, then a transpose through a 64-byte-swizzled
+//              shared-memory tile so that the global stores are coalesced
+//              64-byte row segments.  The accumulator is released as soon as
+//              it has been read, so the next tile's MMAs overlap this tile's
+//              stores.
 #include "internal.h"
 #include "ptx.cuh"
 
 namespace byoc {
 
-template <int BN, int BK>
+template <int BN, int BK, bool RES>
 struct GemmShape {
     static constexpr int BM = kGemmBM;
     static constexpr int A_BYTES = BM * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int RING_BUDGET = 192 * 1024;
-    static constexpr int STAGES_RAW = RING_BUDGET / STAGE_BYTES;
-    static constexpr int STAGES = STAGES_RAW > 16 ? 16 : STAGES_RAW;
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
-    // Epilogue staging per warp: one output and one residual 32x32 bf16 tile.
+    // residual tile: BN/64 boxes of 64 columns x 128 rows, 128-byte swizzle
+    static constexpr int RES_BOX = BM * 64 * 2;
+    static constexpr int RES_TILE = RES ? BM * BN * 2 : 0;
+    static constexpr int BIAS_BYTES = BN * 4;
+    static constexpr int BIAS_REGION = (2 * BIAS_BYTES + 1023) / 1024 * 1024;
+    // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
-    static constexpr int EPI_WARP_BYTES = 2 * EPI_TILE;
-    static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_WARP_BYTES;
-    static constexpr int NUM_BARS = 2 * STAGES + 5;
-    static constexpr int CTRL_BYTES = 8 * NUM_BARS + 16;
-    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + EPI_BYTES + CTRL_BYTES;
+    static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE;
+    static constexpr int CTRL_BYTES = 512;
+    static constexpr int FIXED = 1024 + 2 * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
+    static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
+    static constexpr int STAGES = STAGES_RAW > 16 ? 16 : STAGES_RAW;
+    static constexpr int NUM_BARS = 2 * STAGES + 9;
+    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 2 * RES_TILE + EPI_BYTES +
+                                      BIAS_REGION + CTRL_BYTES;
+    static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
+    static_assert(STAGES >= 2, "ring depth");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
     static_assert(A_BYTES % 1024 == 0 && B_BYTES % 1024 == 0, "tiles must keep 1 KB alignment");
     static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "BN");
+    static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
 };
 
@@ -59,24 +71,29 @@ __device__ __forceinline__ float apply_act(float v, int act) {
     }
 }
 
-template <int BN, int BK, bool IM2COL>
+template <int BN, int BK, bool IM2COL, bool RES>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA,
-                        const __grid_constant__ CUtensorMap tmB, const GemmArgs a) {
-    using S = GemmShape<BN, BK>;
+                        const __grid_constant__ CUtensorMap tmB,
+                        const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
+    using S = GemmShape<BN, BK, RES>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t *smem = smem_raw + (base - raw);
     const uint32_t sA = base;
-    const uint32_t sB = base + S::STAGES * S::A_BYTES;
-    const uint32_t sEpi = base + S::STAGES * S::STAGE_BYTES;
-    const uint32_t bars = sEpi + S::EPI_BYTES;
-    const uint32_t tfull = bars + 8u * (2 * S::STAGES);  // 2 barriers
-    const uint32_t tempty = tfull + 16u;                 // 2 barriers
-    const uint32_t drain = tempty + 16u;
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(
-        smem + S::STAGES * S::STAGE_BYTES + S::EPI_BYTES + 8 * S::NUM_BARS);
+    const uint32_t sB = sA + S::STAGES * S::A_BYTES;
+    const uint32_t sRes = sB + S::STAGES * S::B_BYTES;     // 2 x RES_TILE
+    const uint32_t sEpi = sRes + 2 * S::RES_TILE;          // EPI_BYTES
+    const uint32_t sBias = sEpi + S::EPI_BYTES;            // 2 x BIAS_BYTES
+    const uint32_t ctrl = sBias + S::BIAS_REGION;
+    const uint32_t bars = ctrl;                            // full[S], empty[S]
+    const uint32_t tfull = bars + 8u * (2 * S::STAGES);    // 2: accumulator ready
+    const uint32_t tempty = tfull + 16u;                   // 2: accumulator drained
+    const uint32_t ofull = tempty + 16u;                   // 2: epilogue operands loaded
+    const uint32_t oempty = ofull + 16u;                   // 2: epilogue operands consumed
+    const uint32_t drain = oempty + 16u;
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
     const int warp = threadIdx.x >> 5;
@@ -88,8 +105,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(bars + 8u * (S::STAGES + s), 1);    // empty[s]: MMA commit
         }
         for (int b = 0; b < 2; ++b) {
-            mbar_init(tfull + 8u * b, 1);   // accumulator ready: MMA commit
-            mbar_init(tempty + 8u * b, kGemmEpiWarps);  // drained: one arrive per epilogue warp
+            mbar_init(tfull + 8u * b, 1);                 // MMA commit
+            mbar_init(tempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
+            mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
+            mbar_init(oempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -98,6 +117,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
+        if (RES) tma_prefetch_desc(&tmR);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), S::TMEM_COLS);
@@ -110,30 +130,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            // ------------------------------------------------ TMA producer
-            // The residual tile of the tile RES_L2_AHEAD steps ahead is pulled
-            // into L2 when a tile's loads start, so the epilogue's residual
-            // reads hit L2 instead of waiting on HBM.
-            constexpr int RES_L2_AHEAD = 2;
-            auto prefetch_residual = [&](int tile_i) {
-                if (!a.residual || tile_i >= a.num_tiles) return;
-                const int pm0 = (tile_i / a.tiles_n) * S::BM;
-                const int pn0 = (tile_i % a.tiles_n) * BN;
-                const int rows = min(S::BM, a.M - pm0);
-                const int cols = min(BN, a.N - pn0);
-                const __nv_bfloat16 *base = a.residual + (size_t)pm0 * a.N + pn0;
-                if (cols == a.N) {
-                    bulk_prefetch_l2(base, (uint32_t)rows * (uint32_t)a.N * 2u);
-                } else {
-                    for (int r = 0; r < rows; ++r)
-                        bulk_prefetch_l2(base + (size_t)r * a.N, (uint32_t)cols * 2u);
-                }
-            };
-            for (int d = 0; d < RES_L2_AHEAD; ++d) prefetch_residual(blockIdx.x + d * gridDim.x);
+            // ------------------------------------------------ mainloop producer
             int it = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x) {
-                prefetch_residual(tile + RES_L2_AHEAD * gridDim.x);
                 const int m0 = (tile / a.tiles_n) * S::BM;
                 const int n0 = (tile % a.tiles_n) * BN;
                 int img = 0, h0 = 0, w0 = 0;
@@ -175,6 +175,28 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 for (int j = first; j < it; ++j)
                     mbar_wait_drain(bars + 8u * (j % S::STAGES), (uint32_t)(j / S::STAGES) & 1u);
             }
+        } else if (lane == 1) {
+            // ------------------------------------------------ epilogue-operand producer
+            int t = 0;
+            for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
+                const int ob = t & 1;
+                const uint32_t oph = (uint32_t)(t >> 1) & 1u;
+                if (!mbar_wait(oempty + 8u * ob, oph ^ 1u, abort_flag, a.err, kErrTimeoutProducer))
+                    break;
+                const int m0 = (tile / a.tiles_n) * S::BM;
+                const int n0 = (tile % a.tiles_n) * BN;
+                mbar_arrive_expect_tx(ofull + 8u * ob, S::BIAS_BYTES + S::RES_TILE);
+                bulk_load_1d(sBias + ob * S::BIAS_BYTES, a.bias + n0, S::BIAS_BYTES, ofull + 8u * ob);
+                if (RES) {
+#pragma unroll
+                    for (int j = 0; j < BN / 64; ++j)
+                        tma_load_2d(sRes + ob * S::RES_TILE + j * S::RES_BOX, &tmR, ofull + 8u * ob,
+                                    n0 + 64 * j, m0);
+                }
+            }
+            // Let the last operand loads land before the CTA can exit.
+            if (t > 0) mbar_wait_drain(ofull + 8u * ((t - 1) & 1), (uint32_t)((t - 1) >> 1) & 1u);
+            if (t > 1) mbar_wait_drain(ofull + 8u * ((t - 2) & 1), (uint32_t)((t - 2) >> 1) & 1u);
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -222,71 +244,41 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         const int quarter = warp & 3;      // TMEM lanes (= tile rows) this warp may access
         const int half = e >> 2;           // takes chunks ci with ci % 2 == half
         constexpr int NCH = BN / 32;       // 32-column chunks per tile
-        const uint32_t stg_out = sEpi + (uint32_t)e * S::EPI_WARP_BYTES;
-        const uint32_t stg_res = stg_out + S::EPI_TILE;
-        const bool has_res = a.residual != nullptr;
-        // 64-byte swizzle of the 32x32 bf16 staging tiles: 16-byte piece c of row
-        // r sits at piece c ^ ((r >> 1) & 3), so both the row-per-thread and
-        // the coalesced access patterns below are free of bank conflicts.
+        const uint32_t stg = sEpi + (uint32_t)e * S::EPI_TILE;
+        const int trow = quarter * 32 + lane;  // this thread's row within the tile
+        // 64-byte swizzle of the 32x32 bf16 staging tile: 16-byte piece c of
+        // row r sits at piece c ^ ((r >> 1) & 3), so both the row-per-thread
+        // writes and the coalesced reads below are free of bank conflicts.
         const uint32_t sw_own = ((uint32_t)lane >> 1) & 3u;
-        // coalesced pattern: access k (0..3) covers rows 8k + lane/4, piece lane%4
-        const int cl_row = lane >> 2, cl_piece = lane & 3;
-
-        // The warp's chunk sequence: tiles blockIdx.x + i*gridDim.x, chunks
-        // half, half+2, ... of each.  The residual of the next assignment is
-        // loaded (coalesced) while the current one is processed.
-        auto res_load = [&](int tile_i, int ci, uint4 (&r)[4]) {
-#pragma unroll
-            for (int k = 0; k < 4; ++k) r[k] = make_uint4(0u, 0u, 0u, 0u);
-            if (tile_i >= a.num_tiles) return;
-            const int rrow0 = (tile_i / a.tiles_n) * S::BM + quarter * 32;
-            const int rcol = (tile_i % a.tiles_n) * BN + ci * 32 + cl_piece * 8;
-            if (rcol >= a.N) return;
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int row = rrow0 + 8 * k + cl_row;
-                if (row < a.M)
-                    r[k] = __ldg(reinterpret_cast<const uint4 *>(a.residual + (size_t)row * a.N + rcol));
-            }
-        };
-        auto advance = [&](int &tile_i, int &ci) {
-            ci += 2;
-            if (ci >= NCH) {
-                ci = half;
-                tile_i += gridDim.x;
-            }
-        };
-        uint4 rcur[4];
-        int pf_tile = blockIdx.x, pf_ci = half;  // assignment whose residual rcur holds
-        if (has_res && half < NCH) res_load(pf_tile, pf_ci, rcur);
+        const int cl_row = lane >> 2, cl_piece = lane & 3;  // coalesced: rows 8k + lane/4
         int t = 0;
         for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
             const int buf = t & 1;
             const uint32_t aph = (uint32_t)(t >> 1) & 1u;
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
+            if (!mbar_wait(ofull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
             tc_fence_after();
             const int m0 = (tile / a.tiles_n) * S::BM;
             const int n0 = (tile % a.tiles_n) * BN;
             const int row0 = m0 + quarter * 32;
             const uint32_t tbase =
                 tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
+            const uint32_t bias_s = sBias + (uint32_t)(buf * S::BIAS_BYTES);
+            const uint32_t res_s = sRes + (uint32_t)(buf * S::RES_TILE);
             if (half >= NCH) {  // no chunk for this warp in this tile (BN = 32)
                 tc_fence_before();
                 __syncwarp();
-                if (lane == 0) mbar_arrive(tempty + 8u * buf);
+                if (lane == 0) {
+                    mbar_arrive(tempty + 8u * buf);
+                    mbar_arrive(oempty + 8u * buf);
+                }
                 continue;
             }
 #pragma unroll 1
             for (int ci = half; ci < NCH; ci += 2) {
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
-                tmem_ld_32cols_nowait(tbase + (uint32_t)(ci * 32), v);
-                uint4 rnext[4];
-                if (has_res) {
-                    advance(pf_tile, pf_ci);
-                    res_load(pf_tile, pf_ci, rnext);
-                }
-                tmem_ld_wait_regs(v);
+                tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);  // includes tcgen05.wait::ld
                 if (ci + 2 >= NCH) {  // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
@@ -294,39 +286,27 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 }
                 float f[32];
 #pragma unroll
-                for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]);
-                if (a.bias) {
-                    const float4 *bp = reinterpret_cast<const float4 *>(a.bias + col0);
-#pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        const float4 b4 = __ldg(bp + j);
-                        f[4 * j] += b4.x;
-                        f[4 * j + 1] += b4.y;
-                        f[4 * j + 2] += b4.z;
-                        f[4 * j + 3] += b4.w;
-                    }
+                for (int j = 0; j < 8; ++j) {  // bias: same address in every lane (broadcast)
+                    float4 b4;
+                    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                                 : "=f"(b4.x), "=f"(b4.y), "=f"(b4.z), "=f"(b4.w)
+                                 : "r"(bias_s + (uint32_t)(ci * 32 + 4 * j) * 4u));
+                    f[4 * j] = __uint_as_float(v[4 * j]) + b4.x;
+                    f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4.y;
+                    f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4.z;
+                    f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4.w;
                 }
-                if (has_res) {
-                    // coalesced registers -> swizzled staging -> this thread's row
-                    __syncwarp();
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) {
-                        const uint32_t r = (uint32_t)(8 * k + cl_row);
-                        const uint32_t addr =
-                            stg_res + r * 64u + ((((uint32_t)cl_piece) ^ ((r >> 1) & 3u)) << 4);
-                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr),
-                                     "r"(rcur[k].x), "r"(rcur[k].y), "r"(rcur[k].z), "r"(rcur[k].w)
-                                     : "memory");
-                    }
-                    __syncwarp();
+                if (RES) {
+                    // residual row `trow`, columns ci*32.. of the 128B-swizzled box ci/2
+                    const uint32_t rbox =
+                        res_s + (uint32_t)((ci >> 1) * S::RES_BOX) + (uint32_t)trow * 128u;
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
+                        const uint32_t piece = (uint32_t)((ci & 1) * 4 + q) ^ ((uint32_t)trow & 7u);
                         uint4 r4;
-                        const uint32_t addr = stg_res + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
                         asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
                                      : "=r"(r4.x), "=r"(r4.y), "=r"(r4.z), "=r"(r4.w)
-                                     : "r"(addr)
-                                     : "memory");
+                                     : "r"(rbox + (piece << 4)));
                         const uint32_t rr[4] = {r4.x, r4.y, r4.z, r4.w};
 #pragma unroll
                         for (int e2 = 0; e2 < 4; ++e2) {
@@ -334,8 +314,6 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                             f[8 * q + 2 * e2 + 1] += bf16hi(rr[e2]);
                         }
                     }
-#pragma unroll
-                    for (int k = 0; k < 4; ++k) rcur[k] = rnext[k];
                 }
 #pragma unroll
                 for (int j = 0; j < 32; ++j) f[j] = apply_act(f[j], a.act);
@@ -347,7 +325,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
                     const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
                     const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
-                    const uint32_t addr = stg_out + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
+                    const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
                     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0),
                                  "r"(w1), "r"(w2), "r"(w3)
                                  : "memory");
@@ -358,7 +336,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 for (int k = 0; k < 4; ++k) {
                     const uint32_t r = (uint32_t)(8 * k + cl_row);
                     const uint32_t addr =
-                        stg_out + r * 64u + ((((uint32_t)cl_piece) ^ ((r >> 1) & 3u)) << 4);
+                        stg + r * 64u + ((((uint32_t)cl_piece) ^ ((r >> 1) & 3u)) << 4);
                     uint4 o;
                     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
                                  : "=r"(o.x), "=r"(o.y), "=r"(o.z), "=r"(o.w)
@@ -369,6 +347,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         *reinterpret_cast<uint4 *>(a.out + (size_t)row * a.N + gcol) = o;
                 }
             }
+            // bias / residual reads of this tile are done (ordered by __syncwarp)
+            __syncwarp();
+            if (lane == 0) mbar_arrive(oempty + 8u * buf);
         }
     }
 
@@ -383,72 +364,79 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
 // ---------------------------------------------------------------- dispatch
 
-template <int BN, int BK, bool IM2COL>
-static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const GemmArgs &a,
-                            int grid, cudaStream_t st) {
-    using S = GemmShape<BN, BK>;
-    gemm_tcgen05_kernel<BN, BK, IM2COL><<<grid, kGemmThreads, S::SMEM_BYTES, st>>>(tmA, tmB, a);
+template <int BN, int BK, bool IM2COL, bool RES>
+static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap &tmR,
+                            const GemmArgs &a, int grid, cudaStream_t st) {
+    using S = GemmShape<BN, BK, RES>;
+    gemm_tcgen05_kernel<BN, BK, IM2COL, RES>
+        <<<grid, kGemmThreads, S::SMEM_BYTES, st>>>(tmA, tmB, tmR, a);
     return cudaGetLastError();
 }
 
-template <int BN, int BK, bool IM2COL>
+template <int BN, int BK, bool IM2COL, bool RES>
 static cudaError_t prepare_t() {
-    using S = GemmShape<BN, BK>;
-    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, IM2COL>,
+    using S = GemmShape<BN, BK, RES>;
+    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, IM2COL, RES>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, S::SMEM_BYTES);
 }
 
-// The instantiated (BN, BK, im2col) combinations.
-#define BYOC_GEMM_CONFIGS(X) \
-    X(32, 64, false)         \
-    X(64, 64, false)         \
-    X(128, 64, false)        \
-    X(256, 64, false)        \
-    X(32, 64, true)          \
-    X(64, 64, true)          \
-    X(128, 64, true)         \
-    X(256, 64, true)         \
-    X(64, 16, true)          \
-    X(64, 32, true)          \
-    X(128, 32, true)
+// The instantiated (BN, BK, im2col, residual) combinations.
+#define BYOC_GEMM_CONFIGS(X)  \
+    X(32, 64, false, false)   \
+    X(64, 64, false, false)   \
+    X(128, 64, false, false)  \
+    X(256, 64, false, false)  \
+    X(32, 64, true, false)    \
+    X(64, 64, true, false)    \
+    X(128, 64, true, false)   \
+    X(256, 64, true, false)   \
+    X(64, 16, true, false)    \
+    X(64, 32, true, false)    \
+    X(128, 32, true, false)   \
+    X(64, 64, false, true)    \
+    X(128, 64, false, true)   \
+    X(64, 64, true, true)     \
+    X(128, 64, true, true)
 
 bool gemm_config_supported(const GemmConfig &c) {
-#define X(BN_, BK_, IM_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_) return true;
+#define X(BN_, BK_, IM_, RES_) \
+    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) return true;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return false;
 }
 
 size_t gemm_smem_bytes(const GemmConfig &c) {
-#define X(BN_, BK_, IM_) \
-    if (c.bn == BN_ && c.bk == BK_) return (size_t)GemmShape<BN_, BK_>::SMEM_BYTES;
+#define X(BN_, BK_, IM_, RES_)                                 \
+    if (c.bn == BN_ && c.bk == BK_ && c.res == RES_) \
+        return (size_t)GemmShape<BN_, BK_, RES_>::SMEM_BYTES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 int gemm_stages(const GemmConfig &c) {
-#define X(BN_, BK_, IM_) \
-    if (c.bn == BN_ && c.bk == BK_) return GemmShape<BN_, BK_>::STAGES;
+#define X(BN_, BK_, IM_, RES_) \
+    if (c.bn == BN_ && c.bk == BK_ && c.res == RES_) return GemmShape<BN_, BK_, RES_>::STAGES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 cudaError_t gemm_prepare(const GemmConfig &c) {
-#define X(BN_, BK_, IM_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_) return prepare_t<BN_, BK_, IM_>();
+#define X(BN_, BK_, IM_, RES_)                                              \
+    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) \
+        return prepare_t<BN_, BK_, IM_, RES_>();
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_gemm(const GemmConfig &c, const CUtensorMap &tmA, const CUtensorMap &tmB,
-                        const GemmArgs &a, int grid, cudaStream_t st) {
-#define X(BN_, BK_, IM_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_) \
-        return launch_t<BN_, BK_, IM_>(tmA, tmB, a, grid, st);
+                        const CUtensorMap &tmR, const GemmArgs &a, int grid, cudaStream_t st) {
+#define X(BN_, BK_, IM_, RES_)                                              \
+    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) \
+        return launch_t<BN_, BK_, IM_, RES_>(tmA, tmB, tmR, a, grid, st);
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;

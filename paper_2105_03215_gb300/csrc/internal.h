@@ -30,7 +30,7 @@ struct GemmArgs {
     int tiles_n;    // number of BN-wide column tiles
     int num_tiles;  // tiles_m * tiles_n
     int act;        // Act
-    const float *bias;                // [tiles_n * BN], zero padded; may be null
+    const float *bias;                // [tiles_n * BN], zero padded; required
     const __nv_bfloat16 *residual;    // [M, N] or null
     __nv_bfloat16 *out;               // [M, N]
     int *err;                         // device error word
@@ -40,6 +40,7 @@ struct GemmConfig {
     int bn;       // tile width in output channels: 32, 64, 128, 256
     int bk;       // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
     bool im2col;  // A operand through an im2col tensor map
+    bool res;     // epilogue adds a residual tile (bn 64 or 128)
 };
 
 constexpr int kGemmBM = 128;
@@ -50,8 +51,10 @@ bool gemm_config_supported(const GemmConfig &cfg);
 size_t gemm_smem_bytes(const GemmConfig &cfg);
 int gemm_stages(const GemmConfig &cfg);
 cudaError_t gemm_prepare(const GemmConfig &cfg);  // raises the dynamic smem limit
+// tmR: residual [M, N] bf16 in 64-column x 128-row boxes, 128-byte swizzle
+// (read only when cfg.res).  a.bias must cover tiles_n * bn floats.
 cudaError_t launch_gemm(const GemmConfig &cfg, const CUtensorMap &tmA, const CUtensorMap &tmB,
-                        const GemmArgs &a, int grid, cudaStream_t st);
+                        const CUtensorMap &tmR, const GemmArgs &a, int grid, cudaStream_t st);
 
 // Depthwise conv (groups = C), square kernel k in {3}, NHWC bf16, folded
 // weights fp32 [k*k][C] (tap-major), bias fp32 [C], fused activation.

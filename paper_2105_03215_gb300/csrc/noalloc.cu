@@ -61,7 +61,7 @@ byoc_status cuda_fail(cudaError_t e, const char *what) {
 void setup_device(DeviceState &d, int dev) {
     cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&d.scratch), g_ffn_scratch);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = byoc::gemm_prepare(byoc::GemmConfig{kTileN, 64, false});
+    if (e == cudaSuccess) e = byoc::gemm_prepare(byoc::GemmConfig{kTileN, 64, false, false});
     d.err = e;
 }
 
@@ -125,7 +125,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
         encode(&b2m, w2, (uint64_t)D, (uint64_t)F, kTileN) != CUDA_SUCCESS)
         return fail(BYOC_ERR_CUDA, "byoc_ffn_noalloc: encoding a TMA descriptor failed");
 
-    const byoc::GemmConfig cfg{kTileN, 64, false};
+    const byoc::GemmConfig cfg{kTileN, 64, false, false};
     const int tiles_m = (M + byoc::kGemmBM - 1) / byoc::kGemmBM;
     byoc::GemmArgs g{};
     g.M = M;
@@ -143,7 +143,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.residual = nullptr;
     g.out = hidden;
     g.err = err_word;
-    if ((e = byoc::launch_gemm(cfg, a1, b1m, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a1, b1m, a1, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: first GEMM launch");
     g.N = D;
@@ -154,7 +154,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.act = byoc::kActNone;
     g.bias = b2;
     g.out = static_cast<__nv_bfloat16 *>(y);
-    if ((e = byoc::launch_gemm(cfg, a2, b2m, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a2, b2m, a2, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: second GEMM launch");
     return BYOC_OK;

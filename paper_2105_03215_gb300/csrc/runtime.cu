@@ -152,7 +152,7 @@ struct LaunchPlan {
     int x = -1, y = -1, res = -1;  // tensor ids (may index internal scratch tensors)
     int act = byoc::kActNone;
     // GEMM
-    GemmConfig cfg{64, 64, false};
+    GemmConfig cfg{64, 64, false, false};
     GemmArgs args{};
     int grid = 0;
     int n_pad = 0, k_pack = 0;
@@ -343,11 +343,11 @@ int pick_bk(int64_t C) {
 //                        per accumulator row block work in parallel).
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
 // time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
-int pick_bn(int64_t M, int64_t N, int64_t kblocks, int bk, bool im2col, int num_sms) {
+int pick_bn(int64_t M, int64_t N, int64_t kblocks, int bk, bool im2col, bool res, int num_sms) {
     int best = -1;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
-        GemmConfig c{bn, bk, im2col};
+        GemmConfig c{bn, bk, im2col, res};
         if (!byoc::gemm_config_supported(c)) continue;
         const int64_t tiles = ((M + 127) / 128) * ((N + bn - 1) / bn);
         const int64_t grid = std::min<int64_t>(tiles, num_sms);
@@ -600,11 +600,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         taps = kh * kw;
         bk = op.kind == BYOC_OP_DENSE ? 64 : pick_bk(C);
         chunks = (int)((C + bk - 1) / bk);
-        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks, bk, im2col, P.num_sms);
+        const bool has_res = res >= 0;
+        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks, bk, im2col, has_res, P.num_sms);
         if (bn < 0)
-            return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d im2col=%d", o, bk,
-                        (int)im2col);
-        L.cfg = GemmConfig{bn, bk, im2col};
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d im2col=%d residual=%d",
+                        o, bk, (int)im2col, (int)has_res);
+        L.cfg = GemmConfig{bn, bk, im2col, has_res};
         L.n_pad = (int)((Cout + bn - 1) / bn * bn);
         L.k_pack = taps * chunks * bk;
         Kreal = (int64_t)taps * C;
@@ -709,6 +710,8 @@ struct byoc_handle {
     std::vector<CUtensorMap> tmB;         // per launch (GEMM only)
     std::vector<CUtensorMap> tmA;         // per launch, cached
     std::vector<const void *> tmA_ptr;    // pointer each cached A map encodes
+    std::vector<CUtensorMap> tmR;         // per launch: residual map, cached
+    std::vector<const void *> tmR_ptr;
     std::vector<void *> ptrs;             // scratch: resolved tensor pointers
 };
 
@@ -820,6 +823,8 @@ byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
     h->tmB.resize(nl);
     h->tmA.resize(nl);
     h->tmA_ptr.assign(nl, nullptr);
+    h->tmR.resize(nl);
+    h->tmR_ptr.assign(nl, nullptr);
     h->ptrs.assign(P.tensors.size(), nullptr);
     for (size_t i = 0; i < nl; ++i) {
         LaunchPlan &L = P.launches[i];
@@ -887,7 +892,17 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             GemmArgs a = L.args;
             a.out = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
             a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
-            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a, L.grid, st);
+            if (a.residual && h->tmR_ptr[i] != a.residual) {
+                // residual [M, N]: 64-column x 128-row boxes, 128-byte swizzle
+                CUresult r = encode_2d(&h->tmR[i], a.residual, (uint64_t)a.M, (uint64_t)a.N,
+                                       byoc::kGemmBM, 64, 64);
+                if (r != CUDA_SUCCESS)
+                    return fail(BYOC_ERR_CUDA, "launch %zu: encoding the residual TMA map failed (%d)",
+                                i, (int)r);
+                h->tmR_ptr[i] = a.residual;
+            }
+            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a.residual ? h->tmR[i] : h->tmA[i], a,
+                                  L.grid, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             byoc::DwArgs a = L.dw;
             a.x = static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]);
