@@ -233,6 +233,8 @@ def main():
     ap.add_argument("--no-regions", action="store_true", help="skip the per-config region figures")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--dump", default=None, help="write the per-region timing breakdown (JSON) here")
+    ap.add_argument("--batch", type=int, default=BATCH,
+                    help="images per step (default 64; smaller only for profiler captures)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     world, rank, local = dist_env()
@@ -250,7 +252,8 @@ def main():
 
     torch.cuda.set_device(local)
     peaks, peak_src = load_peaks()
-    res, inp = E.build_resnet50(N=BATCH, H=IMG, W=IMG)
+    batch = args.batch
+    res, inp = E.build_resnet50(N=batch, H=IMG, W=IMG)
     ex = E.Executor(res)
     host_in = torch.from_numpy(inp["data"]).to(torch.bfloat16).pin_memory()
     host_out = torch.empty(ex.output().shape, dtype=torch.bfloat16).pin_memory()
@@ -284,7 +287,7 @@ def main():
     ex.check()
     step_s = [a.elapsed_time(b) * 1e-3 for a, b in evs]
     total = reduce_max(sum(step_s), world)
-    images = BATCH * args.steps * world
+    images = batch * args.steps * world
     value = images / total
 
     # ------------------------------------------------ per-launch events (roofline)
@@ -371,7 +374,7 @@ def main():
         torch.cuda.synchronize()
         e2e_t.append(time.perf_counter() - t0)
     e2e_total = reduce_max(sum(e2e_t), world)
-    e2e_value = BATCH * len(e2e_t) * world / e2e_total
+    e2e_value = batch * len(e2e_t) * world / e2e_total
 
     regions = None
     if not args.no_regions and rank == 0:
@@ -389,12 +392,12 @@ def main():
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * total / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": "resnet50_v1b_N64_224 (54 offloaded regions, pools on host)",
-                       "global_batch": BATCH * world, "image": IMG, "regions": len(ex.regions),
+            "config": {"workload": f"resnet50_v1b_N{batch}_224 (54 offloaded regions, pools on host)",
+                       "global_batch": batch * world, "image": IMG, "regions": len(ex.regions),
                        "parallelism": f"replicas{world}",
                        "l2": "flushed by a 256 MB write before every timed step",
                        "timing": "CUDA events around CUDA-graph replays"},
-            "tflops": value / BATCH * sum(c.flops for c in ex.compiled) / 1e12,
+            "tflops": value / batch * sum(c.flops for c in ex.compiled) / 1e12,
             "wall_s": wall,
             "clocks": clk,
             "e2e": {"value": e2e_value, "unit": "images/s",
