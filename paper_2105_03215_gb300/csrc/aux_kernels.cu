@@ -68,14 +68,18 @@ __global__ void __launch_bounds__(256, 2) dwconv3x3_kernel(const DwArgs a) {
     const int wc0 = q * STRIDE - a.pad;
     const __nv_bfloat16 *xn = a.x + (size_t)n * a.H * a.W * a.C + c0;
     // one input row under the filter: 3 columns x 4 channels, zero outside the image
+    // Loads are unconditional (from a clamped, in-image address) and zeroed by
+    // a select afterwards, so they can all be in flight at once.
     auto load_row = [&](int h, uint2 (&r)[3]) {
         const bool hv = h >= 0 && h < a.H;
+        const int hc = min(max(h, 0), a.H - 1);
 #pragma unroll
         for (int s = 0; s < 3; ++s) {
             const int wc = wc0 + s;
-            r[s] = (hv && wc >= 0 && wc < a.W)
-                       ? __ldg(reinterpret_cast<const uint2 *>(xn + ((size_t)h * a.W + wc) * a.C))
-                       : make_uint2(0u, 0u);
+            const int wcc = min(max(wc, 0), a.W - 1);
+            const uint2 v = __ldg(reinterpret_cast<const uint2 *>(xn + ((size_t)hc * a.W + wcc) * a.C));
+            const bool ok = hv && wc >= 0 && wc < a.W;
+            r[s] = make_uint2(ok ? v.x : 0u, ok ? v.y : 0u);
         }
     };
     auto unpack_row = [&](const uint2 (&r)[3], float (&f)[3][4]) {
@@ -224,17 +228,19 @@ __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, 
     t /= Wo;
     const int pp = (int)(t % Ho);
     const int n = (int)(t / Ho);
+    // Positions outside the image are replaced by the nearest in-image
+    // position of the same window (padding < k keeps it inside the window),
+    // which leaves the maximum unchanged and makes every load unconditional.
     float m[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) m[j] = -INFINITY;
+    const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
     for (int r = 0; r < k; ++r) {
-        const int h = pp * s - p + r;
-        if (h < 0 || h >= H) continue;
+        const int h = min(max(pp * s - p + r, 0), H - 1);
         for (int c = 0; c < k; ++c) {
-            const int w = q * s - p + c;
-            if (w < 0 || w >= W) continue;
+            const int w = min(max(q * s - p + c, 0), W - 1);
             float f[8];
-            unpack8(ldg_v4(x + (((size_t)n * H + h) * W + w) * C + cv * 8), f);
+            unpack8(ldg_v4(xn + ((size_t)h * W + w) * C), f);
 #pragma unroll
             for (int j = 0; j < 8; ++j) m[j] = fmaxf(m[j], f[j]);
         }
@@ -242,8 +248,51 @@ __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, 
     *reinterpret_cast<uint4 *>(y + (((size_t)n * Ho + pp) * Wo + q) * C + cv * 8) = pack8(m);
 }
 
+// 3x3 window, fully unrolled: all nine loads issue before the first max.
+__global__ void maxpool3_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
+                                int s, int p, int Ho, int Wo) {
+    const int CV = C >> 3;
+    const long long total = (long long)N * Ho * Wo * CV;
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= total) return;
+    const int cv = (int)(idx % CV);
+    long long t = idx / CV;
+    const int q = (int)(t % Wo);
+    t /= Wo;
+    const int pp = (int)(t % Ho);
+    const int n = (int)(t / Ho);
+    const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
+    uint4 v[9];
+#pragma unroll
+    for (int r = 0; r < 3; ++r) {
+        const int h = min(max(pp * s - p + r, 0), H - 1);  // nearest in-window position
+#pragma unroll
+        for (int c = 0; c < 3; ++c) {
+            const int w = min(max(q * s - p + c, 0), W - 1);
+            v[r * 3 + c] = ldg_v4(xn + ((size_t)h * W + w) * C);
+        }
+    }
+    float m[8];
+    unpack8(v[0], m);
+#pragma unroll
+    for (int i = 1; i < 9; ++i) {
+        float f[8];
+        unpack8(v[i], f);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) m[j] = fmaxf(m[j], f[j]);
+    }
+    *reinterpret_cast<uint4 *>(y + (((size_t)n * Ho + pp) * Wo + q) * C + cv * 8) = pack8(m);
+}
+
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            int k, int s, int p, cudaStream_t st) {
+    if (k == 3) {
+        const int Ho = (H + 2 * p - 3) / s + 1;
+        const int Wo = (W + 2 * p - 3) / s + 1;
+        const long long total = (long long)N * Ho * Wo * (C / 8);
+        maxpool3_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C, s, p, Ho, Wo);
+        return cudaGetLastError();
+    }
     const int Ho = (H + 2 * p - k) / s + 1;
     const int Wo = (W + 2 * p - k) / s + 1;
     const long long total = (long long)N * Ho * Wo * (C / 8);

@@ -5,16 +5,21 @@
 // "instruction") makes one pass over HBM.
 //
 // Structure (one persistent CTA per SM, 320 threads):
-//   warp 0 lane 0  TMA producer of the mainloop: per k-block, one A tile (128
-//              rows x BK) and one B tile (BN rows x BK) into a STAGES-deep
-//              shared-memory ring.  A is a 2-D tile of a row-major matrix, or
-//              -- for convolutions -- an im2col tile: 128 consecutive output
-//              pixels of one filter tap and channel chunk, with out-of-image
-//              taps zero-filled by TMA.
+//   warp 0 lane 0  TMA producer of the mainloop.  The A operand (activations)
+//              comes in one of three ways (AMODE):
+//                tile   a 128 x BK tile of a row-major [M, K] matrix;
+//                im2col 128 consecutive output pixels of one filter tap and
+//                       channel chunk (out-of-image taps zero-filled by TMA);
+//                slab   stride-1 convolutions: for each channel chunk one
+//                       4-D tiled box of the padded input rows under the tile
+//                       (the "slab"); each filter tap (r, s) is the same slab
+//                       read from row r * Wp + s on, by shifting the MMA's
+//                       shared-memory descriptor -- one load per chunk instead
+//                       of one per tap.
+//              The B operand (packed weights) is one BN x BK tile per k-block.
 //   warp 0 lane 1  producer of the epilogue operands: per tile, the tile's
 //              bias slice (bulk copy) and, when the region adds a residual,
-//              the 128 x BN residual tile (TMA) into one of two buffers, well
-//              before the epilogue needs them.
+//              the 128 x BN residual tile (TMA) into one of two buffers.
 //   warp 1     allocates TMEM; one lane issues tcgen05.mma (M=128, N=BN, K=16
 //              per instruction) into one of two fp32 accumulators in TMEM and
 //              tcgen05.commit's the ring slots and the finished accumulator.
@@ -31,12 +36,14 @@
 
 namespace byoc {
 
-template <int BN, int BK, bool RES>
+template <int BN, int BK, int AMODE, bool RES>
 struct GemmShape {
     static constexpr int BM = kGemmBM;
-    static constexpr int A_BYTES = BM * BK * 2;
+    static constexpr int ROW_BYTES = BK * 2;  // one K-major operand row (= swizzle width)
+    static constexpr int A_BYTES = AMODE == kAModeSlab ? 0 : BM * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
+    static constexpr int SLAB_BYTES = AMODE == kAModeSlab ? slab_max_bytes(BK) : 0;
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
     // residual tile: BN/64 boxes of 64 columns x 128 rows, 128-byte swizzle
     static constexpr int RES_BOX = BM * 64 * 2;
@@ -47,18 +54,20 @@ struct GemmShape {
     static constexpr int EPI_TILE = 32 * 32 * 2;
     static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE;
     static constexpr int CTRL_BYTES = 512;
-    static constexpr int FIXED = 1024 + 2 * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
+    static constexpr int FIXED =
+        1024 + 2 * SLAB_BYTES + 2 * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 16 ? 16 : STAGES_RAW;
-    static constexpr int NUM_BARS = 2 * STAGES + 9;
-    static constexpr int SMEM_BYTES = 1024 + STAGES * STAGE_BYTES + 2 * RES_TILE + EPI_BYTES +
-                                      BIAS_REGION + CTRL_BYTES;
+    static constexpr int NUM_BARS = 2 * STAGES + 13;
+    static constexpr int SMEM_BYTES = FIXED + STAGES * STAGE_BYTES;
     static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
     static_assert(STAGES >= 2, "ring depth");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
-    static_assert(A_BYTES % 1024 == 0 && B_BYTES % 1024 == 0, "tiles must keep 1 KB alignment");
+    static_assert(A_BYTES % 1024 == 0 && B_BYTES % 1024 == 0 && SLAB_BYTES % 1024 == 0,
+                  "buffers must keep 1 KB alignment");
     static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "BN");
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
+    static_assert(!(RES && AMODE == kAModeSlab), "slab tiles skip pad columns; no residual tile");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
 };
 
@@ -71,19 +80,20 @@ __device__ __forceinline__ float apply_act(float v, int act) {
     }
 }
 
-template <int BN, int BK, bool IM2COL, bool RES>
+template <int BN, int BK, int AMODE, bool RES>
 __global__ void __launch_bounds__(kGemmThreads, 1)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
-    using S = GemmShape<BN, BK, RES>;
+    using S = GemmShape<BN, BK, AMODE, RES>;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
     uint8_t *smem = smem_raw + (base - raw);
     const uint32_t sA = base;
     const uint32_t sB = sA + S::STAGES * S::A_BYTES;
-    const uint32_t sRes = sB + S::STAGES * S::B_BYTES;     // 2 x RES_TILE
+    const uint32_t sSlab = sB + S::STAGES * S::B_BYTES;    // 2 x SLAB_BYTES
+    const uint32_t sRes = sSlab + 2 * S::SLAB_BYTES;       // 2 x RES_TILE
     const uint32_t sEpi = sRes + 2 * S::RES_TILE;          // EPI_BYTES
     const uint32_t sBias = sEpi + S::EPI_BYTES;            // 2 x BIAS_BYTES
     const uint32_t ctrl = sBias + S::BIAS_REGION;
@@ -92,7 +102,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     const uint32_t tempty = tfull + 16u;                   // 2: accumulator drained
     const uint32_t ofull = tempty + 16u;                   // 2: epilogue operands loaded
     const uint32_t oempty = ofull + 16u;                   // 2: epilogue operands consumed
-    const uint32_t drain = oempty + 16u;
+    const uint32_t sfull = oempty + 16u;                   // 2: slab loaded
+    const uint32_t sempty = sfull + 16u;                   // 2: slab consumed
+    const uint32_t drain = sempty + 16u;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -109,6 +121,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mbar_init(tempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
             mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
             mbar_init(oempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
+            mbar_init(sfull + 8u * b, 1);                 // producer + slab bytes
+            mbar_init(sempty + 8u * b, 1);                // MMA commit
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -131,49 +145,94 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     if (warp == 0) {
         if (lane == 0) {
             // ------------------------------------------------ mainloop producer
-            int it = 0;
+            int stage = 0, sl = 0, issued = 0;
+            uint32_t phase = 0;
             bool ok = true;
-            for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x) {
-                const int m0 = (tile / a.tiles_n) * S::BM;
-                const int n0 = (tile % a.tiles_n) * BN;
-                int img = 0, h0 = 0, w0 = 0;
-                if (IM2COL) {
-                    const int hw = a.Ho * a.Wo;
-                    img = m0 / hw;
-                    const int rem = m0 - img * hw;
-                    const int p = rem / a.Wo;
-                    const int q = rem - p * a.Wo;
-                    h0 = p * a.stride_h - a.pad_t;
-                    w0 = q * a.stride_w - a.pad_l;
+            // Wait for ring slot `stage` to be free and announce `bytes` on its full barrier.
+            auto claim = [&](uint32_t bytes) -> bool {
+                if (!mbar_wait(bars + 8u * (S::STAGES + stage), phase ^ 1u, abort_flag, a.err,
+                               kErrTimeoutProducer))
+                    return false;
+                mbar_arrive_expect_tx(bars + 8u * stage, bytes);
+                return true;
+            };
+            auto advance = [&]() {
+                ++issued;
+                if (++stage == S::STAGES) {
+                    stage = 0;
+                    phase ^= 1u;
                 }
-                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
-                    const int s = it % S::STAGES;
-                    const uint32_t ph = (uint32_t)(it / S::STAGES) & 1u;
-                    if (!mbar_wait(bars + 8u * (S::STAGES + s), ph ^ 1u, abort_flag, a.err,
-                                   kErrTimeoutProducer)) {
-                        ok = false;
-                        break;
+            };
+            for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x) {
+                const int mt = tile / a.tiles_n;
+                const int n0 = (tile % a.tiles_n) * BN;
+                if constexpr (AMODE == kAModeSlab) {
+                    const int img = mt / a.tiles_per_img;
+                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
+                    for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
+                        const int ss = sl & 1;
+                        const uint32_t sph = (uint32_t)(sl >> 1) & 1u;
+                        if (!mbar_wait(sempty + 8u * ss, sph ^ 1u, abort_flag, a.err,
+                                       kErrTimeoutProducer)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(sfull + 8u * ss, (uint32_t)a.slab_bytes);
+                        tma_load_4d(sSlab + ss * S::SLAB_BYTES, &tmA, sfull + 8u * ss, cc * BK,
+                                    -a.pad_l, p0 - a.pad_t, img);
+                        for (int tap = 0, kb = cc; tap < a.taps; ++tap, kb += a.chunks) {
+                            if (!claim(S::B_BYTES)) {
+                                ok = false;
+                                break;
+                            }
+                            tma_load_2d(sB + stage * S::B_BYTES, &tmB, bars + 8u * stage, kb * BK, n0);
+                            advance();
+                        }
                     }
-                    const uint32_t full = bars + 8u * s;
-                    mbar_arrive_expect_tx(full, S::STAGE_BYTES);
-                    if (IM2COL) {
-                        const int tap = kb / a.chunks;
-                        const int cc = kb - tap * a.chunks;
-                        const int r = tap / a.kw;
-                        const int sx = tap - r * a.kw;
-                        tma_load_im2col_4d(sA + s * S::A_BYTES, &tmA, full, cc * BK, w0, h0, img,
-                                           (uint16_t)(sx * a.dil_w), (uint16_t)(r * a.dil_h));
-                    } else {
-                        tma_load_2d(sA + s * S::A_BYTES, &tmA, full, kb * BK, m0);
+                } else {
+                    const int m0 = mt * S::BM;
+                    int img = 0, h0 = 0, w0 = 0;
+                    if constexpr (AMODE == kAModeIm2col) {
+                        const int hw = a.Ho * a.Wo;
+                        img = m0 / hw;
+                        const int rem = m0 - img * hw;
+                        const int p = rem / a.Wo;
+                        const int q = rem - p * a.Wo;
+                        h0 = p * a.stride_h - a.pad_t;
+                        w0 = q * a.stride_w - a.pad_l;
                     }
-                    tma_load_2d(sB + s * S::B_BYTES, &tmB, full, kb * BK, n0);
+                    int cc = 0, r = 0, sx = 0;  // (tap r, s; chunk cc) of k-block kb, im2col mode
+                    for (int kb = 0; kb < a.num_kb; ++kb) {
+                        if (!claim(S::STAGE_BYTES)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t full = bars + 8u * stage;
+                        if constexpr (AMODE == kAModeIm2col) {
+                            tma_load_im2col_4d(sA + stage * S::A_BYTES, &tmA, full, cc * BK, w0, h0,
+                                               img, (uint16_t)(sx * a.dil_w),
+                                               (uint16_t)(r * a.dil_h));
+                            if (++cc == a.chunks) {
+                                cc = 0;
+                                if (++sx == a.kw) {
+                                    sx = 0;
+                                    ++r;
+                                }
+                            }
+                        } else {
+                            tma_load_2d(sA + stage * S::A_BYTES, &tmA, full, kb * BK, m0);
+                        }
+                        tma_load_2d(sB + stage * S::B_BYTES, &tmB, full, kb * BK, n0);
+                        advance();
+                    }
                 }
             }
             if (!ok) {
                 // Gave up: let the copies already issued land before exiting.
-                const int first = it - S::STAGES > 0 ? it - S::STAGES : 0;
-                for (int j = first; j < it; ++j)
+                for (int j = issued - S::STAGES > 0 ? issued - S::STAGES : 0; j < issued; ++j)
                     mbar_wait_drain(bars + 8u * (j % S::STAGES), (uint32_t)(j / S::STAGES) & 1u);
+                for (int j = sl - 2 > 0 ? sl - 2 : 0; j < sl; ++j)
+                    mbar_wait_drain(sfull + 8u * (j & 1), (uint32_t)(j >> 1) & 1u);
             }
         } else if (lane == 1) {
             // ------------------------------------------------ epilogue-operand producer
@@ -187,7 +246,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 const int n0 = (tile % a.tiles_n) * BN;
                 mbar_arrive_expect_tx(ofull + 8u * ob, S::BIAS_BYTES + S::RES_TILE);
                 bulk_load_1d(sBias + ob * S::BIAS_BYTES, a.bias + n0, S::BIAS_BYTES, ofull + 8u * ob);
-                if (RES) {
+                if constexpr (RES) {
 #pragma unroll
                     for (int j = 0; j < BN / 64; ++j)
                         tma_load_2d(sRes + ob * S::RES_TILE + j * S::RES_BOX, &tmR, ofull + 8u * ob,
@@ -201,8 +260,17 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     } else if (warp == 1) {
         if (lane == 0) {
             // ------------------------------------------------ MMA issuer
+            // One thread issues every MMA, so its per-k-block path is kept
+            // lean: the ring position advances by compare-and-wrap, shared
+            // memory descriptors advance by adding (byte offset >> 4) to their
+            // 14-bit address field, and filter taps are walked without
+            // division.
             constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
-            int it = 0, t = 0;
+            const uint64_t adesc0 = make_smem_desc(AMODE == kAModeSlab ? sSlab : sA, S::ROW_BYTES);
+            const uint64_t bdesc0 = make_smem_desc(sB, S::ROW_BYTES);
+            int stage = 0;
+            uint32_t phase = 0;
+            int sl = 0, t = 0;
             bool ok = true;
             for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x, ++t) {
                 const int buf = t & 1;
@@ -213,23 +281,65 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
-                for (int kb = 0; kb < a.num_kb; ++kb, ++it) {
-                    const int s = it % S::STAGES;
-                    const uint32_t ph = (uint32_t)(it / S::STAGES) & 1u;
-                    if (!mbar_wait(bars + 8u * s, ph, abort_flag, a.err, kErrTimeoutMma)) {
-                        ok = false;
-                        break;
-                    }
-                    tc_fence_after();
-                    const uint32_t a_s = sA + s * S::A_BYTES;
-                    const uint32_t b_s = sB + s * S::B_BYTES;
+                uint32_t acc = 0u;
+                if constexpr (AMODE == kAModeSlab) {
+                    const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
+                    for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
+                        const int ss = sl & 1;
+                        if (!mbar_wait(sfull + 8u * ss, (uint32_t)(sl >> 1) & 1u, abort_flag, a.err,
+                                       kErrTimeoutMma)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint64_t slab_desc = adesc0 + (uint64_t)((ss * S::SLAB_BYTES) >> 4);
+                        uint32_t roff = 0;  // r * wp * ROW_BYTES
+                        for (int r = 0; ok && r < a.taps / a.kw; ++r, roff += row_step) {
+                            uint32_t toff = roff;  // (r * wp + s) * ROW_BYTES
+                            for (int sx = 0; sx < a.kw; ++sx, toff += S::ROW_BYTES) {
+                                if (!mbar_wait(bars + 8u * stage, phase, abort_flag, a.err,
+                                               kErrTimeoutMma)) {
+                                    ok = false;
+                                    break;
+                                }
+                                tc_fence_after();
+                                const uint64_t ad = slab_desc + (uint64_t)(toff >> 4);
+                                const uint64_t bd = bdesc0 + (uint64_t)((stage * S::B_BYTES) >> 4);
 #pragma unroll
-                    for (int k = 0; k < BK / 16; ++k) {
-                        mma_bf16_ss(d_tmem, make_smem_desc(a_s + 32u * k, BK * 2),
-                                    make_smem_desc(b_s + 32u * k, BK * 2), idesc,
-                                    (kb | k) != 0 ? 1u : 0u);
+                                for (int k = 0; k < BK / 16; ++k) {
+                                    mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k),
+                                                idesc, acc);
+                                    acc = 1u;
+                                }
+                                mma_commit(bars + 8u * (S::STAGES + stage));  // frees the B slot
+                                if (++stage == S::STAGES) {
+                                    stage = 0;
+                                    phase ^= 1u;
+                                }
+                            }
+                        }
+                        if (!ok) break;
+                        mma_commit(sempty + 8u * ss);  // frees the slab
                     }
-                    mma_commit(bars + 8u * (S::STAGES + s));  // frees the ring slot
+                } else {
+                    for (int kb = 0; kb < a.num_kb; ++kb) {
+                        if (!mbar_wait(bars + 8u * stage, phase, abort_flag, a.err, kErrTimeoutMma)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t ad = adesc0 + (uint64_t)((stage * S::A_BYTES) >> 4);
+                        const uint64_t bd = bdesc0 + (uint64_t)((stage * S::B_BYTES) >> 4);
+#pragma unroll
+                        for (int k = 0; k < BK / 16; ++k) {
+                            mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, acc);
+                            acc = 1u;
+                        }
+                        mma_commit(bars + 8u * (S::STAGES + stage));  // frees the ring slot
+                        if (++stage == S::STAGES) {
+                            stage = 0;
+                            phase ^= 1u;
+                        }
+                    }
                 }
                 if (!ok) break;
                 mma_commit(tfull + 8u * buf);  // accumulator complete
@@ -258,9 +368,25 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
             if (!mbar_wait(ofull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
             tc_fence_after();
-            const int m0 = (tile / a.tiles_n) * S::BM;
+            const int mt = tile / a.tiles_n;
             const int n0 = (tile % a.tiles_n) * BN;
-            const int row0 = m0 + quarter * 32;
+            // output pixel (row of out / residual) of the 4 rows this lane stores, or -1
+            int orow[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                const int v = quarter * 32 + 8 * k + cl_row;
+                if constexpr (AMODE == kAModeSlab) {
+                    const int img = mt / a.tiles_per_img;
+                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
+                    const int y = v / a.wp;
+                    const int x = v - y * a.wp;
+                    const bool ok = y < a.slab_t && x < a.Wo && p0 + y < a.Ho;
+                    orow[k] = ok ? (img * a.Ho + p0 + y) * a.Wo + x : -1;
+                } else {
+                    const int row = mt * S::BM + v;
+                    orow[k] = row < a.M ? row : -1;
+                }
+            }
             const uint32_t tbase =
                 tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
             const uint32_t bias_s = sBias + (uint32_t)(buf * S::BIAS_BYTES);
@@ -296,7 +422,7 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4.z;
                     f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4.w;
                 }
-                if (RES) {
+                if constexpr (RES) {
                     // residual row `trow`, columns ci*32.. of the 128B-swizzled box ci/2
                     const uint32_t rbox =
                         res_s + (uint32_t)((ci >> 1) * S::RES_BOX) + (uint32_t)trow * 128u;
@@ -342,9 +468,8 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                                  : "=r"(o.x), "=r"(o.y), "=r"(o.z), "=r"(o.w)
                                  : "r"(addr)
                                  : "memory");
-                    const int row = row0 + (int)r;
-                    if (row < a.M && gcol < a.N)
-                        *reinterpret_cast<uint4 *>(a.out + (size_t)row * a.N + gcol) = o;
+                    if (orow[k] >= 0 && gcol < a.N)
+                        *reinterpret_cast<uint4 *>(a.out + (size_t)orow[k] * a.N + gcol) = o;
                 }
             }
             // bias / residual reads of this tile are done (ordered by __syncwarp)
@@ -364,69 +489,75 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
 
 // ---------------------------------------------------------------- dispatch
 
-template <int BN, int BK, bool IM2COL, bool RES>
+template <int BN, int BK, int AMODE, bool RES>
 static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap &tmR,
                             const GemmArgs &a, int grid, cudaStream_t st) {
-    using S = GemmShape<BN, BK, RES>;
-    gemm_tcgen05_kernel<BN, BK, IM2COL, RES>
+    using S = GemmShape<BN, BK, AMODE, RES>;
+    gemm_tcgen05_kernel<BN, BK, AMODE, RES>
         <<<grid, kGemmThreads, S::SMEM_BYTES, st>>>(tmA, tmB, tmR, a);
     return cudaGetLastError();
 }
 
-template <int BN, int BK, bool IM2COL, bool RES>
+template <int BN, int BK, int AMODE, bool RES>
 static cudaError_t prepare_t() {
-    using S = GemmShape<BN, BK, RES>;
-    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, IM2COL, RES>,
+    using S = GemmShape<BN, BK, AMODE, RES>;
+    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, AMODE, RES>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, S::SMEM_BYTES);
 }
 
-// The instantiated (BN, BK, im2col, residual) combinations.
-#define BYOC_GEMM_CONFIGS(X)  \
-    X(32, 64, false, false)   \
-    X(64, 64, false, false)   \
-    X(128, 64, false, false)  \
-    X(256, 64, false, false)  \
-    X(32, 64, true, false)    \
-    X(64, 64, true, false)    \
-    X(128, 64, true, false)   \
-    X(256, 64, true, false)   \
-    X(64, 16, true, false)    \
-    X(64, 32, true, false)    \
-    X(128, 32, true, false)   \
-    X(64, 64, false, true)    \
-    X(128, 64, false, true)   \
-    X(64, 64, true, true)     \
-    X(128, 64, true, true)
+// The instantiated (BN, BK, A mode, residual) combinations.
+#define BYOC_GEMM_CONFIGS(X)          \
+    X(32, 64, kAModeTile, false)      \
+    X(64, 64, kAModeTile, false)      \
+    X(128, 64, kAModeTile, false)     \
+    X(256, 64, kAModeTile, false)     \
+    X(64, 64, kAModeTile, true)       \
+    X(128, 64, kAModeTile, true)      \
+    X(32, 64, kAModeIm2col, false)    \
+    X(64, 64, kAModeIm2col, false)    \
+    X(128, 64, kAModeIm2col, false)   \
+    X(256, 64, kAModeIm2col, false)   \
+    X(64, 64, kAModeIm2col, true)     \
+    X(128, 64, kAModeIm2col, true)    \
+    X(64, 16, kAModeIm2col, false)    \
+    X(64, 32, kAModeIm2col, false)    \
+    X(128, 32, kAModeIm2col, false)   \
+    X(64, 64, kAModeSlab, false)      \
+    X(128, 64, kAModeSlab, false)     \
+    X(256, 64, kAModeSlab, false)     \
+    X(64, 16, kAModeSlab, false)      \
+    X(64, 32, kAModeSlab, false)
 
 bool gemm_config_supported(const GemmConfig &c) {
-#define X(BN_, BK_, IM_, RES_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) return true;
+#define X(BN_, BK_, AM_, RES_) \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) return true;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return false;
 }
 
 size_t gemm_smem_bytes(const GemmConfig &c) {
-#define X(BN_, BK_, IM_, RES_)                                 \
-    if (c.bn == BN_ && c.bk == BK_ && c.res == RES_) \
-        return (size_t)GemmShape<BN_, BK_, RES_>::SMEM_BYTES;
+#define X(BN_, BK_, AM_, RES_)                                             \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
+        return (size_t)GemmShape<BN_, BK_, AM_, RES_>::SMEM_BYTES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 int gemm_stages(const GemmConfig &c) {
-#define X(BN_, BK_, IM_, RES_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.res == RES_) return GemmShape<BN_, BK_, RES_>::STAGES;
+#define X(BN_, BK_, AM_, RES_)                                             \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
+        return GemmShape<BN_, BK_, AM_, RES_>::STAGES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 cudaError_t gemm_prepare(const GemmConfig &c) {
-#define X(BN_, BK_, IM_, RES_)                                              \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) \
-        return prepare_t<BN_, BK_, IM_, RES_>();
+#define X(BN_, BK_, AM_, RES_)                                             \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
+        return prepare_t<BN_, BK_, AM_, RES_>();
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;
@@ -434,9 +565,9 @@ cudaError_t gemm_prepare(const GemmConfig &c) {
 
 cudaError_t launch_gemm(const GemmConfig &c, const CUtensorMap &tmA, const CUtensorMap &tmB,
                         const CUtensorMap &tmR, const GemmArgs &a, int grid, cudaStream_t st) {
-#define X(BN_, BK_, IM_, RES_)                                              \
-    if (c.bn == BN_ && c.bk == BK_ && c.im2col == IM_ && c.res == RES_) \
-        return launch_t<BN_, BK_, IM_, RES_>(tmA, tmB, tmR, a, grid, st);
+#define X(BN_, BK_, AM_, RES_)                                             \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
+        return launch_t<BN_, BK_, AM_, RES_>(tmA, tmB, tmR, a, grid, st);
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;

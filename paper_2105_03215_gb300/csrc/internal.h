@@ -29,6 +29,14 @@ struct GemmArgs {
     int pad_t, pad_l;
     int tiles_n;    // number of BN-wide column tiles
     int num_tiles;  // tiles_m * tiles_n
+    // slab mode (stride-1 convolution): a tile is slab_t output rows of one
+    // image; tile row v = y * wp + x indexes the padded width wp, and filter
+    // tap (r, s) reads the slab from row r * wp + s on
+    int wp;             // padded input width (W + pad_l + pad_r)
+    int slab_t;         // output rows per tile
+    int tiles_per_img;  // ceil(Ho / slab_t)
+    int slab_bytes;     // bytes of one slab (one channel chunk)
+    int taps;           // kh * kw
     int act;        // Act
     const float *bias;                // [tiles_n * BN], zero padded; required
     const __nv_bfloat16 *residual;    // [M, N] or null
@@ -36,12 +44,21 @@ struct GemmArgs {
     int *err;                         // device error word
 };
 
-struct GemmConfig {
-    int bn;       // tile width in output channels: 32, 64, 128, 256
-    int bk;       // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
-    bool im2col;  // A operand through an im2col tensor map
-    bool res;     // epilogue adds a residual tile (bn 64 or 128)
+enum AMode : int {
+    kAModeTile = 0,    // A is a row-major [M, K] matrix (2-D tiled TMA)
+    kAModeIm2col = 1,  // A through an im2col TMA map: one load per filter tap and chunk
+    kAModeSlab = 2     // stride-1 conv: one 4-D tiled slab per chunk, taps by row shift
 };
+
+struct GemmConfig {
+    int bn;      // tile width in output channels: 32, 64, 128, 256
+    int bk;      // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
+    int amode;   // AMode
+    bool res;    // epilogue adds a residual tile (bn 64 or 128)
+};
+
+// Largest slab (one channel chunk) the slab mode holds, per buffer.
+constexpr int slab_max_bytes(int bk) { return bk == 64 ? 48 * 1024 : 24 * 1024; }
 
 constexpr int kGemmBM = 128;
 constexpr int kGemmEpiWarps = 8;

@@ -61,7 +61,7 @@ byoc_status cuda_fail(cudaError_t e, const char *what) {
 void setup_device(DeviceState &d, int dev) {
     cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&d.scratch), g_ffn_scratch);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
-    if (e == cudaSuccess) e = byoc::gemm_prepare(byoc::GemmConfig{kTileN, 64, false, false});
+    if (e == cudaSuccess) e = byoc::gemm_prepare(byoc::GemmConfig{kTileN, 64, byoc::kAModeTile, false});
     d.err = e;
 }
 
@@ -125,7 +125,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
         encode(&b2m, w2, (uint64_t)D, (uint64_t)F, kTileN) != CUDA_SUCCESS)
         return fail(BYOC_ERR_CUDA, "byoc_ffn_noalloc: encoding a TMA descriptor failed");
 
-    const byoc::GemmConfig cfg{kTileN, 64, false, false};
+    const byoc::GemmConfig cfg{kTileN, 64, byoc::kAModeTile, false};
     const int tiles_m = (M + byoc::kGemmBM - 1) / byoc::kGemmBM;
     byoc::GemmArgs g{};
     g.M = M;

@@ -113,6 +113,16 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *tm,
         : "memory");
 }
 
+// 4-D tiled load; coordinates innermost first (for NHWC: c, w, h, n).
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *tm, uint32_t bar,
+                                            int32_t c0, int32_t c1, int32_t c2, int32_t c3) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3)
+        : "memory");
+}
+
 // 4-D im2col load of an NHWC tensor: coordinates {c, w, h, n} of the first
 // pixel's filter origin, plus the filter-tap offsets {off_w, off_h}.  Loads
 // `pixelsPerColumn` pixels (traversing w, then h, then n inside the tensor
@@ -218,6 +228,16 @@ __device__ __forceinline__ uint64_t make_smem_desc(uint32_t saddr, uint32_t row_
     d |= static_cast<uint64_t>(1u) << 46;
     d |= static_cast<uint64_t>(layout) << 61;
     return d;
+}
+
+// The same descriptor for an operand whose first row starts at an arbitrary
+// row of a swizzled buffer that TMA filled (the buffer 1024-byte aligned).
+// The tensor core applies the swizzle to the absolute shared-memory address
+// bits, as TMA does when writing, so shifting the start address by whole rows
+// is enough; the matrix base-offset field stays 0 (measured on GB300: setting
+// it to the row phase breaks the result, leaving it 0 is bit-exact).
+__device__ __forceinline__ uint64_t make_smem_desc_shifted(uint32_t saddr, uint32_t row_bytes) {
+    return make_smem_desc(saddr, row_bytes);
 }
 
 // Instruction descriptor of tcgen05.mma kind::f16: bf16 x bf16 -> fp32,

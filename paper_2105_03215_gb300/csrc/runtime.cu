@@ -120,6 +120,19 @@ CUresult encode_im2col(CUtensorMap *m, const void *ptr, const Im2colGeom &g, int
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// Tiled 4-D map over an NHWC tensor for slab loads: box = {bk channels, wp
+// columns, rows rows, 1 image}; out-of-image elements read as zero.
+CUresult encode_slab(CUtensorMap *m, const void *ptr, int N, int H, int W, int C, int wp, int rows,
+                     int bk) {
+    cuuint64_t dims[4] = {(cuuint64_t)C, (cuuint64_t)W, (cuuint64_t)H, (cuuint64_t)N};
+    cuuint64_t strides[3] = {(cuuint64_t)C * 2, (cuuint64_t)W * C * 2, (cuuint64_t)H * W * C * 2};
+    cuuint32_t box[4] = {(cuuint32_t)bk, (cuuint32_t)wp, (cuuint32_t)rows, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 // ------------------------------------------------------------ bf16 rounding (host)
 
 uint16_t f32_to_bf16_rne(float f) {
@@ -152,13 +165,14 @@ struct LaunchPlan {
     int x = -1, y = -1, res = -1;  // tensor ids (may index internal scratch tensors)
     int act = byoc::kActNone;
     // GEMM
-    GemmConfig cfg{64, 64, false, false};
+    GemmConfig cfg{64, 64, byoc::kAModeTile, false};
     GemmArgs args{};
     int grid = 0;
     int n_pad = 0, k_pack = 0;
     // A operand geometry
     Im2colGeom geo{};
     int64_t aM = 0, aK = 0;
+    int slab_rows = 0;  // slab mode: padded input rows per slab
     // constants: byte offsets into the constant blob
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
     // depthwise / space-to-depth
@@ -336,23 +350,27 @@ int pick_bk(int64_t C) {
 // Choose the output-channel tile among the compiled configurations by a
 // makespan estimate of the persistent grid, in SM cycles, calibrated on
 // GB300 traces of this kernel:
-//   mainloop per tile  = 300 + k-blocks x max(2.5 bn, 450): a 64-deep k-block
-//                        costs ~450 cycles of TMA delivery at small bn and is
-//                        tensor-core bound (~640 cycles) at bn = 256;
+//   mainloop per tile  = 300 + k-blocks x per-k-block cost: with A loaded per
+//                        k-block (tile, im2col) ~450 cycles of TMA delivery at
+//                        small bn, tensor-core bound (~2.5 bn) at bn = 256;
+//                        in slab mode A arrives once per channel chunk, so a
+//                        k-block costs the MMA time (~2.5 bn, at least 150);
 //   epilogue per tile  = ~600 cycles per pair of 32-column chunks (two warps
 //                        per accumulator row block work in parallel).
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
 // time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
-int pick_bn(int64_t M, int64_t N, int64_t kblocks, int bk, bool im2col, bool res, int num_sms) {
+int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool res, int num_sms) {
     int best = -1;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
-        GemmConfig c{bn, bk, im2col, res};
+        GemmConfig c{bn, bk, amode, res};
         if (!byoc::gemm_config_supported(c)) continue;
-        const int64_t tiles = ((M + 127) / 128) * ((N + bn - 1) / bn);
+        const int64_t tiles = tiles_m * ((N + bn - 1) / bn);
         const int64_t grid = std::min<int64_t>(tiles, num_sms);
         const int64_t rounds = (tiles + grid - 1) / grid;
-        const double mainloop = 300.0 + (double)kblocks * std::max(2.5 * bn, 450.0);
+        const double kb = amode == byoc::kAModeSlab ? std::max(2.5 * bn * bk / 64.0, 150.0)
+                                                    : std::max(2.5 * bn, 450.0);
+        const double mainloop = 300.0 + (double)kblocks * kb;
         const double epilogue = 600.0 * std::max(1, bn / 64);
         const double cost = (double)rounds * std::max(mainloop, epilogue) + std::min(mainloop, epilogue);
         if (cost < best_cost - 1e-9) {
@@ -361,6 +379,27 @@ int pick_bn(int64_t M, int64_t N, int64_t kblocks, int bk, bool im2col, bool res
         }
     }
     return best;
+}
+
+// Slab-mode geometry of a stride-1 convolution: output rows per tile, padded
+// width, slab rows, slab bytes.  Returns false when the slab mode does not fit
+// (padded width over 128, under 70% of the 128 MMA rows carrying outputs, or a
+// slab larger than its buffer).
+struct SlabGeom {
+    int wp, t, rows, bytes;
+};
+bool slab_geometry(int H, int W, int Ho, int Wo, int kh, int kw, int pt, int pl, int pr, int bk,
+                   SlabGeom &g) {
+    (void)H;
+    g.wp = W + pl + pr;
+    if (g.wp > 128 || g.wp > 256) return false;
+    g.t = std::min(128 / g.wp, Ho);
+    if (g.t < 1 || g.t * Wo < 90) return false;
+    const int dmax = (kh - 1) * g.wp + (kw - 1);
+    g.rows = (128 + dmax + g.wp - 1) / g.wp;
+    g.bytes = g.rows * g.wp * bk * 2;
+    (void)pt;
+    return g.rows <= 256 && g.bytes <= byoc::slab_max_bytes(bk);
 }
 
 struct Affine {
@@ -484,6 +523,8 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         int64_t C;
         std::vector<double> wsrc;  // weights as [Cout][kh][kw][C] (channel innermost)
         bool im2col = false;
+        bool slab = false;
+        SlabGeom sgeo{};
         if (op.kind == BYOC_OP_DENSE) {
             C = X.shape[1];
             M = X.shape[0];
@@ -556,6 +597,9 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                 kh = 1;
                 kw = k2;
                 im2col = true;
+                // the 1 x k2 stride-1 conv over the stacked tensor reads well as slabs
+                slab = slab_geometry((int)Z.shape[1], (int)Z.shape[2], (int)Y.shape[1],
+                                     (int)Y.shape[2], 1, k2, 0, 0, 0, pick_bk(Cz), sgeo);
                 L.geo = Im2colGeom{(int)Z.shape[0], (int)Z.shape[1], (int)Z.shape[2], Cz,
                                    1, k2, 1, 1, 0, 0, 0, 0, 1, 1};
                 L.args.stride_h = L.args.stride_w = 1;
@@ -588,6 +632,11 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                     L.geo = Im2colGeom{(int)X.shape[0], (int)X.shape[1], (int)X.shape[2], (int)C,
                                        kh, kw, op.stride[0], op.stride[1], op.pad[0], op.pad[1],
                                        op.pad[2], op.pad[3], op.dilation[0], op.dilation[1]};
+                    slab = op.stride[0] == 1 && op.stride[1] == 1 && op.dilation[0] == 1 &&
+                           op.dilation[1] == 1 && res < 0 &&
+                           slab_geometry((int)X.shape[1], (int)X.shape[2], (int)Y.shape[1],
+                                         (int)Y.shape[2], kh, kw, op.pad[0], op.pad[1], op.pad[3],
+                                         pick_bk(C), sgeo);
                     L.args.stride_h = op.stride[0];
                     L.args.stride_w = op.stride[1];
                     L.args.pad_t = op.pad[0];
@@ -601,11 +650,21 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         bk = op.kind == BYOC_OP_DENSE ? 64 : pick_bk(C);
         chunks = (int)((C + bk - 1) / bk);
         const bool has_res = res >= 0;
-        const int bn = pick_bn(M, Cout, (int64_t)taps * chunks, bk, im2col, has_res, P.num_sms);
+        const int amode = slab ? byoc::kAModeSlab : (im2col ? byoc::kAModeIm2col : byoc::kAModeTile);
+        const int64_t tiles_per_img = slab ? (Y.shape[1] + sgeo.t - 1) / sgeo.t : 0;
+        const int64_t tiles_m = slab ? X.shape[0] * tiles_per_img : (M + 127) / 128;
+        const int bn = pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms);
         if (bn < 0)
-            return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d im2col=%d residual=%d",
-                        o, bk, (int)im2col, (int)has_res);
-        L.cfg = GemmConfig{bn, bk, im2col, has_res};
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
+                        o, bk, amode, (int)has_res);
+        L.cfg = GemmConfig{bn, bk, amode, has_res};
+        if (slab) {
+            L.slab_rows = sgeo.rows;
+            L.args.wp = sgeo.wp;
+            L.args.slab_t = sgeo.t;
+            L.args.tiles_per_img = (int)tiles_per_img;
+            L.args.slab_bytes = sgeo.bytes;
+        }
         L.n_pad = (int)((Cout + bn - 1) / bn * bn);
         L.k_pack = taps * chunks * bk;
         Kreal = (int64_t)taps * C;
@@ -638,7 +697,8 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         A.Ho = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[1];
         A.Wo = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[2];
         A.tiles_n = L.n_pad / bn;
-        A.num_tiles = (int)(((M + 127) / 128) * A.tiles_n);
+        A.num_tiles = (int)(tiles_m * A.tiles_n);
+        A.taps = taps;
         A.act = act;
         L.grid = std::min(A.num_tiles, P.num_sms);
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
@@ -684,7 +744,7 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
         r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : 0;
         r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : 0;
         r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : 0;
-        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? (int)L.cfg.im2col : 0;
+        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.amode : 0;
         r->grid[i] = L.grid;
     }
     r->flops = P.flops;
@@ -879,7 +939,10 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             const void *xa = h->ptrs[L.x];
             if (h->tmA_ptr[i] != xa) {
                 CUresult r;
-                if (L.cfg.im2col)
+                if (L.cfg.amode == byoc::kAModeSlab)
+                    r = encode_slab(&h->tmA[i], xa, L.geo.N, L.geo.H, L.geo.W, L.geo.C, L.args.wp,
+                                    L.slab_rows, L.cfg.bk);
+                else if (L.cfg.amode == byoc::kAModeIm2col)
                     r = encode_im2col(&h->tmA[i], xa, L.geo, L.cfg.bk);
                 else
                     r = encode_2d(&h->tmA[i], xa, (uint64_t)L.aM, (uint64_t)L.aK, byoc::kGemmBM,

@@ -46,7 +46,7 @@ def test_plan_fuses_composites_into_launches():
     assert [rep.n_ops[i] for i in range(3)] == [3, 3, 4]      # conv+bn+relu x2, conv+bn+add+relu
     assert [rep.act[i] for i in range(3)] == [1, 1, 1]
     assert rep.residual[2] == 0 and rep.residual[0] == -1     # residual = region input 0
-    assert [rep.im2col[i] for i in range(3)] == [0, 1, 0]     # 1x1 as GEMM, 3x3 as im2col
+    assert [rep.im2col[i] for i in range(3)] == [0, 2, 0]     # 1x1 as GEMM, 3x3 in slab mode
     rep = _plan(I.bert_ffn(M=64, D=128, F=256)[0])
     assert rep.n_launches == 2 and rep.act[0] == 3 and rep.act[1] == 0
     rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0])
@@ -59,8 +59,8 @@ def test_plan_stem_inserts_space_to_depth():
     rep = R.Region(g, [n.name for n in g.nodes[:3]], "stem").plan()
     assert rep.n_launches == 2
     assert rep.kind[0] == abi.LAUNCH_S2D and rep.kind[1] == abi.LAUNCH_GEMM
-    # 7x7/2 over 3 channels -> 1x4 conv over 4 stacked taps x 16 channels
-    assert rep.gemm_k[1] == 4 * 64 and rep.tile_k[1] == 64 and rep.im2col[1] == 1
+    # 7x7/2 over 3 channels -> 1x4 stride-1 conv over 4 stacked taps x 16 channels (slab mode)
+    assert rep.gemm_k[1] == 4 * 64 and rep.tile_k[1] == 64 and rep.im2col[1] == 2
 
 
 def test_plan_flops_match_mac_count():
