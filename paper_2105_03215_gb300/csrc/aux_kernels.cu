@@ -171,47 +171,111 @@ cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st) {
 // ------------------------------------------------------------ space-to-depth
 // z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]; one
 // thread per 16-channel group (a) of one output pixel, writing 32 bytes.
-__global__ void s2d_kernel(const S2dArgs a) {
-    const long long total = (long long)a.N * a.Hz * a.Wz * a.taps;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= total) return;
-    const int tap = (int)(idx % a.taps);
-    long long t = idx / a.taps;
-    const int j = (int)(t % a.Wz);
-    t /= a.Wz;
-    const int p = (int)(t % a.Hz);
-    const int n = (int)(t / a.Hz);
-    float v[16];
-#pragma unroll
-    for (int k = 0; k < 16; ++k) v[k] = 0.0f;
+// Block (p, n): output row p of image n.  Its input rows 2p-pad ..
+// 2p-pad+2*taps-1 are one contiguous run of x; the block stages them in
+// shared memory (zero rows outside the image; 16-byte loads, four in flight
+// per thread), assembles the output row there -- per (column j, stacked
+// tap) one 16-channel group -- and writes it out with coalesced 16-byte
+// stores.  Staged rows are padded by 8 elements so that the stacked taps of
+// one column fall in different banks.
+// C is a template parameter so that the 16 channel values stay in registers.
+template <int C>
+__global__ void __launch_bounds__(256) s2d_kernel(const S2dArgs a) {
+    extern __shared__ __align__(16) unsigned short smem_s2d[];
+    const int p = blockIdx.x;
+    const int n = blockIdx.y;
+    const int rows = 2 * a.taps;
+    const int row_elems = a.W * C;
+    const int pitch = ((row_elems + 7) & ~7) + 8;  // staged row pitch (elements, 16-byte multiple)
+    unsigned short *srows = smem_s2d;
+    uint4 *sout = reinterpret_cast<uint4 *>(smem_s2d + (size_t)rows * pitch);
+    const int h0 = 2 * p - a.pad;
     const unsigned short *xs = reinterpret_cast<const unsigned short *>(a.x);
+    if ((row_elems & 7) == 0) {
+        const int vec_row = row_elems >> 3;
+        const int total = rows * vec_row;
+        for (int base = threadIdx.x; base < total; base += 4 * blockDim.x) {
+            uint4 v[4];
 #pragma unroll
-    for (int dy = 0; dy < 2; ++dy) {
+            for (int k = 0; k < 4; ++k) {
+                const int i = base + k * (int)blockDim.x;
+                const int r = i / vec_row;
+                const int h = h0 + r;
+                v[k] = make_uint4(0u, 0u, 0u, 0u);
+                if (i < total && h >= 0 && h < a.H)
+                    v[k] = __ldg(reinterpret_cast<const uint4 *>(xs + ((size_t)n * a.H + h) * row_elems) +
+                                 (i - r * vec_row));
+            }
 #pragma unroll
-        for (int dx = 0; dx < 2; ++dx) {
-            const int h = 2 * (p + tap) + dy - a.pad;
-            const int w = 2 * j + dx - a.pad;
-            if (h < 0 || h >= a.H || w < 0 || w >= a.W) continue;
-            const size_t off = (((size_t)n * a.H + h) * a.W + w) * a.C;
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-                if (c < a.C) v[(dy * 2 + dx) * a.C + c] = __uint_as_float((uint32_t)__ldg(xs + off + c) << 16);
+            for (int k = 0; k < 4; ++k) {
+                const int i = base + k * (int)blockDim.x;
+                const int r = i / vec_row;
+                if (i < total)
+                    *reinterpret_cast<uint4 *>(srows + (size_t)r * pitch + 8 * (i - r * vec_row)) = v[k];
+            }
+        }
+    } else {
+        for (int i = threadIdx.x; i < rows * row_elems; i += blockDim.x) {
+            const int r = i / row_elems;
+            const int h = h0 + r;
+            srows[(size_t)r * pitch + (i - r * row_elems)] =
+                (h >= 0 && h < a.H) ? __ldg(xs + ((size_t)n * a.H + h) * row_elems + (i - r * row_elems))
+                                    : (unsigned short)0;
         }
     }
-    uint4 *zp = reinterpret_cast<uint4 *>(a.z + (((size_t)n * a.Hz + p) * a.Wz + j) * a.Cz + tap * 16);
-    float lo[8], hi[8];
+    __syncthreads();
+    const int groups = a.Wz * a.taps;
+    for (int idx = threadIdx.x; idx < groups; idx += blockDim.x) {
+        const int j = idx / a.taps;
+        const int tap = idx - j * a.taps;
+        uint32_t v[16];
 #pragma unroll
-    for (int k = 0; k < 8; ++k) {
-        lo[k] = v[k];
-        hi[k] = v[8 + k];
+        for (int k = 0; k < 16; ++k) v[k] = 0u;
+#pragma unroll
+        for (int dy = 0; dy < 2; ++dy) {
+            const unsigned short *row = srows + (size_t)(2 * tap + dy) * pitch;
+#pragma unroll
+            for (int dx = 0; dx < 2; ++dx) {
+                const int w = 2 * j + dx - a.pad;
+                if (w < 0 || w >= a.W) continue;
+#pragma unroll
+                for (int c = 0; c < C; ++c) v[(dy * 2 + dx) * C + c] = row[w * C + c];
+            }
+        }
+        sout[2 * idx] = make_uint4(v[0] | v[1] << 16, v[2] | v[3] << 16, v[4] | v[5] << 16,
+                                   v[6] | v[7] << 16);
+        sout[2 * idx + 1] = make_uint4(v[8] | v[9] << 16, v[10] | v[11] << 16,
+                                       v[12] | v[13] << 16, v[14] | v[15] << 16);
     }
-    zp[0] = pack8(lo);
-    zp[1] = pack8(hi);
+    __syncthreads();
+    uint4 *zrow = reinterpret_cast<uint4 *>(a.z + ((size_t)n * a.Hz + p) * (size_t)groups * 16);
+    for (int i = threadIdx.x; i < 2 * groups; i += blockDim.x) zrow[i] = sout[i];
+}
+
+size_t s2d_smem_bytes(const S2dArgs &a) {
+    return (size_t)2 * a.taps * (((a.W * a.C + 7) & ~7) + 8) * 2 + (size_t)a.Wz * a.taps * 32;
 }
 
 cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
-    const long long total = (long long)a.N * a.Hz * a.Wz * a.taps;
-    s2d_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(a);
+    const size_t smem = s2d_smem_bytes(a);
+    if (smem > kS2dMaxSmem) return cudaErrorInvalidValue;
+    if (smem > 48 * 1024) {
+        const void *fns[4] = {(const void *)s2d_kernel<1>, (const void *)s2d_kernel<2>,
+                              (const void *)s2d_kernel<3>, (const void *)s2d_kernel<4>};
+        for (const void *f : fns) {
+            cudaError_t e =
+                cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kS2dMaxSmem);
+            if (e != cudaSuccess) return e;
+        }
+    }
+    const dim3 grid((unsigned)a.Hz, (unsigned)a.N);
+    switch (a.C) {
+        case 1: s2d_kernel<1><<<grid, 256, smem, st>>>(a); break;
+        case 2: s2d_kernel<2><<<grid, 256, smem, st>>>(a); break;
+        case 3: s2d_kernel<3><<<grid, 256, smem, st>>>(a); break;
+        case 4: s2d_kernel<4><<<grid, 256, smem, st>>>(a); break;
+        default: return cudaErrorInvalidValue;
+    }
     return cudaGetLastError();
 }
 

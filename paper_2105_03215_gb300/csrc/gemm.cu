@@ -4,9 +4,11 @@
 // (Section 3.1.1: a Conv2D-Add-ReLU style sequence mapped to one
 // "instruction") makes one pass over HBM.
 //
-// Structure (one persistent CTA per SM, 320 threads):
-//   warp 0 lane 0  TMA producer of the mainloop.  The A operand (activations)
-//              comes in one of three ways (AMODE):
+// Structure (one persistent CTA per SM, 352 threads).  Every role that waits
+// on a barrier has a warp of its own: a lane suspended in mbarrier.try_wait
+// holds up the divergent paths of the other lanes of its warp.
+//   warp 0     TMA producer of the mainloop (one elected lane issues).  The A
+//              operand (activations) comes in one of three ways (AMODE):
 //                tile   a 128 x BK tile of a row-major [M, K] matrix;
 //                im2col 128 consecutive output pixels of one filter tap and
 //                       channel chunk (out-of-image taps zero-filled by TMA);
@@ -16,21 +18,25 @@
 //                       read from row r * Wp + s on, by shifting the MMA's
 //                       shared-memory descriptor -- one load per chunk instead
 //                       of one per tap.
-//              The B operand (packed weights) is one BN x BK tile per k-block.
-//   warp 0 lane 1  producer of the epilogue operands: per tile, the tile's
-//              bias slice (bulk copy) and, when the region adds a residual,
-//              the 128 x BN residual tile (TMA) into one of two buffers.
-//   warp 1     allocates TMEM; one lane issues tcgen05.mma (M=128, N=BN, K=16
-//              per instruction) into one of two fp32 accumulators in TMEM and
-//              tcgen05.commit's the ring slots and the finished accumulator.
-//   warps 2-9  epilogue: two warps per 32-row TMEM lane quarter, taking
-//              alternate 32-column chunks.  Per chunk: tcgen05.ld (one row per
+//              The B operand (packed weights) is one BN x BK tile per k-block;
+//              a ring stage holds G k-blocks.
+//   warp 1     allocates TMEM; one elected lane issues tcgen05.mma (M=128,
+//              N=BN, K=16 per instruction) into one of two fp32 accumulators
+//              in TMEM and tcgen05.commit's the ring stages and the finished
+//              accumulator.
+//   warps 2-9  epilogue: two groups of four warps (one per 32-row TMEM lane
+//              quarter).  For BN <= 64 the groups take alternate tiles, so
+//              that two tiles' epilogues overlap; for wider tiles they split
+//              each tile's 32-column chunks.  Per chunk: tcgen05.ld (one row per
 //              thread), + bias and + residual from shared memory, activation,
 //              bf16 rounding, then a transpose through a 64-byte-swizzled
 //              shared-memory tile so that the global stores are coalesced
 //              64-byte row segments.  The accumulator is released as soon as
 //              it has been read, so the next tile's MMAs overlap this tile's
 //              stores.
+//   warp 10    producer of the epilogue operands: per tile, the tile's bias
+//              slice (bulk copy) and, when the region adds a residual, the
+//              128 x BN residual tile (TMA) into one of two buffers.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -53,11 +59,11 @@ struct GemmShape {
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
     static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE;
-    static constexpr int CTRL_BYTES = 512;
+    static constexpr int CTRL_BYTES = 1024;
     static constexpr int FIXED =
         1024 + 2 * SLAB_BYTES + 2 * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
-    static constexpr int STAGES = STAGES_RAW > 16 ? 16 : STAGES_RAW;
+    static constexpr int STAGES = STAGES_RAW > 32 ? 32 : STAGES_RAW;  // ring slots (k-blocks)
     static constexpr int NUM_BARS = 2 * STAGES + 13;
     static constexpr int SMEM_BYTES = FIXED + STAGES * STAGE_BYTES;
     static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
@@ -81,11 +87,14 @@ __device__ __forceinline__ float apply_act(float v, int act) {
 }
 
 template <int BN, int BK, int AMODE, bool RES>
-__global__ void __launch_bounds__(kGemmThreads, 1)
+// 168 registers: 11 warps put three on some SM sub-partitions, and three
+// warps x 32 lanes x 168 fit a sub-partition's 16384 registers.
+__global__ void __maxnreg__(168)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
     using S = GemmShape<BN, BK, AMODE, RES>;
+    constexpr int kEpiArrivals = BN <= 64 ? kGemmEpiWarps / 2 : kGemmEpiWarps;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -118,9 +127,9 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull + 8u * b, 1);                 // MMA commit
-            mbar_init(tempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
+            mbar_init(tempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
             mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
-            mbar_init(oempty + 8u * b, kGemmEpiWarps);    // one arrive per epilogue warp
+            mbar_init(oempty + 8u * b, kEpiArrivals);
             mbar_init(sfull + 8u * b, 1);                 // producer + slab bytes
             mbar_init(sempty + 8u * b, 1);                // MMA commit
         }
@@ -141,25 +150,34 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // Ring stages of G k-blocks each; at least two stages.
+    const int G = a.group < 1 ? 1 : (a.group > S::STAGES / 2 ? S::STAGES / 2 : a.group);
+    const int nst = S::STAGES / G;
 
     if (warp == 0) {
-        if (lane == 0) {
-            // ------------------------------------------------ mainloop producer
-            int stage = 0, sl = 0, issued = 0;
+        // -------------------------------------------------- mainloop producer
+        // Like the MMA warp, one lane chosen by elect.sync runs the whole
+        // loop.  A ring stage holds G consecutive k-blocks (slab mode: G
+        // filter taps of one channel chunk): one barrier handshake per stage.
+        if (elect_one()) {
+            auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
+                return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutProducer);
+            };
+            int stage = 0, slot0 = 0, sl = 0, issued = 0;
             uint32_t phase = 0;
             bool ok = true;
-            // Wait for ring slot `stage` to be free and announce `bytes` on its full barrier.
+            // Wait for `stage` to be free and announce `bytes` on its full barrier.
             auto claim = [&](uint32_t bytes) -> bool {
-                if (!mbar_wait(bars + 8u * (S::STAGES + stage), phase ^ 1u, abort_flag, a.err,
-                               kErrTimeoutProducer))
-                    return false;
+                if (!wait(bars + 8u * (S::STAGES + stage), phase ^ 1u)) return false;
                 mbar_arrive_expect_tx(bars + 8u * stage, bytes);
                 return true;
             };
             auto advance = [&]() {
                 ++issued;
-                if (++stage == S::STAGES) {
+                slot0 += G;
+                if (++stage == nst) {
                     stage = 0;
+                    slot0 = 0;
                     phase ^= 1u;
                 }
             };
@@ -172,20 +190,23 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
                         const int ss = sl & 1;
                         const uint32_t sph = (uint32_t)(sl >> 1) & 1u;
-                        if (!mbar_wait(sempty + 8u * ss, sph ^ 1u, abort_flag, a.err,
-                                       kErrTimeoutProducer)) {
+                        if (!wait(sempty + 8u * ss, sph ^ 1u)) {
                             ok = false;
                             break;
                         }
                         mbar_arrive_expect_tx(sfull + 8u * ss, (uint32_t)a.slab_bytes);
                         tma_load_4d(sSlab + ss * S::SLAB_BYTES, &tmA, sfull + 8u * ss, cc * BK,
                                     -a.pad_l, p0 - a.pad_t, img);
-                        for (int tap = 0, kb = cc; tap < a.taps; ++tap, kb += a.chunks) {
-                            if (!claim(S::B_BYTES)) {
+                        for (int tap = 0, kb = cc; tap < a.taps; tap += G) {
+                            const int gn = a.taps - tap < G ? a.taps - tap : G;
+                            if (!claim((uint32_t)(gn * S::B_BYTES))) {
                                 ok = false;
                                 break;
                             }
-                            tma_load_2d(sB + stage * S::B_BYTES, &tmB, bars + 8u * stage, kb * BK, n0);
+                            for (int g = 0; g < gn; ++g)
+                                tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, bars + 8u * stage,
+                                            (kb + g * a.chunks) * BK, n0);
+                            kb += gn * a.chunks;
                             advance();
                         }
                     }
@@ -202,39 +223,45 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                         w0 = q * a.stride_w - a.pad_l;
                     }
                     int cc = 0, r = 0, sx = 0;  // (tap r, s; chunk cc) of k-block kb, im2col mode
-                    for (int kb = 0; kb < a.num_kb; ++kb) {
-                        if (!claim(S::STAGE_BYTES)) {
+                    for (int kb = 0; kb < a.num_kb; kb += G) {
+                        const int gn = a.num_kb - kb < G ? a.num_kb - kb : G;
+                        if (!claim((uint32_t)(gn * S::STAGE_BYTES))) {
                             ok = false;
                             break;
                         }
                         const uint32_t full = bars + 8u * stage;
-                        if constexpr (AMODE == kAModeIm2col) {
-                            tma_load_im2col_4d(sA + stage * S::A_BYTES, &tmA, full, cc * BK, w0, h0,
-                                               img, (uint16_t)(sx * a.dil_w),
-                                               (uint16_t)(r * a.dil_h));
-                            if (++cc == a.chunks) {
-                                cc = 0;
-                                if (++sx == a.kw) {
-                                    sx = 0;
-                                    ++r;
+                        for (int g = 0; g < gn; ++g) {
+                            const uint32_t dA = sA + (slot0 + g) * S::A_BYTES;
+                            if constexpr (AMODE == kAModeIm2col) {
+                                tma_load_im2col_4d(dA, &tmA, full, cc * BK, w0, h0, img,
+                                                   (uint16_t)(sx * a.dil_w), (uint16_t)(r * a.dil_h));
+                                if (++cc == a.chunks) {
+                                    cc = 0;
+                                    if (++sx == a.kw) {
+                                        sx = 0;
+                                        ++r;
+                                    }
                                 }
+                            } else {
+                                tma_load_2d(dA, &tmA, full, (kb + g) * BK, m0);
                             }
-                        } else {
-                            tma_load_2d(sA + stage * S::A_BYTES, &tmA, full, kb * BK, m0);
+                            tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, full, (kb + g) * BK, n0);
                         }
-                        tma_load_2d(sB + stage * S::B_BYTES, &tmB, full, kb * BK, n0);
                         advance();
                     }
                 }
             }
             if (!ok) {
                 // Gave up: let the copies already issued land before exiting.
-                for (int j = issued - S::STAGES > 0 ? issued - S::STAGES : 0; j < issued; ++j)
-                    mbar_wait_drain(bars + 8u * (j % S::STAGES), (uint32_t)(j / S::STAGES) & 1u);
+                for (int j = issued - nst > 0 ? issued - nst : 0; j < issued; ++j)
+                    mbar_wait_drain(bars + 8u * (j % nst), (uint32_t)(j / nst) & 1u);
                 for (int j = sl - 2 > 0 ? sl - 2 : 0; j < sl; ++j)
                     mbar_wait_drain(sfull + 8u * (j & 1), (uint32_t)(j >> 1) & 1u);
             }
-        } else if (lane == 1) {
+        }
+        __syncwarp();
+    } else if (warp == kGemmOperandWarp) {
+        if (elect_one()) {
             // ------------------------------------------------ epilogue-operand producer
             int t = 0;
             for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
@@ -258,24 +285,38 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             if (t > 1) mbar_wait_drain(ofull + 8u * ((t - 2) & 1), (uint32_t)((t - 2) >> 1) & 1u);
         }
     } else if (warp == 1) {
-        if (lane == 0) {
-            // ------------------------------------------------ MMA issuer
-            // One thread issues every MMA, so its per-k-block path is kept
-            // lean: the ring position advances by compare-and-wrap, shared
-            // memory descriptors advance by adding (byte offset >> 4) to their
-            // 14-bit address field, and filter taps are walked without
-            // division.
+        // ---------------------------------------------------- MMA issuer
+        // One lane chosen by elect.sync runs the whole loop: waits, MMAs and
+        // commits.  Issued this way tcgen05.mma keeps the tensor pipe fed
+        // (measured: a voted wait or a __syncwarp per stage starves it), and
+        // the compiler knows that a single lane issues.  The path per
+        // k-block is kept lean: the ring position advances by
+        // compare-and-wrap, descriptors advance by adding (byte offset >> 4)
+        // to their 14-bit address field, and filter taps are walked without
+        // division.
+        if (elect_one()) {
+            auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
+                return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutMma);
+            };
             constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
             const uint64_t adesc0 = make_smem_desc(AMODE == kAModeSlab ? sSlab : sA, S::ROW_BYTES);
             const uint64_t bdesc0 = make_smem_desc(sB, S::ROW_BYTES);
-            int stage = 0;
+            int stage = 0, slot0 = 0;
             uint32_t phase = 0;
             int sl = 0, t = 0;
             bool ok = true;
+            auto advance = [&]() {
+                slot0 += G;
+                if (++stage == nst) {
+                    stage = 0;
+                    slot0 = 0;
+                    phase ^= 1u;
+                }
+            };
             for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x, ++t) {
                 const int buf = t & 1;
                 const uint32_t aph = (uint32_t)(t >> 1) & 1u;
-                if (!mbar_wait(tempty + 8u * buf, aph ^ 1u, abort_flag, a.err, kErrTimeoutMma)) {
+                if (!wait(tempty + 8u * buf, aph ^ 1u)) {
                     ok = false;
                     break;
                 }
@@ -286,59 +327,60 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                     const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
                         const int ss = sl & 1;
-                        if (!mbar_wait(sfull + 8u * ss, (uint32_t)(sl >> 1) & 1u, abort_flag, a.err,
-                                       kErrTimeoutMma)) {
+                        if (!wait(sfull + 8u * ss, (uint32_t)(sl >> 1) & 1u)) {
                             ok = false;
                             break;
                         }
                         const uint64_t slab_desc = adesc0 + (uint64_t)((ss * S::SLAB_BYTES) >> 4);
-                        uint32_t roff = 0;  // r * wp * ROW_BYTES
-                        for (int r = 0; ok && r < a.taps / a.kw; ++r, roff += row_step) {
-                            uint32_t toff = roff;  // (r * wp + s) * ROW_BYTES
-                            for (int sx = 0; sx < a.kw; ++sx, toff += S::ROW_BYTES) {
-                                if (!mbar_wait(bars + 8u * stage, phase, abort_flag, a.err,
-                                               kErrTimeoutMma)) {
-                                    ok = false;
-                                    break;
-                                }
-                                tc_fence_after();
-                                const uint64_t ad = slab_desc + (uint64_t)(toff >> 4);
-                                const uint64_t bd = bdesc0 + (uint64_t)((stage * S::B_BYTES) >> 4);
+                        uint32_t roff = 0;  // r * wp * ROW_BYTES of the current tap (r, sx)
+                        int sx = 0;
+                        for (int tap = 0; tap < a.taps; tap += G) {
+                            const int gn = a.taps - tap < G ? a.taps - tap : G;
+                            if (!wait(bars + 8u * stage, phase)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                            uint64_t bd = bdesc0 + (uint64_t)((slot0 * S::B_BYTES) >> 4);
+                            for (int g = 0; g < gn; ++g, bd += (uint64_t)(S::B_BYTES >> 4)) {
+                                const uint64_t ad =
+                                    slab_desc + (uint64_t)((roff + (uint32_t)sx * S::ROW_BYTES) >> 4);
 #pragma unroll
-                                for (int k = 0; k < BK / 16; ++k) {
+                                for (int k = 0; k < BK / 16; ++k)
                                     mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k),
-                                                idesc, acc);
-                                    acc = 1u;
-                                }
-                                mma_commit(bars + 8u * (S::STAGES + stage));  // frees the B slot
-                                if (++stage == S::STAGES) {
-                                    stage = 0;
-                                    phase ^= 1u;
+                                                idesc, acc | (uint32_t)k);
+                                acc = 1u;
+                                if (++sx == a.kw) {
+                                    sx = 0;
+                                    roff += row_step;
                                 }
                             }
+                            mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
+                            advance();
                         }
                         if (!ok) break;
                         mma_commit(sempty + 8u * ss);  // frees the slab
                     }
                 } else {
-                    for (int kb = 0; kb < a.num_kb; ++kb) {
-                        if (!mbar_wait(bars + 8u * stage, phase, abort_flag, a.err, kErrTimeoutMma)) {
+                    for (int kb = 0; kb < a.num_kb; kb += G) {
+                        const int gn = a.num_kb - kb < G ? a.num_kb - kb : G;
+                        if (!wait(bars + 8u * stage, phase)) {
                             ok = false;
                             break;
                         }
                         tc_fence_after();
-                        const uint64_t ad = adesc0 + (uint64_t)((stage * S::A_BYTES) >> 4);
-                        const uint64_t bd = bdesc0 + (uint64_t)((stage * S::B_BYTES) >> 4);
+                        uint64_t ad = adesc0 + (uint64_t)((slot0 * S::A_BYTES) >> 4);
+                        uint64_t bd = bdesc0 + (uint64_t)((slot0 * S::B_BYTES) >> 4);
+                        for (int g = 0; g < gn; ++g, ad += (uint64_t)(S::A_BYTES >> 4),
+                                 bd += (uint64_t)(S::B_BYTES >> 4)) {
 #pragma unroll
-                        for (int k = 0; k < BK / 16; ++k) {
-                            mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, acc);
+                            for (int k = 0; k < BK / 16; ++k)
+                                mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                            acc | (uint32_t)k);
                             acc = 1u;
                         }
-                        mma_commit(bars + 8u * (S::STAGES + stage));  // frees the ring slot
-                        if (++stage == S::STAGES) {
-                            stage = 0;
-                            phase ^= 1u;
-                        }
+                        mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
+                        advance();
                     }
                 }
                 if (!ok) break;
@@ -348,12 +390,18 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
             mma_commit(drain);
             mbar_wait_drain(drain, 0);
         }
+        __syncwarp();
     } else {
         // ---------------------------------------------------- epilogue
         const int e = warp - 2;            // 0..7
         const int quarter = warp & 3;      // TMEM lanes (= tile rows) this warp may access
-        const int half = e >> 2;           // takes chunks ci with ci % 2 == half
         constexpr int NCH = BN / 32;       // 32-column chunks per tile
+        // BN <= 64: the two groups take alternate tiles (accumulator t % 2), all
+        // chunks each.  BN >= 128: both groups take every tile, group `grp`
+        // the chunks ci with ci % 2 == grp, so that a tile's accumulator is
+        // read, and released to the MMAs, twice as fast.
+        constexpr bool ALT = BN <= 64;
+        const int grp = e >> 2;
         const uint32_t stg = sEpi + (uint32_t)e * S::EPI_TILE;
         const int trow = quarter * 32 + lane;  // this thread's row within the tile
         // 64-byte swizzle of the 32x32 bf16 staging tile: 16-byte piece c of
@@ -361,8 +409,10 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
         // writes and the coalesced reads below are free of bank conflicts.
         const uint32_t sw_own = ((uint32_t)lane >> 1) & 3u;
         const int cl_row = lane >> 2, cl_piece = lane & 3;  // coalesced: rows 8k + lane/4
-        int t = 0;
-        for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
+        const int t_first = ALT ? grp : 0, t_step = ALT ? 2 : 1;
+        const int c_first = ALT ? 0 : grp, c_step = ALT ? 1 : 2;
+        for (int tile = blockIdx.x + t_first * (int)gridDim.x, t = t_first; tile < a.num_tiles;
+             tile += t_step * (int)gridDim.x, t += t_step) {
             const int buf = t & 1;
             const uint32_t aph = (uint32_t)(t >> 1) & 1u;
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
@@ -391,21 +441,12 @@ __global__ void __launch_bounds__(kGemmThreads, 1)
                 tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
             const uint32_t bias_s = sBias + (uint32_t)(buf * S::BIAS_BYTES);
             const uint32_t res_s = sRes + (uint32_t)(buf * S::RES_TILE);
-            if (half >= NCH) {  // no chunk for this warp in this tile (BN = 32)
-                tc_fence_before();
-                __syncwarp();
-                if (lane == 0) {
-                    mbar_arrive(tempty + 8u * buf);
-                    mbar_arrive(oempty + 8u * buf);
-                }
-                continue;
-            }
 #pragma unroll 1
-            for (int ci = half; ci < NCH; ci += 2) {
+            for (int ci = c_first; ci < NCH; ci += c_step) {
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);  // includes tcgen05.wait::ld
-                if (ci + 2 >= NCH) {  // this warp's last read of the accumulator
+                if (ci + c_step >= NCH) {  // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty + 8u * buf);

@@ -37,6 +37,8 @@ struct GemmArgs {
     int tiles_per_img;  // ceil(Ho / slab_t)
     int slab_bytes;     // bytes of one slab (one channel chunk)
     int taps;           // kh * kw
+    int group;      // k-blocks (slab mode: filter taps) per ring stage, >= 1; the
+                    // kernel lowers it so that at least two stages fit the ring
     int act;        // Act
     const float *bias;                // [tiles_n * BN], zero padded; required
     const __nv_bfloat16 *residual;    // [M, N] or null
@@ -62,7 +64,21 @@ constexpr int slab_max_bytes(int bk) { return bk == 64 ? 48 * 1024 : 24 * 1024; 
 
 constexpr int kGemmBM = 128;
 constexpr int kGemmEpiWarps = 8;
-constexpr int kGemmThreads = 64 + 32 * kGemmEpiWarps;  // warp 0 TMA, warp 1 MMA, warps 2-9 epilogue
+// warp 0 mainloop TMA, warp 1 MMA, warps 2-9 epilogue, warp 10 epilogue operands
+constexpr int kGemmOperandWarp = 2 + kGemmEpiWarps;
+constexpr int kGemmThreads = 32 * (kGemmOperandWarp + 1);
+
+// k-blocks per ring stage for a run of `n` k-blocks (slab mode: the taps of
+// one channel chunk): enough MMA work per barrier handshake (bn * bk * group
+// >= 256 * 64, about 600 tensor-core cycles at M = 128) that the single
+// issuing thread stays ahead of the tensor pipe, then evened out over n.
+inline int gemm_group(int bn, int bk, int n) {
+    int g = (256 * 64 + bn * bk - 1) / (bn * bk);
+    if (g > 8) g = 8;
+    if (n < 1) return 1;
+    const int stages = (n + g - 1) / g;
+    return (n + stages - 1) / stages;
+}
 
 bool gemm_config_supported(const GemmConfig &cfg);
 size_t gemm_smem_bytes(const GemmConfig &cfg);
@@ -90,14 +106,22 @@ cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st);
 // (space-to-depth with zero padding, vertical filter taps stacked):
 //   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
 // for a < taps, zero outside the image and in channels a*16 + [4C, 16).
+// Space-to-depth of a stride-2 stem (C <= 4 channels) with the `taps`
+// vertical filter taps stacked into the channel dimension:
+//   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
+// zero outside x and in channels 4C..15 of each 16-channel group.
 struct S2dArgs {
-    const __nv_bfloat16 *x;
-    __nv_bfloat16 *z;
-    int N, H, W, C;   // input
-    int Hz, Wz, Cz;   // output: Hz = output rows, Cz = 16 * taps
+    const __nv_bfloat16 *x;  // [N, H, W, C]
+    __nv_bfloat16 *z;        // [N, Hz, Wz, 16 * taps]
+    int N, H, W, C;
+    int Hz, Wz;              // N, Hz <= 65535
     int taps;
     int pad;
 };
+// The transform stages 2 * taps input rows (W * C elements each) in shared
+// memory; the planner rejects stems whose rows need more than kS2dMaxSmem.
+constexpr size_t kS2dMaxSmem = 200 * 1024;
+size_t s2d_smem_bytes(const S2dArgs &a);
 cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st);
 
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,

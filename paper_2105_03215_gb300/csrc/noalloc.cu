@@ -138,6 +138,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.stride_h = g.stride_w = 1;
     g.tiles_n = F / kTileN;
     g.num_tiles = tiles_m * g.tiles_n;
+    g.group = byoc::gemm_group(kTileN, 64, g.num_kb);
     g.act = byoc::kActGelu;
     g.bias = b1;
     g.residual = nullptr;
@@ -151,6 +152,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.chunks = g.num_kb;
     g.tiles_n = D / kTileN;
     g.num_tiles = tiles_m * g.tiles_n;
+    g.group = byoc::gemm_group(kTileN, 64, g.num_kb);
     g.act = byoc::kActNone;
     g.bias = b2;
     g.out = static_cast<__nv_bfloat16 *>(y);

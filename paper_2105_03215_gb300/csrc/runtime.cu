@@ -163,6 +163,7 @@ struct LaunchPlan {
     int kind = BYOC_LAUNCH_GEMM;
     int first_op = -1, n_ops = 0;
     int x = -1, y = -1, res = -1;  // tensor ids (may index internal scratch tensors)
+    size_t x_off = 0, y_off = 0;   // byte offsets into tensors x and y (image chunks)
     int act = byoc::kActNone;
     // GEMM
     GemmConfig cfg{64, 64, byoc::kAModeTile, false};
@@ -519,6 +520,8 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
 
         // ---------------- GEMM (conv2d groups=1, or dense)
         int64_t M, Kreal;
+        int64_t stem_k = 0;     // > 0: the stem conv's reduction length before space-to-depth
+        int64_t stem_imgs = 0;  // stem: images per (space-to-depth, GEMM) launch pair
         int kh = 1, kw = 1, taps = 1, chunks, bk;
         int64_t C;
         std::vector<double> wsrc;  // weights as [Cout][kh][kw][C] (channel innermost)
@@ -547,9 +550,14 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                 // turns the k x k stride-2 conv over C channels into a k2 x k2
                 // stride-1 conv over 4C (<= 16) channels, k2 = (k+1)/2, and also
                 // stacks the k2 vertical taps into the channel dimension, so the
-                // GEMM is a 1 x k2 conv over 16*k2 channels:
+                // GEMM is a 1 x k2 conv over 16*k2 channels (128-byte operand rows
+                // for k2 = 4):
                 //   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
                 //   w''[k][b][a*16 + (dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx]
+                // The stacked tensor is k2 times larger than the image, so the
+                // pair of launches runs over chunks of images whose z fits in
+                // L2 (about 32 MiB): z is written and read back without a DRAM
+                // round trip.
                 if (!(square && op.stride[0] == 2 && op.dilation[0] == 1 && C <= 4 && (kh % 2) == 1))
                     return fail(BYOC_ERR_UNSUPPORTED,
                                 "op %d: %lld input channels: only a stride-2 odd square stem with "
@@ -557,9 +565,16 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                                 o, (long long)C);
                 const int k2 = (kh + 1) / 2;
                 const int Cz = 16 * k2;
+                if (X.shape[0] > 65535 || Y.shape[1] > 65535)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem batch or height above 65535", o);
+                const int64_t z_img = Y.shape[1] * (Y.shape[2] + k2 - 1) * Cz * 2;
+                int64_t nck = (X.shape[0] * z_img + (32ll << 20) - 1) / (32ll << 20);
+                const int64_t room = (BYOC_PLAN_MAX_LAUNCHES - 1 - (int64_t)P.launches.size()) / 2;
+                nck = std::max<int64_t>(1, std::min<int64_t>({nck, room, X.shape[0]}));
+                stem_imgs = (X.shape[0] + nck - 1) / nck;
                 TensorInfo Z;
                 Z.ndim = 4;
-                Z.shape[0] = X.shape[0];
+                Z.shape[0] = stem_imgs;
                 Z.shape[1] = Y.shape[1];
                 Z.shape[2] = Y.shape[2] + k2 - 1;
                 Z.shape[3] = Cz;
@@ -575,10 +590,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                 S.s2d.C = (int)C;
                 S.s2d.Hz = (int)Z.shape[1];
                 S.s2d.Wz = (int)Z.shape[2];
-                S.s2d.Cz = Cz;
                 S.s2d.taps = k2;
                 S.s2d.pad = op.pad[0];
-                S.bytes = (double)X.bytes() + (double)Z.bytes();
+                S.bytes = (double)X.bytes();  // z is internal: not algorithmic traffic
+                if (byoc::s2d_smem_bytes(S.s2d) > byoc::kS2dMaxSmem)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem rows too wide (%lld x %lld)", o,
+                                (long long)X.shape[2], (long long)C);
                 P.launches.push_back(S);
                 wsrc.assign((size_t)Cout * k2 * Cz, 0.0);
                 for (int64_t k = 0; k < Cout; ++k)
@@ -592,6 +609,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                                         wsrc[((size_t)k * k2 + b) * Cz + a * 16 + (dy * 2 + dx) * C + c] =
                                             op.consts[0][((k * C + c) * kh + r) * kw + s];
                                     }
+                stem_k = (int64_t)kh * kw * C;  // the conv's own reduction length
                 L.x = zid;
                 C = Cz;
                 kh = 1;
@@ -667,7 +685,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         }
         L.n_pad = (int)((Cout + bn - 1) / bn * bn);
         L.k_pack = taps * chunks * bk;
-        Kreal = (int64_t)taps * C;
+        Kreal = stem_k > 0 ? stem_k : (int64_t)taps * C;
         // Folded, bf16-rounded, K-major packed weights [n_pad][k_pack].
         std::vector<uint16_t> wp((size_t)L.n_pad * L.k_pack, 0);
         for (int64_t k = 0; k < Cout; ++k)
@@ -699,14 +717,42 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         A.tiles_n = L.n_pad / bn;
         A.num_tiles = (int)(tiles_m * A.tiles_n);
         A.taps = taps;
+        A.group = byoc::gemm_group(bn, bk, amode == byoc::kAModeSlab ? taps : A.num_kb);
         A.act = act;
         L.grid = std::min(A.num_tiles, P.num_sms);
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
-        const double in_bytes = L.x < P.n_region_tensors ? (double)X.bytes()
-                                                         : (double)P.tensors[L.x].bytes();
+        const double in_bytes = stem_k > 0 ? 0.0  // z: counted as x by the transform
+                                : L.x < P.n_region_tensors ? (double)X.bytes()
+                                                           : (double)P.tensors[L.x].bytes();
         L.bytes = in_bytes + (double)Y.bytes() + (double)Cout * Kreal * 2 + (double)Cout * 4 +
                   (res >= 0 ? (double)P.tensors[res].bytes() : 0.0);
         P.launches.push_back(L);
+        if (stem_k > 0) {
+            // one (space-to-depth, GEMM) pair per chunk of stem_imgs images
+            const LaunchPlan S0 = P.launches[P.launches.size() - 2];
+            const LaunchPlan G0 = L;
+            P.launches.resize(P.launches.size() - 2);
+            const int64_t N = X.shape[0];
+            const int64_t hw = Y.shape[1] * Y.shape[2];
+            for (int64_t n0 = 0; n0 < N; n0 += stem_imgs) {
+                const int64_t nc = std::min(stem_imgs, N - n0);
+                const double frac = (double)nc / (double)N;
+                LaunchPlan S = S0;
+                S.s2d.N = (int)nc;
+                S.x_off = (size_t)(n0 * X.shape[1] * X.shape[2] * X.shape[3] * 2);
+                S.bytes = S0.bytes * frac;
+                P.launches.push_back(S);
+                LaunchPlan G = G0;
+                G.geo.N = (int)nc;
+                G.args.M = (int)(nc * hw);
+                G.args.num_tiles = (int)(nc * G.args.tiles_per_img * G.args.tiles_n);
+                G.grid = std::min(G.args.num_tiles, P.num_sms);
+                G.y_off = (size_t)(n0 * hw * Cout * 2);
+                G.flops = G0.flops * frac;
+                G.bytes = G0.bytes * frac;
+                P.launches.push_back(G);
+            }
+        }
         o = j;
     }
     // Workspace: every tensor that is neither a region input nor output.
@@ -936,7 +982,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
         LaunchPlan &L = P.launches[i];
         cudaError_t e = cudaSuccess;
         if (L.kind == BYOC_LAUNCH_GEMM) {
-            const void *xa = h->ptrs[L.x];
+            const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
                 CUresult r;
                 if (L.cfg.amode == byoc::kAModeSlab)
@@ -953,7 +999,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                 h->tmA_ptr[i] = xa;
             }
             GemmArgs a = L.args;
-            a.out = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            a.out = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
             a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
             if (a.residual && h->tmR_ptr[i] != a.residual) {
                 // residual [M, N]: 64-column x 128-row boxes, 128-byte swizzle
@@ -973,8 +1019,9 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             e = byoc::launch_dwconv(a, P.num_sms, st);
         } else {
             byoc::S2dArgs a = L.s2d;
-            a.x = static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]);
-            a.z = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            a.x = reinterpret_cast<const __nv_bfloat16 *>(static_cast<const char *>(h->ptrs[L.x]) +
+                                                           L.x_off);
+            a.z = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
             e = byoc::launch_s2d(a, st);
         }
         if (e != cudaSuccess) return cuda_fail(e, "kernel launch");

@@ -63,6 +63,42 @@ def test_plan_stem_inserts_space_to_depth():
     assert rep.gemm_k[1] == 4 * 64 and rep.tile_k[1] == 64 and rep.im2col[1] == 2
 
 
+def test_stem_weights_follow_the_space_to_depth_definition():
+    # w''[k][b][a*16 + (dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx], zero where 2a+dy or 2b+dx >= 7
+    g, _ = I.resnet50(N=1, H=32, W=32)
+    reg = R.Region(g, [n.name for n in g.nodes[:3]], "stem")
+    rep = reg.plan()
+    w = g.nodes[0].consts["weight"].astype(np.float64)            # [64, 3, 7, 7]
+    bn = g.nodes[1]
+    scale = bn.consts["gamma"].astype(np.float64) / np.sqrt(
+        bn.consts["moving_var"].astype(np.float64) + 1e-5)
+    packed = np.frombuffer(reg.plan_constants(1, 0), dtype=np.uint16).reshape(-1, rep.gemm_k[1])
+    expect = np.zeros((64, 4, 4, 16), dtype=np.float64)            # [k][b][a][group]
+    for a in range(4):
+        for b in range(4):
+            for dy in range(2):
+                for dx in range(2):
+                    r, s_ = 2 * a + dy, 2 * b + dx
+                    if r < 7 and s_ < 7:
+                        expect[:, b, a, (dy * 2 + dx) * 3:(dy * 2 + dx) * 3 + 3] = w[:, :, r, s_]
+    expect *= scale[:, None, None, None]
+    want = I.bf16_bits(expect.reshape(64, -1).astype(np.float32))
+    assert np.array_equal(packed[:64], want)
+    # the flop count is the 7x7x3 convolution's, not the padded GEMM's
+    assert rep.flops == pytest.approx(2.0 * 64 * 16 * 16 * 7 * 7 * 3, rel=1e-12)
+
+
+def test_stem_runs_in_image_chunks_that_fit_l2():
+    g, _ = I.stem(N=64, H=224, W=224)
+    rep = R.whole_graph_region(g).plan()
+    # stacked z: 112 x 115 x 64 bf16 = 1.65 MB per image -> 4 chunks of 16 images
+    assert rep.n_launches == 8
+    assert [rep.kind[i] for i in range(8)] == [abi.LAUNCH_S2D, abi.LAUNCH_GEMM] * 4
+    assert all(rep.gemm_m[i] == 16 * 112 * 112 for i in range(1, 8, 2))
+    assert rep.workspace_bytes <= 256 + 16 * 112 * 115 * 64 * 2 + 256
+    assert rep.flops == pytest.approx(2.0 * 64 * 112 * 112 * 64 * 7 * 7 * 3, rel=1e-12)
+
+
 def test_plan_flops_match_mac_count():
     for g, _ in [I.bert_ffn(), I.resnet_bottleneck(), I.conv_bias_relu()]:
         assert _plan(g).flops == pytest.approx(I.region_flops(g), rel=1e-12)

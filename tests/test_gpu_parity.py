@@ -133,6 +133,15 @@ def test_stem_variants(k, cout, C):
     _check_graph(g, inp, what=f"stem{k}x{k}")
 
 
+def test_stem_in_image_chunks_with_a_ragged_last_chunk():
+    # 21 images of 224 x 224: the stacked space-to-depth tensor (1.65 MB per
+    # image) is processed as two launch pairs, of 11 and 10 images
+    g, inp = I.stem(N=21, H=224, W=224, seed=17)
+    rep = R.whole_graph_region(g).plan()
+    assert rep.n_launches == 4 and rep.gemm_m[1] == 11 * 112 * 112 and rep.gemm_m[3] == 10 * 112 * 112
+    _check_graph(g, inp, what="stem in chunks")
+
+
 def test_region_can_run_twice_with_new_pointers():
     import torch
     from .parity import to_dev
