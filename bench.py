@@ -178,16 +178,25 @@ def run_reference(args, world, rank):
 # ---------------------------------------------------------------- region micro-benchmarks
 
 def time_region(cr, ins, outs, flush, reps=20):
+    """Median device time of one region call: the call is captured in a CUDA
+    graph and replayed between events, so host-side launch work is excluded;
+    L2 is flushed before every replay."""
     import torch
-    st = torch.cuda.current_stream()
-    for _ in range(3):
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        for _ in range(3):
+            cr.run(ins, outs, st)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=st):
         cr.run(ins, outs, st)
+    cur = torch.cuda.current_stream()
     evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
     for a, b in evs:
         flush.zero_()
-        a.record(st)
-        cr.run(ins, outs, st)
-        b.record(st)
+        a.record(cur)
+        graph.replay()
+        b.record(cur)
     torch.cuda.synchronize()
     cr.check()
     return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3  # seconds

@@ -7,6 +7,8 @@
 //     which the paper leaves on the host (Section 3.4, CUDA as the host).
 // All tensors are bf16 NHWC; every thread moves 8 channels (16 bytes) at a
 // time so that a warp's accesses are contiguous along C.
+#include <algorithm>
+
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -37,140 +39,262 @@ __device__ __forceinline__ uint4 ldg_v4(const void *p) {
 // Thread <-> (image n, output column q, 4-channel group, ROWS consecutive
 // output rows).  The channel group varies fastest across threads, so a warp
 // reads and writes one contiguous 256-byte run of an image row per access.
-// The 3 x 3 input window lives in registers as fp32 and slides down the
-// column: each output row loads one new input row (stride 1; two for stride
-// 2), and the next row is loaded before the current one is computed, so two
-// rows of loads are in flight per thread.  Registers stay under 80, so a
-// multiprocessor holds enough warps to keep HBM busy.
-template <int STRIDE, int ROWS>
-__global__ void __launch_bounds__(256, 2) dwconv3x3_kernel(const DwArgs a) {
-    const int CG = a.C >> 2;  // 4-channel groups
-    const int PB = (a.Ho + ROWS - 1) / ROWS;
-    const long long total = (long long)a.N * PB * a.Wo * CG;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= total) return;
-    const int cg = (int)(idx % CG);
-    long long t = idx / CG;
-    const int q = (int)(t % a.Wo);
-    t /= a.Wo;
-    const int pb = (int)(t % PB);
-    const int n = (int)(t / PB);
-    const int c0 = cg * 4;
+// One persistent CTA per SM walks the tiles (chunk slowest, so a CTA mostly
+// keeps one channel chunk and its weights).  Thread t owns the 4-channel
+// vector v = t % V (V = cc / 4), whose 9 x 4 folded weights stay in
+// registers, and computes blocks of kDwBlockH x kDwBlockW outputs (blocks
+// t / V + k * lanes): each input vector under a block is read from shared
+// memory once (8 bytes), unpacked once and fed to every output of the block
+// that uses it, with packed two-lane fp32 FMAs.  A 4 x 2 block reads 24 input
+// vectors for 8 outputs at stride 1 and keeps a thread under 128 registers,
+// so 16 warps per SM overlap the load, unpack and FMA latencies.  The
+// activation is applied to the packed bf16 pairs (exact: rounding is
+// monotonic and 0 and 6 are bf16 values).  The next tile's box loads (TMA)
+// while this one is computed.
+__device__ __forceinline__ void fma2(uint64_t &acc, uint64_t x, uint64_t w) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(x), "l"(w));
+}
+// Register-pair moves (mov.b64 {lo, hi}) so that packing and unpacking the
+// two lanes costs no arithmetic.
+__device__ __forceinline__ uint64_t pair(uint32_t lo, uint32_t hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+    return r;
+}
+__device__ __forceinline__ uint64_t f32x2_of_bf16x2(uint32_t u) {
+    // low half -> lane 0, high half -> lane 1 (a bf16 is the top half of its fp32)
+    return pair(u << 16, u & 0xFFFF0000u);
+}
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+    return pair(__float_as_uint(lo), __float_as_uint(hi));
+}
+__device__ __forceinline__ float lane0(uint64_t v) {
+    uint32_t lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
+    return __uint_as_float(lo);
+}
+__device__ __forceinline__ float lane1(uint64_t v) {
+    uint32_t lo, hi;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
+    return __uint_as_float(hi);
+}
 
-    float w[9][4];
-#pragma unroll
-    for (int tap = 0; tap < 9; ++tap) {
-        const float4 v = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c0));
-        w[tap][0] = v.x; w[tap][1] = v.y; w[tap][2] = v.z; w[tap][3] = v.w;
-    }
-    const float4 b4 = __ldg(reinterpret_cast<const float4 *>(a.bias + c0));
-
-    const int wc0 = q * STRIDE - a.pad;
-    const __nv_bfloat16 *xn = a.x + (size_t)n * a.H * a.W * a.C + c0;
-    // one input row under the filter: 3 columns x 4 channels, zero outside the image
-    // Loads are unconditional (from a clamped, in-image address) and zeroed by
-    // a select afterwards, so they can all be in flight at once.
-    auto load_row = [&](int h, uint2 (&r)[3]) {
-        const bool hv = h >= 0 && h < a.H;
-        const int hc = min(max(h, 0), a.H - 1);
-#pragma unroll
-        for (int s = 0; s < 3; ++s) {
-            const int wc = wc0 + s;
-            const int wcc = min(max(wc, 0), a.W - 1);
-            const uint2 v = __ldg(reinterpret_cast<const uint2 *>(xn + ((size_t)hc * a.W + wcc) * a.C));
-            const bool ok = hv && wc >= 0 && wc < a.W;
-            r[s] = make_uint2(ok ? v.x : 0u, ok ? v.y : 0u);
-        }
-    };
-    auto unpack_row = [&](const uint2 (&r)[3], float (&f)[3][4]) {
-#pragma unroll
-        for (int s = 0; s < 3; ++s) {
-            f[s][0] = bf16lo(r[s].x); f[s][1] = bf16hi(r[s].x);
-            f[s][2] = bf16lo(r[s].y); f[s][3] = bf16hi(r[s].y);
-        }
-    };
-
-    const int p0 = pb * ROWS;
-    float win[3][3][4];
-    uint2 raw[3], nxt[3];
-    load_row(p0 * STRIDE - a.pad, raw);
-    unpack_row(raw, win[0]);
-    load_row(p0 * STRIDE - a.pad + 1, raw);
-    unpack_row(raw, win[1]);
-    load_row(p0 * STRIDE - a.pad + 2, nxt);
-#pragma unroll
-    for (int i = 0; i < ROWS; ++i) {
-        const int p = p0 + i;
-        if (p >= a.Ho) break;
-        const int hb = p * STRIDE - a.pad;
-        unpack_row(nxt, win[2]);
-        // prefetch what the next output row needs beyond the rows kept
-        uint2 mid[3];
-        if (i + 1 < ROWS) {
-            if (STRIDE == 1) {
-                load_row(hb + 3, nxt);
-            } else {
-                load_row(hb + 3, mid);
-                load_row(hb + 4, nxt);
-            }
-        }
-        float acc[4] = {b4.x, b4.y, b4.z, b4.w};
-#pragma unroll
-        for (int r = 0; r < 3; ++r)
-#pragma unroll
-            for (int s = 0; s < 3; ++s)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) acc[j] = fmaf(win[r][s][j], w[r * 3 + s][j], acc[j]);
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            float v = acc[j];
-            if (a.act == kActRelu) v = fmaxf(v, 0.0f);
-            else if (a.act == kActRelu6) v = fminf(fmaxf(v, 0.0f), 6.0f);
-            else if (a.act == kActGelu) v = 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
-            acc[j] = v;
-        }
-        uint2 o;
-        o.x = pack_bf16x2(acc[0], acc[1]);
-        o.y = pack_bf16x2(acc[2], acc[3]);
-        *reinterpret_cast<uint2 *>(a.y + (((size_t)n * a.Ho + p) * a.Wo + q) * a.C + c0) = o;
-        // slide the window
-        if (STRIDE == 1) {
-#pragma unroll
-            for (int s = 0; s < 3; ++s)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) {
-                    win[0][s][j] = win[1][s][j];
-                    win[1][s][j] = win[2][s][j];
-                }
-        } else {
-#pragma unroll
-            for (int s = 0; s < 3; ++s)
-#pragma unroll
-                for (int j = 0; j < 4; ++j) win[0][s][j] = win[2][s][j];
-            if (i + 1 < ROWS) unpack_row(mid, win[1]);
-        }
+// act(x) for a pair of outputs, rounded to a bf16 pair; ReLU and ReLU6 are
+// applied after rounding, on the packed pair.
+template <int ACT>
+__device__ __forceinline__ uint32_t dw_act2(float lo, float hi) {
+    if constexpr (ACT == kActRelu || ACT == kActRelu6) {
+        uint32_t r = pack_bf16x2(lo, hi);
+        asm("max.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0u));
+        if constexpr (ACT == kActRelu6) asm("min.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0x40C040C0u));
+        return r;
+    } else if constexpr (ACT == kActGelu) {
+        return pack_bf16x2(0.5f * lo * (1.0f + erff(lo * 0.70710678118654752f)),
+                           0.5f * hi * (1.0f + erff(hi * 0.70710678118654752f)));
+    } else {
+        return pack_bf16x2(lo, hi);
     }
 }
 
-cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st) {
-    (void)num_sms;
-    const int CG = a.C / 4;
-    const int threads = 256;
-    if (a.stride == 1) {
-        constexpr int R = 8;
-        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CG;
-        dwconv3x3_kernel<1, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
-    } else {
-        constexpr int R = 4;
-        const long long total = (long long)a.N * ((a.Ho + R - 1) / R) * a.Wo * CG;
-        dwconv3x3_kernel<2, R><<<(unsigned)((total + threads - 1) / threads), threads, 0, st>>>(a);
+
+template <int STRIDE, int ACT>
+__global__ void __launch_bounds__(kDwMaxThreads, 1)
+    dwconv3x3_kernel(const __grid_constant__ CUtensorMap tmX, const DwArgs a) {
+    constexpr int BH = kDwBlockH, BW = kDwBlockW;      // outputs per thread block
+    constexpr int IR = (BH - 1) * STRIDE + 3;          // input rows under a block
+    constexpr int IC = (BW - 1) * STRIDE + 3;          // input columns under a block
+    extern __shared__ __align__(128) uint8_t smem_dw[];
+    const uint32_t raw = smem_u32(smem_dw);
+    const uint32_t base = (raw + 127u) & ~127u;
+    uint8_t *sbase = smem_dw + (base - raw);
+    const uint32_t bars = base + 2u * (uint32_t)a.buf_bytes;  // 2 full barriers
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(sbase + 2 * a.buf_bytes + 16);
+    const int tid = threadIdx.x;
+    const int V = a.cc >> 2;
+    const int lanes = a.threads / V;
+    const int v = tid % V;
+    const int g = tid / V;
+    if (tid == 0) {
+        mbar_init(bars, 1);
+        mbar_init(bars + 8u, 1);
+        *abort_flag = 0;
+        fence_barrier_init();
+        tma_prefetch_desc(&tmX);
     }
-    return cudaGetLastError();
+    __syncthreads();
+    pdl_launch_dependents();
+    pdl_wait();
+    const int per_chunk = a.N * a.tiles_h * a.tiles_w;
+    auto issue = [&](int tile, int b) {
+        const int ch = tile / per_chunk;
+        int r = tile - ch * per_chunk;
+        const int n = r / (a.tiles_h * a.tiles_w);
+        r -= n * a.tiles_h * a.tiles_w;
+        const int ph = r / a.tiles_w;
+        const int pw = r - ph * a.tiles_w;
+        const uint32_t bar = bars + 8u * (uint32_t)b;
+        mbar_arrive_expect_tx(bar, (uint32_t)(a.in_rows * a.in_cols * a.cc * 2));
+        tma_load_4d(base + (uint32_t)(b * a.buf_bytes), &tmX, bar, ch * a.cc,
+                    pw * a.tw * STRIDE - a.pad, ph * a.th * STRIDE - a.pad, n);
+    };
+    if (tid == 0) {
+        if ((int)blockIdx.x < a.num_tiles) issue(blockIdx.x, 0);
+        if ((int)(blockIdx.x + gridDim.x) < a.num_tiles) issue(blockIdx.x + gridDim.x, 1);
+    }
+    uint64_t w[9][2];  // folded weights, channel pairs
+    float bias[4];
+    int wc = -1;       // channel of the weights in registers
+    const int bcols = a.tw / BW, blocks = (a.th / BH) * bcols;
+    int i = 0;
+    for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++i) {
+        const int b = i & 1;
+        const bool ok = mbar_wait(bars + 8u * (uint32_t)b, (uint32_t)(i >> 1) & 1u, abort_flag, a.err,
+                                  kErrTimeoutProducer);
+        if (__syncthreads_or(!ok)) {
+            // gave up: let this CTA's copies in flight land before exiting
+            if (tid == 0)
+                for (int k = 0; k < 2; ++k)
+                    if (tile + k * (int)gridDim.x < a.num_tiles)
+                        mbar_wait_drain(bars + 8u * (uint32_t)((i + k) & 1), (uint32_t)((i + k) >> 1) & 1u);
+            break;
+        }
+        const int ch = tile / per_chunk;
+        int r = tile - ch * per_chunk;
+        const int n = r / (a.tiles_h * a.tiles_w);
+        r -= n * a.tiles_h * a.tiles_w;
+        const int ph = r / a.tiles_w;
+        const int pw = r - ph * a.tiles_w;
+        const int c = ch * a.cc + v * 4;  // this thread's first channel
+        if (c < a.C && c != wc) {
+#pragma unroll
+            for (int tap = 0; tap < 9; ++tap) {
+                const float4 q = __ldg(reinterpret_cast<const float4 *>(a.w + (size_t)tap * a.C + c));
+                w[tap][0] = f32x2(q.x, q.y);
+                w[tap][1] = f32x2(q.z, q.w);
+            }
+            const float4 q = __ldg(reinterpret_cast<const float4 *>(a.bias + c));
+            bias[0] = q.x; bias[1] = q.y; bias[2] = q.z; bias[3] = q.w;
+            wc = c;
+        }
+        if (c < a.C) {
+            // plain loads (not volatile asm), so the compiler can hoist them
+            // ahead of the FMAs; the barrier wait above orders them after the copy
+            const uint8_t *buf = sbase + (size_t)b * a.buf_bytes + (size_t)v * 8;
+            const uint32_t col_step = (uint32_t)a.cc * 2u;
+            const uint32_t row_step = (uint32_t)a.in_cols * col_step;
+            const int p0 = ph * a.th, q0 = pw * a.tw;
+            __nv_bfloat16 *yimg = a.y + (size_t)n * a.Ho * a.Wo * a.C + c;
+            for (int blk = g; blk < blocks; blk += lanes) {
+                const int br = blk / bcols;
+                const int bc = blk - br * bcols;
+                uint64_t acc[BH][BW][2];
+#pragma unroll
+                for (int oy = 0; oy < BH; ++oy)
+#pragma unroll
+                    for (int ox = 0; ox < BW; ++ox) {
+                        acc[oy][ox][0] = f32x2(bias[0], bias[1]);
+                        acc[oy][ox][1] = f32x2(bias[2], bias[3]);
+                    }
+                const uint8_t *sblk = buf + (size_t)(br * BH * STRIDE) * row_step +
+                                      (size_t)(bc * BW * STRIDE) * col_step;
+#pragma unroll
+                for (int ir = 0; ir < IR; ++ir)
+#pragma unroll
+                    for (int ic = 0; ic < IC; ++ic) {
+                        const uint2 u = *reinterpret_cast<const uint2 *>(
+                            sblk + (size_t)ir * row_step + (size_t)ic * col_step);
+                        const uint64_t x0 = f32x2_of_bf16x2(u.x), x1 = f32x2_of_bf16x2(u.y);
+#pragma unroll
+                        for (int oy = 0; oy < BH; ++oy)
+#pragma unroll
+                            for (int ox = 0; ox < BW; ++ox) {
+                                const int dy = ir - oy * STRIDE, dx = ic - ox * STRIDE;
+                                if (dy < 0 || dy > 2 || dx < 0 || dx > 2) continue;
+                                fma2(acc[oy][ox][0], x0, w[dy * 3 + dx][0]);
+                                fma2(acc[oy][ox][1], x1, w[dy * 3 + dx][1]);
+                            }
+                    }
+                const int pb = p0 + br * BH, qb = q0 + bc * BW;
+                __nv_bfloat16 *yb = yimg + ((size_t)pb * a.Wo + qb) * a.C;
+#pragma unroll
+                for (int oy = 0; oy < BH; ++oy) {
+                    if (pb + oy >= a.Ho) break;
+#pragma unroll
+                    for (int ox = 0; ox < BW; ++ox) {
+                        if (qb + ox >= a.Wo) break;
+                        uint2 o;
+                        o.x = dw_act2<ACT>(lane0(acc[oy][ox][0]), lane1(acc[oy][ox][0]));
+                        o.y = dw_act2<ACT>(lane0(acc[oy][ox][1]), lane1(acc[oy][ox][1]));
+                        *reinterpret_cast<uint2 *>(yb + ((size_t)oy * a.Wo + ox) * a.C) = o;
+                    }
+                }
+            }
+        }
+        __syncthreads();  // buffer b consumed
+        if (tid == 0 && tile + 2 * (int)gridDim.x < a.num_tiles) issue(tile + 2 * (int)gridDim.x, b);
+    }
+}
+
+size_t dw_smem_bytes(const DwArgs &a) { return 128 + 2 * (size_t)a.buf_bytes + 64; }
+
+bool dw_plan(DwArgs &a, int num_sms) {
+    if (a.C % 8 || (a.stride != 1 && a.stride != 2)) return false;
+    a.chunks = (a.C + 255) / 256;
+    a.cc = ((a.C + a.chunks - 1) / a.chunks + 7) / 8 * 8;
+    const int V = a.cc / 4;
+    const int lanes = kDwMaxThreads / V;
+    a.threads = V * lanes;
+    // Tiles are whole kDwBlockH x kDwBlockW output blocks.  Full output width
+    // (rounded up to the block) when its input columns fit one box (<= 256).
+    constexpr int B = kDwBlockH, BW = kDwBlockW;
+    const int tw_max = ((256 - 3) / a.stride + 1) / BW * BW;
+    a.tw = std::min((a.Wo + BW - 1) / BW * BW, tw_max);
+    a.tiles_w = (a.Wo + a.tw - 1) / a.tw;
+    a.in_cols = (a.tw - 1) * a.stride + 3;
+    const size_t row_bytes = (size_t)a.in_cols * a.cc * 2;
+    const size_t budget = 108 * 1024;  // per buffer; two buffers per CTA
+    auto rows_in = [&](int th) { return (th - 1) * a.stride + 3; };
+    const int ho_blocks = (a.Ho + B - 1) / B * B;
+    int th = B;
+    while (th + B <= ho_blocks && (size_t)rows_in(th + B) * row_bytes <= budget && rows_in(th + B) <= 256)
+        th += B;
+    // fewer rows per tile while there would be under two tiles per SM
+    while (th > B && (long long)a.chunks * a.N * ((a.Ho + th - 1) / th) * a.tiles_w < 2ll * num_sms)
+        th -= B;
+    a.th = th;
+    a.in_rows = rows_in(th);
+    if ((size_t)a.in_rows * row_bytes > budget || a.in_rows > 256) return false;
+    a.tiles_h = (a.Ho + th - 1) / th;
+    a.num_tiles = a.chunks * a.N * a.tiles_h * a.tiles_w;
+    a.buf_bytes = (int)(((size_t)a.in_rows * row_bytes + 127) / 128 * 128);
+    return true;
+}
+
+template <int STRIDE>
+static auto dw_kernel_for(int act) -> decltype(&dwconv3x3_kernel<1, kActNone>) {
+    switch (act) {
+        case kActRelu: return dwconv3x3_kernel<STRIDE, kActRelu>;
+        case kActRelu6: return dwconv3x3_kernel<STRIDE, kActRelu6>;
+        case kActGelu: return dwconv3x3_kernel<STRIDE, kActGelu>;
+        default: return dwconv3x3_kernel<STRIDE, kActNone>;
+    }
+}
+
+static auto dw_kernel(const DwArgs &a) -> decltype(&dwconv3x3_kernel<1, kActNone>) {
+    return a.stride == 1 ? dw_kernel_for<1>(a.act) : dw_kernel_for<2>(a.act);
+}
+
+cudaError_t dw_prepare(const DwArgs &a) {
+    return cudaFuncSetAttribute(dw_kernel(a), cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                (int)dw_smem_bytes(a));
+}
+
+cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cudaStream_t st) {
+    return launch_pdl(dw_kernel(a), dim3(grid), dim3(a.threads), dw_smem_bytes(a), st, tmX, a);
 }
 
 // ------------------------------------------------------------ space-to-depth
-// z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]; one
-// thread per 16-channel group (a) of one output pixel, writing 32 bytes.
+// z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c].
 // Block (p, n): output row p of image n.  Its input rows 2p-pad ..
 // 2p-pad+2*taps-1 are one contiguous run of x; the block stages them in
 // shared memory (zero rows outside the image; 16-byte loads, four in flight
@@ -181,6 +305,8 @@ cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st) {
 // C is a template parameter so that the 16 channel values stay in registers.
 template <int C>
 __global__ void __launch_bounds__(256) s2d_kernel(const S2dArgs a) {
+    pdl_launch_dependents();
+    pdl_wait();
     extern __shared__ __align__(16) unsigned short smem_s2d[];
     const int p = blockIdx.x;
     const int n = blockIdx.y;
@@ -270,18 +396,19 @@ cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
     }
     const dim3 grid((unsigned)a.Hz, (unsigned)a.N);
     switch (a.C) {
-        case 1: s2d_kernel<1><<<grid, 256, smem, st>>>(a); break;
-        case 2: s2d_kernel<2><<<grid, 256, smem, st>>>(a); break;
-        case 3: s2d_kernel<3><<<grid, 256, smem, st>>>(a); break;
-        case 4: s2d_kernel<4><<<grid, 256, smem, st>>>(a); break;
+        case 1: return launch_pdl(s2d_kernel<1>, grid, dim3(256), smem, st, a);
+        case 2: return launch_pdl(s2d_kernel<2>, grid, dim3(256), smem, st, a);
+        case 3: return launch_pdl(s2d_kernel<3>, grid, dim3(256), smem, st, a);
+        case 4: return launch_pdl(s2d_kernel<4>, grid, dim3(256), smem, st, a);
         default: return cudaErrorInvalidValue;
     }
-    return cudaGetLastError();
 }
 
 // ------------------------------------------------------------ max pool
 __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                                int k, int s, int p, int Ho, int Wo) {
+    pdl_launch_dependents();
+    pdl_wait();
     const int CV = C >> 3;
     const long long total = (long long)N * Ho * Wo * CV;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -315,6 +442,8 @@ __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, 
 // 3x3 window, fully unrolled: all nine loads issue before the first max.
 __global__ void maxpool3_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                                 int s, int p, int Ho, int Wo) {
+    pdl_launch_dependents();
+    pdl_wait();
     const int CV = C >> 3;
     const long long total = (long long)N * Ho * Wo * CV;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -354,19 +483,21 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
         const int Ho = (H + 2 * p - 3) / s + 1;
         const int Wo = (W + 2 * p - 3) / s + 1;
         const long long total = (long long)N * Ho * Wo * (C / 8);
-        maxpool3_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C, s, p, Ho, Wo);
-        return cudaGetLastError();
+        return launch_pdl(maxpool3_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y,
+                          N, H, W, C, s, p, Ho, Wo);
     }
     const int Ho = (H + 2 * p - k) / s + 1;
     const int Wo = (W + 2 * p - k) / s + 1;
     const long long total = (long long)N * Ho * Wo * (C / 8);
-    maxpool_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C, k, s, p, Ho, Wo);
-    return cudaGetLastError();
+    return launch_pdl(maxpool_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y, N,
+                      H, W, C, k, s, p, Ho, Wo);
 }
 
 // ------------------------------------------------------------ global average pool
 __global__ void avgpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W,
                                int C) {
+    pdl_launch_dependents();
+    pdl_wait();
     const int CV = C >> 3;
     const long long total = (long long)N * CV;
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
@@ -392,8 +523,8 @@ __global__ void avgpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, 
 cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            cudaStream_t st) {
     const long long total = (long long)N * (C / 8);
-    avgpool_kernel<<<(unsigned)((total + 255) / 256), 256, 0, st>>>(x, y, N, H, W, C);
-    return cudaGetLastError();
+    return launch_pdl(avgpool_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y, N,
+                      H, W, C);
 }
 
 }  // namespace byoc

@@ -150,6 +150,10 @@ __global__ void __maxnreg__(168)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
+    // Set-up done: the next kernel may be scheduled; global memory is touched
+    // only after the previous kernel has completed.
+    pdl_launch_dependents();
+    pdl_wait();
     // Ring stages of G k-blocks each; at least two stages.
     const int G = a.group < 1 ? 1 : (a.group > S::STAGES / 2 ? S::STAGES / 2 : a.group);
     const int nst = S::STAGES / G;
@@ -534,9 +538,8 @@ template <int BN, int BK, int AMODE, bool RES>
 static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap &tmR,
                             const GemmArgs &a, int grid, cudaStream_t st) {
     using S = GemmShape<BN, BK, AMODE, RES>;
-    gemm_tcgen05_kernel<BN, BK, AMODE, RES>
-        <<<grid, kGemmThreads, S::SMEM_BYTES, st>>>(tmA, tmB, tmR, a);
-    return cudaGetLastError();
+    return launch_pdl(gemm_tcgen05_kernel<BN, BK, AMODE, RES>, dim3(grid), dim3(kGemmThreads),
+                      (size_t)S::SMEM_BYTES, st, tmA, tmB, tmR, a);
 }
 
 template <int BN, int BK, int AMODE, bool RES>

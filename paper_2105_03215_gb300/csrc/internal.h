@@ -12,6 +12,29 @@ namespace byoc {
 
 enum Act : int { kActNone = 0, kActRelu = 1, kActRelu6 = 2, kActGelu = 3 };
 
+// Every kernel of the library is launched with programmatic stream
+// serialisation: it may be scheduled while the previous kernel in the stream
+// is still running.  Each kernel signals pdl_launch_dependents() as it starts
+// and calls pdl_wait() -- which returns once the previous grid has completed
+// and its memory operations are visible -- before its first global memory
+// access, so only set-up work (barrier init, TMEM allocation, descriptor
+// prefetch) overlaps the previous kernel's tail.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+
 // Implicit-GEMM problem: out[M, N] = act(A[M, K] . B[N, K]^T + bias [+ residual]).
 //  A is either a row-major [M, K] matrix (dense, 1x1 stride-1 conv) read with a
 //  2-D tiled tensor map, or the implicit im2col matrix of an NHWC activation
@@ -91,16 +114,32 @@ cudaError_t launch_gemm(const GemmConfig &cfg, const CUtensorMap &tmA, const CUt
 
 // Depthwise conv (groups = C), square kernel k in {3}, NHWC bf16, folded
 // weights fp32 [k*k][C] (tap-major), bias fp32 [C], fused activation.
+// Depthwise 3x3 convolution + folded BN/bias + activation, NHWC.  A tile is
+// th output rows x tw output columns x cc channels of one image; its input
+// (in_rows x in_cols x cc, halo included, zero outside the image) is one TMA
+// box.  Persistent CTAs loop over the tiles with two input buffers.
 struct DwArgs {
-    const __nv_bfloat16 *x;
-    const float *w;
-    const float *bias;
-    __nv_bfloat16 *y;
+    const float *w;      // [9][C] folded weights, fp32
+    const float *bias;   // [C]
+    __nv_bfloat16 *y;    // [N, Ho, Wo, C]
     int N, H, W, C, Ho, Wo;
     int stride, pad;
     int act;
+    int th, tw, cc;               // output tile rows, columns; channels per chunk (multiple of 8)
+    int in_rows, in_cols;         // input box: (th-1)*stride+3, (tw-1)*stride+3
+    int tiles_h, tiles_w, chunks;
+    int num_tiles;                // chunks * N * tiles_h * tiles_w (chunk slowest)
+    int buf_bytes;                // one input buffer, 128-byte multiple
+    int threads;                  // (cc / 4) * lanes, <= kDwMaxThreads
+    int *err;                     // device error word
 };
-cudaError_t launch_dwconv(const DwArgs &a, int num_sms, cudaStream_t st);
+constexpr int kDwMaxThreads = 512;
+constexpr int kDwBlockH = 4, kDwBlockW = 2;  // outputs a thread computes (tiles are multiples)
+// Tiling for the depthwise kernel; false when no tile fits shared memory.
+bool dw_plan(DwArgs &a, int num_sms);
+size_t dw_smem_bytes(const DwArgs &a);
+cudaError_t dw_prepare(const DwArgs &a);  // raises the kernel's dynamic smem limit
+cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cudaStream_t st);
 
 // Boundary layout transform for a stride-2 stem with few input channels
 // (space-to-depth with zero padding, vertical filter taps stacked):

@@ -251,6 +251,13 @@ __host__ __device__ constexpr uint32_t make_idesc_bf16(int M, int N) {
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T, issued by one thread.
+// Programmatic dependent launch (see launch_pdl): let the next kernel in the
+// stream be scheduled, and wait for the previous one to complete.
+__device__ __forceinline__ void pdl_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
 // True in exactly one lane of the (fully converged) warp.
 __device__ __forceinline__ bool elect_one() {
     uint32_t pred;

@@ -133,6 +133,19 @@ CUresult encode_slab(CUtensorMap *m, const void *ptr, int N, int H, int W, int C
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// Depthwise input box: in_rows x in_cols pixels x cc channels, no swizzle
+// (the kernel reads it with plain 16-byte shared-memory loads).
+CUresult encode_dw(CUtensorMap *m, const void *ptr, const byoc::DwArgs &a) {
+    cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N};
+    cuuint64_t strides[3] = {(cuuint64_t)a.C * 2, (cuuint64_t)a.W * a.C * 2,
+                             (cuuint64_t)a.H * a.W * a.C * 2};
+    cuuint32_t box[4] = {(cuuint32_t)a.cc, (cuuint32_t)a.in_cols, (cuuint32_t)a.in_rows, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 // ------------------------------------------------------------ bf16 rounding (host)
 
 uint16_t f32_to_bf16_rne(float f) {
@@ -511,6 +524,9 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
             L.dw.stride = op.stride[0];
             L.dw.pad = op.pad[0];
             L.dw.act = act;
+            if (!byoc::dw_plan(L.dw, P.num_sms))
+                return fail(BYOC_ERR_UNSUPPORTED, "op %d: depthwise tile does not fit shared memory", o);
+            L.grid = std::min(L.dw.num_tiles, P.num_sms);
             L.flops = 2.0 * (double)Y.elems() * 9.0;
             L.bytes = (double)X.bytes() + (double)Y.bytes() + (double)(w.size() + b.size()) * 4;
             P.launches.push_back(L);
@@ -951,6 +967,11 @@ byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             L.dw.w = reinterpret_cast<const float *>(h->d_const + L.w_off);
             L.dw.bias = reinterpret_cast<const float *>(h->d_const + L.b_off);
+            L.dw.err = h->d_err;
+            if ((e = byoc::dw_prepare(L.dw)) != cudaSuccess) {
+                byoc_release(h);
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            }
         }
     }
     *out = h;
@@ -1013,10 +1034,17 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a.residual ? h->tmR[i] : h->tmA[i], a,
                                   L.grid, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
+            const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
+            if (h->tmA_ptr[i] != xa) {
+                CUresult r = encode_dw(&h->tmA[i], xa, L.dw);
+                if (r != CUDA_SUCCESS)
+                    return fail(BYOC_ERR_CUDA, "launch %zu: encoding the depthwise TMA map failed (%d)",
+                                i, (int)r);
+                h->tmA_ptr[i] = xa;
+            }
             byoc::DwArgs a = L.dw;
-            a.x = static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]);
-            a.y = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
-            e = byoc::launch_dwconv(a, P.num_sms, st);
+            a.y = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
+            e = byoc::launch_dwconv(h->tmA[i], a, L.grid, st);
         } else {
             byoc::S2dArgs a = L.s2d;
             a.x = reinterpret_cast<const __nv_bfloat16 *>(static_cast<const char *>(h->ptrs[L.x]) +

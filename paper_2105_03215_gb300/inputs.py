@@ -336,6 +336,14 @@ MOBILENET_V2_BLOCKS = ((1, 16, 1, 1), (6, 24, 2, 2), (6, 32, 3, 2), (6, 64, 4, 2
                        (6, 160, 3, 2), (6, 320, 1, 1))
 
 
+def depthwise(N=2, H=20, W=17, C=144, stride=1, seed=3):
+    """Depthwise 3x3 conv (pad 1) + BN + ReLU6 alone."""
+    b = _Builder(f"depthwise{C}s{stride}")
+    x = b.input("x", (N, H, W, C))
+    y = b.relu6(b.batch_norm(b.conv2d(x, C, 3, stride=stride, groups=C)))
+    return _finish(b, [y], seed)
+
+
 def mobilenet_v2(N=1, H=224, W=224, num_classes=1000, seed=7, draw=False):
     """MobileNetV2 1.0: inverted residual blocks (expand 1x1, depthwise 3x3,
     project 1x1, residual add when shapes allow), ReLU6 activations."""

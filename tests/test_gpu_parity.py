@@ -97,6 +97,20 @@ def test_mbv2_dw_pw_full():
     _check_graph(g, inp)
 
 
+@pytest.mark.parametrize("N,H,W,C,stride", [
+    (2, 9, 7, 960, 1),     # channels in 4 chunks of 240
+    (1, 11, 13, 264, 2),   # 2 chunks of 136, the last one ragged
+    (1, 5, 300, 16, 1),    # output wider than one box: column tiles
+    (1, 6, 190, 24, 2),    # stride 2, column tiles
+    (3, 1, 1, 8, 1),       # 1 x 1 image, 8 channels
+    (2, 2, 3, 32, 2),      # output 1 x 2
+    (1, 57, 56, 144, 1),   # ragged last row tile
+])
+def test_depthwise_tiles(N, H, W, C, stride):
+    g, inp = I.depthwise(N=N, H=H, W=W, C=C, stride=stride, seed=N * 7 + C)
+    _check_graph(g, inp, what=f"depthwise {N}x{H}x{W}x{C} s{stride}")
+
+
 def test_depthwise_stride2():
     g, inp = I.mbv2_dw_pw(N=2, H=21, W=20, C=96, Cout=32, seed=9, stride=2)
     _check_graph(g, inp)
