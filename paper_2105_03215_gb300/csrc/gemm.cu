@@ -151,8 +151,22 @@ __global__ void __maxnreg__(168)
     tc_fence_after();
     const uint32_t tmem_base = *tmem_slot;
     // Set-up done: the next kernel may be scheduled; global memory is touched
-    // only after the previous kernel has completed.
+    // only after the previous kernel has completed -- except for the packed
+    // weights, constant for the handle's lifetime: the operand warp
+    // prefetches this CTA's first tile's weight rows into L2 while the
+    // previous kernel finishes.
     pdl_launch_dependents();
+    if (warp == kGemmOperandWarp && a.w != nullptr && (int)blockIdx.x < a.num_tiles) {
+        if (elect_one()) {
+            const size_t row_bytes = (size_t)a.k_pack * 2;
+            const uint8_t *src =
+                static_cast<const uint8_t *>(a.w) + (size_t)((int)blockIdx.x % a.tiles_n) * BN * row_bytes;
+            const size_t bytes = (size_t)BN * row_bytes;
+            for (size_t off = 0; off < bytes; off += 32768)
+                bulk_prefetch_l2(src + off, (uint32_t)(bytes - off < 32768 ? bytes - off : 32768));
+        }
+        __syncwarp();
+    }
     pdl_wait();
     // Ring stages of G k-blocks each; at least two stages.
     const int G = a.group < 1 ? 1 : (a.group > S::STAGES / 2 ? S::STAGES / 2 : a.group);

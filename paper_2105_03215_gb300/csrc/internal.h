@@ -62,6 +62,10 @@ struct GemmArgs {
     int taps;           // kh * kw
     int group;      // k-blocks (slab mode: filter taps) per ring stage, >= 1; the
                     // kernel lowers it so that at least two stages fit the ring
+    // packed weights [n_pad][k_pack] (bf16), or null: before waiting for the
+    // previous kernel, a CTA prefetches its first tile's weight rows into L2
+    const void *w;
+    int k_pack;
     int act;        // Act
     const float *bias;                // [tiles_n * BN], zero padded; required
     const __nv_bfloat16 *residual;    // [M, N] or null

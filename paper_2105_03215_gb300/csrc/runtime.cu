@@ -953,6 +953,8 @@ byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
         if (L.kind == BYOC_LAUNCH_GEMM) {
             L.args.bias = reinterpret_cast<const float *>(h->d_const + L.b_off);
             L.args.err = h->d_err;
+            L.args.w = h->d_const + L.w_off;
+            L.args.k_pack = L.k_pack;
             CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
                                    (uint64_t)L.k_pack, (uint32_t)L.cfg.bn, (uint32_t)L.cfg.bk,
                                    L.cfg.bk);

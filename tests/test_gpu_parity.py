@@ -156,6 +156,35 @@ def test_stem_in_image_chunks_with_a_ragged_last_chunk():
     _check_graph(g, inp, what="stem in chunks")
 
 
+def test_gelu_epilogue_within_one_bf16_ulp():
+    # identity weights and zero bias: the region computes GELU(x) of bf16
+    # inputs swept over [-8, 8], so the epilogue's GELU is compared with the
+    # exact one (oracle, erf in fp64) after rounding both to bf16
+    import numpy as np
+    b = I._Builder("gelu_sweep")
+    x = b.input("x", (128, 128))
+    y = b.gelu(b.bias_add(b.dense(x, 128)))
+    g, _ = I._finish(b, [y], seed=3)
+    g.nodes[0].consts["weight"] = np.eye(128, dtype=np.float32)
+    g.nodes[1].consts["bias"] = np.zeros(128, dtype=np.float32)
+    xs = I.bf16_round(np.linspace(-8.0, 8.0, 128 * 128, dtype=np.float32).reshape(128, 128))
+    inp = {"x": xs}
+    reg = R.whole_graph_region(g)
+    got, cr = run_region(reg, inp)
+    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    gv = got[g.outputs[0]].astype(np.float64)
+    got_b = I.bf16_bits(gv.astype(np.float32)).astype(np.int32)
+    ref_b = I.bf16_bits(ref.astype(np.float32)).astype(np.int32)
+    # where |GELU| >= 1e-3 the bf16 results agree to one ulp (bf16 patterns are
+    # ordered like their values within one sign); below that, 1 + erf(z)
+    # cancels in fp32 for large negative inputs, so compare absolutely
+    big = np.abs(ref) >= 1e-3
+    assert ((got_b < 0x8000) == (ref_b < 0x8000))[big].all()
+    assert np.abs(got_b - ref_b)[big].max() <= 1
+    assert np.abs(gv - ref)[~big].max() <= 1e-5
+    cr.release()
+
+
 def test_region_can_run_twice_with_new_pointers():
     import torch
     from .parity import to_dev
