@@ -20,6 +20,8 @@ def main():
     ap.add_argument("--workload", default="resnet50",
                     choices=["resnet50", "conv3x3", "bert_ffn", "mbv2_dw_pw", "mbv2_dw", "bottleneck"])
     ap.add_argument("--batch", type=int, default=64)
+    ap.add_argument("--n", type=int, default=None,
+                    help="batch of the other workloads (default: the workload's own)")
     ap.add_argument("--region", type=int, default=0)
     ap.add_argument("--reps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=2)
@@ -60,11 +62,12 @@ def main():
                                 moving_mean=np.zeros(C, "float32"), moving_var=np.ones(C, "float32"))
         reg = R.Region(g, names, f"resnet50_region{args.region}")
     else:
-        g, _ = {"conv3x3": lambda: I.conv_bias_relu(seed=0),
+        nk = {} if args.n is None else {"N": args.n}
+        g, _ = {"conv3x3": lambda: I.conv_bias_relu(seed=0, **nk),
                 "bert_ffn": lambda: I.bert_ffn(seed=1),
-                "mbv2_dw_pw": lambda: I.mbv2_dw_pw(seed=2),
-                "mbv2_dw": lambda: I.mbv2_dw_pw(seed=2),
-                "bottleneck": lambda: I.resnet_bottleneck(seed=3)}[args.workload]()
+                "mbv2_dw_pw": lambda: I.mbv2_dw_pw(seed=2, **nk),
+                "mbv2_dw": lambda: I.mbv2_dw_pw(seed=2, **nk),
+                "bottleneck": lambda: I.resnet_bottleneck(seed=3, **nk)}[args.workload]()
         if args.workload == "mbv2_dw":
             reg = R.Region(g, [n.name for n in g.nodes[:3]], "mbv2_dw")
         else:
