@@ -54,17 +54,20 @@ struct GemmShape {
     // residual tile: BN/64 boxes of 64 columns x 128 rows, 128-byte swizzle
     static constexpr int RES_BOX = BM * 64 * 2;
     static constexpr int RES_TILE = RES ? BM * BN * 2 : 0;
+    // epilogue-operand buffers (bias slice, residual tile): residual regions
+    // are HBM-bound and keep more residual tiles in flight
+    static constexpr int OPB = RES ? (BN >= 128 ? 3 : 4) : 2;
     static constexpr int BIAS_BYTES = BN * 4;
-    static constexpr int BIAS_REGION = (2 * BIAS_BYTES + 1023) / 1024 * 1024;
+    static constexpr int BIAS_REGION = (OPB * BIAS_BYTES + 1023) / 1024 * 1024;
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
     static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE;
     static constexpr int CTRL_BYTES = 1024;
     static constexpr int FIXED =
-        1024 + 2 * SLAB_BYTES + 2 * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
+        1024 + 2 * SLAB_BYTES + OPB * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 32 ? 32 : STAGES_RAW;  // ring slots (k-blocks)
-    static constexpr int NUM_BARS = 2 * STAGES + 13;
+    static constexpr int NUM_BARS = 2 * STAGES + 9 + 2 * OPB;
     static constexpr int SMEM_BYTES = FIXED + STAGES * STAGE_BYTES;
     static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
     static_assert(STAGES >= 2, "ring depth");
@@ -102,16 +105,16 @@ __global__ void __maxnreg__(168)
     const uint32_t sA = base;
     const uint32_t sB = sA + S::STAGES * S::A_BYTES;
     const uint32_t sSlab = sB + S::STAGES * S::B_BYTES;    // 2 x SLAB_BYTES
-    const uint32_t sRes = sSlab + 2 * S::SLAB_BYTES;       // 2 x RES_TILE
-    const uint32_t sEpi = sRes + 2 * S::RES_TILE;          // EPI_BYTES
+    const uint32_t sRes = sSlab + 2 * S::SLAB_BYTES;       // OPB x RES_TILE
+    const uint32_t sEpi = sRes + S::OPB * S::RES_TILE;     // EPI_BYTES
     const uint32_t sBias = sEpi + S::EPI_BYTES;            // 2 x BIAS_BYTES
     const uint32_t ctrl = sBias + S::BIAS_REGION;
     const uint32_t bars = ctrl;                            // full[S], empty[S]
     const uint32_t tfull = bars + 8u * (2 * S::STAGES);    // 2: accumulator ready
     const uint32_t tempty = tfull + 16u;                   // 2: accumulator drained
-    const uint32_t ofull = tempty + 16u;                   // 2: epilogue operands loaded
-    const uint32_t oempty = ofull + 16u;                   // 2: epilogue operands consumed
-    const uint32_t sfull = oempty + 16u;                   // 2: slab loaded
+    const uint32_t ofull = tempty + 16u;                   // OPB: epilogue operands loaded
+    const uint32_t oempty = ofull + 8u * S::OPB;           // OPB: epilogue operands consumed
+    const uint32_t sfull = oempty + 8u * S::OPB;           // 2: slab loaded
     const uint32_t sempty = sfull + 16u;                   // 2: slab consumed
     const uint32_t drain = sempty + 16u;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
@@ -128,10 +131,12 @@ __global__ void __maxnreg__(168)
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull + 8u * b, 1);                 // MMA commit
             mbar_init(tempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
-            mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
-            mbar_init(oempty + 8u * b, kEpiArrivals);
             mbar_init(sfull + 8u * b, 1);                 // producer + slab bytes
             mbar_init(sempty + 8u * b, 1);                // MMA commit
+        }
+        for (int b = 0; b < S::OPB; ++b) {
+            mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
+            mbar_init(oempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -283,8 +288,8 @@ __global__ void __maxnreg__(168)
             // ------------------------------------------------ epilogue-operand producer
             int t = 0;
             for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
-                const int ob = t & 1;
-                const uint32_t oph = (uint32_t)(t >> 1) & 1u;
+                const int ob = t % S::OPB;
+                const uint32_t oph = (uint32_t)(t / S::OPB) & 1u;
                 if (!mbar_wait(oempty + 8u * ob, oph ^ 1u, abort_flag, a.err, kErrTimeoutProducer))
                     break;
                 const int m0 = (tile / a.tiles_n) * S::BM;
@@ -299,8 +304,8 @@ __global__ void __maxnreg__(168)
                 }
             }
             // Let the last operand loads land before the CTA can exit.
-            if (t > 0) mbar_wait_drain(ofull + 8u * ((t - 1) & 1), (uint32_t)((t - 1) >> 1) & 1u);
-            if (t > 1) mbar_wait_drain(ofull + 8u * ((t - 2) & 1), (uint32_t)((t - 2) >> 1) & 1u);
+            for (int j = t - S::OPB > 0 ? t - S::OPB : 0; j < t; ++j)
+                mbar_wait_drain(ofull + 8u * (j % S::OPB), (uint32_t)(j / S::OPB) & 1u);
         }
     } else if (warp == 1) {
         // ---------------------------------------------------- MMA issuer
@@ -434,7 +439,10 @@ __global__ void __maxnreg__(168)
             const int buf = t & 1;
             const uint32_t aph = (uint32_t)(t >> 1) & 1u;
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
-            if (!mbar_wait(ofull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
+            const int ob = t % S::OPB;  // epilogue-operand buffer
+            if (!mbar_wait(ofull + 8u * ob, (uint32_t)(t / S::OPB) & 1u, abort_flag, a.err,
+                           kErrTimeoutEpilogue))
+                break;
             tc_fence_after();
             const int mt = tile / a.tiles_n;
             const int n0 = (tile % a.tiles_n) * BN;
@@ -457,8 +465,8 @@ __global__ void __maxnreg__(168)
             }
             const uint32_t tbase =
                 tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
-            const uint32_t bias_s = sBias + (uint32_t)(buf * S::BIAS_BYTES);
-            const uint32_t res_s = sRes + (uint32_t)(buf * S::RES_TILE);
+            const uint32_t bias_s = sBias + (uint32_t)(ob * S::BIAS_BYTES);
+            const uint32_t res_s = sRes + (uint32_t)(ob * S::RES_TILE);
 #pragma unroll 1
             for (int ci = c_first; ci < NCH; ci += c_step) {
                 const int col0 = n0 + ci * 32;
@@ -533,7 +541,7 @@ __global__ void __maxnreg__(168)
             }
             // bias / residual reads of this tile are done (ordered by __syncwarp)
             __syncwarp();
-            if (lane == 0) mbar_arrive(oempty + 8u * buf);
+            if (lane == 0) mbar_arrive(oempty + 8u * ob);
         }
     }
 
