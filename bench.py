@@ -238,6 +238,31 @@ def region_figures(flush, peaks):
                 "hbm_frac_of_measured": dcr.bytes / td / 1e9 / peaks["hbm_gbs"]}
             dcr.release()
         cr.release()
+    # MobileNetV2 1.0 end to end (53 regions, global average pool on the host):
+    # the other image-classification model whose regions the path covers
+    from paper_2105_03215_gb300 import executor as E
+    mres, minp = E.build_mobilenet_v2(N=BATCH, H=IMG, W=IMG)
+    mex = E.Executor(mres)
+    mex.set_input("data", torch.from_numpy(minp["data"]).to(torch.bfloat16).cuda())
+    mex.capture()
+    for _ in range(3):
+        mex.replay()
+    torch.cuda.synchronize()
+    st = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(20)]
+    for a, b in evs:
+        flush.zero_()
+        a.record(st)
+        mex.replay()
+        b.record(st)
+    torch.cuda.synchronize()
+    mex.check()
+    tm = statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3
+    mflops = sum(c.flops for c in mex.compiled)
+    out[f"mobilenet_v2_N{BATCH}_224"] = {"images_per_s": BATCH / tm, "ms_per_step": tm * 1e3,
+                                         "tflops": mflops / tm / 1e12, "regions": len(mex.regions),
+                                         "launches": mex.n_launches}
+    mex.release()
     return out
 
 

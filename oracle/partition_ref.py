@@ -22,6 +22,8 @@ from typing import Dict, List, Optional, Sequence, Set, Tuple
 REF_PATTERNS: List[Tuple[str, List[List[str]]]] = [
     ("conv2d_bn_add_relu", [["nn.relu", "add", "nn.batch_norm", "nn.bias_add", "nn.conv2d"],
                             ["nn.relu", "add", "nn.batch_norm", "nn.conv2d"]]),
+    ("conv2d_bn_add", [["add", "nn.batch_norm", "nn.bias_add", "nn.conv2d"],
+                       ["add", "nn.batch_norm", "nn.conv2d"]]),
     ("conv2d_bn_act", [["nn.relu", "nn.batch_norm", "nn.bias_add", "nn.conv2d"],
                        ["nn.relu", "nn.batch_norm", "nn.conv2d"],
                        ["clip", "nn.batch_norm", "nn.bias_add", "nn.conv2d"],

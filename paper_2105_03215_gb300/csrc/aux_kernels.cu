@@ -248,12 +248,16 @@ bool dw_plan(DwArgs &a, int num_sms) {
     // (rounded up to the block) when its input columns fit one box (<= 256).
     constexpr int B = kDwBlockH, BW = kDwBlockW;
     const int tw_max = ((256 - 3) / a.stride + 1) / BW * BW;
+    const size_t budget = kDwBufBudget;
+    auto rows_in = [&](int th) { return (th - 1) * a.stride + 3; };
+    // Narrower column tiles where even the shortest row tile of the full
+    // width would overflow one buffer (wide rows of many channels).
     a.tw = std::min((a.Wo + BW - 1) / BW * BW, tw_max);
+    while (a.tw > BW && (size_t)rows_in(B) * ((a.tw - 1) * a.stride + 3) * a.cc * 2 > budget)
+        a.tw -= BW;
     a.tiles_w = (a.Wo + a.tw - 1) / a.tw;
     a.in_cols = (a.tw - 1) * a.stride + 3;
     const size_t row_bytes = (size_t)a.in_cols * a.cc * 2;
-    const size_t budget = 108 * 1024;  // per buffer; two buffers per CTA
-    auto rows_in = [&](int th) { return (th - 1) * a.stride + 3; };
     const int ho_blocks = (a.Ho + B - 1) / B * B;
     int th = B;
     while (th + B <= ho_blocks && (size_t)rows_in(th + B) * row_bytes <= budget && rows_in(th + B) <= 256)
@@ -285,8 +289,10 @@ static auto dw_kernel(const DwArgs &a) -> decltype(&dwconv3x3_kernel<1, kActNone
 }
 
 cudaError_t dw_prepare(const DwArgs &a) {
+    DwArgs largest = a;
+    largest.buf_bytes = (int)kDwBufBudget;
     return cudaFuncSetAttribute(dw_kernel(a), cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                (int)dw_smem_bytes(a));
+                                (int)dw_smem_bytes(largest));
 }
 
 cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cudaStream_t st) {

@@ -578,6 +578,12 @@ static cudaError_t prepare_t() {
     X(128, 64, kAModeTile, false)     \
     X(256, 64, kAModeTile, false)     \
     X(64, 64, kAModeTile, true)       \
+    X(32, 16, kAModeTile, false)      \
+    X(64, 16, kAModeTile, false)      \
+    X(128, 16, kAModeTile, false)     \
+    X(32, 32, kAModeTile, false)      \
+    X(64, 32, kAModeTile, false)      \
+    X(128, 32, kAModeTile, false)     \
     X(128, 64, kAModeTile, true)      \
     X(32, 64, kAModeIm2col, false)    \
     X(64, 64, kAModeIm2col, false)    \

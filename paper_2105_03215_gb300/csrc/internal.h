@@ -139,10 +139,14 @@ struct DwArgs {
 };
 constexpr int kDwMaxThreads = 512;
 constexpr int kDwBlockH = 4, kDwBlockW = 2;  // outputs a thread computes (tiles are multiples)
+constexpr size_t kDwBufBudget = 108 * 1024;   // bytes per input buffer; two buffers per CTA
 // Tiling for the depthwise kernel; false when no tile fits shared memory.
 bool dw_plan(DwArgs &a, int num_sms);
 size_t dw_smem_bytes(const DwArgs &a);
-cudaError_t dw_prepare(const DwArgs &a);  // raises the kernel's dynamic smem limit
+// Raises the kernel's dynamic smem limit to the largest size dw_plan can
+// choose: the limit belongs to the kernel, not the launch, so several regions
+// sharing one instantiation must all fit under it.
+cudaError_t dw_prepare(const DwArgs &a);
 cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cudaStream_t st);
 
 // Boundary layout transform for a stride-2 stem with few input channels

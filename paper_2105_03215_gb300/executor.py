@@ -192,3 +192,15 @@ def build_resnet50(N: int = 64, H: int = 224, W: int = 224, seed: int = 4, max_o
         inp = None
     res = P.partition(graph, P.PATTERN_TABLE, target=P.TARGET, max_ops=max_ops)
     return res, inp
+
+
+def build_mobilenet_v2(N: int = 64, H: int = 224, W: int = 224, seed: int = 7,
+                       max_ops: Optional[int] = 1):
+    """MobileNetV2 1.0 partitioned for this library (global average pool on the
+    host); with ``max_ops=1`` every conv2d / dense composite is its own region
+    (52 conv composites, depthwise included, + the classifier)."""
+    from . import inputs as I
+    from . import partition as P
+    graph, inp = I.mobilenet_v2(N=N, H=H, W=W, seed=seed, draw=True)
+    res = P.partition(graph, P.PATTERN_TABLE, target=P.TARGET, max_ops=max_ops)
+    return res, inp

@@ -412,6 +412,12 @@ def conv2d_bn_add_relu_pattern():
     return is_op("nn.relu")(is_op("add")(_conv_bn(), wildcard()))
 
 
+def conv2d_bn_add_pattern():
+    """A linear projection conv + BN whose output is added to a residual
+    (MobileNetV2's inverted-residual blocks)."""
+    return is_op("add")(_conv_bn(), wildcard())
+
+
 def conv2d_bn_act_pattern():
     return Alt(is_op("nn.relu")(_conv_bn()), is_op("clip")(_conv_bn()))
 
@@ -433,6 +439,7 @@ def dense_bias_act_pattern():
 
 PATTERN_TABLE = [
     ("conv2d_bn_add_relu", conv2d_bn_add_relu_pattern),
+    ("conv2d_bn_add", conv2d_bn_add_pattern),
     ("conv2d_bn_act", conv2d_bn_act_pattern),
     ("conv2d_bn", conv2d_bn_pattern),
     ("conv2d_bias_act", conv2d_bias_act_pattern),

@@ -171,3 +171,18 @@ def test_unsupported_chains_are_rejected_not_run_elsewhere():
     with pytest.raises(abi.ByocError) as e:
         R.whole_graph_region(g).plan()
     assert e.value.status == abi.ERR_UNSUPPORTED
+
+
+def test_every_mobilenet_v2_region_plans_at_224():
+    # The stride-2 depthwise over 112 x 112 x 96 needs 9 input rows x 113
+    # columns x 96 channels = 195 KB for a full-width tile of 4 output rows:
+    # the planner narrows the column tile until one buffer holds it.
+    from paper_2105_03215_gb300 import partition as P
+    g, _ = I.mobilenet_v2(N=64, H=224, W=224, draw=True)
+    res = P.partition(g, P.PATTERN_TABLE, target=P.TARGET, max_ops=1)
+    regions = res.region_objects()
+    assert len(regions) == 53
+    for r in regions:
+        rep = r.plan()
+        assert rep.n_launches >= 1
+    assert sum(r.plan().flops for r in regions) == pytest.approx(I.region_flops(g), rel=1e-9)

@@ -105,6 +105,7 @@ def test_mbv2_dw_pw_full():
     (3, 1, 1, 8, 1),       # 1 x 1 image, 8 channels
     (2, 2, 3, 32, 2),      # output 1 x 2
     (1, 57, 56, 144, 1),   # ragged last row tile
+    (1, 112, 112, 96, 2),  # full-width tile overflows a buffer: narrowed column tiles
 ])
 def test_depthwise_tiles(N, H, W, C, stride):
     g, inp = I.depthwise(N=N, H=H, W=W, C=C, stride=stride, seed=N * 7 + C)
@@ -200,3 +201,24 @@ def test_region_can_run_twice_with_new_pointers():
         cr.check()
         assert_close(y.float().cpu().numpy(), ref, "rerun")
     cr.release()
+
+
+def test_depthwise_regions_sharing_a_kernel_run_in_any_compile_order():
+    # The dynamic shared-memory limit belongs to the kernel, not the launch:
+    # compiling a region with a small tile after one with a large tile must
+    # not shrink the limit the first one launches under.
+    import torch
+    from .parity import to_dev
+    big_g, big_inp = I.depthwise(N=1, H=57, W=56, C=144, stride=1, seed=4)
+    small_g, small_inp = I.depthwise(N=3, H=1, W=1, C=8, stride=1, seed=5)
+    big = R.whole_graph_region(big_g).compile()
+    small = R.whole_graph_region(small_g).compile()
+    for g, inp, cr in [(big_g, big_inp, big), (small_g, small_inp, small)]:
+        x = to_dev(inp["x"])
+        y = torch.full(g.shape_of(g.outputs[0]), float("nan"), dtype=torch.bfloat16, device="cuda")
+        cr.run([x], [y])
+        torch.cuda.synchronize()
+        cr.check()
+        assert_close(y.float().cpu().numpy(), ograph.evaluate(g, inp)[g.outputs[0]], g.name)
+    big.release()
+    small.release()

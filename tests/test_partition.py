@@ -68,6 +68,21 @@ def test_composites_match_reference_on_resnet50():
     assert names.count("dense_bias_act") == 1
 
 
+def test_mobilenet_v2_composites_and_regions_match_reference():
+    # every inverted-residual block with a shortcut ends in conv + BN + add
+    g, _ = I.mobilenet_v2(draw=False)
+    mine = [(c.name, c.members) for c in P.merge_composite(g, P.PATTERN_TABLE)]
+    assert mine == ref.composites(g)
+    names = [c[0] for c in mine]
+    assert names.count("conv2d_bn_add") == 10
+    res = P.partition(g, P.PATTERN_TABLE, target=P.TARGET, max_ops=1)
+    regs = _regions(res)
+    assert regs == ref.partition(g, set(P.annotations(P.TARGET)), max_ops=1)
+    assert len(regs) == 53  # 52 conv composites + the classifier; global avg pool on the host
+    on_host = [n.op for n in g.nodes if not any(n.name in r for r in regs)]
+    assert on_host == ["nn.global_avg_pool2d"]
+
+
 # ------------------------------------------------------------ Table 2 pins
 
 @pytest.mark.parametrize("builder", [I.resnet18, I.resnet50, I.mobilenet_v2, I.vgg19])
