@@ -51,34 +51,6 @@ __device__ __forceinline__ uint4 ldg_v4(const void *p) {
 // activation is applied to the packed bf16 pairs (exact: rounding is
 // monotonic and 0 and 6 are bf16 values).  The next tile's box loads (TMA)
 // while this one is computed.
-__device__ __forceinline__ void fma2(uint64_t &acc, uint64_t x, uint64_t w) {
-    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(x), "l"(w));
-}
-// Register-pair moves (mov.b64 {lo, hi}) so that packing and unpacking the
-// two lanes costs no arithmetic.
-__device__ __forceinline__ uint64_t pair(uint32_t lo, uint32_t hi) {
-    uint64_t r;
-    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
-    return r;
-}
-__device__ __forceinline__ uint64_t f32x2_of_bf16x2(uint32_t u) {
-    // low half -> lane 0, high half -> lane 1 (a bf16 is the top half of its fp32)
-    return pair(u << 16, u & 0xFFFF0000u);
-}
-__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
-    return pair(__float_as_uint(lo), __float_as_uint(hi));
-}
-__device__ __forceinline__ float lane0(uint64_t v) {
-    uint32_t lo, hi;
-    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
-    return __uint_as_float(lo);
-}
-__device__ __forceinline__ float lane1(uint64_t v) {
-    uint32_t lo, hi;
-    asm("mov.b64 {%0, %1}, %2;" : "=r"(lo), "=r"(hi) : "l"(v));
-    return __uint_as_float(hi);
-}
-
 // act(x) for a pair of outputs, rounded to a bf16 pair; ReLU and ReLU6 are
 // applied after rounding, on the packed pair.
 template <int ACT>
@@ -89,8 +61,8 @@ __device__ __forceinline__ uint32_t dw_act2(float lo, float hi) {
         if constexpr (ACT == kActRelu6) asm("min.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0x40C040C0u));
         return r;
     } else if constexpr (ACT == kActGelu) {
-        return pack_bf16x2(0.5f * lo * (1.0f + erff(lo * 0.70710678118654752f)),
-                           0.5f * hi * (1.0f + erff(hi * 0.70710678118654752f)));
+        const uint64_t g = gelu2(f32x2(lo, hi));
+        return pack_bf16x2(lane0(g), lane1(g));
     } else {
         return pack_bf16x2(lo, hi);
     }

@@ -80,11 +80,11 @@ struct GemmShape {
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
 };
 
+// ReLU, ReLU6 or none; GELU is applied to lane pairs (gelu2) by the caller.
 __device__ __forceinline__ float apply_act(float v, int act) {
     switch (act) {
         case kActRelu: return fmaxf(v, 0.0f);
         case kActRelu6: return fminf(fmaxf(v, 0.0f), 6.0f);
-        case kActGelu: return 0.5f * v * (1.0f + erff(v * 0.70710678118654752f));
         default: return v;
     }
 }
@@ -508,8 +508,17 @@ __global__ void __maxnreg__(168)
                         }
                     }
                 }
+                if (a.act == kActGelu) {
 #pragma unroll
-                for (int j = 0; j < 32; ++j) f[j] = apply_act(f[j], a.act);
+                    for (int j = 0; j < 16; ++j) {
+                        const uint64_t g = gelu2(f32x2(f[2 * j], f[2 * j + 1]));
+                        f[2 * j] = lane0(g);
+                        f[2 * j + 1] = lane1(g);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) f[j] = apply_act(f[j], a.act);
+                }
                 // this thread's row -> swizzled staging -> coalesced global stores
                 __syncwarp();
 #pragma unroll

@@ -345,4 +345,102 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 __device__ __forceinline__ float bf16lo(uint32_t u) { return __uint_as_float(u << 16); }
 __device__ __forceinline__ float bf16hi(uint32_t u) { return __uint_as_float(u & 0xFFFF0000u); }
 
+// ---------------------------------------------------------------- packed fp32 pairs
+// Two fp32 lanes in one 64-bit register pair, for the two-lane fp32
+// instructions (fma / mul / add .f32x2).  Packing and unpacking are register
+// pair moves (mov.b64 {lo, hi}) and cost no arithmetic.
+
+__device__ __forceinline__ uint64_t pair(uint32_t lo, uint32_t hi) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
+    return r;
+}
+__device__ __forceinline__ uint64_t f32x2(float lo, float hi) {
+    return pair(__float_as_uint(lo), __float_as_uint(hi));
+}
+__device__ __forceinline__ uint64_t f32x2_of_bf16x2(uint32_t u) {
+    // low half -> lane 0, high half -> lane 1 (a bf16 is the top half of its fp32)
+    return pair(u << 16, u & 0xFFFF0000u);
+}
+__device__ __forceinline__ void lanes(uint64_t v, float &lo, float &hi) {
+    uint32_t l, h;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(l), "=r"(h) : "l"(v));
+    lo = __uint_as_float(l);
+    hi = __uint_as_float(h);
+}
+__device__ __forceinline__ float lane0(uint64_t v) {
+    float lo, hi;
+    lanes(v, lo, hi);
+    return lo;
+}
+__device__ __forceinline__ float lane1(uint64_t v) {
+    float lo, hi;
+    lanes(v, lo, hi);
+    return hi;
+}
+__device__ __forceinline__ void fma2(uint64_t &acc, uint64_t x, uint64_t w) {
+    asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(acc) : "l"(x), "l"(w));
+}
+__device__ __forceinline__ uint64_t fma2r(uint64_t x, uint64_t w, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(x), "l"(w), "l"(c));
+    return r;
+}
+__device__ __forceinline__ uint64_t mul2(uint64_t x, uint64_t y) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(x), "l"(y));
+    return r;
+}
+__device__ __forceinline__ uint64_t add2(uint64_t x, uint64_t y) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(x), "l"(y));
+    return r;
+}
+__device__ __forceinline__ float rcp_approx(float x) {
+    float r;
+    asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
+// GELU(x) = x * Phi(x), Phi(x) = (1 + erf(x / sqrt 2)) / 2, for a pair of
+// lanes.  erf comes from Abramowitz & Stegun, Handbook of Mathematical
+// Functions, formula 7.1.28: for z >= 0
+//     erf(z) = 1 - (1 + a1 z + a2 z^2 + ... + a6 z^6)^-16,  |error| <= 3e-7.
+// In that form the lower tail is a product, not a difference:
+//     Phi(-|x|) = (1/2) p(|x| / sqrt 2)^-16,
+// so GELU(x) = x * Phi(-|x|) for x < 0 and x - x * Phi(-|x|) for x >= 0,
+// with no cancellation for large negative x.  The factor 1/2 is folded into
+// the polynomial as 2^(1/16) * p.  Cost per pair: 7 fma + 6 mul (two-lane)
+// and 2 reciprocals.
+namespace gelu_as {
+constexpr double kScale = 1.0442737824274138;  // 2^(1/16)
+constexpr float c0 = (float)(kScale * 1.0);
+constexpr float c1 = (float)(kScale * 0.0705230784);
+constexpr float c2 = (float)(kScale * 0.0422820123);
+constexpr float c3 = (float)(kScale * 0.0092705272);
+constexpr float c4 = (float)(kScale * 0.0001520143);
+constexpr float c5 = (float)(kScale * 0.0002765672);
+constexpr float c6 = (float)(kScale * 0.0000430638);
+}  // namespace gelu_as
+
+__device__ __forceinline__ uint64_t gelu2(uint64_t x) {
+    using namespace gelu_as;
+    const float x0 = lane0(x), x1 = lane1(x);
+    const uint64_t z = mul2(f32x2(fabsf(x0), fabsf(x1)), f32x2(0.70710678118654752f, 0.70710678118654752f));
+    uint64_t p = fma2r(z, f32x2(c6, c6), f32x2(c5, c5));
+    p = fma2r(p, z, f32x2(c4, c4));
+    p = fma2r(p, z, f32x2(c3, c3));
+    p = fma2r(p, z, f32x2(c2, c2));
+    p = fma2r(p, z, f32x2(c1, c1));
+    p = fma2r(p, z, f32x2(c0, c0));
+    uint64_t r = f32x2(rcp_approx(lane0(p)), rcp_approx(lane1(p)));
+    r = mul2(r, r);   // ^2
+    r = mul2(r, r);   // ^4
+    r = mul2(r, r);   // ^8
+    r = mul2(r, r);   // ^16: Phi(-|x|)
+    const uint64_t t = mul2(x, r);  // x * Phi(-|x|)
+    const uint64_t u = fma2r(t, f32x2(-1.0f, -1.0f), x);  // x - t
+    return f32x2(x0 < 0.0f ? lane0(t) : lane0(u), x1 < 0.0f ? lane1(t) : lane1(u));
+}
+
 }  // namespace byoc
