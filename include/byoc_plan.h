@@ -40,6 +40,8 @@ typedef struct {
     int32_t tile_k[BYOC_PLAN_MAX_LAUNCHES];     /* BK */
     int32_t im2col[BYOC_PLAN_MAX_LAUNCHES];     /* 1 if A is read through an im2col map */
     int32_t grid[BYOC_PLAN_MAX_LAUNCHES];       /* CTAs launched */
+    int32_t resident_b[BYOC_PLAN_MAX_LAUNCHES]; /* 1: the weights are loaded once per CTA (slab mode) */
+    int32_t slab_slots[BYOC_PLAN_MAX_LAUNCHES]; /* slab buffers in flight (slab mode), else 0 */
     double flops;
     double bytes;
     size_t const_bytes;

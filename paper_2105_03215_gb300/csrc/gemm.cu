@@ -45,11 +45,17 @@ namespace byoc {
 template <int BN, int BK, int AMODE, bool RES>
 struct GemmShape {
     static constexpr int BM = kGemmBM;
+    static constexpr bool SLAB = AMODE == kAModeSlab || AMODE == kAModeSlabRes;
+    static constexpr bool WRES = AMODE == kAModeSlabRes;  // weights resident
     static constexpr int ROW_BYTES = BK * 2;  // one K-major operand row (= swizzle width)
-    static constexpr int A_BYTES = AMODE == kAModeSlab ? 0 : BM * BK * 2;
+    static constexpr int A_BYTES = SLAB ? 0 : BM * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int SLAB_BYTES = AMODE == kAModeSlab ? slab_max_bytes(BK) : 0;
+    static constexpr int SLAB_BYTES = SLAB ? slab_max_bytes(BK) : 0;
+    // slab barriers: two slots beside a weight ring; up to kMaxSlabSlots
+    // beside resident weights (the ring and the two largest slabs form one
+    // pool, split at run time)
+    static constexpr int SLOTS_MAX = WRES ? kMaxSlabSlots : 2;
     static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
     // residual tile: BN/64 boxes of 64 columns x 128 rows, 128-byte swizzle
     static constexpr int RES_BOX = BM * 64 * 2;
@@ -67,7 +73,8 @@ struct GemmShape {
         1024 + 2 * SLAB_BYTES + OPB * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 32 ? 32 : STAGES_RAW;  // ring slots (k-blocks)
-    static constexpr int NUM_BARS = 2 * STAGES + 9 + 2 * OPB;
+    static constexpr int POOL_BYTES = STAGES * STAGE_BYTES + 2 * SLAB_BYTES;
+    static constexpr int NUM_BARS = 2 * STAGES + 5 + 2 * SLOTS_MAX + 2 * OPB;
     static constexpr int SMEM_BYTES = FIXED + STAGES * STAGE_BYTES;
     static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
     static_assert(STAGES >= 2, "ring depth");
@@ -76,7 +83,7 @@ struct GemmShape {
                   "buffers must keep 1 KB alignment");
     static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "BN");
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
-    static_assert(!(RES && AMODE == kAModeSlab), "slab tiles skip pad columns; no residual tile");
+    static_assert(!(RES && SLAB), "slab tiles skip pad columns; no residual tile");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
 };
 
@@ -104,8 +111,10 @@ __global__ void __maxnreg__(168)
     uint8_t *smem = smem_raw + (base - raw);
     const uint32_t sA = base;
     const uint32_t sB = sA + S::STAGES * S::A_BYTES;
-    const uint32_t sSlab = sB + S::STAGES * S::B_BYTES;    // 2 x SLAB_BYTES
-    const uint32_t sRes = sSlab + 2 * S::SLAB_BYTES;       // OPB x RES_TILE
+    const uint32_t sPoolEnd = sB + S::STAGES * S::B_BYTES + 2 * S::SLAB_BYTES;
+    // slabs: 2 x SLAB_BYTES after the ring, or (resident weights) slab_slots x slab_pitch
+    const uint32_t sSlab = S::WRES ? sB + (uint32_t)a.slab_off : sB + S::STAGES * S::B_BYTES;
+    const uint32_t sRes = sPoolEnd;                        // OPB x RES_TILE
     const uint32_t sEpi = sRes + S::OPB * S::RES_TILE;     // EPI_BYTES
     const uint32_t sBias = sEpi + S::EPI_BYTES;            // 2 x BIAS_BYTES
     const uint32_t ctrl = sBias + S::BIAS_REGION;
@@ -114,9 +123,9 @@ __global__ void __maxnreg__(168)
     const uint32_t tempty = tfull + 16u;                   // 2: accumulator drained
     const uint32_t ofull = tempty + 16u;                   // OPB: epilogue operands loaded
     const uint32_t oempty = ofull + 8u * S::OPB;           // OPB: epilogue operands consumed
-    const uint32_t sfull = oempty + 8u * S::OPB;           // 2: slab loaded
-    const uint32_t sempty = sfull + 16u;                   // 2: slab consumed
-    const uint32_t drain = sempty + 16u;
+    const uint32_t sfull = oempty + 8u * S::OPB;           // SLOTS_MAX: slab loaded
+    const uint32_t sempty = sfull + 8u * S::SLOTS_MAX;     // SLOTS_MAX: slab consumed
+    const uint32_t drain = sempty + 8u * S::SLOTS_MAX;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -131,6 +140,8 @@ __global__ void __maxnreg__(168)
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull + 8u * b, 1);                 // MMA commit
             mbar_init(tempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
+        }
+        for (int b = 0; b < S::SLOTS_MAX; ++b) {
             mbar_init(sfull + 8u * b, 1);                 // producer + slab bytes
             mbar_init(sempty + 8u * b, 1);                // MMA commit
         }
@@ -204,10 +215,38 @@ __global__ void __maxnreg__(168)
                     phase ^= 1u;
                 }
             };
+            int ss = 0;        // resident weights: slab slot of slab sl, and its phase
+            uint32_t sph = 0;
+            if constexpr (S::WRES) {
+                // the whole weight matrix once, on ring stage 0
+                if (claim((uint32_t)(a.num_kb * S::B_BYTES))) {
+                    for (int kb = 0; kb < a.num_kb; ++kb)
+                        tma_load_2d(sB + kb * S::B_BYTES, &tmB, bars, kb * BK, 0);
+                    advance();
+                } else {
+                    ok = false;
+                }
+            }
             for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x) {
                 const int mt = tile / a.tiles_n;
                 const int n0 = (tile % a.tiles_n) * BN;
-                if constexpr (AMODE == kAModeSlab) {
+                if constexpr (S::WRES) {
+                    const int img = mt / a.tiles_per_img;
+                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
+                    for (int cc = 0; cc < a.chunks; ++cc, ++sl) {
+                        if (!wait(sempty + 8u * ss, sph ^ 1u)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(sfull + 8u * ss, (uint32_t)a.slab_bytes);
+                        tma_load_4d(sSlab + (uint32_t)(ss * a.slab_pitch), &tmA, sfull + 8u * ss,
+                                    cc * BK, -a.pad_l, p0 - a.pad_t, img);
+                        if (++ss == a.slab_slots) {
+                            ss = 0;
+                            sph ^= 1u;
+                        }
+                    }
+                } else if constexpr (AMODE == kAModeSlab) {
                     const int img = mt / a.tiles_per_img;
                     const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
@@ -278,8 +317,9 @@ __global__ void __maxnreg__(168)
                 // Gave up: let the copies already issued land before exiting.
                 for (int j = issued - nst > 0 ? issued - nst : 0; j < issued; ++j)
                     mbar_wait_drain(bars + 8u * (j % nst), (uint32_t)(j / nst) & 1u);
-                for (int j = sl - 2 > 0 ? sl - 2 : 0; j < sl; ++j)
-                    mbar_wait_drain(sfull + 8u * (j & 1), (uint32_t)(j >> 1) & 1u);
+                const int nsl = S::WRES ? a.slab_slots : 2;
+                for (int j = sl - nsl > 0 ? sl - nsl : 0; j < sl; ++j)
+                    mbar_wait_drain(sfull + 8u * (j % nsl), (uint32_t)(j / nsl) & 1u);
             }
         }
         __syncwarp();
@@ -322,12 +362,18 @@ __global__ void __maxnreg__(168)
                 return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutMma);
             };
             constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
-            const uint64_t adesc0 = make_smem_desc(AMODE == kAModeSlab ? sSlab : sA, S::ROW_BYTES);
+            const uint64_t adesc0 = make_smem_desc(S::SLAB ? sSlab : sA, S::ROW_BYTES);
             const uint64_t bdesc0 = make_smem_desc(sB, S::ROW_BYTES);
             int stage = 0, slot0 = 0;
             uint32_t phase = 0;
             int sl = 0, t = 0;
+            int ss = 0;        // resident weights: slab slot and its phase
+            uint32_t sph = 0;
             bool ok = true;
+            if constexpr (S::WRES) {  // the resident weights, once per CTA
+                ok = wait(bars, 0u);
+                tc_fence_after();
+            }
             auto advance = [&]() {
                 slot0 += G;
                 if (++stage == nst) {
@@ -346,7 +392,41 @@ __global__ void __maxnreg__(168)
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
                 uint32_t acc = 0u;
-                if constexpr (AMODE == kAModeSlab) {
+                if constexpr (S::WRES) {
+                    // k-block of filter tap t and chunk cc sits at t * chunks + cc
+                    const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
+                    const uint64_t bstep = (uint64_t)((uint32_t)(a.chunks * S::B_BYTES) >> 4);
+                    for (int cc = 0; ok && cc < a.chunks; ++cc) {
+                        if (!wait(sfull + 8u * ss, sph)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint64_t slab_desc =
+                            adesc0 + (uint64_t)((uint32_t)(ss * a.slab_pitch) >> 4);
+                        uint32_t roff = 0;  // r * wp * ROW_BYTES of the current tap (r, sx)
+                        int sx = 0;
+                        uint64_t bd = bdesc0 + (uint64_t)((uint32_t)(cc * S::B_BYTES) >> 4);
+                        for (int tap = 0; tap < a.taps; ++tap, bd += bstep) {
+                            const uint64_t ad =
+                                slab_desc + (uint64_t)((roff + (uint32_t)sx * S::ROW_BYTES) >> 4);
+#pragma unroll
+                            for (int k = 0; k < BK / 16; ++k)
+                                mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                            acc | (uint32_t)k);
+                            acc = 1u;
+                            if (++sx == a.kw) {
+                                sx = 0;
+                                roff += row_step;
+                            }
+                        }
+                        mma_commit(sempty + 8u * ss);  // frees the slab
+                        if (++ss == a.slab_slots) {
+                            ss = 0;
+                            sph ^= 1u;
+                        }
+                    }
+                } else if constexpr (AMODE == kAModeSlab) {
                     const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
                         const int ss = sl & 1;
@@ -451,7 +531,7 @@ __global__ void __maxnreg__(168)
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int v = quarter * 32 + 8 * k + cl_row;
-                if constexpr (AMODE == kAModeSlab) {
+                if constexpr (S::SLAB) {
                     const int img = mt / a.tiles_per_img;
                     const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
                     const int y = v / a.wp;
@@ -607,7 +687,11 @@ static cudaError_t prepare_t() {
     X(128, 64, kAModeSlab, false)     \
     X(256, 64, kAModeSlab, false)     \
     X(64, 16, kAModeSlab, false)      \
-    X(64, 32, kAModeSlab, false)
+    X(64, 32, kAModeSlab, false)      \
+    X(64, 64, kAModeSlabRes, false)   \
+    X(128, 64, kAModeSlabRes, false)  \
+    X(64, 16, kAModeSlabRes, false)   \
+    X(64, 32, kAModeSlabRes, false)
 
 bool gemm_config_supported(const GemmConfig &c) {
 #define X(BN_, BK_, AM_, RES_) \
@@ -615,6 +699,35 @@ bool gemm_config_supported(const GemmConfig &c) {
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return false;
+}
+
+static void slab_pool_shape(const GemmConfig &c, int &pool, int &bbytes) {
+    pool = bbytes = 0;
+#define X(BN_, BK_, AM_, RES_)                                            \
+    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) { \
+        pool = GemmShape<BN_, BK_, AM_, RES_>::POOL_BYTES;                \
+        bbytes = GemmShape<BN_, BK_, AM_, RES_>::B_BYTES;                 \
+    }
+    BYOC_GEMM_CONFIGS(X)
+#undef X
+}
+
+bool gemm_slab_res_fits(const GemmConfig &c, int num_kb, int slab_bytes) {
+    int pool, bbytes;
+    slab_pool_shape(c, pool, bbytes);
+    const int pitch = (slab_bytes + 1023) / 1024 * 1024;
+    return c.amode == kAModeSlabRes && pool > 0 && num_kb * bbytes + 2 * pitch <= pool;
+}
+
+void gemm_slab_pool(const GemmConfig &c, GemmArgs &a) {
+    a.slab_off = a.slab_pitch = a.slab_slots = 0;
+    if (c.amode != kAModeSlabRes) return;
+    int pool, bbytes;
+    slab_pool_shape(c, pool, bbytes);
+    a.slab_pitch = (a.slab_bytes + 1023) / 1024 * 1024;
+    a.slab_off = a.num_kb * bbytes;
+    const int slots = (pool - a.slab_off) / a.slab_pitch;
+    a.slab_slots = slots > kMaxSlabSlots ? kMaxSlabSlots : slots;
 }
 
 size_t gemm_smem_bytes(const GemmConfig &c) {

@@ -60,6 +60,12 @@ struct GemmArgs {
     int tiles_per_img;  // ceil(Ho / slab_t)
     int slab_bytes;     // bytes of one slab (one channel chunk)
     int taps;           // kh * kw
+    // resident-weight slab mode: the packed weights (every k-block, one
+    // column tile) sit at the start of the shared-memory pool, loaded once
+    // per CTA; the slabs take the rest, set by gemm_slab_pool()
+    int slab_off;       // bytes from the start of the pool to the first slab slot
+    int slab_pitch;     // bytes per slot, a multiple of 1024
+    int slab_slots;     // 2 .. kMaxSlabSlots
     int group;      // k-blocks (slab mode: filter taps) per ring stage, >= 1; the
                     // kernel lowers it so that at least two stages fit the ring
     // packed weights [n_pad][k_pack] (bf16), or null: before waiting for the
@@ -76,7 +82,8 @@ struct GemmArgs {
 enum AMode : int {
     kAModeTile = 0,    // A is a row-major [M, K] matrix (2-D tiled TMA)
     kAModeIm2col = 1,  // A through an im2col TMA map: one load per filter tap and chunk
-    kAModeSlab = 2     // stride-1 conv: one 4-D tiled slab per chunk, taps by row shift
+    kAModeSlab = 2,    // stride-1 conv: one 4-D tiled slab per chunk, taps by row shift
+    kAModeSlabRes = 3  // slab mode, one column tile, all weights resident in shared memory
 };
 
 struct GemmConfig {
@@ -88,6 +95,7 @@ struct GemmConfig {
 
 // Largest slab (one channel chunk) the slab mode holds, per buffer.
 constexpr int slab_max_bytes(int bk) { return bk == 64 ? 48 * 1024 : 24 * 1024; }
+constexpr int kMaxSlabSlots = 8;
 
 constexpr int kGemmBM = 128;
 constexpr int kGemmEpiWarps = 8;
@@ -110,6 +118,11 @@ inline int gemm_group(int bn, int bk, int n) {
 bool gemm_config_supported(const GemmConfig &cfg);
 size_t gemm_smem_bytes(const GemmConfig &cfg);
 int gemm_stages(const GemmConfig &cfg);
+// Resident-weight slab mode: whether num_kb weight k-blocks and two slabs of
+// slab_bytes fit the configuration's pool, and the split of the pool
+// (a.slab_off, slab_pitch, slab_slots from a.num_kb and a.slab_bytes).
+bool gemm_slab_res_fits(const GemmConfig &cfg, int num_kb, int slab_bytes);
+void gemm_slab_pool(const GemmConfig &cfg, GemmArgs &a);
 cudaError_t gemm_prepare(const GemmConfig &cfg);  // raises the dynamic smem limit
 // tmR: residual [M, N] bf16 in 64-column x 128-row boxes, 128-byte swizzle
 // (read only when cfg.res).  a.bias must cover tiles_n * bn floats.

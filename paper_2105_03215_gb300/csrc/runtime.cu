@@ -692,6 +692,13 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
                         o, bk, amode, (int)has_res);
         L.cfg = GemmConfig{bn, bk, amode, has_res};
+        if (slab && Cout <= bn) {
+            // one column tile: keep the whole weight matrix in shared memory
+            // when it fits beside two slabs
+            const GemmConfig rc{bn, bk, byoc::kAModeSlabRes, false};
+            if (byoc::gemm_config_supported(rc) && byoc::gemm_slab_res_fits(rc, taps * chunks, sgeo.bytes))
+                L.cfg = rc;
+        }
         if (slab) {
             L.slab_rows = sgeo.rows;
             L.args.wp = sgeo.wp;
@@ -734,6 +741,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         A.num_tiles = (int)(tiles_m * A.tiles_n);
         A.taps = taps;
         A.group = byoc::gemm_group(bn, bk, amode == byoc::kAModeSlab ? taps : A.num_kb);
+        byoc::gemm_slab_pool(L.cfg, A);
         A.act = act;
         L.grid = std::min(A.num_tiles, P.num_sms);
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
@@ -806,8 +814,13 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
         r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : 0;
         r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : 0;
         r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : 0;
-        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.amode : 0;
+        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? std::min(L.cfg.amode, (int)byoc::kAModeSlab) : 0;
         r->grid[i] = L.grid;
+        r->resident_b[i] = L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeSlabRes ? 1 : 0;
+        r->slab_slots[i] = L.kind != BYOC_LAUNCH_GEMM ? 0
+                           : L.cfg.amode == byoc::kAModeSlabRes ? L.args.slab_slots
+                           : L.cfg.amode == byoc::kAModeSlab    ? 2
+                                                                : 0;
     }
     r->flops = P.flops;
     r->bytes = P.bytes;
@@ -1008,7 +1021,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
                 CUresult r;
-                if (L.cfg.amode == byoc::kAModeSlab)
+                if (L.cfg.amode == byoc::kAModeSlab || L.cfg.amode == byoc::kAModeSlabRes)
                     r = encode_slab(&h->tmA[i], xa, L.geo.N, L.geo.H, L.geo.W, L.geo.C, L.args.wp,
                                     L.slab_rows, L.cfg.bk);
                 else if (L.cfg.amode == byoc::kAModeIm2col)

@@ -186,3 +186,22 @@ def test_every_mobilenet_v2_region_plans_at_224():
         rep = r.plan()
         assert rep.n_launches >= 1
     assert sum(r.plan().flops for r in regions) == pytest.approx(I.region_flops(g), rel=1e-9)
+
+
+def test_slab_pool_keeps_small_weight_matrices_resident():
+    # one column tile whose packed weights fit beside two slabs: loaded once
+    # per CTA; the slabs take the rest of the pool, up to 8 in flight
+    g, _ = I.conv_bias_relu(N=2, H=56, W=56, C=64, K=64)
+    rep = _plan(g)
+    assert rep.im2col[0] == 2 and rep.tile_n[0] == 64 and rep.gemm_k[0] == 576
+    assert rep.resident_b[0] == 1 and 2 <= rep.slab_slots[0] <= 8
+    g, _ = I.resnet50(N=1, H=32, W=32)
+    rep = R.Region(g, [n.name for n in g.nodes[:3]], "stem").plan()
+    assert rep.resident_b[1] == 1 and rep.slab_slots[1] >= 4     # 1 x 115-pixel slabs of 16 KB
+    # 3x3 over 128 channels to 128: 18 k-blocks x 16 KB do not fit; ringed, slabs double-buffered or more
+    g, _ = I.conv_bias_relu(N=2, H=28, W=28, C=128, K=128)
+    rep = _plan(g)
+    assert rep.im2col[0] == 2 and rep.resident_b[0] == 0 and rep.slab_slots[0] >= 2
+    # other modes carry no slab pool
+    rep = _plan(I.bert_ffn(M=64, D=128, F=256)[0])
+    assert rep.resident_b[0] == 0 and rep.slab_slots[0] == 0
