@@ -170,6 +170,34 @@ const char *byoc_last_error(void);
 byoc_status byoc_query(const byoc_handle *h, byoc_info *info);
 
 /* ---------------------------------------------------------------------------
+ * Serialised regions: codegen option 3 of Section 3.3, where the backend's
+ * output is serialised into the module so that deployment loads it instead
+ * of running the code generator again (the paper's TensorRT engines and
+ * Vitis-AI artifacts).  Here the output is the compiled plan: the launch
+ * list with its tile choices and arguments, the folded, rounded and packed
+ * constants, and the workspace layout.  Host byte order; a layout tag ties
+ * the bytes to the library build that wrote them.
+ * ------------------------------------------------------------------------- */
+
+/* Write the compiled region h into dst (host memory).
+ *   dst       : buffer of dst_bytes bytes, or NULL to query the size only.
+ *   needed    : receives the serialised size (always set on success and on a
+ *               too-small buffer).
+ * Synchronous, touches no device memory.
+ * Errors: INVALID_ARG (null handle / size pointer, buffer too small). */
+byoc_status byoc_serialize(const byoc_handle *h, void *dst, size_t dst_bytes, size_t *needed);
+
+/* Rebuild a handle from byoc_serialize's bytes on the current CUDA device:
+ * uploads the constants, allocates the workspace and encodes the weight
+ * descriptors -- no validation of a graph, no batch-norm folding, no packing.
+ * src is read only during the call; the new handle behaves exactly like the
+ * one that was serialised (same kernels, same results bit for bit).
+ * Errors: INVALID_ARG (truncated, corrupted -- checksum -- or inconsistent
+ *         bytes), UNSUPPORTED (bytes from another library build; device not
+ *         sm_103), OOM, CUDA. */
+byoc_status byoc_deserialize(const void *src, size_t src_bytes, byoc_handle **out);
+
+/* ---------------------------------------------------------------------------
  * Host-side operators.  In the paper, operators that stay outside every
  * region run on the host through the compiler's own code generation, and CUDA
  * may serve as the host (Section 3.4, footnote on the metadata module;

@@ -61,6 +61,14 @@ byoc_status byoc_plan(const byoc_region_desc *desc, int32_t num_sms, byoc_plan_r
 byoc_status byoc_plan_constants(const byoc_region_desc *desc, int32_t num_sms, int32_t launch,
                                 int32_t what, void *dst, size_t dst_bytes, size_t *needed);
 
+/* The host halves of byoc_serialize / byoc_deserialize, for tests without a
+ * GPU: plan the region for `num_sms` SMs and serialise the plan (dst NULL:
+ * size query), or parse serialised bytes and report the plan they hold.
+ * Same formats and errors as byoc_serialize / byoc_deserialize. */
+byoc_status byoc_plan_serialize(const byoc_region_desc *desc, int32_t num_sms, void *dst,
+                                size_t dst_bytes, size_t *needed);
+byoc_status byoc_plan_deserialize(const void *src, size_t src_bytes, byoc_plan_report *rep);
+
 #ifdef __cplusplus
 }
 #endif

@@ -85,6 +85,11 @@ _SIGNATURES = {
     "byoc_plan": (c_int32, [POINTER(RegionDesc), c_int32, POINTER(PlanReport)]),
     "byoc_plan_constants": (c_int32, [POINTER(RegionDesc), c_int32, c_int32, c_int32, c_void_p,
                                       c_size_t, POINTER(c_size_t)]),
+    "byoc_serialize": (c_int32, [c_void_p, c_void_p, c_size_t, POINTER(c_size_t)]),
+    "byoc_deserialize": (c_int32, [c_void_p, c_size_t, POINTER(c_void_p)]),
+    "byoc_plan_serialize": (c_int32, [POINTER(RegionDesc), c_int32, c_void_p, c_size_t,
+                                      POINTER(c_size_t)]),
+    "byoc_plan_deserialize": (c_int32, [c_void_p, c_size_t, POINTER(PlanReport)]),
 }
 
 _lib = None

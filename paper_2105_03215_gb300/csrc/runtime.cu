@@ -26,6 +26,7 @@
 #include <mutex>
 #include <new>
 #include <string>
+#include <type_traits>
 #include <vector>
 
 #include "byoc.h"
@@ -915,23 +916,28 @@ void byoc_release(byoc_handle *h) {
     delete h;
 }
 
-byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
-    if (!out) return fail(BYOC_ERR_INVALID_ARG, "null output handle pointer");
-    *out = nullptr;
-    int32_t sms = 0, ccM = 0, ccm = 0;
-    byoc_status st = byoc_device_info(&sms, &ccM, &ccm);
+}  // extern "C"
+
+namespace {
+
+// The current device must be an sm_103 GPU; returns its SM count.
+byoc_status check_device(int32_t *sms) {
+    int32_t ccM = 0, ccm = 0;
+    byoc_status st = byoc_device_info(sms, &ccM, &ccm);
     if (st != BYOC_OK) return st;
     if (ccM != 10 || ccm != 3)
         return fail(BYOC_ERR_UNSUPPORTED, "device is sm_%d%d; this library is built for sm_103a", ccM, ccm);
     cudaError_t e = load_driver();
     if (e != cudaSuccess) return cuda_fail(e, "driver entry points for TMA descriptors");
-    byoc_handle *h = new (std::nothrow) byoc_handle();
-    if (!h) return fail(BYOC_ERR_OOM, "host allocation");
-    st = plan_region(desc, sms, h->P);
-    if (st != BYOC_OK) {
-        delete h;
-        return st;
-    }
+    return BYOC_OK;
+}
+
+// Device half of byoc_compile / byoc_deserialize: h->P is a complete plan.
+// Uploads the constants, allocates the workspace, binds the device pointers
+// into the launch arguments, encodes the weight TMA descriptors and raises
+// the kernels' shared-memory limits.  Releases h on failure.
+byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
+    cudaError_t e;
     cudaGetDevice(&h->device);
     Plan &P = h->P;
     if (!P.blob.empty()) {
@@ -990,6 +996,235 @@ byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
         }
     }
     *out = h;
+    return BYOC_OK;
+}
+
+// ------------------------------------------------------------ serialised plans
+//
+// Section 3.3, codegen option 3: the backend's output serialised so that
+// deployment loads it without compiling.  Layout (host byte order):
+//   magic "BYOCPLN1" | u32 format | u32 abi_version | u64 layout tag |
+//   i32 num_sms | i32 n_region_tensors | u32 tensors, inputs, outputs,
+//   launches | u64 blob bytes | u64 workspace bytes | f64 flops, bytes |
+//   TensorInfo[] | i32 inputs[] | i32 outputs[] | LaunchPlan[] |
+//   u64 ws_off[] | blob | u64 FNV-1a 64 of everything before it.
+// Launch records are stored as this build's structs; the layout tag (the
+// sizes of the structs, the format and ABI versions) rejects bytes written by
+// a build with a different layout.  Device pointers inside the records are
+// rebound when the plan is instantiated.
+
+static_assert(std::is_trivially_copyable<LaunchPlan>::value && std::is_trivially_copyable<TensorInfo>::value,
+              "launch records are stored byte for byte");
+constexpr char kPlanMagic[8] = {'B', 'Y', 'O', 'C', 'P', 'L', 'N', '1'};
+constexpr uint32_t kPlanFormat = 1;
+
+uint64_t fnv1a(const uint8_t *p, size_t n, uint64_t h = 1469598103934665603ull) {
+    for (size_t i = 0; i < n; ++i) {
+        h ^= p[i];
+        h *= 1099511628211ull;
+    }
+    return h;
+}
+
+uint64_t layout_tag() {
+    const uint64_t sizes[] = {sizeof(TensorInfo), sizeof(LaunchPlan), sizeof(GemmArgs),
+                              sizeof(byoc::DwArgs), sizeof(byoc::S2dArgs), sizeof(Im2colGeom),
+                              kPlanFormat, BYOC_ABI_VERSION};
+    return fnv1a(reinterpret_cast<const uint8_t *>(sizes), sizeof(sizes));
+}
+
+struct PlanHeader {
+    char magic[8];
+    uint32_t format, abi_version;
+    uint64_t tag;
+    int32_t num_sms, n_region_tensors;
+    uint32_t n_tensors, n_inputs, n_outputs, n_launches;
+    uint64_t blob_bytes, ws_bytes;
+    double flops, bytes;
+};
+
+// Records are written with their padding zeroed, so that the bytes depend
+// only on the plan (no stray host memory in a serialised region).
+template <typename T>
+void put(std::vector<uint8_t> &out, const T *v, size_t n) {
+    for (size_t i = 0; i < n; ++i) {
+        T c = v[i];
+        __builtin_clear_padding(&c);
+        const uint8_t *b = reinterpret_cast<const uint8_t *>(&c);
+        out.insert(out.end(), b, b + sizeof(T));
+    }
+}
+
+void serialize_plan(const Plan &P, std::vector<uint8_t> &out) {
+    PlanHeader hd{};
+    std::memcpy(hd.magic, kPlanMagic, 8);
+    hd.format = kPlanFormat;
+    hd.abi_version = BYOC_ABI_VERSION;
+    hd.tag = layout_tag();
+    hd.num_sms = P.num_sms;
+    hd.n_region_tensors = P.n_region_tensors;
+    hd.n_tensors = (uint32_t)P.tensors.size();
+    hd.n_inputs = (uint32_t)P.inputs.size();
+    hd.n_outputs = (uint32_t)P.outputs.size();
+    hd.n_launches = (uint32_t)P.launches.size();
+    hd.blob_bytes = P.blob.size();
+    hd.ws_bytes = P.ws_bytes;
+    hd.flops = P.flops;
+    hd.bytes = P.bytes;
+    out.clear();
+    put(out, &hd, 1);
+    put(out, P.tensors.data(), P.tensors.size());
+    put(out, P.inputs.data(), P.inputs.size());
+    put(out, P.outputs.data(), P.outputs.size());
+    put(out, P.launches.data(), P.launches.size());
+    std::vector<uint64_t> ws(P.ws_off.begin(), P.ws_off.end());
+    put(out, ws.data(), ws.size());
+    put(out, P.blob.data(), P.blob.size());
+    const uint64_t sum = fnv1a(out.data(), out.size());
+    put(out, &sum, 1);
+}
+
+byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
+    if (!src) return fail(BYOC_ERR_INVALID_ARG, "null serialised plan");
+    const uint8_t *b = static_cast<const uint8_t *>(src);
+    PlanHeader hd;
+    if (n < sizeof(hd) + 8) return fail(BYOC_ERR_INVALID_ARG, "serialised plan truncated (%zu bytes)", n);
+    std::memcpy(&hd, b, sizeof(hd));
+    if (std::memcmp(hd.magic, kPlanMagic, 8) != 0) return fail(BYOC_ERR_INVALID_ARG, "not a serialised plan");
+    if (hd.format != kPlanFormat || hd.abi_version != BYOC_ABI_VERSION || hd.tag != layout_tag())
+        return fail(BYOC_ERR_UNSUPPORTED, "serialised plan from another library build (format %u, abi %u)",
+                    hd.format, hd.abi_version);
+    const uint64_t limit = (uint64_t)1 << 40;
+    if (hd.n_tensors > 4096 || hd.n_inputs > hd.n_tensors || hd.n_outputs > hd.n_tensors ||
+        hd.n_launches > 4096 || hd.blob_bytes > limit || hd.ws_bytes > limit ||
+        hd.n_region_tensors < 0 || (uint32_t)hd.n_region_tensors > hd.n_tensors)
+        return fail(BYOC_ERR_INVALID_ARG, "serialised plan: counts out of range");
+    const uint64_t body = (uint64_t)hd.n_tensors * sizeof(TensorInfo) +
+                          (uint64_t)(hd.n_inputs + hd.n_outputs) * sizeof(int) +
+                          (uint64_t)hd.n_launches * sizeof(LaunchPlan) + (uint64_t)hd.n_tensors * 8 +
+                          hd.blob_bytes;
+    if ((uint64_t)n != sizeof(hd) + body + 8)
+        return fail(BYOC_ERR_INVALID_ARG, "serialised plan: %zu bytes, header describes %llu", n,
+                    (unsigned long long)(sizeof(hd) + body + 8));
+    uint64_t sum;
+    std::memcpy(&sum, b + n - 8, 8);
+    if (sum != fnv1a(b, n - 8)) return fail(BYOC_ERR_INVALID_ARG, "serialised plan: checksum mismatch");
+    size_t off = sizeof(hd);
+    auto take = [&](void *dst, size_t bytes) {
+        if (bytes) std::memcpy(dst, b + off, bytes);
+        off += bytes;
+    };
+    P = Plan();
+    P.num_sms = hd.num_sms;
+    P.n_region_tensors = hd.n_region_tensors;
+    P.tensors.resize(hd.n_tensors);
+    take(P.tensors.data(), P.tensors.size() * sizeof(TensorInfo));
+    P.inputs.resize(hd.n_inputs);
+    take(P.inputs.data(), P.inputs.size() * sizeof(int));
+    P.outputs.resize(hd.n_outputs);
+    take(P.outputs.data(), P.outputs.size() * sizeof(int));
+    P.launches.resize(hd.n_launches);
+    take(P.launches.data(), P.launches.size() * sizeof(LaunchPlan));
+    std::vector<uint64_t> ws(hd.n_tensors);
+    take(ws.data(), ws.size() * 8);
+    P.ws_off.assign(ws.begin(), ws.end());
+    P.blob.resize(hd.blob_bytes);
+    take(P.blob.data(), P.blob.size());
+    P.ws_bytes = hd.ws_bytes;
+    P.flops = hd.flops;
+    P.bytes = hd.bytes;
+    // references inside the records must stay within the plan
+    const int nt = (int)hd.n_tensors;
+    for (int id : P.inputs)
+        if (id < 0 || id >= nt) return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad input id");
+    for (int id : P.outputs)
+        if (id < 0 || id >= nt) return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad output id");
+    for (int t = 0; t < nt; ++t)
+        if (P.ws_off[t] != SIZE_MAX && P.ws_off[t] + P.tensors[t].bytes() > P.ws_bytes)
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: workspace layout out of range");
+    for (const LaunchPlan &L : P.launches) {
+        if (L.kind != BYOC_LAUNCH_GEMM && L.kind != BYOC_LAUNCH_DEPTHWISE && L.kind != BYOC_LAUNCH_S2D)
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad launch kind");
+        if (L.x < 0 || L.x >= nt || L.y < 0 || L.y >= nt || L.res >= nt)
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad tensor id in a launch");
+        if (L.w_off + L.w_bytes > P.blob.size() || L.b_off + L.b_bytes > P.blob.size())
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: constants out of range");
+        if (L.kind == BYOC_LAUNCH_GEMM && !byoc::gemm_config_supported(L.cfg))
+            return fail(BYOC_ERR_UNSUPPORTED, "serialised plan: tile configuration not in this build");
+    }
+    return BYOC_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+byoc_status byoc_compile(const byoc_region_desc *desc, byoc_handle **out) {
+    if (!out) return fail(BYOC_ERR_INVALID_ARG, "null output handle pointer");
+    *out = nullptr;
+    int32_t sms = 0;
+    byoc_status st = check_device(&sms);
+    if (st != BYOC_OK) return st;
+    byoc_handle *h = new (std::nothrow) byoc_handle();
+    if (!h) return fail(BYOC_ERR_OOM, "host allocation");
+    st = plan_region(desc, sms, h->P);
+    if (st != BYOC_OK) {
+        delete h;
+        return st;
+    }
+    return instantiate(h, out);
+}
+
+byoc_status byoc_serialize(const byoc_handle *h, void *dst, size_t dst_bytes, size_t *needed) {
+    if (!h || !needed) return fail(BYOC_ERR_INVALID_ARG, "null handle or size pointer");
+    std::vector<uint8_t> buf;
+    serialize_plan(h->P, buf);
+    *needed = buf.size();
+    if (!dst) return BYOC_OK;
+    if (dst_bytes < buf.size())
+        return fail(BYOC_ERR_INVALID_ARG, "buffer of %zu bytes, %zu needed", dst_bytes, buf.size());
+    std::memcpy(dst, buf.data(), buf.size());
+    return BYOC_OK;
+}
+
+byoc_status byoc_deserialize(const void *src, size_t src_bytes, byoc_handle **out) {
+    if (!out) return fail(BYOC_ERR_INVALID_ARG, "null output handle pointer");
+    *out = nullptr;
+    int32_t sms = 0;
+    byoc_status st = check_device(&sms);
+    if (st != BYOC_OK) return st;
+    byoc_handle *h = new (std::nothrow) byoc_handle();
+    if (!h) return fail(BYOC_ERR_OOM, "host allocation");
+    st = deserialize_plan(src, src_bytes, h->P);
+    if (st != BYOC_OK) {
+        delete h;
+        return st;
+    }
+    return instantiate(h, out);
+}
+
+byoc_status byoc_plan_serialize(const byoc_region_desc *desc, int32_t num_sms, void *dst,
+                                size_t dst_bytes, size_t *needed) {
+    if (!needed) return fail(BYOC_ERR_INVALID_ARG, "null size pointer");
+    Plan P;
+    byoc_status st = plan_region(desc, num_sms, P);
+    if (st != BYOC_OK) return st;
+    std::vector<uint8_t> buf;
+    serialize_plan(P, buf);
+    *needed = buf.size();
+    if (!dst) return BYOC_OK;
+    if (dst_bytes < buf.size())
+        return fail(BYOC_ERR_INVALID_ARG, "buffer of %zu bytes, %zu needed", dst_bytes, buf.size());
+    std::memcpy(dst, buf.data(), buf.size());
+    return BYOC_OK;
+}
+
+byoc_status byoc_plan_deserialize(const void *src, size_t src_bytes, byoc_plan_report *rep) {
+    if (!rep) return fail(BYOC_ERR_INVALID_ARG, "null report");
+    Plan P;
+    byoc_status st = deserialize_plan(src, src_bytes, P);
+    if (st != BYOC_OK) return st;
+    fill_report(P, rep);
     return BYOC_OK;
 }
 

@@ -24,7 +24,12 @@ HOST_OPS = ("nn.max_pool2d", "nn.global_avg_pool2d", "nn.batch_flatten")
 
 
 class Executor:
-    def __init__(self, result: PartitionResult):
+    def __init__(self, result: PartitionResult, serialized: Optional[List[bytes]] = None):
+        """Compile every region of ``result`` -- or, given ``serialized`` (one
+        ``CompiledRegion.serialize()`` blob per region, from ``serialize()``),
+        load them without compiling (Section 3.3, option 3).  ``init_s`` is
+        the wall time of that step (the engine initialisation of Section 4.1)."""
+        import time
         import torch
         self.torch = torch
         self.result = result
@@ -33,7 +38,14 @@ class Executor:
         self.by_name = {n.name: n for n in g.nodes}
         # steps: ("region", index) or ("host", node name), in a topological order
         self.regions = result.region_objects()
-        self.compiled = [r.compile() for r in self.regions]
+        t0 = time.perf_counter()
+        if serialized is None:
+            self.compiled = [r.compile() for r in self.regions]
+        else:
+            if len(serialized) != len(self.regions):
+                raise ValueError(f"{len(serialized)} serialised regions for {len(self.regions)} regions")
+            self.compiled = [r.load(b) for r, b in zip(self.regions, serialized)]
+        self.init_s = time.perf_counter() - t0
         self.steps = self._order_steps()
         # data entries
         needed = set(g.outputs) | set(g.inputs)
@@ -59,6 +71,10 @@ class Executor:
         self._graph = None
         self.n_launches = sum(c.n_launches for c in self.compiled) + sum(
             1 for k, x in self.steps if k == "host" and self.by_name[x].op != "nn.batch_flatten")
+
+    def serialize(self) -> List[bytes]:
+        """Every compiled region as bytes, in region order."""
+        return [c.serialize() for c in self.compiled]
 
     # ------------------------------------------------------------------ planning
     def _order_key(self, name: str) -> int:

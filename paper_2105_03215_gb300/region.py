@@ -149,6 +149,34 @@ class Region:
         abi.check(abi.lib().byoc_compile(ctypes.byref(desc), ctypes.byref(h)))
         return CompiledRegion(h, self)
 
+    def plan_serialized(self, num_sms: int = 148) -> bytes:
+        """The serialised plan of this region for ``num_sms`` SMs, made on the
+        host (no GPU); ``load_plan_report`` parses it back."""
+        desc, keep = self.to_desc()
+        need = ctypes.c_size_t()
+        L = abi.lib()
+        abi.check(L.byoc_plan_serialize(ctypes.byref(desc), num_sms, None, 0, ctypes.byref(need)))
+        buf = ctypes.create_string_buffer(need.value)
+        abi.check(L.byoc_plan_serialize(ctypes.byref(desc), num_sms, buf, need.value,
+                                        ctypes.byref(need)))
+        return buf.raw
+
+    def load(self, blob: bytes) -> "CompiledRegion":
+        """A compiled region rebuilt from ``CompiledRegion.serialize()`` bytes
+        (Section 3.3, option 3): no planning, folding or packing."""
+        h = ctypes.c_void_p()
+        buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+        abi.check(abi.lib().byoc_deserialize(buf, len(blob), ctypes.byref(h)))
+        return CompiledRegion(h, self)
+
+
+def load_plan_report(blob: bytes) -> abi.PlanReport:
+    """Parse serialised region bytes on the host and report the plan they hold."""
+    rep = abi.PlanReport()
+    buf = ctypes.create_string_buffer(bytes(blob), len(blob))
+    abi.check(abi.lib().byoc_plan_deserialize(buf, len(blob), ctypes.byref(rep)))
+    return rep
+
 
 class CompiledRegion:
     """A compiled, cached engine for one region (owns device constants)."""
@@ -181,6 +209,15 @@ class CompiledRegion:
     def check(self) -> None:
         """Raise if a kernel of this region hit a bounded-wait timeout."""
         abi.check(abi.lib().byoc_check(self._h))
+
+    def serialize(self) -> bytes:
+        """The compiled region as bytes (``Region.load`` rebuilds it)."""
+        need = ctypes.c_size_t()
+        L = abi.lib()
+        abi.check(L.byoc_serialize(self._h, None, 0, ctypes.byref(need)))
+        buf = ctypes.create_string_buffer(need.value)
+        abi.check(L.byoc_serialize(self._h, buf, need.value, ctypes.byref(need)))
+        return buf.raw
 
     def release(self) -> None:
         if self._h:

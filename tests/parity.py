@@ -31,10 +31,11 @@ def to_dev(a):
     return torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16).cuda()
 
 
-def run_region(region, inputs, poison=True):
-    """Compile and run ``region`` once; returns {output name: float32 array}."""
+def run_region(region, inputs, poison=True, compiled=None):
+    """Compile (unless ``compiled`` is given) and run ``region`` once; returns
+    ({output name: float32 array}, the compiled region)."""
     import torch
-    cr = region.compile()
+    cr = compiled if compiled is not None else region.compile()
     try:
         ins = [to_dev(inputs[n]) for n in region.inputs]
         outs = []

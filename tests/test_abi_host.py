@@ -205,3 +205,51 @@ def test_slab_pool_keeps_small_weight_matrices_resident():
     # other modes carry no slab pool
     rep = _plan(I.bert_ffn(M=64, D=128, F=256)[0])
     assert rep.resident_b[0] == 0 and rep.slab_slots[0] == 0
+
+
+def _report_tuple(rep):
+    n = rep.n_launches
+    fields = ["kind", "first_op", "n_ops", "act", "residual", "gemm_m", "gemm_n", "gemm_k", "tile_n",
+              "tile_k", "im2col", "grid", "resident_b", "slab_slots"]
+    return (n, tuple(tuple(getattr(rep, f)[:n]) for f in fields), rep.flops, rep.bytes,
+            rep.const_bytes, rep.workspace_bytes)
+
+
+@pytest.mark.parametrize("make", [
+    lambda: R.whole_graph_region(I.resnet_bottleneck(N=2, H=14, W=14, C=256, width=64)[0]),
+    lambda: R.whole_graph_region(I.bert_ffn(M=64, D=128, F=256)[0]),
+    lambda: R.whole_graph_region(I.mbv2_dw_pw(N=1, H=8, W=8)[0]),
+    lambda: R.Region(I.resnet50(N=1, H=32, W=32)[0], [n.name for n in I.resnet50(N=1, H=32, W=32)[0].nodes[:3]], "stem"),
+])
+def test_serialized_plan_round_trips(make):
+    # Section 3.3 option 3: the serialised plan holds the same launches,
+    # figures and constants as the plan it was written from
+    reg = make()
+    blob = reg.plan_serialized(152)
+    assert blob[:8] == b"BYOCPLN1"
+    assert _report_tuple(R.load_plan_report(blob)) == _report_tuple(reg.plan(152))
+    # the packed constants of every launch are in the blob byte for byte
+    rep = reg.plan(152)
+    for i in range(rep.n_launches):
+        if rep.kind[i] == abi.LAUNCH_S2D:
+            continue
+        w = reg.plan_constants(i, 0, 152)
+        assert blob.find(w) > 0
+    # deterministic: planning twice gives the same bytes
+    assert reg.plan_serialized(152) == blob
+
+
+def test_serialized_plan_rejects_damaged_bytes():
+    reg = R.whole_graph_region(I.conv_bias_relu(N=1, H=8, W=8, C=64, K=64)[0])
+    blob = bytearray(reg.plan_serialized(152))
+    for bad, status in [
+        (blob[:-1], abi.ERR_INVALID_ARG),                               # truncated
+        (blob + b"\0", abi.ERR_INVALID_ARG),                            # trailing bytes
+        (b"NOTAPLAN" + blob[8:], abi.ERR_INVALID_ARG),                  # magic
+        (blob[:200] + bytes([blob[200] ^ 1]) + blob[201:], abi.ERR_INVALID_ARG),  # checksum
+        (blob[:8] + (99).to_bytes(4, "little") + blob[12:], abi.ERR_UNSUPPORTED),  # format
+        (b"", abi.ERR_INVALID_ARG),
+    ]:
+        with pytest.raises(abi.ByocError) as e:
+            R.load_plan_report(bytes(bad))
+        assert e.value.status == status

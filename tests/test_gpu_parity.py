@@ -222,3 +222,25 @@ def test_depthwise_regions_sharing_a_kernel_run_in_any_compile_order():
         assert_close(y.float().cpu().numpy(), ograph.evaluate(g, inp)[g.outputs[0]], g.name)
     big.release()
     small.release()
+
+
+@pytest.mark.parametrize("make", [
+    lambda: I.resnet_bottleneck(N=2, H=14, W=14, C=256, width=64, seed=5),
+    lambda: I.mbv2_dw_pw(N=2, H=12, W=12, C=96, Cout=32, seed=6),
+    lambda: I.bert_ffn(M=96, D=128, F=256, seed=7),
+])
+def test_deserialized_region_runs_bit_identically(make):
+    # Section 3.3 option 3: a region rebuilt from its serialised bytes runs the
+    # same kernels on the same constants as the compiled one
+    g, inp = make()
+    reg = R.whole_graph_region(g)
+    got, cr = run_region(reg, inp)
+    blob = cr.serialize()
+    cr.release()
+    cr2 = reg.load(blob)
+    assert cr2.serialize() == blob
+    got2, _ = run_region(reg, inp, compiled=cr2)
+    for name in g.outputs:
+        assert np.array_equal(got[name].view(np.uint32), got2[name].view(np.uint32)), name
+    assert_close(got2[g.outputs[0]], ograph.evaluate(g, inp)[g.outputs[0]], g.name)
+    cr2.release()
