@@ -263,10 +263,79 @@ def region_figures(flush, peaks):
                                          "tflops": mflops / tm / 1e12, "regions": len(mex.regions),
                                          "launches": mex.n_launches}
     mex.release()
+    # the boundary layout transformation (Section 3.2) of the ResNet-50 input:
+    # NCHW fp32 [64,3,224,224] -> NHWC bf16, one launch, HBM-bound
+    from paper_2105_03215_gb300 import abi
+    xs = torch.randn(BATCH, 3, IMG, IMG, device="cuda")
+    ys = torch.empty(BATCH, IMG, IMG, 3, dtype=torch.bfloat16, device="cuda")
+    tb = []
+    for _ in range(23):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(st)
+        abi.check(abi.lib().byoc_nchw_to_nhwc_bf16(xs.data_ptr(), ys.data_ptr(), BATCH, 3, IMG, IMG, 3,
+                                                   abi._stream_ptr(st)))
+        b.record(st)
+        torch.cuda.synchronize()
+        tb.append(a.elapsed_time(b) * 1e-3)
+    tb = statistics.median(tb[3:])
+    nbytes = xs.numel() * 4 + ys.numel() * 2
+    out[f"boundary_nchw_f32_to_nhwc_bf16_{BATCH}x3x{IMG}x{IMG}"] = {
+        "us": tb * 1e6, "gbps": nbytes / tb / 1e9, "hbm_frac_of_measured": nbytes / tb / 1e9 / peaks["hbm_gbs"]}
     return out
 
 
 # ---------------------------------------------------------------- main (ours)
+
+def partition_study(graph, data, flush, reps=10):
+    """Region granularity against invocation overhead (the paper's Table 2 /
+    Figs 7-8 question asked of this GPU): ResNet-50 partitioned with at most
+    K composites per region.  The same kernels run in every case; what
+    changes is how many external calls (byoc_run) the host makes.  Per K:
+    regions, kernel launches, compile time, the forward pass replayed as one
+    CUDA graph, and enqueued eagerly from Python (host work per call
+    included); logits must be bit-identical to K=1."""
+    import torch
+    from paper_2105_03215_gb300 import executor as E
+    x = torch.from_numpy(data).to(torch.bfloat16).cuda()
+    out, ref = {}, None
+    for mo in (1, 4, 16, None):
+        res, _ = E.build_resnet50(max_ops=mo, graph=graph)
+        ex = E.Executor(res)
+        ex.set_input("data", x)
+        ex.run_steps()
+        torch.cuda.synchronize()
+        ex.check()
+        logits = ex.output().clone()
+        ref = logits if ref is None else ref
+
+        def timed(fn):
+            ts, hs = [], []
+            for _ in range(reps):
+                flush.zero_()
+                a = torch.cuda.Event(enable_timing=True)
+                b = torch.cuda.Event(enable_timing=True)
+                torch.cuda.synchronize()
+                a.record()
+                h0 = time.perf_counter()
+                fn()
+                hs.append(time.perf_counter() - h0)
+                b.record()
+                torch.cuda.synchronize()
+                ts.append(a.elapsed_time(b))
+            return statistics.median(ts), statistics.median(hs) * 1e3
+
+        eager_ms, host_ms = timed(ex.run_steps)
+        ex.capture()
+        graph_ms, _ = timed(ex.replay)
+        out["all" if mo is None else str(mo)] = {
+            "regions": len(ex.regions), "launches": ex.n_launches, "compile_ms": ex.init_s * 1e3,
+            "graph_ms": graph_ms, "eager_ms": eager_ms, "eager_host_enqueue_ms": host_ms,
+            "logits_bit_identical": bool(torch.equal(logits, ref))}
+        ex.release()
+    return out
+
 
 def main():
     ap = argparse.ArgumentParser()
@@ -460,6 +529,10 @@ def main():
                        "loaded_output_bit_identical": bool(torch.equal(ex.output(), ex2.output()))}
         ex2.release()
 
+    study = None
+    if not args.no_regions and rank == 0:
+        study = partition_study(res.graph, inp["data"], flush)
+
     cpu = None
     if not args.no_cpu_baseline and rank == 0 and world == 1:
         # a bounded sample: two images to estimate the rate, then enough
@@ -499,6 +572,7 @@ def main():
                          "gemm_gbps": gemm_b / gemm_t / 1e9},
             "cpu_baseline": cpu,
             "engine_init": engine_init,
+            "partition_study": study,
             "regions": regions,
         }
         print(json.dumps(line), flush=True)

@@ -216,6 +216,14 @@ byoc_status byoc_max_pool2d_nhwc(const void *x, void *y, int32_t N, int32_t H, i
 byoc_status byoc_global_avg_pool_nhwc(const void *x, void *y, int32_t N, int32_t H, int32_t W,
                                       int32_t C, void *cuda_stream);
 
+/* Layout transformation at a region boundary (Section 3.2): the framework's
+ * NCHW fp32 tensor x [N,C,H,W] -> the NHWC bf16 tensor y [N,H,W,c_pad] the
+ * regions read, y[n,h,w,c] = x[n,c,h,w] rounded to nearest even, and 0 for
+ * C <= c < c_pad.  Requires c_pad >= C and W * c_pad <= 16384; pointers
+ * 16-byte aligned.  Asynchronous on cuda_stream.  Errors: INVALID_ARG, CUDA. */
+byoc_status byoc_nchw_to_nhwc_bf16(const void *x, void *y, int32_t N, int32_t C, int32_t H, int32_t W,
+                                   int32_t c_pad, void *cuda_stream);
+
 /* ---------------------------------------------------------------------------
  * Allocation-free entry point.  The paper has no counterpart: it exists for
  * callers that cannot allocate device memory -- code running inside a memory

@@ -18,7 +18,8 @@
 extern "C" {
 #endif
 
-#define BYOC_PLAN_MAX_LAUNCHES 16
+/* launches of one region (a whole ResNet-50 body plans to 61) */
+#define BYOC_PLAN_MAX_LAUNCHES 128
 
 typedef enum {
     BYOC_LAUNCH_GEMM = 0,      /* tcgen05 implicit-GEMM conv2d / dense + fused epilogue */

@@ -159,3 +159,31 @@ def global_avg_pool_nhwc(x):
     y = np.empty((N, C), dtype=np.float64)
     lib().oracle_global_avg_pool_nhwc(_p(x), _I(N), _I(H), _I(W), _I(C), _p(y))
     return y
+
+
+def round_bf16(x):
+    """Round to the nearest bfloat16 value, ties to even (8 significant bits,
+    fp32's exponent range): the cast at a region boundary (Section 3.2,
+    "partial quantization" read as fp32 -> bf16).  Written from the
+    definition: x = m 2^e with 1/2 <= |m| < 1, so the bf16 neighbours of x are
+    the multiples of 2^(e-8) and np.rint picks the nearest, ties to the even
+    multiple.  Below 2^-126 the spacing stays 2^-133 (subnormals); beyond the
+    largest finite bf16 the result is infinite.  Returns float64."""
+    x = _f64(x)
+    m, e = np.frexp(x)
+    e = np.maximum(e, -125)                      # subnormal range: fixed spacing 2^-133
+    q = np.rint(np.ldexp(x, 8 - e))
+    r = np.ldexp(q, e - 8)
+    bf16_max = (2.0 - 2.0 ** -7) * 2.0 ** 127
+    r = np.where(np.abs(r) > bf16_max, np.copysign(np.inf, x), r)
+    return np.where(np.isfinite(x), r, x)
+
+
+def nchw_to_nhwc(x, c_pad):
+    """Layout transformation at a region boundary (Section 3.2): NCHW ->
+    NHWC with channels zero-padded to c_pad, values rounded to bf16."""
+    x = _f64(x)
+    N, C, H, W = x.shape
+    y = np.zeros((N, H, W, c_pad))
+    y[..., :C] = np.transpose(x, (0, 2, 3, 1))
+    return round_bf16(y)

@@ -23,7 +23,7 @@ LAYOUT_NHWC, LAYOUT_NC = 0, 1
 OP_CONV2D, OP_DENSE, OP_BIAS_ADD, OP_BATCH_NORM, OP_RELU, OP_RELU6, OP_GELU, OP_ADD = range(8)
 
 LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D = range(3)
-PLAN_MAX_LAUNCHES = 16
+PLAN_MAX_LAUNCHES = 128
 
 
 class ByocError(RuntimeError):
@@ -85,6 +85,7 @@ _SIGNATURES = {
     "byoc_plan": (c_int32, [POINTER(RegionDesc), c_int32, POINTER(PlanReport)]),
     "byoc_plan_constants": (c_int32, [POINTER(RegionDesc), c_int32, c_int32, c_int32, c_void_p,
                                       c_size_t, POINTER(c_size_t)]),
+    "byoc_nchw_to_nhwc_bf16": (c_int32, [c_void_p, c_void_p] + [c_int32] * 5 + [c_void_p]),
     "byoc_serialize": (c_int32, [c_void_p, c_void_p, c_size_t, POINTER(c_size_t)]),
     "byoc_deserialize": (c_int32, [c_void_p, c_size_t, POINTER(c_void_p)]),
     "byoc_plan_serialize": (c_int32, [POINTER(RegionDesc), c_int32, c_void_p, c_size_t,

@@ -382,6 +382,80 @@ cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
     }
 }
 
+// ------------------------------------------------------------ boundary layout transform
+// y[n, h, w, c] = bf16_rne(x[n, c, h, w]) for c < C, 0 for C <= c < Cp: the
+// NCHW fp32 layout of the framework side to the NHWC bf16 layout the regions
+// use (a layout transformation at a region boundary, Section 3.2).  Block
+// (row group, n) converts `rows` image rows: it reads C planes' rows of W
+// floats (coalesced along w), stages the rows x W x Cp bf16 output in shared
+// memory and writes it with 16-byte stores (output rows of one image are
+// contiguous).  HBM-bound: 4 C + 2 Cp bytes per pixel.
+__global__ void __launch_bounds__(256) nchw_to_nhwc_kernel(const float *x, __nv_bfloat16 *y, int C, int H,
+                                                           int W, int Cp, int rows) {
+    pdl_launch_dependents();
+    pdl_wait();
+    extern __shared__ __align__(16) unsigned short sxf[];
+    const int n = blockIdx.y;
+    const int h0 = blockIdx.x * rows;
+    const int nr = H - h0 < rows ? H - h0 : rows;
+    const size_t plane = (size_t)H * W;
+    const float *xn = x + (size_t)n * C * plane + (size_t)h0 * W;
+    const int per_row = W * Cp;
+    const int elems = nr * per_row;
+    if (Cp > C)  // padded channels are zero
+        for (int i = threadIdx.x; i < elems; i += blockDim.x) sxf[i] = 0;
+    __syncthreads();
+    // the nr rows of one plane are one contiguous run of nr * W floats
+    const int run = nr * W;
+    if ((W & 3) == 0) {
+        const int run4 = run >> 2;
+        for (int c = 0; c < C; ++c) {
+            const float4 *src = reinterpret_cast<const float4 *>(xn + (size_t)c * plane);
+#pragma unroll 4
+            for (int i = threadIdx.x; i < run4; i += blockDim.x) {
+                const float4 v = __ldg(src + i);
+                unsigned short *d = sxf + (size_t)(4 * i) * Cp + c;  // pixel 4i of the run
+                __nv_bfloat16 b0 = __float2bfloat16_rn(v.x), b1 = __float2bfloat16_rn(v.y);
+                __nv_bfloat16 b2 = __float2bfloat16_rn(v.z), b3 = __float2bfloat16_rn(v.w);
+                d[0] = *reinterpret_cast<unsigned short *>(&b0);
+                d[Cp] = *reinterpret_cast<unsigned short *>(&b1);
+                d[2 * Cp] = *reinterpret_cast<unsigned short *>(&b2);
+                d[3 * Cp] = *reinterpret_cast<unsigned short *>(&b3);
+            }
+        }
+    } else {
+        for (int c = 0; c < C; ++c) {
+            const float *src = xn + (size_t)c * plane;
+            for (int i = threadIdx.x; i < run; i += blockDim.x) {
+                __nv_bfloat16 b = __float2bfloat16_rn(__ldg(src + i));
+                sxf[(size_t)i * Cp + c] = *reinterpret_cast<unsigned short *>(&b);
+            }
+        }
+    }
+    __syncthreads();
+    unsigned short *yo = reinterpret_cast<unsigned short *>(y) + ((size_t)n * H + h0) * per_row;
+    if ((per_row & 7) == 0) {  // rows of 16-byte multiples: the run starts 16-byte aligned
+        const uint4 *src = reinterpret_cast<const uint4 *>(sxf);
+        uint4 *dst = reinterpret_cast<uint4 *>(yo);
+        for (int i = threadIdx.x; i < (elems >> 3); i += blockDim.x) dst[i] = src[i];
+    } else {
+        for (int i = threadIdx.x; i < elems; i += blockDim.x) yo[i] = sxf[i];
+    }
+}
+
+int nchw_rows_per_block(int W, int Cp) {
+    const int r = kNchwStageElems / (W * Cp);
+    return r < 1 ? 1 : (r > 32 ? 32 : r);
+}
+
+cudaError_t launch_nchw_to_nhwc(const float *x, __nv_bfloat16 *y, int N, int C, int H, int W, int Cp,
+                                cudaStream_t st) {
+    const int rows = nchw_rows_per_block(W, Cp);
+    const size_t smem = (size_t)rows * W * Cp * 2;
+    const dim3 grid((unsigned)((H + rows - 1) / rows), (unsigned)N);
+    return launch_pdl(nchw_to_nhwc_kernel, grid, dim3(256), smem, st, x, y, C, H, W, Cp, rows);
+}
+
 // ------------------------------------------------------------ max pool
 __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                                int k, int s, int p, int Ho, int Wo) {

@@ -189,6 +189,12 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
 // Sets the thread-local message byoc_last_error() returns.
 void set_last_error(const char *msg);
 
+// NCHW fp32 -> NHWC bf16 (channels zero-padded to Cp) at a region boundary.
+// Requires W * Cp <= kNchwStageElems; y 16-byte aligned when its rows are.
+constexpr int kNchwStageElems = 16384;
+int nchw_rows_per_block(int W, int Cp);
+cudaError_t launch_nchw_to_nhwc(const float *x, __nv_bfloat16 *y, int N, int C, int H, int W, int Cp,
+                                cudaStream_t st);
 cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            cudaStream_t st);
 

@@ -1357,4 +1357,16 @@ byoc_status byoc_global_avg_pool_nhwc(const void *x, void *y, int32_t N, int32_t
     return e == cudaSuccess ? BYOC_OK : cuda_fail(e, "global_avg_pool launch");
 }
 
+byoc_status byoc_nchw_to_nhwc_bf16(const void *x, void *y, int32_t N, int32_t C, int32_t H, int32_t W,
+                                   int32_t c_pad, void *cuda_stream) {
+    if (!x || !y || ((reinterpret_cast<uintptr_t>(x) | reinterpret_cast<uintptr_t>(y)) & 15u))
+        return fail(BYOC_ERR_INVALID_ARG, "nchw_to_nhwc: null or misaligned pointer");
+    if (N < 1 || C < 1 || H < 1 || W < 1 || c_pad < C || (int64_t)W * c_pad > byoc::kNchwStageElems)
+        return fail(BYOC_ERR_INVALID_ARG, "nchw_to_nhwc: bad shape (need c_pad >= C, W * c_pad <= %d)",
+                    byoc::kNchwStageElems);
+    cudaError_t e = byoc::launch_nchw_to_nhwc(static_cast<const float *>(x), static_cast<__nv_bfloat16 *>(y),
+                                              N, C, H, W, c_pad, static_cast<cudaStream_t>(cuda_stream));
+    return e == cudaSuccess ? BYOC_OK : cuda_fail(e, "nchw_to_nhwc launch");
+}
+
 }  // extern "C"

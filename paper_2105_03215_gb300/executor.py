@@ -162,6 +162,19 @@ class Executor:
     def set_input(self, name: str, src, non_blocking: bool = True) -> None:
         self.entries[name].copy_(src, non_blocking=non_blocking)
 
+    def set_input_nchw(self, name: str, x, stream=None) -> None:
+        """Fill the NHWC bf16 data entry ``name`` from a framework-layout
+        NCHW fp32 CUDA tensor, through the boundary layout transformation
+        (Section 3.2) of this library; channels beyond x's are zero."""
+        dst = self.entries[name]
+        N, H, W, Cp = dst.shape
+        if x.dtype != self.torch.float32 or not x.is_cuda or not x.is_contiguous():
+            raise ValueError("x must be a contiguous fp32 CUDA tensor")
+        if tuple(x.shape) != (N, x.shape[1], H, W) or x.shape[1] > Cp:
+            raise ValueError(f"x {tuple(x.shape)} does not match entry {tuple(dst.shape)} as NCHW")
+        abi.check(abi.lib().byoc_nchw_to_nhwc_bf16(x.data_ptr(), dst.data_ptr(), N, x.shape[1], H, W, Cp,
+                                                   abi._stream_ptr(stream)))
+
     def output(self, name: Optional[str] = None):
         return self.entries[name or self.graph.outputs[0]]
 

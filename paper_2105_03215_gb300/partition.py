@@ -125,9 +125,17 @@ class PartitionResult:
             names.update(self.units[u])
         return [n.name for n in self.graph.nodes if n.name in names]
 
+    def region_nodes_by_unit(self, r: int) -> List[str]:
+        """The nodes of region r unit by unit (units in topological order,
+        each composite's members together in graph order): the op order of
+        the region's descriptor, so that the engine fuses exactly the
+        composites the patterns found, whatever the region's size."""
+        order = {n.name: i for i, n in enumerate(self.graph.nodes)}
+        return [m for u in self.regions[r] for m in sorted(self.units[u], key=order.__getitem__)]
+
     def region_objects(self):
         from .region import Region
-        return [Region(self.graph, self.region_nodes(r), f"{self.target}_{r}")
+        return [Region(self.graph, self.region_nodes_by_unit(r), f"{self.target}_{r}")
                 for r in range(len(self.regions))]
 
     def offload_ratio(self) -> Tuple[float, float]:

@@ -49,9 +49,17 @@ class Region:
                  outputs: Optional[Sequence[str]] = None):
         self.graph = graph
         members = set(node_names)
-        self.nodes: List[Node] = [n for n in graph.nodes if n.name in members]
-        if len(self.nodes) != len(members):
-            raise KeyError(f"unknown nodes in region {name}")
+        # ops keep the given order (the descriptor's op order, which decides
+        # what the engine fuses); it must be topological within the region
+        by_name = {n.name: n for n in graph.nodes}
+        if len(members) != len(node_names) or not members <= by_name.keys():
+            raise KeyError(f"unknown or repeated nodes in region {name}")
+        self.nodes: List[Node] = [by_name[m] for m in node_names]
+        seen = set()
+        for n in self.nodes:
+            if any(i in members and i not in seen for i in n.inputs):
+                raise ValueError(f"region {name}: {n.name} comes before one of its inputs")
+            seen.add(n.name)
         self.name = name
         produced = {n.name for n in self.nodes}
         ins: List[str] = []

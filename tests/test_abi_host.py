@@ -253,3 +253,27 @@ def test_serialized_plan_rejects_damaged_bytes():
         with pytest.raises(abi.ByocError) as e:
             R.load_plan_report(bytes(bad))
         assert e.value.status == status
+
+
+def test_fusion_follows_the_composites_at_every_region_size():
+    # the engine fuses a region's ops greedily in descriptor order; regions
+    # list their ops composite by composite, so a downsample block fuses the
+    # same way (conv3 + BN + add + ReLU, residual = the downsample output)
+    # whether it is one region per composite or part of a larger region
+    from collections import Counter
+    from paper_2105_03215_gb300 import partition as P
+    g, _ = I.resnet50(N=1, H=64, W=64)
+
+    def launches(max_ops):
+        res = P.partition(g, P.PATTERN_TABLE, target=P.TARGET, max_ops=max_ops)
+        c = Counter()
+        for r in res.region_objects():
+            rep = r.plan(152)
+            for i in range(rep.n_launches):
+                c[(rep.kind[i], rep.gemm_m[i], rep.gemm_n[i], rep.gemm_k[i], rep.act[i],
+                   rep.residual[i] >= 0, rep.n_ops[i], rep.tile_n[i])] += 1
+        return c
+
+    base = launches(1)
+    for mo in (4, 16, None):
+        assert launches(mo) == base, mo

@@ -244,3 +244,34 @@ def test_deserialized_region_runs_bit_identically(make):
         assert np.array_equal(got[name].view(np.uint32), got2[name].view(np.uint32)), name
     assert_close(got2[g.outputs[0]], ograph.evaluate(g, inp)[g.outputs[0]], g.name)
     cr2.release()
+
+
+@pytest.mark.parametrize("N,C,H,W,Cp", [
+    (2, 3, 37, 224, 3),    # ResNet-50 input rows; 24-row blocks and a ragged last block
+    (1, 3, 9, 224, 8),     # channels zero-padded to 8
+    (3, 3, 4, 5, 3),       # rows of 15 values: the unvectorised store path
+    (1, 16, 7, 1024, 16),  # one row per block (W * Cp = 16384)
+])
+def test_nchw_fp32_to_nhwc_bf16_boundary_transform_bit_exact(N, C, H, W, Cp):
+    # Section 3.2: the layout transformation and cast at a region boundary;
+    # every output is one rounding of one input, so the comparison is exact
+    import torch
+    from oracle import ops
+    from paper_2105_03215_gb300 import abi
+    rng = np.random.default_rng(N * 100 + C + W)
+    x = (rng.standard_normal((N, C, H, W)) * np.exp2(rng.integers(-8, 8, (N, C, H, W)))).astype(np.float32)
+    xd = torch.from_numpy(x).cuda()
+    y = torch.full((N, H, W, Cp), float("nan"), dtype=torch.bfloat16, device="cuda")
+    abi.check(abi.lib().byoc_nchw_to_nhwc_bf16(xd.data_ptr(), y.data_ptr(), N, C, H, W, Cp, None))
+    torch.cuda.synchronize()
+    ref = ops.nchw_to_nhwc(x, Cp)
+    assert np.array_equal(y.float().cpu().numpy().astype(np.float64), ref)
+
+
+def test_nchw_boundary_rejects_bad_shapes_on_the_host():
+    import torch
+    from paper_2105_03215_gb300 import abi
+    x = torch.zeros(1, 4, 2, 2, device="cuda")
+    y = torch.zeros(1, 2, 2, 8, dtype=torch.bfloat16, device="cuda")
+    assert abi.lib().byoc_nchw_to_nhwc_bf16(x.data_ptr(), y.data_ptr(), 1, 4, 2, 2, 3, None) == abi.ERR_INVALID_ARG
+    assert abi.lib().byoc_nchw_to_nhwc_bf16(x.data_ptr(), y.data_ptr(), 1, 4, 2, 20000, 8, None) == abi.ERR_INVALID_ARG

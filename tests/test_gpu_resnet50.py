@@ -81,6 +81,26 @@ def test_resnet50_graph_replay_equals_eager():
     ex.release()
 
 
+@pytest.mark.parametrize("max_ops", [4, None])
+def test_resnet50_region_granularity_does_not_change_results(max_ops):
+    # Section 3.1.3: capping a region at K composites (or not at all) changes
+    # how many external calls the host makes, not what they compute: the same
+    # kernels run on the same values, so the logits match bit for bit
+    import torch
+    outs = []
+    for mo in (1, max_ops):
+        res, inp = E.build_resnet50(N=2, H=64, W=64, max_ops=mo)
+        ex = E.Executor(res)
+        ex.set_input("data", torch.from_numpy(inp["data"]).to(torch.bfloat16).cuda())
+        ex.run_steps()
+        torch.cuda.synchronize()
+        ex.check()
+        outs.append((len(ex.regions), ex.output().clone()))
+        ex.release()
+    assert outs[0][0] == 54 and outs[1][0] < 54
+    assert torch.equal(outs[0][1], outs[1][1])
+
+
 def _sampled_region_ref(g, r, feed, out_name, rng, count):
     """Oracle value of a single-composite region at `count` random outputs."""
     nodes = r.nodes

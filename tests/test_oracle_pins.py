@@ -293,3 +293,43 @@ def test_bf16_rounding_is_round_to_nearest_even():
                  dtype=np.float32)
     r = I.bf16_round(v)
     assert list(r) == [1.0, 1.0, 1.0 + 2 ** -6, 1.0 + 2 ** -7, -2.5]
+
+
+# ------------------------------------------------------------ bf16 rounding (boundary cast)
+
+def test_round_bf16_ties_to_even_and_keeps_representable_values():
+    from oracle import ops
+    one = 1.0
+    # spacing at 1 is 2^-7; midpoints go to the even neighbour
+    assert ops.round_bf16(np.array([one + 2.0 ** -8]))[0] == 1.0
+    assert ops.round_bf16(np.array([one + 3 * 2.0 ** -8]))[0] == 1.0 + 2.0 ** -6
+    assert ops.round_bf16(np.array([-(one + 3 * 2.0 ** -8)]))[0] == -(1.0 + 2.0 ** -6)
+    assert ops.round_bf16(np.array([one + 2.0 ** -8 + 2.0 ** -20]))[0] == 1.0 + 2.0 ** -7
+    rep = np.array([0.0, 1.0, -2.5, 3.0 * 2.0 ** 100, 2.0 ** -126, 1.5 * 2.0 ** -130])
+    assert np.array_equal(ops.round_bf16(rep), rep)
+    assert np.isinf(ops.round_bf16(np.array([3.5e38]))[0])
+
+
+def test_round_bf16_is_the_nearest_bf16_value():
+    # brute force: the result carries at most 8 significant bits and no other
+    # such value at the same binade spacing is closer
+    from oracle import ops
+    rng = np.random.default_rng(5)
+    x = rng.standard_normal(20000) * np.exp2(rng.integers(-20, 20, 20000))
+    r = ops.round_bf16(x)
+    m, e = np.frexp(r)
+    assert np.all(np.ldexp(m, 8) == np.rint(np.ldexp(m, 8)))     # 8 significant bits
+    ulp = np.ldexp(1.0, np.frexp(x)[1] - 8)
+    assert np.all(np.abs(x - r) <= ulp / 2)
+    for d in (-1, 1):
+        assert np.all(np.abs(x - r) <= np.abs(x - (r + d * ulp)))
+
+
+def test_nchw_to_nhwc_moves_every_value_and_pads_with_zeros():
+    from oracle import ops
+    x = np.arange(2 * 3 * 4 * 5, dtype=np.float64).reshape(2, 3, 4, 5)   # small integers: exact in bf16
+    y = ops.nchw_to_nhwc(x, 8)
+    assert y.shape == (2, 4, 5, 8)
+    for n, c, h, w in [(0, 0, 0, 0), (1, 2, 3, 4), (0, 1, 2, 3)]:
+        assert y[n, h, w, c] == x[n, c, h, w]
+    assert not y[..., 3:].any()

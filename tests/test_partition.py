@@ -127,6 +127,19 @@ def test_bottleneck_cap_three_gives_one_region_per_block():
     assert _regions(res) == ref.partition(g, set(P.annotations(P.TARGET)), max_ops=4)
 
 
+@pytest.mark.parametrize("max_ops,count", [(16, 6), (None, 3)])
+def test_resnet50_granularities_of_the_partition_study(max_ops, count):
+    # the region counts the granularity study runs: every cut matches the
+    # reference checker and keeps every region convex
+    g, _ = I.resnet50(N=1, draw=False)
+    res = P.partition(g, P.PATTERN_TABLE, target=P.TARGET, max_ops=max_ops)
+    regs = _regions(res)
+    assert regs == ref.partition(g, set(P.annotations(P.TARGET)), max_ops=max_ops)
+    assert len(regs) == count
+    for r in regs:
+        assert ref.is_convex(g, r)
+
+
 # ------------------------------------------------------------ Fig. 3 reconstruction
 
 def test_figure3_counts_reconstruction():
