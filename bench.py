@@ -226,6 +226,14 @@ def region_figures(flush, peaks):
                      "tensor_frac_of_measured": tf / peaks["bf16_tflops"],
                      "hbm_frac_of_measured": gb / peaks["hbm_gbs"]}
         if name.startswith("mbv2"):
+            # the same region as one fused kernel (depthwise output kept on chip)
+            os.environ["BYOC_FUSE_DW_PW"] = "1"
+            fcr = reg.compile()
+            os.environ.pop("BYOC_FUSE_DW_PW")
+            tfz = time_region(fcr, ins, outs, flush)
+            out[name + "_fused"] = {"us": tfz * 1e6, "gbps": fcr.bytes / tfz / 1e9, "launches": fcr.n_launches,
+                                    "hbm_frac_of_measured": fcr.bytes / tfz / 1e9 / peaks["hbm_gbs"]}
+            fcr.release()
             # the depthwise launch alone (the bandwidth-bound composite)
             dwg, dwi = I.mbv2_dw_pw(seed=2)
             dreg = R.Region(dwg, [n.name for n in dwg.nodes[:3]], "dw")
@@ -240,29 +248,35 @@ def region_figures(flush, peaks):
         cr.release()
     # MobileNetV2 1.0 end to end (53 regions, global average pool on the host):
     # the other image-classification model whose regions the path covers
+    # (one composite per region, and the whole network as one region, where
+    # 11 of the 17 depthwise -> 1x1 pairs run fused)
     from paper_2105_03215_gb300 import executor as E
-    mres, minp = E.build_mobilenet_v2(N=BATCH, H=IMG, W=IMG)
-    mex = E.Executor(mres)
-    mex.set_input("data", torch.from_numpy(minp["data"]).to(torch.bfloat16).cuda())
-    mex.capture()
-    for _ in range(3):
-        mex.replay()
-    torch.cuda.synchronize()
     st = torch.cuda.current_stream()
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(20)]
-    for a, b in evs:
-        flush.zero_()
-        a.record(st)
-        mex.replay()
-        b.record(st)
-    torch.cuda.synchronize()
-    mex.check()
-    tm = statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3
-    mflops = sum(c.flops for c in mex.compiled)
-    out[f"mobilenet_v2_N{BATCH}_224"] = {"images_per_s": BATCH / tm, "ms_per_step": tm * 1e3,
-                                         "tflops": mflops / tm / 1e12, "regions": len(mex.regions),
-                                         "launches": mex.n_launches}
-    mex.release()
+    for tag, mo in (("", 1), ("_fused", None)):
+        mres, minp = E.build_mobilenet_v2(N=BATCH, H=IMG, W=IMG, max_ops=mo)
+        if tag:
+            os.environ["BYOC_FUSE_DW_PW"] = "1"
+        mex = E.Executor(mres)
+        os.environ.pop("BYOC_FUSE_DW_PW", None)
+        mex.set_input("data", torch.from_numpy(minp["data"]).to(torch.bfloat16).cuda())
+        mex.capture()
+        for _ in range(3):
+            mex.replay()
+        torch.cuda.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(20)]
+        for a, b in evs:
+            flush.zero_()
+            a.record(st)
+            mex.replay()
+            b.record(st)
+        torch.cuda.synchronize()
+        mex.check()
+        tm = statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3
+        mflops = sum(c.flops for c in mex.compiled)
+        out[f"mobilenet_v2_N{BATCH}_224{tag}"] = {"images_per_s": BATCH / tm, "ms_per_step": tm * 1e3,
+                                                  "tflops": mflops / tm / 1e12, "regions": len(mex.regions),
+                                                  "launches": mex.n_launches}
+        mex.release()
     # the boundary layout transformation (Section 3.2) of the ResNet-50 input:
     # NCHW fp32 [64,3,224,224] -> NHWC bf16, one launch, HBM-bound
     from paper_2105_03215_gb300 import abi

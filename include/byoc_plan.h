@@ -24,7 +24,8 @@ extern "C" {
 typedef enum {
     BYOC_LAUNCH_GEMM = 0,      /* tcgen05 implicit-GEMM conv2d / dense + fused epilogue */
     BYOC_LAUNCH_DEPTHWISE = 1, /* depthwise 3x3 conv + fused epilogue */
-    BYOC_LAUNCH_S2D = 2        /* space-to-depth boundary transform of a stride-2 stem */
+    BYOC_LAUNCH_S2D = 2,       /* space-to-depth boundary transform of a stride-2 stem */
+    BYOC_LAUNCH_DWPW = 3       /* depthwise 3x3 + epilogue fused with the 1x1 conv + epilogue after it */
 } byoc_launch_kind;
 
 typedef struct {
@@ -58,6 +59,8 @@ byoc_status byoc_plan(const byoc_region_desc *desc, int32_t num_sms, byoc_plan_r
  *             column k = (filter tap, channel) K-major, zero padded;
  *             depthwise: fp32 [9][C] tap-major.
  *   what = 1: bias (fp32, folded batch norm shift), zero padded.
+ *   what = 2, 3 (fused depthwise -> 1x1 launches only): the 1x1 conv's
+ *             weights, bf16 [n_pad][64 * ceil(C / 64)] K-major, and bias.
  * *needed receives the byte size; dst may be NULL to query it. */
 byoc_status byoc_plan_constants(const byoc_region_desc *desc, int32_t num_sms, int32_t launch,
                                 int32_t what, void *dst, size_t dst_bytes, size_t *needed);

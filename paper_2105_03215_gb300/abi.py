@@ -22,7 +22,7 @@ LAYOUT_NHWC, LAYOUT_NC = 0, 1
 
 OP_CONV2D, OP_DENSE, OP_BIAS_ADD, OP_BATCH_NORM, OP_RELU, OP_RELU6, OP_GELU, OP_ADD = range(8)
 
-LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D = range(3)
+LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D, LAUNCH_DWPW = range(4)
 PLAN_MAX_LAUNCHES = 128
 
 

@@ -51,24 +51,6 @@ __device__ __forceinline__ uint4 ldg_v4(const void *p) {
 // activation is applied to the packed bf16 pairs (exact: rounding is
 // monotonic and 0 and 6 are bf16 values).  The next tile's box loads (TMA)
 // while this one is computed.
-// act(x) for a pair of outputs, rounded to a bf16 pair; ReLU and ReLU6 are
-// applied after rounding, on the packed pair.
-template <int ACT>
-__device__ __forceinline__ uint32_t dw_act2(float lo, float hi) {
-    if constexpr (ACT == kActRelu || ACT == kActRelu6) {
-        uint32_t r = pack_bf16x2(lo, hi);
-        asm("max.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0u));
-        if constexpr (ACT == kActRelu6) asm("min.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0x40C040C0u));
-        return r;
-    } else if constexpr (ACT == kActGelu) {
-        const uint64_t g = gelu2(f32x2(lo, hi));
-        return pack_bf16x2(lane0(g), lane1(g));
-    } else {
-        return pack_bf16x2(lo, hi);
-    }
-}
-
-
 template <int STRIDE, int ACT>
 __global__ void __launch_bounds__(kDwMaxThreads, 1)
     dwconv3x3_kernel(const __grid_constant__ CUtensorMap tmX, const DwArgs a) {

@@ -189,6 +189,37 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
 // Sets the thread-local message byoc_last_error() returns.
 void set_last_error(const char *msg);
 
+// Depthwise 3x3 (pad 1, stride 1|2) + folded BN + activation fused with the
+// 1x1 conv + folded BN (+ residual) (+ activation) that consumes it (dwpw.cu).
+struct DwPwArgs {
+    const float *dw_w;                // [9][C] folded depthwise weights, tap-major
+    const float *dw_b;                // [C]
+    const float *pw_b;                // [n_pad] folded pointwise bias, zero padded
+    const __nv_bfloat16 *residual;    // [N, Ho, Wo, Cout] or null
+    __nv_bfloat16 *out;               // [N, Ho, Wo, Cout]
+    int *err;
+    int N, H, W, C, Ho, Wo, stride, pad;
+    int dw_act, act;                  // activations after the depthwise and after the pointwise
+    int Cout, n_pad, chunks;          // n_pad: Cout rounded up to 16 (the MMA's N); chunks of 64 channels
+    int tr;                           // output rows per tile (tr * Wo <= 128)
+    int bh;                           // depthwise output rows per thread block (1 or 2)
+    int tiles_per_img, num_tiles;
+    int in_rows, in_cols, in_bytes, in_pitch;  // input box per (tile, chunk) and its buffer
+    int in_stages;                    // input buffers in the ring (2 .. kDpMaxInStages)
+    int b_bytes, w_off, a_off, in_off, ctrl_off, smem_bytes;  // shared-memory layout (bytes)
+    int acc_stride, tmem_cols;        // TMEM columns per accumulator (>= 32) and allocated
+};
+constexpr int kDpThreads = 704;
+constexpr int kDpMaxInStages = 4;
+constexpr int kDpChunk = 64;
+constexpr int kDpABytes = 128 * 128;  // A operand: 128 pixels x 64 channels bf16
+constexpr int kDpMaxBBytes = 96 * 1024;
+constexpr int kDpSmemMax = 232448;
+bool dwpw_plan(DwPwArgs &a, int num_sms);  // false: the pair does not fit this kernel
+cudaError_t dwpw_prepare(const DwPwArgs &a);
+cudaError_t launch_dwpw(const CUtensorMap &tmX, const CUtensorMap &tmB, const DwPwArgs &a, int grid,
+                        cudaStream_t st);
+
 // NCHW fp32 -> NHWC bf16 (channels zero-padded to Cp) at a region boundary.
 // Requires W * Cp <= kNchwStageElems; y 16-byte aligned when its rows are.
 constexpr int kNchwStageElems = 16384;

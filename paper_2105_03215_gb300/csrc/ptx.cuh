@@ -12,6 +12,8 @@
 #include <cuda_bf16.h>
 #include <stdint.h>
 
+#include "internal.h"
+
 namespace byoc {
 
 // Error codes written to the per-handle device error word.
@@ -441,6 +443,23 @@ __device__ __forceinline__ uint64_t gelu2(uint64_t x) {
     const uint64_t t = mul2(x, r);  // x * Phi(-|x|)
     const uint64_t u = fma2r(t, f32x2(-1.0f, -1.0f), x);  // x - t
     return f32x2(x0 < 0.0f ? lane0(t) : lane0(u), x1 < 0.0f ? lane1(t) : lane1(u));
+}
+
+// act(x) for a pair of outputs, rounded to a bf16 pair; ReLU and ReLU6 are
+// applied after rounding, on the packed pair.
+template <int ACT>
+__device__ __forceinline__ uint32_t dw_act2(float lo, float hi) {
+    if constexpr (ACT == kActRelu || ACT == kActRelu6) {
+        uint32_t r = pack_bf16x2(lo, hi);
+        asm("max.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0u));
+        if constexpr (ACT == kActRelu6) asm("min.bf16x2 %0, %0, %1;" : "+r"(r) : "r"(0x40C040C0u));
+        return r;
+    } else if constexpr (ACT == kActGelu) {
+        const uint64_t g = gelu2(f32x2(lo, hi));
+        return pack_bf16x2(lane0(g), lane1(g));
+    } else {
+        return pack_bf16x2(lo, hi);
+    }
 }
 
 }  // namespace byoc

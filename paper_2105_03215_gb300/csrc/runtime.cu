@@ -22,6 +22,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <mutex>
 #include <new>
@@ -147,6 +148,19 @@ CUresult encode_dw(CUtensorMap *m, const void *ptr, const byoc::DwArgs &a) {
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// Input boxes of the fused depthwise -> 1x1 kernel: 64 channels x in_cols x
+// in_rows of one image, no swizzle (read by CUDA cores), zero outside.
+CUresult encode_dwpw_input(CUtensorMap *m, const void *ptr, const byoc::DwPwArgs &a) {
+    cuuint64_t dims[4] = {(cuuint64_t)a.C, (cuuint64_t)a.W, (cuuint64_t)a.H, (cuuint64_t)a.N};
+    cuuint64_t strides[3] = {(cuuint64_t)a.C * 2, (cuuint64_t)a.W * a.C * 2,
+                             (cuuint64_t)a.H * a.W * a.C * 2};
+    cuuint32_t box[4] = {(cuuint32_t)byoc::kDpChunk, (cuuint32_t)a.in_cols, (cuuint32_t)a.in_rows, 1};
+    cuuint32_t es[4] = {1, 1, 1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 // ------------------------------------------------------------ bf16 rounding (host)
 
 uint16_t f32_to_bf16_rne(float f) {
@@ -190,9 +204,11 @@ struct LaunchPlan {
     int slab_rows = 0;  // slab mode: padded input rows per slab
     // constants: byte offsets into the constant blob
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
-    // depthwise / space-to-depth
+    // depthwise / space-to-depth / fused depthwise -> 1x1
     byoc::DwArgs dw{};
     byoc::S2dArgs s2d{};
+    byoc::DwPwArgs dp{};
+    size_t w2_off = 0, w2_bytes = 0, b2_off = 0, b2_bytes = 0;  // fused: the 1x1 conv's constants
     double flops = 0, bytes = 0;
 };
 
@@ -421,6 +437,17 @@ struct Affine {
     std::vector<double> scale, shift;
 };
 
+// Whether a depthwise composite and the 1x1 composite that consumes it, in
+// one region, are planned as one fused launch (dwpw.cu) rather than two.
+// Off unless BYOC_FUSE_DW_PW=1: on GB300 the fused kernel moves a third of
+// the bytes but its depthwise arithmetic, not HBM, bounds it, and the two
+// launches measure faster on the MobileNetV2 shapes.  Read at planning time,
+// so a compiled (or serialised) region keeps the choice it was made with.
+bool fuse_dw_pw() {
+    const char *f = std::getenv("BYOC_FUSE_DW_PW");
+    return f && f[0] == '1';
+}
+
 // Builds the launch list (no device work).
 byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
     P = Plan();
@@ -449,38 +476,52 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         const TensorInfo Yp = P.tensors[op.out];
         const int64_t Cout = Yp.channels();
         // ---------------- epilogue chain
-        Affine af;
-        af.scale.assign(Cout, 1.0);
-        af.shift.assign(Cout, 0.0);
-        int cur = op.out, res = -1, act = byoc::kActNone, stage = 0, j = o + 1;
-        for (; j < d->n_ops; ++j) {
-            const byoc_op &nx = d->ops[j];
-            const bool reads_cur = nx.in[0] == cur || (nx.kind == BYOC_OP_ADD && nx.in[1] == cur);
-            if (!reads_cur || consumers[cur] != 1 || is_output[cur]) break;
-            if (nx.kind == BYOC_OP_BIAS_ADD && stage == 0) {
-                for (int64_t c = 0; c < Cout; ++c) af.shift[c] += (double)nx.consts[0][c];
-            } else if (nx.kind == BYOC_OP_BATCH_NORM && stage == 0) {
-                for (int64_t c = 0; c < Cout; ++c) {
-                    const double s = (double)nx.consts[0][c] /
-                                     std::sqrt((double)nx.consts[3][c] + (double)nx.eps);
-                    af.scale[c] *= s;
-                    af.shift[c] = af.shift[c] * s + ((double)nx.consts[1][c] - s * (double)nx.consts[2][c]);
+        // Epilogue chain of the conv2d/dense at op `first`: the bias / batch
+        // norm (folded into af), residual add and activation ops that follow
+        // it, each the single consumer of the previous one.  Returns the index
+        // of the first op after the chain.
+        auto walk_chain = [&](int first, Affine &af, int &cur, int &res, int &act) -> int {
+            const int64_t Co = P.tensors[d->ops[first].out].channels();
+            af.scale.assign(Co, 1.0);
+            af.shift.assign(Co, 0.0);
+            cur = d->ops[first].out;
+            res = -1;
+            act = byoc::kActNone;
+            int stage = 0, jj = first + 1;
+            for (; jj < d->n_ops; ++jj) {
+                const byoc_op &nx = d->ops[jj];
+                const bool reads_cur = nx.in[0] == cur || (nx.kind == BYOC_OP_ADD && nx.in[1] == cur);
+                if (!reads_cur || consumers[cur] != 1 || is_output[cur]) break;
+                if (nx.kind == BYOC_OP_BIAS_ADD && stage == 0) {
+                    for (int64_t c = 0; c < Co; ++c) af.shift[c] += (double)nx.consts[0][c];
+                } else if (nx.kind == BYOC_OP_BATCH_NORM && stage == 0) {
+                    for (int64_t c = 0; c < Co; ++c) {
+                        const double s = (double)nx.consts[0][c] /
+                                         std::sqrt((double)nx.consts[3][c] + (double)nx.eps);
+                        af.scale[c] *= s;
+                        af.shift[c] = af.shift[c] * s + ((double)nx.consts[1][c] - s * (double)nx.consts[2][c]);
+                    }
+                } else if (nx.kind == BYOC_OP_ADD && stage == 0) {
+                    const int r2 = nx.in[0] == cur ? nx.in[1] : nx.in[0];
+                    if (r2 == cur) break;  // x + x: not a residual pattern
+                    res = r2;
+                    stage = 1;
+                } else if ((nx.kind == BYOC_OP_RELU || nx.kind == BYOC_OP_RELU6 ||
+                            nx.kind == BYOC_OP_GELU) && stage <= 1) {
+                    act = nx.kind == BYOC_OP_RELU ? byoc::kActRelu
+                                                  : (nx.kind == BYOC_OP_RELU6 ? byoc::kActRelu6
+                                                                              : byoc::kActGelu);
+                    stage = 2;
+                } else {
+                    break;
                 }
-            } else if (nx.kind == BYOC_OP_ADD && stage == 0) {
-                res = nx.in[0] == cur ? nx.in[1] : nx.in[0];
-                if (res == cur) break;  // x + x: not a residual pattern
-                stage = 1;
-            } else if ((nx.kind == BYOC_OP_RELU || nx.kind == BYOC_OP_RELU6 ||
-                        nx.kind == BYOC_OP_GELU) && stage <= 1) {
-                act = nx.kind == BYOC_OP_RELU ? byoc::kActRelu
-                                              : (nx.kind == BYOC_OP_RELU6 ? byoc::kActRelu6
-                                                                          : byoc::kActGelu);
-                stage = 2;
-            } else {
-                break;
+                cur = nx.out;
             }
-            cur = nx.out;
-        }
+            return jj;
+        };
+        Affine af;
+        int cur, res, act;
+        const int j = walk_chain(o, af, cur, res, act);
         const TensorInfo Y = P.tensors[cur];
         LaunchPlan L;
         L.first_op = o;
@@ -505,13 +546,76 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                 return fail(BYOC_ERR_UNSUPPORTED,
                             "op %d: depthwise supports 3x3, stride 1|2, symmetric padding", o);
             if (res >= 0) return fail(BYOC_ERR_UNSUPPORTED, "op %d: residual add after depthwise", o);
-            L.kind = BYOC_LAUNCH_DEPTHWISE;
             std::vector<float> w(9 * C), b(C);
             for (int64_t c = 0; c < C; ++c) {
                 for (int t = 0; t < 9; ++t)
                     w[t * C + c] = (float)((double)op.consts[0][c * 9 + t] * af.scale[c]);
                 b[c] = (float)af.shift[c];
             }
+            // Depthwise -> 1x1 conv in one launch (dwpw.cu) when the 1x1 conv
+            // is the depthwise output's only consumer: the intermediate stays
+            // in shared memory (the gain of merging the two composites into
+            // one region).
+            if (fuse_dw_pw() && j < d->n_ops && consumers[cur] == 1 && !is_output[cur] &&
+                act != byoc::kActGelu) {
+                const byoc_op &pw = d->ops[j];
+                if (pw.kind == BYOC_OP_CONV2D && pw.in[0] == cur && pw.groups == 1 && pw.kernel[0] == 1 &&
+                    pw.kernel[1] == 1 && pw.stride[0] == 1 && pw.stride[1] == 1 && pw.dilation[0] == 1 &&
+                    pw.dilation[1] == 1 && pw.pad[0] == 0 && pw.pad[1] == 0 && pw.pad[2] == 0 && pw.pad[3] == 0) {
+                    Affine af2;
+                    int cur2, res2, act2;
+                    const int j2 = walk_chain(j, af2, cur2, res2, act2);
+                    const TensorInfo Y2 = P.tensors[cur2];
+                    const int64_t Cout2 = Y2.channels();
+                    byoc::DwPwArgs dp{};
+                    dp.N = (int)X.shape[0];
+                    dp.H = (int)X.shape[1];
+                    dp.W = (int)X.shape[2];
+                    dp.C = (int)C;
+                    dp.Ho = (int)Y.shape[1];
+                    dp.Wo = (int)Y.shape[2];
+                    dp.stride = op.stride[0];
+                    dp.pad = op.pad[0];
+                    dp.dw_act = act;
+                    dp.act = act2;
+                    dp.Cout = (int)Cout2;
+                    if (act2 != byoc::kActGelu && byoc::dwpw_plan(dp, P.num_sms)) {
+                        L.kind = BYOC_LAUNCH_DWPW;
+                        L.n_ops = j2 - o;
+                        L.y = cur2;
+                        L.res = res2;
+                        L.act = act2;
+                        L.w_off = blob_append(P.blob, w.data(), w.size() * 4);
+                        L.w_bytes = w.size() * 4;
+                        L.b_off = blob_append(P.blob, b.data(), b.size() * 4);
+                        L.b_bytes = b.size() * 4;
+                        // 1x1 weights: folded, bf16 RNE, [n_pad][chunks * 64] K-major, zero padded
+                        L.n_pad = dp.n_pad;
+                        L.k_pack = dp.chunks * byoc::kDpChunk;
+                        std::vector<uint16_t> w2((size_t)L.n_pad * L.k_pack, 0);
+                        for (int64_t k = 0; k < Cout2; ++k)
+                            for (int64_t c = 0; c < C; ++c)
+                                w2[(size_t)k * L.k_pack + c] =
+                                    f32_to_bf16_rne((float)((double)pw.consts[0][k * C + c] * af2.scale[k]));
+                        std::vector<float> b2((size_t)L.n_pad, 0.0f);
+                        for (int64_t k = 0; k < Cout2; ++k) b2[k] = (float)af2.shift[k];
+                        L.w2_off = blob_append(P.blob, w2.data(), w2.size() * 2);
+                        L.w2_bytes = w2.size() * 2;
+                        L.b2_off = blob_append(P.blob, b2.data(), b2.size() * 4);
+                        L.b2_bytes = b2.size() * 4;
+                        L.dp = dp;
+                        L.grid = std::min(dp.num_tiles, P.num_sms);
+                        L.flops = 2.0 * (double)Y.elems() * 9.0 + 2.0 * (double)Y2.elems() * (double)C;
+                        L.bytes = (double)X.bytes() + (double)Y2.bytes() +
+                                  (res2 >= 0 ? (double)P.tensors[res2].bytes() : 0.0) +
+                                  (double)(w.size() + b.size()) * 4 + (double)Cout2 * C * 2 + (double)Cout2 * 4;
+                        P.launches.push_back(L);
+                        o = j2;
+                        continue;
+                    }
+                }
+            }
+            L.kind = BYOC_LAUNCH_DEPTHWISE;
             L.w_off = blob_append(P.blob, w.data(), w.size() * 4);
             L.w_bytes = w.size() * 4;
             L.b_off = blob_append(P.blob, b.data(), b.size() * 4);
@@ -810,11 +914,12 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
         r->n_ops[i] = L.n_ops;
         r->act[i] = L.act;
         r->residual[i] = L.res;
-        r->gemm_m[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.M : 0;
-        r->gemm_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.N : 0;
-        r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : 0;
-        r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : 0;
-        r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : 0;
+        const bool dp = L.kind == BYOC_LAUNCH_DWPW;
+        r->gemm_m[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.M : (dp ? L.dp.N * L.dp.Ho * L.dp.Wo : 0);
+        r->gemm_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.args.N : (dp ? L.dp.Cout : 0);
+        r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : (dp ? L.dp.C : 0);
+        r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : (dp ? L.dp.n_pad : 0);
+        r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : (dp ? byoc::kDpChunk : 0);
         r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? std::min(L.cfg.amode, (int)byoc::kAModeSlab) : 0;
         r->grid[i] = L.grid;
         r->resident_b[i] = L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeSlabRes ? 1 : 0;
@@ -873,8 +978,10 @@ byoc_status byoc_plan_constants(const byoc_region_desc *desc, int32_t num_sms, i
         return fail(BYOC_ERR_INVALID_ARG, "launch %d out of range", launch);
     const LaunchPlan &L = P.launches[launch];
     if (L.kind == BYOC_LAUNCH_S2D) return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants", launch);
-    const size_t off = what == 0 ? L.w_off : L.b_off;
-    const size_t n = what == 0 ? L.w_bytes : L.b_bytes;
+    if ((what < 0 || what > 3) || (what > 1 && L.kind != BYOC_LAUNCH_DWPW))
+        return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants of kind %d", launch, what);
+    const size_t off = what == 0 ? L.w_off : what == 1 ? L.b_off : what == 2 ? L.w2_off : L.b2_off;
+    const size_t n = what == 0 ? L.w_bytes : what == 1 ? L.b_bytes : what == 2 ? L.w2_bytes : L.b2_bytes;
     if (needed) *needed = n;
     if (!dst) return BYOC_OK;
     if (dst_bytes < n) return fail(BYOC_ERR_INVALID_ARG, "destination too small (%zu < %zu)", dst_bytes, n);
@@ -982,6 +1089,22 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
                 return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(weights) = %d", i, (int)r);
             }
             if ((e = byoc::gemm_prepare(L.cfg)) != cudaSuccess) {
+                byoc_release(h);
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            }
+        } else if (L.kind == BYOC_LAUNCH_DWPW) {
+            L.dp.dw_w = reinterpret_cast<const float *>(h->d_const + L.w_off);
+            L.dp.dw_b = reinterpret_cast<const float *>(h->d_const + L.b_off);
+            L.dp.pw_b = reinterpret_cast<const float *>(h->d_const + L.b2_off);
+            L.dp.err = h->d_err;
+            // the 1x1 weights: 64-channel x n_pad boxes, 128-byte swizzle (the MMA's B operand)
+            CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w2_off, (uint64_t)L.n_pad, (uint64_t)L.k_pack,
+                                   (uint32_t)L.n_pad, (uint32_t)byoc::kDpChunk, byoc::kDpChunk);
+            if (r != CUDA_SUCCESS) {
+                byoc_release(h);
+                return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(1x1 weights) = %d", i, (int)r);
+            }
+            if ((e = byoc::dwpw_prepare(L.dp)) != cudaSuccess) {
                 byoc_release(h);
                 return cuda_fail(e, "cudaFuncSetAttribute");
             }
@@ -1143,11 +1266,13 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
         if (P.ws_off[t] != SIZE_MAX && P.ws_off[t] + P.tensors[t].bytes() > P.ws_bytes)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: workspace layout out of range");
     for (const LaunchPlan &L : P.launches) {
-        if (L.kind != BYOC_LAUNCH_GEMM && L.kind != BYOC_LAUNCH_DEPTHWISE && L.kind != BYOC_LAUNCH_S2D)
+        if (L.kind != BYOC_LAUNCH_GEMM && L.kind != BYOC_LAUNCH_DEPTHWISE && L.kind != BYOC_LAUNCH_S2D &&
+            L.kind != BYOC_LAUNCH_DWPW)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad launch kind");
         if (L.x < 0 || L.x >= nt || L.y < 0 || L.y >= nt || L.res >= nt)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad tensor id in a launch");
-        if (L.w_off + L.w_bytes > P.blob.size() || L.b_off + L.b_bytes > P.blob.size())
+        if (L.w_off + L.w_bytes > P.blob.size() || L.b_off + L.b_bytes > P.blob.size() ||
+            L.w2_off + L.w2_bytes > P.blob.size() || L.b2_off + L.b2_bytes > P.blob.size())
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: constants out of range");
         if (L.kind == BYOC_LAUNCH_GEMM && !byoc::gemm_config_supported(L.cfg))
             return fail(BYOC_ERR_UNSUPPORTED, "serialised plan: tile configuration not in this build");
@@ -1295,6 +1420,19 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             byoc::DwArgs a = L.dw;
             a.y = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
             e = byoc::launch_dwconv(h->tmA[i], a, L.grid, st);
+        } else if (L.kind == BYOC_LAUNCH_DWPW) {
+            const void *xa = h->ptrs[L.x];
+            if (h->tmA_ptr[i] != xa) {
+                CUresult r = encode_dwpw_input(&h->tmA[i], xa, L.dp);
+                if (r != CUDA_SUCCESS)
+                    return fail(BYOC_ERR_CUDA, "launch %zu: encoding the depthwise input TMA map failed (%d)",
+                                i, (int)r);
+                h->tmA_ptr[i] = xa;
+            }
+            byoc::DwPwArgs a = L.dp;
+            a.out = static_cast<__nv_bfloat16 *>(h->ptrs[L.y]);
+            a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
+            e = byoc::launch_dwpw(h->tmA[i], h->tmB[i], a, L.grid, st);
         } else {
             byoc::S2dArgs a = L.s2d;
             a.x = reinterpret_cast<const __nv_bfloat16 *>(static_cast<const char *>(h->ptrs[L.x]) +

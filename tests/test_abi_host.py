@@ -50,7 +50,22 @@ def test_plan_fuses_composites_into_launches():
     rep = _plan(I.bert_ffn(M=64, D=128, F=256)[0])
     assert rep.n_launches == 2 and rep.act[0] == 3 and rep.act[1] == 0
     rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0])
-    assert [rep.kind[i] for i in range(2)] == [abi.LAUNCH_DEPTHWISE, abi.LAUNCH_GEMM]
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_DEPTHWISE, abi.LAUNCH_GEMM]
+    assert rep.act[0] == 2
+
+
+def test_plan_fuses_depthwise_into_the_pointwise_when_asked(monkeypatch):
+    # depthwise + BN + ReLU6 -> 1x1 + BN: one fused launch (the depthwise output stays on chip)
+    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
+    rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0])
+    assert rep.n_launches == 1 and rep.kind[0] == abi.LAUNCH_DWPW
+    assert rep.n_ops[0] == 5 and rep.act[0] == 0
+    assert (rep.gemm_m[0], rep.gemm_n[0], rep.gemm_k[0], rep.tile_n[0]) == (64, 24, 144, 32)
+    # a depthwise whose output is also a region output stays a launch of its own
+    g, _ = I.mbv2_dw_pw(N=1, H=8, W=8)
+    reg = R.Region(g, [n.name for n in g.nodes], "both", outputs=[g.nodes[2].name, g.outputs[0]])
+    rep = reg.plan()
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_DEPTHWISE, abi.LAUNCH_GEMM]
     assert rep.act[0] == 2
 
 
@@ -104,7 +119,8 @@ def test_plan_flops_match_mac_count():
         assert _plan(g).flops == pytest.approx(I.region_flops(g), rel=1e-12)
 
 
-def test_packed_weights_are_folded_rounded_and_k_major():
+def test_packed_weights_are_folded_rounded_and_k_major(monkeypatch):
+    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
     g, _ = I.conv_bias_relu(N=1, H=8, W=8, C=64, K=32, seed=3)
     g2, _ = I.mbv2_dw_pw(N=1, H=8, W=8, C=64, Cout=32)
     # conv -> bn (from the pointwise part of g2) : fold checked on the GEMM launch
@@ -115,12 +131,12 @@ def test_packed_weights_are_folded_rounded_and_k_major():
     s = bn.consts["gamma"].astype(np.float64) / np.sqrt(bn.consts["moving_var"].astype(np.float64) + 1e-5)
     shift = bn.consts["beta"] - s * bn.consts["moving_mean"]
     w = pw.consts["weight"][:, :, 0, 0].astype(np.float64) * s[:, None]
-    raw = np.frombuffer(reg.plan_constants(1, 0), dtype=np.uint16)
-    Kp = rep.gemm_k[1]
-    packed = raw.reshape(-1, Kp)
+    assert rep.kind[0] == abi.LAUNCH_DWPW
+    raw = np.frombuffer(reg.plan_constants(0, 2), dtype=np.uint16)   # the fused launch's 1x1 weights
+    packed = raw.reshape(rep.tile_n[0], -1)
+    assert packed.shape == (32, 64)
     assert np.array_equal(packed[:32, :64], I.bf16_bits(w.astype(np.float32)))
-    assert not packed[:32, 64:].any() and not packed[32:].any()
-    bias = np.frombuffer(reg.plan_constants(1, 1), dtype=np.float32)
+    bias = np.frombuffer(reg.plan_constants(0, 3), dtype=np.float32)
     np.testing.assert_allclose(bias[:32], shift, rtol=1e-6, atol=1e-7)
     # 3x3 conv: column index = (tap r*3+s) * Cin_pad + c
     reg = R.whole_graph_region(g)

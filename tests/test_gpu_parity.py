@@ -275,3 +275,54 @@ def test_nchw_boundary_rejects_bad_shapes_on_the_host():
     y = torch.zeros(1, 2, 2, 8, dtype=torch.bfloat16, device="cuda")
     assert abi.lib().byoc_nchw_to_nhwc_bf16(x.data_ptr(), y.data_ptr(), 1, 4, 2, 2, 3, None) == abi.ERR_INVALID_ARG
     assert abi.lib().byoc_nchw_to_nhwc_bf16(x.data_ptr(), y.data_ptr(), 1, 4, 2, 20000, 8, None) == abi.ERR_INVALID_ARG
+
+
+def _dw_pw_graph(N, H, W, C, Cout, stride, residual, seed, small_int=False):
+    b = I._Builder("dw_pw_case")
+    x = b.input("x", (N, H, W, C))
+    d = b.relu6(b.batch_norm(b.conv2d(x, C, 3, stride=stride, groups=C)))
+    y = b.batch_norm(b.conv2d(d, Cout, 1))
+    if residual:
+        Ho, Wo = (H - 1) // stride + 1, (W - 1) // stride + 1
+        r = b.input("r", (N, Ho, Wo, Cout))
+        y = b.add(y, r)
+    return I._finish(b, [y], seed)
+
+
+@pytest.mark.parametrize("N,H,W,C,Cout,stride,residual", [
+    (2, 13, 9, 48, 16, 1, False),     # fewer than 64 channels, ragged row tile
+    (1, 30, 30, 160, 40, 2, False),   # three channel chunks (64, 64, 32), stride 2, N padded to 48
+    (3, 7, 7, 96, 8, 1, True),        # 7x7 maps, one tile per image, residual, N padded to 16
+    (1, 112, 112, 32, 16, 1, False),  # 112-wide rows: one output row per tile
+    (2, 28, 28, 192, 64, 2, False),   # stride 2 at 28x28 (MobileNetV2 block 3 shape)
+    (2, 14, 14, 384, 64, 1, True),    # 6 chunks, 64 outputs, residual
+])
+def test_fused_depthwise_pointwise(N, H, W, C, Cout, stride, residual, monkeypatch):
+    # depthwise + BN + ReLU6 -> 1x1 + BN (+ residual) in one kernel against the
+    # oracle of the unfused chain
+    from paper_2105_03215_gb300 import abi
+    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
+    g, inp = _dw_pw_graph(N, H, W, C, Cout, stride, residual, seed=N + C + Cout)
+    rep = R.whole_graph_region(g).plan(152)
+    assert rep.n_launches == 1 and rep.kind[0] == abi.LAUNCH_DWPW
+    _check_graph(g, inp, what=f"dw_pw {N}x{H}x{W}x{C}->{Cout} s{stride} res{residual}")
+
+
+def test_fused_depthwise_pointwise_equals_the_two_launches_bit_for_bit(monkeypatch):
+    # the fused kernel rounds the depthwise output to bf16 and accumulates the
+    # 1x1 conv's K steps in the same order as the two separate launches, so the
+    # outputs agree bit for bit (separate launches: the depthwise output is
+    # also a region output, which keeps it out of the fusion)
+    import torch
+    from .parity import to_dev
+    g, inp = I.mbv2_dw_pw(N=4, H=28, W=28, C=144, Cout=24, seed=12)
+    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
+    fused = R.whole_graph_region(g)
+    split = R.Region(g, [n.name for n in g.nodes], "split", outputs=[g.nodes[2].name, g.outputs[0]])
+    got_f, cf = run_region(fused, inp)
+    got_s, cs = run_region(split, inp)
+    assert cf.n_launches == 1 and cs.n_launches == 2
+    a, b = got_f[g.outputs[0]], got_s[g.outputs[0]]
+    assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
+    cf.release()
+    cs.release()
