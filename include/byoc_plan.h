@@ -44,6 +44,7 @@ typedef struct {
     int32_t grid[BYOC_PLAN_MAX_LAUNCHES];       /* CTAs launched */
     int32_t resident_b[BYOC_PLAN_MAX_LAUNCHES]; /* 1: the weights are loaded once per CTA (slab mode) */
     int32_t slab_slots[BYOC_PLAN_MAX_LAUNCHES]; /* slab buffers in flight (slab mode), else 0 */
+    int32_t splits[BYOC_PLAN_MAX_LAUNCHES];     /* GEMM: CTAs sharing each tile's k-blocks (split-K), else 0 */
     double flops;
     double bytes;
     size_t const_bytes;

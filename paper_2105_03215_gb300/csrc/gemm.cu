@@ -105,6 +105,11 @@ __global__ void __maxnreg__(168)
                         const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
     using S = GemmShape<BN, BK, AMODE, RES>;
     constexpr int kEpiArrivals = BN <= 64 ? kGemmEpiWarps / 2 : kGemmEpiWarps;
+    // split-K: a work unit is (tile, split); split sp covers k-blocks
+    // [sp * num_kb / SPL, (sp + 1) * num_kb / SPL)
+    constexpr bool SPLITK = AMODE == kAModeTileSplit;
+    const int SPL = SPLITK ? a.splits : 1;
+    const int num_units = a.num_tiles * SPL;
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -172,7 +177,7 @@ __global__ void __maxnreg__(168)
     // prefetches this CTA's first tile's weight rows into L2 while the
     // previous kernel finishes.
     pdl_launch_dependents();
-    if (warp == kGemmOperandWarp && a.w != nullptr && (int)blockIdx.x < a.num_tiles) {
+    if (!SPLITK && warp == kGemmOperandWarp && a.w != nullptr && (int)blockIdx.x < a.num_tiles) {
         if (elect_one()) {
             const size_t row_bytes = (size_t)a.k_pack * 2;
             const uint8_t *src =
@@ -227,7 +232,9 @@ __global__ void __maxnreg__(168)
                     ok = false;
                 }
             }
-            for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x) {
+            for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
+                const int tile = unit / SPL;
+                const int sp = unit - tile * SPL;
                 const int mt = tile / a.tiles_n;
                 const int n0 = (tile % a.tiles_n) * BN;
                 if constexpr (S::WRES) {
@@ -285,8 +292,10 @@ __global__ void __maxnreg__(168)
                         w0 = q * a.stride_w - a.pad_l;
                     }
                     int cc = 0, r = 0, sx = 0;  // (tap r, s; chunk cc) of k-block kb, im2col mode
-                    for (int kb = 0; kb < a.num_kb; kb += G) {
-                        const int gn = a.num_kb - kb < G ? a.num_kb - kb : G;
+                    const int kb_lo = SPLITK ? sp * a.num_kb / SPL : 0;
+                    const int kb_hi = SPLITK ? (sp + 1) * a.num_kb / SPL : a.num_kb;
+                    for (int kb = kb_lo; kb < kb_hi; kb += G) {
+                        const int gn = kb_hi - kb < G ? kb_hi - kb : G;
                         if (!claim((uint32_t)(gn * S::STAGE_BYTES))) {
                             ok = false;
                             break;
@@ -327,7 +336,8 @@ __global__ void __maxnreg__(168)
         if (elect_one()) {
             // ------------------------------------------------ epilogue-operand producer
             int t = 0;
-            for (int tile = blockIdx.x; tile < a.num_tiles; tile += gridDim.x, ++t) {
+            for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++t) {
+                const int tile = unit / SPL;
                 const int ob = t % S::OPB;
                 const uint32_t oph = (uint32_t)(t / S::OPB) & 1u;
                 if (!mbar_wait(oempty + 8u * ob, oph ^ 1u, abort_flag, a.err, kErrTimeoutProducer))
@@ -382,7 +392,8 @@ __global__ void __maxnreg__(168)
                     phase ^= 1u;
                 }
             };
-            for (int tile = blockIdx.x; ok && tile < a.num_tiles; tile += gridDim.x, ++t) {
+            for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++t) {
+                const int sp = unit - (unit / SPL) * SPL;
                 const int buf = t & 1;
                 const uint32_t aph = (uint32_t)(t >> 1) & 1u;
                 if (!wait(tempty + 8u * buf, aph ^ 1u)) {
@@ -465,8 +476,10 @@ __global__ void __maxnreg__(168)
                         mma_commit(sempty + 8u * ss);  // frees the slab
                     }
                 } else {
-                    for (int kb = 0; kb < a.num_kb; kb += G) {
-                        const int gn = a.num_kb - kb < G ? a.num_kb - kb : G;
+                    const int kb_lo = SPLITK ? sp * a.num_kb / SPL : 0;
+                    const int kb_hi = SPLITK ? (sp + 1) * a.num_kb / SPL : a.num_kb;
+                    for (int kb = kb_lo; kb < kb_hi; kb += G) {
+                        const int gn = kb_hi - kb < G ? kb_hi - kb : G;
                         if (!wait(bars + 8u * stage, phase)) {
                             ok = false;
                             break;
@@ -514,8 +527,9 @@ __global__ void __maxnreg__(168)
         const int cl_row = lane >> 2, cl_piece = lane & 3;  // coalesced: rows 8k + lane/4
         const int t_first = ALT ? grp : 0, t_step = ALT ? 2 : 1;
         const int c_first = ALT ? 0 : grp, c_step = ALT ? 1 : 2;
-        for (int tile = blockIdx.x + t_first * (int)gridDim.x, t = t_first; tile < a.num_tiles;
-             tile += t_step * (int)gridDim.x, t += t_step) {
+        for (int unit = blockIdx.x + t_first * (int)gridDim.x, t = t_first; unit < num_units;
+             unit += t_step * (int)gridDim.x, t += t_step) {
+            const int tile = unit / SPL;
             const int buf = t & 1;
             const uint32_t aph = (uint32_t)(t >> 1) & 1u;
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
@@ -547,8 +561,54 @@ __global__ void __maxnreg__(168)
                 tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
             const uint32_t bias_s = sBias + (uint32_t)(ob * S::BIAS_BYTES);
             const uint32_t res_s = sRes + (uint32_t)(ob * S::RES_TILE);
+            // split-K: every split writes its fp32 partial of this warp's rows
+            // and columns, then counts itself in on the tile's counter for this
+            // warp's slot; the split that completes the count sums all partials
+            // in split order (the same bits whichever split finishes last) and
+            // runs the epilogue.  No split waits for another.
+            const int sp = unit - tile * SPL;
+            // Partials are laid out the way the warp reads TMEM, not as the
+            // output matrix: per (tile, warp slot, chunk) 32 x 32 fp32 with
+            // the 16-byte piece q of lane l at (q * 32 + l) * 16 bytes, so
+            // every store (and every load of the last split) is a contiguous
+            // 512-byte run.  Only the same (slot, lane) of another split ever
+            // reads it.
+            const int slot = ALT ? quarter : quarter * 2 + grp;
+            constexpr int kSlotFloats = (ALT ? NCH : NCH / 2) * 1024;
+            const size_t pbase = SPLITK ? (size_t)tile * (size_t)(S::BM * BN) + (size_t)slot * kSlotFloats +
+                                              (size_t)lane * 4
+                                        : 0;
+            const size_t pstride = SPLITK ? (size_t)a.num_tiles * (size_t)(S::BM * BN) : 0;  // one split
+            if constexpr (SPLITK) {
 #pragma unroll 1
-            for (int ci = c_first; ci < NCH; ci += c_step) {
+                for (int ci = c_first, k = 0; ci < NCH; ci += c_step, ++k) {
+                    uint32_t v[32];
+                    tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
+                    float *dst = a.partial + (size_t)sp * pstride + pbase + (size_t)k * 1024;
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        *reinterpret_cast<uint4 *>(dst + q * 128) =
+                            make_uint4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+                }
+                __threadfence();
+                __syncwarp();
+                unsigned old = 0u;
+                if (lane == 0) old = atomicAdd(a.counters + (size_t)tile * 8 + slot, 1u);
+                old = __shfl_sync(0xffffffffu, old, 0);
+                if (old % (unsigned)SPL != (unsigned)(SPL - 1)) {
+                    // not the last split of this tile: release the accumulator and operands
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(tempty + 8u * buf);
+                        mbar_arrive(oempty + 8u * ob);
+                    }
+                    continue;
+                }
+                __threadfence();  // the other splits' partials are read after the count
+            }
+#pragma unroll 1
+            for (int ci = c_first, kk = 0; ci < NCH; ci += c_step, ++kk) {
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);  // includes tcgen05.wait::ld
@@ -556,6 +616,30 @@ __global__ void __maxnreg__(168)
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty + 8u * buf);
+                }
+                if constexpr (SPLITK) {
+                    float sum[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) sum[j] = 0.0f;
+                    for (int s2 = 0; s2 < SPL; ++s2) {
+                        if (s2 == sp) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) sum[j] += __uint_as_float(v[j]);
+                        } else {
+                            const float *src = a.partial + (size_t)s2 * pstride + pbase + (size_t)kk * 1024;
+#pragma unroll
+                            for (int q = 0; q < 8; ++q) {
+                                // L2: written by other CTAs
+                                const float4 p4 = __ldcg(reinterpret_cast<const float4 *>(src + q * 128));
+                                sum[4 * q] += p4.x;
+                                sum[4 * q + 1] += p4.y;
+                                sum[4 * q + 2] += p4.z;
+                                sum[4 * q + 3] += p4.w;
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
                 }
                 float f[32];
 #pragma unroll
@@ -688,6 +772,9 @@ static cudaError_t prepare_t() {
     X(256, 64, kAModeSlab, false)     \
     X(64, 16, kAModeSlab, false)      \
     X(64, 32, kAModeSlab, false)      \
+    X(64, 64, kAModeTileSplit, false) \
+    X(128, 64, kAModeTileSplit, false) \
+    X(256, 64, kAModeTileSplit, false) \
     X(64, 64, kAModeSlabRes, false)   \
     X(128, 64, kAModeSlabRes, false)  \
     X(64, 16, kAModeSlabRes, false)   \

@@ -66,6 +66,12 @@ struct GemmArgs {
     int slab_off;       // bytes from the start of the pool to the first slab slot
     int slab_pitch;     // bytes per slot, a multiple of 1024
     int slab_slots;     // 2 .. kMaxSlabSlots
+    // split-K (kAModeTileSplit): fp32 partials [splits][m_pad][n_pad] and one
+    // arrival counter per (tile, epilogue warp slot), zeroed once, counted
+    // modulo `splits`
+    int splits, m_pad, n_pad;
+    float *partial;
+    unsigned *counters;
     int group;      // k-blocks (slab mode: filter taps) per ring stage, >= 1; the
                     // kernel lowers it so that at least two stages fit the ring
     // packed weights [n_pad][k_pack] (bf16), or null: before waiting for the
@@ -83,7 +89,8 @@ enum AMode : int {
     kAModeTile = 0,    // A is a row-major [M, K] matrix (2-D tiled TMA)
     kAModeIm2col = 1,  // A through an im2col TMA map: one load per filter tap and chunk
     kAModeSlab = 2,    // stride-1 conv: one 4-D tiled slab per chunk, taps by row shift
-    kAModeSlabRes = 3  // slab mode, one column tile, all weights resident in shared memory
+    kAModeSlabRes = 3,  // slab mode, one column tile, all weights resident in shared memory
+    kAModeTileSplit = 4  // tile mode with the k-blocks of every tile split over `splits` CTAs
 };
 
 struct GemmConfig {

@@ -202,6 +202,8 @@ struct LaunchPlan {
     Im2colGeom geo{};
     int64_t aM = 0, aK = 0;
     int slab_rows = 0;  // slab mode: padded input rows per slab
+    // split-K scratch (handle workspace): fp32 partials and arrival counters
+    size_t part_off = 0, part_bytes = 0, cnt_off = 0, cnt_bytes = 0;
     // constants: byte offsets into the constant blob
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
     // depthwise / space-to-depth / fused depthwise -> 1x1
@@ -390,25 +392,42 @@ int pick_bk(int64_t C) {
 //                        per accumulator row block work in parallel).
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
 // time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
-int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool res, int num_sms) {
-    int best = -1;
+//   split-K (tile mode, no residual, one wave of units only): S splits of
+//                        kblocks / S each; every split writes and fences its
+//                        fp32 partial (~26 bn cycles, traced) and the last one
+//                        reads the other S - 1 back (~10 bn cycles each)
+//                        before the epilogue.
+int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool res, int num_sms,
+            int *splits_out = nullptr) {
+    int best = -1, best_s = 1;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
         GemmConfig c{bn, bk, amode, res};
         if (!byoc::gemm_config_supported(c)) continue;
         const int64_t tiles = tiles_m * ((N + bn - 1) / bn);
-        const int64_t grid = std::min<int64_t>(tiles, num_sms);
-        const int64_t rounds = (tiles + grid - 1) / grid;
         const double kb = amode == byoc::kAModeSlab ? std::max(2.5 * bn * bk / 64.0, 150.0)
                                                     : std::max(2.5 * bn, 450.0);
-        const double mainloop = 300.0 + (double)kblocks * kb;
         const double epilogue = 600.0 * std::max(1, bn / 64);
-        const double cost = (double)rounds * std::max(mainloop, epilogue) + std::min(mainloop, epilogue);
-        if (cost < best_cost - 1e-9) {
-            best_cost = cost;
-            best = bn;
+        for (int S = 1; S <= 4; ++S) {
+            if (S > 1 && (!splits_out || amode != byoc::kAModeTile || res || kblocks < 4 * S ||
+                          tiles * S > num_sms ||
+                          !byoc::gemm_config_supported(GemmConfig{bn, bk, byoc::kAModeTileSplit, false})))
+                continue;
+            const int64_t units = tiles * S;
+            const int64_t grid = std::min<int64_t>(units, num_sms);
+            const int64_t rounds = (units + grid - 1) / grid;
+            const double mainloop = 300.0 + (double)((kblocks + S - 1) / S) * kb;
+            const double cost =
+                S == 1 ? (double)rounds * std::max(mainloop, epilogue) + std::min(mainloop, epilogue)
+                       : mainloop + 26.0 * bn + 10.0 * bn * (S - 1) + epilogue;
+            if (cost < best_cost - 1e-9) {
+                best_cost = cost;
+                best = bn;
+                best_s = S;
+            }
         }
     }
+    if (splits_out) *splits_out = best_s;
     return best;
 }
 
@@ -792,11 +811,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         const int amode = slab ? byoc::kAModeSlab : (im2col ? byoc::kAModeIm2col : byoc::kAModeTile);
         const int64_t tiles_per_img = slab ? (Y.shape[1] + sgeo.t - 1) / sgeo.t : 0;
         const int64_t tiles_m = slab ? X.shape[0] * tiles_per_img : (M + 127) / 128;
-        const int bn = pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms);
+        int splits = 1;
+        const int bn = pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms, &splits);
         if (bn < 0)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
                         o, bk, amode, (int)has_res);
-        L.cfg = GemmConfig{bn, bk, amode, has_res};
+        L.cfg = GemmConfig{bn, bk, splits > 1 ? byoc::kAModeTileSplit : amode, has_res};
         if (slab && Cout <= bn) {
             // one column tile: keep the whole weight matrix in shared memory
             // when it fits beside two slabs
@@ -845,10 +865,17 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         A.tiles_n = L.n_pad / bn;
         A.num_tiles = (int)(tiles_m * A.tiles_n);
         A.taps = taps;
-        A.group = byoc::gemm_group(bn, bk, amode == byoc::kAModeSlab ? taps : A.num_kb);
+        A.group = byoc::gemm_group(bn, bk, amode == byoc::kAModeSlab ? taps : (A.num_kb + splits - 1) / splits);
         byoc::gemm_slab_pool(L.cfg, A);
+        A.splits = splits;
+        A.m_pad = (int)(tiles_m * byoc::kGemmBM);
+        A.n_pad = L.n_pad;
+        if (splits > 1) {
+            L.part_bytes = (size_t)splits * A.m_pad * A.n_pad * 4;
+            L.cnt_bytes = (size_t)A.num_tiles * 8 * 4;
+        }
+        L.grid = std::min(A.num_tiles * splits, P.num_sms);
         A.act = act;
-        L.grid = std::min(A.num_tiles, P.num_sms);
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
         const double in_bytes = stem_k > 0 ? 0.0  // z: counted as x by the transform
                                 : L.x < P.n_region_tensors ? (double)X.bytes()
@@ -896,6 +923,14 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         P.ws_off[t] = ws;
         ws = align_up(ws + P.tensors[t].bytes(), 256);
     }
+    for (LaunchPlan &L : P.launches) {
+        if (L.part_bytes) {
+            L.part_off = ws;
+            ws = align_up(ws + L.part_bytes, 256);
+            L.cnt_off = ws;
+            ws = align_up(ws + L.cnt_bytes, 256);
+        }
+    }
     P.ws_bytes = ws;
     for (const LaunchPlan &L : P.launches) {
         P.flops += L.flops;
@@ -920,7 +955,10 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
         r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : (dp ? L.dp.C : 0);
         r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : (dp ? L.dp.n_pad : 0);
         r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : (dp ? byoc::kDpChunk : 0);
-        r->im2col[i] = L.kind == BYOC_LAUNCH_GEMM ? std::min(L.cfg.amode, (int)byoc::kAModeSlab) : 0;
+        r->im2col[i] = L.kind != BYOC_LAUNCH_GEMM || L.cfg.amode == byoc::kAModeTileSplit
+                           ? 0
+                           : std::min(L.cfg.amode, (int)byoc::kAModeSlab);
+        r->splits[i] = L.kind == BYOC_LAUNCH_GEMM ? std::max(1, L.args.splits) : 0;
         r->grid[i] = L.grid;
         r->resident_b[i] = L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeSlabRes ? 1 : 0;
         r->slab_slots[i] = L.kind != BYOC_LAUNCH_GEMM ? 0
@@ -1081,6 +1119,14 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
             L.args.err = h->d_err;
             L.args.w = h->d_const + L.w_off;
             L.args.k_pack = L.k_pack;
+            if (L.part_bytes) {
+                L.args.partial = reinterpret_cast<float *>(h->d_ws + L.part_off);
+                L.args.counters = reinterpret_cast<unsigned *>(h->d_ws + L.cnt_off);
+                if ((e = cudaMemset(h->d_ws + L.cnt_off, 0, L.cnt_bytes)) != cudaSuccess) {
+                    byoc_release(h);
+                    return cuda_fail(e, "cudaMemset(split-K counters)");
+                }
+            }
             CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
                                    (uint64_t)L.k_pack, (uint32_t)L.cfg.bn, (uint32_t)L.cfg.bk,
                                    L.cfg.bk);
@@ -1274,6 +1320,8 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
         if (L.w_off + L.w_bytes > P.blob.size() || L.b_off + L.b_bytes > P.blob.size() ||
             L.w2_off + L.w2_bytes > P.blob.size() || L.b2_off + L.b2_bytes > P.blob.size())
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: constants out of range");
+        if (L.part_off + L.part_bytes > P.ws_bytes || L.cnt_off + L.cnt_bytes > P.ws_bytes)
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: split-K scratch out of range");
         if (L.kind == BYOC_LAUNCH_GEMM && !byoc::gemm_config_supported(L.cfg))
             return fail(BYOC_ERR_UNSUPPORTED, "serialised plan: tile configuration not in this build");
     }

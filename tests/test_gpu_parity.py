@@ -326,3 +326,33 @@ def test_fused_depthwise_pointwise_equals_the_two_launches_bit_for_bit(monkeypat
     assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
     cf.release()
     cs.release()
+
+
+@pytest.mark.parametrize("M,Iw,U", [(100, 3072, 256), (1024, 3072, 768), (64, 2048, 1000), (7, 1024, 40)])
+def test_split_k_dense_matches_and_is_deterministic(M, Iw, U):
+    # deep reductions over few tiles run split-K: every split writes an fp32
+    # partial, the last to arrive sums them in split order -- within tolerance
+    # of the oracle, and the same bits on every run
+    import torch
+    from .parity import to_dev
+    b = I._Builder("dense_deep")
+    x = b.input("x", (M, Iw))
+    y = b.bias_add(b.dense(x, U))
+    g, inp = I._finish(b, [y], seed=M + U)
+    reg = R.whole_graph_region(g)
+    rep = reg.plan(152)
+    got, cr = run_region(reg, inp)
+    assert_close(got[g.outputs[0]], ograph.evaluate(g, inp)[g.outputs[0]], f"dense {M}x{Iw}->{U}")
+    out = torch.empty(g.shape_of(g.outputs[0]), dtype=torch.bfloat16, device="cuda")
+    xs = [to_dev(inp["x"])]
+    ref_bits = None
+    for _ in range(3):
+        cr.run(xs, [out])
+        torch.cuda.synchronize()
+        bits = out.view(torch.int16).cpu().numpy().copy()
+        ref_bits = bits if ref_bits is None else ref_bits
+        assert np.array_equal(bits, ref_bits)
+    cr.check()
+    cr.release()
+    if (M, Iw, U) == (1024, 3072, 768):
+        assert rep.splits[0] == 3
