@@ -174,8 +174,10 @@ __global__ void __maxnreg__(168)
     // Set-up done: the next kernel may be scheduled; global memory is touched
     // only after the previous kernel has completed -- except for the packed
     // weights, constant for the handle's lifetime: the operand warp
-    // prefetches this CTA's first tile's weight rows into L2 while the
-    // previous kernel finishes.
+    // prefetches this CTA's first tile's weight rows into L2, and the
+    // producer loads the first ring stages' weights (resident-weight mode:
+    // all of them) into shared memory, while the previous kernel finishes;
+    // the producer waits for it only before its first activation load.
     pdl_launch_dependents();
     if (!SPLITK && warp == kGemmOperandWarp && a.w != nullptr && (int)blockIdx.x < a.num_tiles) {
         if (elect_one()) {
@@ -188,7 +190,7 @@ __global__ void __maxnreg__(168)
         }
         __syncwarp();
     }
-    pdl_wait();
+    if (warp != 0) pdl_wait();
     // Ring stages of G k-blocks each; at least two stages.
     const int G = a.group < 1 ? 1 : (a.group > S::STAGES / 2 ? S::STAGES / 2 : a.group);
     const int nst = S::STAGES / G;
@@ -232,6 +234,30 @@ __global__ void __maxnreg__(168)
                     ok = false;
                 }
             }
+            // Tile / im2col / split modes: claim the first unit's first ring
+            // stages and load their weights before waiting for the previous
+            // kernel; their activations follow the wait (same stage barriers).
+            // (measured: the same for the ringed slab mode's first chunk costs
+            // ~2 us on the ResNet-50 step, so that mode waits first)
+            int pre = 0;
+            if constexpr (!S::SLAB) {
+                if ((int)blockIdx.x < num_units) {
+                    const int u0 = blockIdx.x;
+                    const int t0 = u0 / SPL, sp0 = u0 - (u0 / SPL) * SPL;
+                    const int n00 = (t0 % a.tiles_n) * BN;
+                    const int lo = SPLITK ? sp0 * a.num_kb / SPL : 0;
+                    const int hi = SPLITK ? (sp0 + 1) * a.num_kb / SPL : a.num_kb;
+                    for (int kb = lo; kb < hi && pre < nst; kb += G, ++pre) {
+                        const int gn = hi - kb < G ? hi - kb : G;
+                        // fresh ring: stage pre is free; the full barrier expects A and B
+                        mbar_arrive_expect_tx(bars + 8u * pre, (uint32_t)(gn * S::STAGE_BYTES));
+                        for (int g = 0; g < gn; ++g)
+                            tma_load_2d(sB + (pre * G + g) * S::B_BYTES, &tmB, bars + 8u * pre, (kb + g) * BK,
+                                        n00);
+                    }
+                }
+            }
+            pdl_wait();
             for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
                 const int tile = unit / SPL;
                 const int sp = unit - tile * SPL;
@@ -296,7 +322,10 @@ __global__ void __maxnreg__(168)
                     const int kb_hi = SPLITK ? (sp + 1) * a.num_kb / SPL : a.num_kb;
                     for (int kb = kb_lo; kb < kb_hi; kb += G) {
                         const int gn = kb_hi - kb < G ? kb_hi - kb : G;
-                        if (!claim((uint32_t)(gn * S::STAGE_BYTES))) {
+                        const bool preloaded = pre > 0;  // claimed, weights issued before the wait
+                        if (preloaded) {
+                            --pre;
+                        } else if (!claim((uint32_t)(gn * S::STAGE_BYTES))) {
                             ok = false;
                             break;
                         }
@@ -316,7 +345,8 @@ __global__ void __maxnreg__(168)
                             } else {
                                 tma_load_2d(dA, &tmA, full, (kb + g) * BK, m0);
                             }
-                            tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, full, (kb + g) * BK, n0);
+                            if (!preloaded)
+                                tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, full, (kb + g) * BK, n0);
                         }
                         advance();
                     }
