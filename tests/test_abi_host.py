@@ -104,14 +104,18 @@ def test_stem_weights_follow_the_space_to_depth_definition():
 
 
 def test_stem_runs_in_image_chunks_that_fit_l2():
+    # stacked z: 112 x 115 x 64 bf16 = 1.65 MB per image; chunks of <= 128 MB
     g, _ = I.stem(N=64, H=224, W=224)
     rep = R.whole_graph_region(g).plan()
-    # stacked z: 112 x 115 x 64 bf16 = 1.65 MB per image -> 4 chunks of 16 images
-    assert rep.n_launches == 8
-    assert [rep.kind[i] for i in range(8)] == [abi.LAUNCH_S2D, abi.LAUNCH_GEMM] * 4
-    assert all(rep.gemm_m[i] == 16 * 112 * 112 for i in range(1, 8, 2))
-    assert rep.workspace_bytes <= 256 + 16 * 112 * 115 * 64 * 2 + 256
+    assert rep.n_launches == 2 and rep.gemm_m[1] == 64 * 112 * 112
     assert rep.flops == pytest.approx(2.0 * 64 * 112 * 112 * 64 * 7 * 7 * 3, rel=1e-12)
+    g, _ = I.stem(N=170, H=224, W=224)
+    rep = R.whole_graph_region(g).plan()
+    # 170 x 1,648,640 bytes = 2.09 x 128 MiB -> 3 chunks of 57, 57, 56 images
+    assert rep.n_launches == 6
+    assert [rep.kind[i] for i in range(6)] == [abi.LAUNCH_S2D, abi.LAUNCH_GEMM] * 3
+    assert [rep.gemm_m[i] for i in (1, 3, 5)] == [57 * 12544, 57 * 12544, 56 * 12544]
+    assert rep.workspace_bytes <= 256 + 57 * 112 * 115 * 64 * 2 + 256
 
 
 def test_plan_flops_match_mac_count():

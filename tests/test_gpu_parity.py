@@ -149,12 +149,31 @@ def test_stem_variants(k, cout, C):
 
 
 def test_stem_in_image_chunks_with_a_ragged_last_chunk():
-    # 21 images of 224 x 224: the stacked space-to-depth tensor (1.65 MB per
-    # image) is processed as two launch pairs, of 11 and 10 images
-    g, inp = I.stem(N=21, H=224, W=224, seed=17)
-    rep = R.whole_graph_region(g).plan()
-    assert rep.n_launches == 4 and rep.gemm_m[1] == 11 * 112 * 112 and rep.gemm_m[3] == 10 * 112 * 112
-    _check_graph(g, inp, what="stem in chunks")
+    # 83 images of 224 x 224: the stacked space-to-depth tensor (1.65 MB per
+    # image, 137 MB) runs as two launch pairs, of 42 and 41 images; the oracle
+    # checks 3000 sampled outputs, half of them in the second chunk
+    import torch
+    from oracle import ops
+    from .parity import to_dev
+    g, inp = I.stem(N=83, H=224, W=224, seed=17)
+    reg = R.whole_graph_region(g)
+    rep = reg.plan()
+    assert rep.n_launches == 4 and rep.gemm_m[1] == 42 * 112 * 112 and rep.gemm_m[3] == 41 * 112 * 112
+    got, cr = run_region(reg, inp)
+    y = got[g.outputs[0]].reshape(-1, 64)
+    rng = np.random.default_rng(3)
+    half = 42 * 112 * 112
+    pix = np.concatenate([rng.integers(0, half, 1500), rng.integers(half, 83 * 112 * 112, 1500)])
+    ks = rng.integers(0, 64, 3000)
+    conv, bn = g.nodes[0], g.nodes[1]
+    a = conv.attrs
+    v = ops.conv2d_nhwc_sampled(inp["data"], conv.consts["weight"], pix, ks, a["strides"], a["padding"],
+                                a["dilation"], a["groups"]).reshape(1, -1)
+    v = ops.batch_norm(v, bn.consts["gamma"][ks], bn.consts["beta"][ks], bn.consts["moving_mean"][ks],
+                       bn.consts["moving_var"][ks], bn.attrs.get("epsilon", 1e-5))
+    ref = ops.relu(v).ravel()
+    assert_close(y[pix, ks], ref, "stem chunks (sampled)")
+    cr.release()
 
 
 def test_gelu_epilogue_within_one_bf16_ulp():
