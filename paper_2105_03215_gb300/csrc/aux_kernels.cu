@@ -473,42 +473,67 @@ __global__ void maxpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, 
     *reinterpret_cast<uint4 *>(y + (((size_t)n * Ho + pp) * Wo + q) * C + cv * 8) = pack8(m);
 }
 
-// 3x3 window, fully unrolled: all nine loads issue before the first max.
+// 3x3 window (stride s, padding p): a thread computes two horizontally
+// adjacent outputs of one 8-channel vector; their windows share a column at
+// stride 2, so 15 loads (all issued before the first max) serve both.  The
+// max of bf16 values is one of them, so it is taken on the packed pairs
+// (max.bf16x2), with no conversion.  Out-of-image positions are clamped to
+// the nearest in-window position (the padding never wins).
+__device__ __forceinline__ uint4 max8(const uint4 &a, const uint4 &b) {
+    uint4 r;
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r.x) : "r"(a.x), "r"(b.x));
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r.y) : "r"(a.y), "r"(b.y));
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r.z) : "r"(a.z), "r"(b.z));
+    asm("max.bf16x2 %0, %1, %2;" : "=r"(r.w) : "r"(a.w), "r"(b.w));
+    return r;
+}
+
 __global__ void maxpool3_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                                 int s, int p, int Ho, int Wo) {
     pdl_launch_dependents();
     pdl_wait();
     const int CV = C >> 3;
-    const long long total = (long long)N * Ho * Wo * CV;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    const int Wq = (Wo + 1) >> 1;  // output column pairs
+    const int total = N * Ho * Wq * CV;
+    const int idx = (int)(blockIdx.x * blockDim.x + threadIdx.x);
     if (idx >= total) return;
-    const int cv = (int)(idx % CV);
-    long long t = idx / CV;
-    const int q = (int)(t % Wo);
-    t /= Wo;
-    const int pp = (int)(t % Ho);
-    const int n = (int)(t / Ho);
+    const int cv = idx % CV;
+    int t = idx / CV;
+    const int qp = t % Wq;
+    t /= Wq;
+    const int pp = t % Ho;
+    const int n = t / Ho;
+    const int q0 = 2 * qp;
+    const bool two = q0 + 1 < Wo;
     const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
-    uint4 v[9];
+    // columns of the two windows: q0*s - p + {0, 1, 2} and (q0+1)*s - p + {0, 1, 2}
+    int col[6];
+#pragma unroll
+    for (int c = 0; c < 3; ++c) {
+        col[c] = min(max(q0 * s - p + c, 0), W - 1);
+        col[3 + c] = min(max((two ? q0 + 1 : q0) * s - p + c, 0), W - 1);
+    }
+    uint4 m0 = make_uint4(0, 0, 0, 0), m1 = m0;
 #pragma unroll
     for (int r = 0; r < 3; ++r) {
-        const int h = min(max(pp * s - p + r, 0), H - 1);  // nearest in-window position
+        const int h = min(max(pp * s - p + r, 0), H - 1);  // nearest in-window row
+        const __nv_bfloat16 *row = xn + (size_t)h * W * C;
+        uint4 v[6];
 #pragma unroll
-        for (int c = 0; c < 3; ++c) {
-            const int w = min(max(q * s - p + c, 0), W - 1);
-            v[r * 3 + c] = ldg_v4(xn + ((size_t)h * W + w) * C);
+        for (int c = 0; c < 6; ++c) {
+            // at stride 2 the second window's first column is the first window's last
+            if (c == 3 && s == 2) continue;
+            v[c] = ldg_v4(row + (size_t)col[c] * C);
         }
+        if (s == 2) v[3] = v[2];
+        const uint4 a = max8(max8(v[0], v[1]), v[2]);
+        const uint4 b = max8(max8(v[3], v[4]), v[5]);
+        m0 = r == 0 ? a : max8(m0, a);
+        m1 = r == 0 ? b : max8(m1, b);
     }
-    float m[8];
-    unpack8(v[0], m);
-#pragma unroll
-    for (int i = 1; i < 9; ++i) {
-        float f[8];
-        unpack8(v[i], f);
-#pragma unroll
-        for (int j = 0; j < 8; ++j) m[j] = fmaxf(m[j], f[j]);
-    }
-    *reinterpret_cast<uint4 *>(y + (((size_t)n * Ho + pp) * Wo + q) * C + cv * 8) = pack8(m);
+    __nv_bfloat16 *yo = y + (((size_t)n * Ho + pp) * Wo + q0) * C + cv * 8;
+    *reinterpret_cast<uint4 *>(yo) = m0;
+    if (two) *reinterpret_cast<uint4 *>(yo + C) = m1;
 }
 
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
@@ -516,9 +541,10 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
     if (k == 3) {
         const int Ho = (H + 2 * p - 3) / s + 1;
         const int Wo = (W + 2 * p - 3) / s + 1;
-        const long long total = (long long)N * Ho * Wo * (C / 8);
-        return launch_pdl(maxpool3_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y,
-                          N, H, W, C, s, p, Ho, Wo);
+        const long long total = (long long)N * Ho * ((Wo + 1) / 2) * (C / 8);
+        if (total < (1ll << 31))
+            return launch_pdl(maxpool3_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y,
+                              N, H, W, C, s, p, Ho, Wo);
     }
     const int Ho = (H + 2 * p - k) / s + 1;
     const int Wo = (W + 2 * p - k) / s + 1;

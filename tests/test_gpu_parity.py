@@ -375,3 +375,22 @@ def test_split_k_dense_matches_and_is_deterministic(M, Iw, U):
     cr.release()
     if (M, Iw, U) == (1024, 3072, 768):
         assert rep.splits[0] == 3
+
+
+@pytest.mark.parametrize("N,H,W,C,s", [(2, 15, 13, 64, 2), (1, 9, 10, 16, 1), (3, 112, 112, 64, 2), (1, 7, 1, 8, 2)])
+def test_max_pool_3x3_host_operator_bit_exact(N, H, W, C, s):
+    # the host max pool (padding 1): two outputs per thread, packed bf16 max --
+    # the max of bf16 values is one of them, so the result is exact
+    import torch
+    from oracle import ops
+    from paper_2105_03215_gb300 import abi
+    from .parity import to_dev
+    rng = np.random.default_rng(N * 31 + W)
+    x = I.bf16_round(rng.standard_normal((N, H, W, C)).astype(np.float32))
+    Ho, Wo = (H + 2 - 3) // s + 1, (W + 2 - 3) // s + 1
+    xd = to_dev(x)
+    y = torch.full((N, Ho, Wo, C), float("nan"), dtype=torch.bfloat16, device="cuda")
+    abi.check(abi.lib().byoc_max_pool2d_nhwc(xd.data_ptr(), y.data_ptr(), N, H, W, C, 3, s, 1, None))
+    torch.cuda.synchronize()
+    ref = ops.max_pool2d_nhwc(x, (3, 3), (s, s), (1, 1, 1, 1))
+    assert_bit_exact(y.float().cpu().numpy(), ref, f"maxpool {N}x{H}x{W}x{C} s{s}")
