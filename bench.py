@@ -471,7 +471,7 @@ def main():
             continue
         c = ex.compiled[x]
         if c.n_launches != 1:
-            continue  # the stem region also runs its space-to-depth transform
+            continue  # the stem region also runs its input layout transform
         gemm_t += t
         gemm_f += c.flops
         gemm_b += c.bytes

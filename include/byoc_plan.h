@@ -24,7 +24,7 @@ extern "C" {
 typedef enum {
     BYOC_LAUNCH_GEMM = 0,      /* tcgen05 implicit-GEMM conv2d / dense + fused epilogue */
     BYOC_LAUNCH_DEPTHWISE = 1, /* depthwise 3x3 conv + fused epilogue */
-    BYOC_LAUNCH_S2D = 2,       /* space-to-depth boundary transform of a stride-2 stem */
+    BYOC_LAUNCH_S2D = 2,       /* layout transform of a stride-2 few-channel stem (4-channel, zero-padded pixel pairs) */
     BYOC_LAUNCH_DWPW = 3       /* depthwise 3x3 + epilogue fused with the 1x1 conv + epilogue after it */
 } byoc_launch_kind;
 
@@ -45,6 +45,8 @@ typedef struct {
     int32_t resident_b[BYOC_PLAN_MAX_LAUNCHES]; /* 1: the weights are loaded once per CTA (slab mode) */
     int32_t slab_slots[BYOC_PLAN_MAX_LAUNCHES]; /* slab buffers in flight (slab mode), else 0 */
     int32_t splits[BYOC_PLAN_MAX_LAUNCHES];     /* GEMM: CTAs sharing each tile's k-blocks (split-K), else 0 */
+    int32_t pair_units[BYOC_PLAN_MAX_LAUNCHES]; /* 1: slab-mode units of two adjacent 128-row tiles
+                                                   sharing each weight k-block, else 0 */
     double flops;
     double bytes;
     size_t const_bytes;

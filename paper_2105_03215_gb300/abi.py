@@ -65,7 +65,7 @@ class PlanReport(ctypes.Structure):
                 ("gemm_m", c_int32 * _L), ("gemm_n", c_int32 * _L), ("gemm_k", c_int32 * _L),
                 ("tile_n", c_int32 * _L), ("tile_k", c_int32 * _L), ("im2col", c_int32 * _L),
                 ("grid", c_int32 * _L), ("resident_b", c_int32 * _L), ("slab_slots", c_int32 * _L),
-                ("splits", c_int32 * _L),
+                ("splits", c_int32 * _L), ("pair_units", c_int32 * _L),
                 ("flops", c_double), ("bytes", c_double),
                 ("const_bytes", c_size_t), ("workspace_bytes", c_size_t)]
 

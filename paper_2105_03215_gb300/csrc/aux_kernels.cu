@@ -253,114 +253,78 @@ cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cud
     return launch_pdl(dw_kernel(a), dim3(grid), dim3(a.threads), dw_smem_bytes(a), st, tmX, a);
 }
 
-// ------------------------------------------------------------ space-to-depth
-// z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c].
-// Block (p, n): output row p of image n.  Its input rows 2p-pad ..
-// 2p-pad+2*taps-1 are one contiguous run of x; the block stages them in
-// shared memory (zero rows outside the image; 16-byte loads, four in flight
-// per thread), assembles the output row there -- per (column j, stacked
-// tap) one 16-channel group -- and writes it out with coalesced 16-byte
-// stores.  Staged rows are padded by 8 elements so that the stacked taps of
-// one column fall in different banks.
-// C is a template parameter so that the 16 channel values stay in registers.
+// ------------------------------------------------------------ stem input layout
+// xq[n, u, v, c] = x[n, u - pad, v - pad, c] for c < C inside x, else 0 (see
+// StemArgs).  Block (u-block, n): kStemRows rows of xq.  The input rows under
+// them are staged in shared memory first -- 16-byte loads when a row is a
+// whole number of 16-byte pieces, all of a block's loads in flight at once,
+// since the transform is bound by memory latency -- then each thread writes
+// 16-byte pixel pairs (coalesced across the warp).  C is a template parameter
+// so that the pair assembly unrolls.
+constexpr int kStemRows = 8;
+
 template <int C>
-__global__ void __launch_bounds__(256) s2d_kernel(const S2dArgs a) {
+__global__ void __launch_bounds__(256) stem_layout_kernel(const StemArgs a, int vec) {
     pdl_launch_dependents();
     pdl_wait();
-    extern __shared__ __align__(16) unsigned short smem_s2d[];
-    const int p = blockIdx.x;
+    extern __shared__ __align__(16) unsigned short srow[];  // [kStemRows][W * C]
     const int n = blockIdx.y;
-    const int rows = 2 * a.taps;
+    const int u0 = blockIdx.x * kStemRows;
     const int row_elems = a.W * C;
-    const int pitch = ((row_elems + 7) & ~7) + 8;  // staged row pitch (elements, 16-byte multiple)
-    unsigned short *srows = smem_s2d;
-    uint4 *sout = reinterpret_cast<uint4 *>(smem_s2d + (size_t)rows * pitch);
-    const int h0 = 2 * p - a.pad;
-    const unsigned short *xs = reinterpret_cast<const unsigned short *>(a.x);
-    if ((row_elems & 7) == 0) {
-        const int vec_row = row_elems >> 3;
-        const int total = rows * vec_row;
-        for (int base = threadIdx.x; base < total; base += 4 * blockDim.x) {
-            uint4 v[4];
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int i = base + k * (int)blockDim.x;
-                const int r = i / vec_row;
-                const int h = h0 + r;
-                v[k] = make_uint4(0u, 0u, 0u, 0u);
-                if (i < total && h >= 0 && h < a.H)
-                    v[k] = __ldg(reinterpret_cast<const uint4 *>(xs + ((size_t)n * a.H + h) * row_elems) +
-                                 (i - r * vec_row));
-            }
-#pragma unroll
-            for (int k = 0; k < 4; ++k) {
-                const int i = base + k * (int)blockDim.x;
-                const int r = i / vec_row;
-                if (i < total)
-                    *reinterpret_cast<uint4 *>(srows + (size_t)r * pitch + 8 * (i - r * vec_row)) = v[k];
-            }
+    const unsigned short *xs = reinterpret_cast<const unsigned short *>(a.x) + (size_t)n * a.H * row_elems;
+    if (vec) {
+        const int pieces = row_elems >> 3;
+        for (int i = threadIdx.x; i < kStemRows * pieces; i += blockDim.x) {
+            const int r = i / pieces, q = i - r * pieces;
+            const int h = u0 + r - a.pad;
+            if (u0 + r < a.Hq && h >= 0 && h < a.H)
+                reinterpret_cast<uint4 *>(srow + (size_t)r * row_elems)[q] =
+                    __ldg(reinterpret_cast<const uint4 *>(xs + (size_t)h * row_elems) + q);
         }
     } else {
-        for (int i = threadIdx.x; i < rows * row_elems; i += blockDim.x) {
-            const int r = i / row_elems;
-            const int h = h0 + r;
-            srows[(size_t)r * pitch + (i - r * row_elems)] =
-                (h >= 0 && h < a.H) ? __ldg(xs + ((size_t)n * a.H + h) * row_elems + (i - r * row_elems))
-                                    : (unsigned short)0;
+        for (int i = threadIdx.x; i < kStemRows * row_elems; i += blockDim.x) {
+            const int r = i / row_elems, q = i - r * row_elems;
+            const int h = u0 + r - a.pad;
+            if (u0 + r < a.Hq && h >= 0 && h < a.H) srow[(size_t)r * row_elems + q] = __ldg(xs + (size_t)h * row_elems + q);
         }
     }
     __syncthreads();
-    const int groups = a.Wz * a.taps;
-    for (int idx = threadIdx.x; idx < groups; idx += blockDim.x) {
-        const int j = idx / a.taps;
-        const int tap = idx - j * a.taps;
-        uint32_t v[16];
+    const int pairs = a.Wq >> 1;
+    for (int i = threadIdx.x; i < kStemRows * pairs; i += blockDim.x) {
+        const int r = i / pairs, j = i - r * pairs;
+        const int u = u0 + r;
+        if (u >= a.Hq) break;  // i grows with r: the rest of this thread's items are past Hq too
+        const int h = u - a.pad;
+        const bool row_in = h >= 0 && h < a.H;
+        const unsigned short *sr = srow + (size_t)r * row_elems;
+        uint32_t v[8];
 #pragma unroll
-        for (int k = 0; k < 16; ++k) v[k] = 0u;
+        for (int dx = 0; dx < 2; ++dx) {
+            const int w = 2 * j + dx - a.pad;
+            const bool in = row_in && w >= 0 && w < a.W;
 #pragma unroll
-        for (int dy = 0; dy < 2; ++dy) {
-            const unsigned short *row = srows + (size_t)(2 * tap + dy) * pitch;
-#pragma unroll
-            for (int dx = 0; dx < 2; ++dx) {
-                const int w = 2 * j + dx - a.pad;
-                if (w < 0 || w >= a.W) continue;
-#pragma unroll
-                for (int c = 0; c < C; ++c) v[(dy * 2 + dx) * C + c] = row[w * C + c];
-            }
+            for (int c = 0; c < 4; ++c) v[dx * 4 + c] = (in && c < C) ? (uint32_t)sr[w * C + c] : 0u;
         }
-        sout[2 * idx] = make_uint4(v[0] | v[1] << 16, v[2] | v[3] << 16, v[4] | v[5] << 16,
-                                   v[6] | v[7] << 16);
-        sout[2 * idx + 1] = make_uint4(v[8] | v[9] << 16, v[10] | v[11] << 16,
-                                       v[12] | v[13] << 16, v[14] | v[15] << 16);
+        reinterpret_cast<uint4 *>(a.xq + ((size_t)n * a.Hq + u) * a.Wq * 4)[j] =
+            make_uint4(v[0] | v[1] << 16, v[2] | v[3] << 16, v[4] | v[5] << 16, v[6] | v[7] << 16);
     }
-    __syncthreads();
-    uint4 *zrow = reinterpret_cast<uint4 *>(a.z + ((size_t)n * a.Hz + p) * (size_t)groups * 16);
-    for (int i = threadIdx.x; i < 2 * groups; i += blockDim.x) zrow[i] = sout[i];
 }
 
-size_t s2d_smem_bytes(const S2dArgs &a) {
-    return (size_t)2 * a.taps * (((a.W * a.C + 7) & ~7) + 8) * 2 + (size_t)a.Wz * a.taps * 32;
-}
+size_t stem_layout_smem_bytes(const StemArgs &a) { return (size_t)kStemRows * a.W * a.C * 2; }
 
-cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st) {
-    const size_t smem = s2d_smem_bytes(a);
-    if (smem > kS2dMaxSmem) return cudaErrorInvalidValue;
-    if (smem > 48 * 1024) {
-        const void *fns[4] = {(const void *)s2d_kernel<1>, (const void *)s2d_kernel<2>,
-                              (const void *)s2d_kernel<3>, (const void *)s2d_kernel<4>};
-        for (const void *f : fns) {
-            cudaError_t e =
-                cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kS2dMaxSmem);
-            if (e != cudaSuccess) return e;
-        }
-    }
-    const dim3 grid((unsigned)a.Hz, (unsigned)a.N);
+cudaError_t launch_stem_layout(const StemArgs &a, cudaStream_t st) {
+    const size_t smem = stem_layout_smem_bytes(a);
+    if (a.Hq < 1 || a.N < 1 || a.N > 65535 || (a.Wq & 1) || a.Wq < 2 || a.C < 1 || a.C > 4 ||
+        smem > kStemLayoutMaxSmem)
+        return cudaErrorInvalidValue;
+    // 16-byte staging loads when every input row starts on a 16-byte boundary
+    const int vec = (a.W * a.C) % 8 == 0 && (reinterpret_cast<uintptr_t>(a.x) & 15) == 0;
+    const dim3 grid((unsigned)((a.Hq + kStemRows - 1) / kStemRows), (unsigned)a.N);
     switch (a.C) {
-        case 1: return launch_pdl(s2d_kernel<1>, grid, dim3(256), smem, st, a);
-        case 2: return launch_pdl(s2d_kernel<2>, grid, dim3(256), smem, st, a);
-        case 3: return launch_pdl(s2d_kernel<3>, grid, dim3(256), smem, st, a);
-        case 4: return launch_pdl(s2d_kernel<4>, grid, dim3(256), smem, st, a);
-        default: return cudaErrorInvalidValue;
+        case 1: return launch_pdl(stem_layout_kernel<1>, grid, dim3(256), smem, st, a, vec);
+        case 2: return launch_pdl(stem_layout_kernel<2>, grid, dim3(256), smem, st, a, vec);
+        case 3: return launch_pdl(stem_layout_kernel<3>, grid, dim3(256), smem, st, a, vec);
+        default: return launch_pdl(stem_layout_kernel<4>, grid, dim3(256), smem, st, a, vec);
     }
 }
 

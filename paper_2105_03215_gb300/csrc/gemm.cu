@@ -45,18 +45,23 @@ namespace byoc {
 template <int BN, int BK, int AMODE, bool RES>
 struct GemmShape {
     static constexpr int BM = kGemmBM;
-    static constexpr bool SLAB = AMODE == kAModeSlab || AMODE == kAModeSlabRes;
-    static constexpr bool WRES = AMODE == kAModeSlabRes;  // weights resident
+    static constexpr bool SLAB = amode_slab(AMODE);
+    static constexpr bool WRES = amode_wres(AMODE);  // weights resident
+    static constexpr bool PAIR = amode_pair(AMODE);  // two tiles (halves) per unit
+    static constexpr int HALVES = PAIR ? 2 : 1;
+    static_assert(!PAIR || WRES, "pair units keep their weights resident");
     static constexpr int ROW_BYTES = BK * 2;  // one K-major operand row (= swizzle width)
     static constexpr int A_BYTES = SLAB ? 0 : BM * BK * 2;
     static constexpr int B_BYTES = BN * BK * 2;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
-    static constexpr int SLAB_BYTES = SLAB ? slab_max_bytes(BK) : 0;
+    static constexpr int SLAB_BYTES = SLAB ? slab_max_bytes(BK, PAIR) : 0;
     // slab barriers: two slots beside a weight ring; up to kMaxSlabSlots
     // beside resident weights (the ring and the two largest slabs form one
     // pool, split at run time)
     static constexpr int SLOTS_MAX = WRES ? kMaxSlabSlots : 2;
-    static constexpr int TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;
+    // two accumulators (double buffer), each HALVES x BN columns
+    static constexpr int ACC_COLS = HALVES * BN;
+    static constexpr int TMEM_COLS = 2 * ACC_COLS < 32 ? 32 : 2 * ACC_COLS;
     // residual tile: BN/64 boxes of 64 columns x 128 rows, 128-byte swizzle
     static constexpr int RES_BOX = BM * 64 * 2;
     static constexpr int RES_TILE = RES ? BM * BN * 2 : 0;
@@ -82,10 +87,34 @@ struct GemmShape {
     static_assert(A_BYTES % 1024 == 0 && B_BYTES % 1024 == 0 && SLAB_BYTES % 1024 == 0,
                   "buffers must keep 1 KB alignment");
     static_assert(BN % 32 == 0 && BN >= 32 && BN <= 256, "BN");
+    static_assert(TMEM_COLS <= 512, "TMEM: two accumulators of HALVES x BN columns");
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
     static_assert(!(RES && SLAB), "slab tiles skip pad columns; no residual tile");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
 };
+
+// Slab modes: image, first output row and tile count (halves) of m-unit mt.
+// Single-tile modes: tile mt of tiles_per_img per image.  Pair modes: tiles
+// 2u and 2u + 1 of an image, the second absent past the image's last tile.
+struct SlabUnit {
+    int img, p0, nh;
+};
+template <bool PAIR>
+__device__ __forceinline__ SlabUnit slab_unit(const GemmArgs &a, int mt) {
+    SlabUnit u;
+    if constexpr (PAIR) {
+        const int upi = (a.tiles_per_img + 1) >> 1;
+        u.img = mt / upi;
+        const int pu = mt - u.img * upi;
+        u.p0 = 2 * pu * a.slab_t;
+        u.nh = 2 * pu + 1 < a.tiles_per_img ? 2 : 1;
+    } else {
+        u.img = mt / a.tiles_per_img;
+        u.p0 = (mt - u.img * a.tiles_per_img) * a.slab_t;
+        u.nh = 1;
+    }
+    return u;
+}
 
 // ReLU, ReLU6 or none; GELU is applied to lane pairs (gelu2) by the caller.
 __device__ __forceinline__ float apply_act(float v, int act) {
@@ -104,7 +133,11 @@ __global__ void __maxnreg__(168)
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
     using S = GemmShape<BN, BK, AMODE, RES>;
-    constexpr int kEpiArrivals = BN <= 64 ? kGemmEpiWarps / 2 : kGemmEpiWarps;
+    constexpr bool PAIR = S::PAIR;
+    // epilogue warps that read each accumulator: one group of four for
+    // narrow single tiles (groups alternate tiles), both groups otherwise
+    // (wide tiles: alternate 32-column chunks; pair units: one half each)
+    constexpr int kEpiArrivals = BN <= 64 && !PAIR ? kGemmEpiWarps / 2 : kGemmEpiWarps;
     // split-K: a work unit is (tile, split); split sp covers k-blocks
     // [sp * num_kb / SPL, (sp + 1) * num_kb / SPL)
     constexpr bool SPLITK = AMODE == kAModeTileSplit;
@@ -264,24 +297,28 @@ __global__ void __maxnreg__(168)
                 const int mt = tile / a.tiles_n;
                 const int n0 = (tile % a.tiles_n) * BN;
                 if constexpr (S::WRES) {
-                    const int img = mt / a.tiles_per_img;
-                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
+                    const SlabUnit su = slab_unit<PAIR>(a, mt);
+                    const int img = su.img, p0 = su.p0;
                     for (int cc = 0; cc < a.chunks; ++cc, ++sl) {
                         if (!wait(sempty + 8u * ss, sph ^ 1u)) {
                             ok = false;
                             break;
                         }
                         mbar_arrive_expect_tx(sfull + 8u * ss, (uint32_t)a.slab_bytes);
-                        tma_load_4d(sSlab + (uint32_t)(ss * a.slab_pitch), &tmA, sfull + 8u * ss,
-                                    cc * BK, -a.pad_l, p0 - a.pad_t, img);
+                        if (a.stem_rows > 0)  // stem layout: one chunk
+                            tma_load_5d(sSlab + (uint32_t)(ss * a.slab_pitch), &tmA, sfull + 8u * ss, 0, 0, p0, 0,
+                                        img);
+                        else
+                            tma_load_4d(sSlab + (uint32_t)(ss * a.slab_pitch), &tmA, sfull + 8u * ss,
+                                        cc * BK, -a.pad_l, p0 - a.pad_t, img);
                         if (++ss == a.slab_slots) {
                             ss = 0;
                             sph ^= 1u;
                         }
                     }
-                } else if constexpr (AMODE == kAModeSlab) {
-                    const int img = mt / a.tiles_per_img;
-                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
+                } else if constexpr (S::SLAB) {
+                    const SlabUnit su = slab_unit<PAIR>(a, mt);
+                    const int img = su.img, p0 = su.p0;
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
                         const int ss = sl & 1;
                         const uint32_t sph = (uint32_t)(sl >> 1) & 1u;
@@ -290,8 +327,11 @@ __global__ void __maxnreg__(168)
                             break;
                         }
                         mbar_arrive_expect_tx(sfull + 8u * ss, (uint32_t)a.slab_bytes);
-                        tma_load_4d(sSlab + ss * S::SLAB_BYTES, &tmA, sfull + 8u * ss, cc * BK,
-                                    -a.pad_l, p0 - a.pad_t, img);
+                        if (a.stem_rows > 0)  // stem layout: one chunk
+                            tma_load_5d(sSlab + ss * S::SLAB_BYTES, &tmA, sfull + 8u * ss, 0, 0, p0, 0, img);
+                        else
+                            tma_load_4d(sSlab + ss * S::SLAB_BYTES, &tmA, sfull + 8u * ss, cc * BK,
+                                        -a.pad_l, p0 - a.pad_t, img);
                         for (int tap = 0, kb = cc; tap < a.taps; tap += G) {
                             const int gn = a.taps - tap < G ? a.taps - tap : G;
                             if (!claim((uint32_t)(gn * S::B_BYTES))) {
@@ -402,7 +442,16 @@ __global__ void __maxnreg__(168)
                 return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutMma);
             };
             constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
-            const uint64_t adesc0 = make_smem_desc(S::SLAB ? sSlab : sA, S::ROW_BYTES);
+            // Slab operands, in descriptor units (16 bytes): pos_u per slab
+            // position (= operand row) and k_u per K16 slice.  TMA-swizzled
+            // slabs: rows of ROW_BYTES, a slice 32 bytes on.  Stem slabs (row
+            // planes, no swizzle): rows 16 bytes apart, a slice two planes on.
+            const bool planes = S::SLAB && a.stem_rows > 0;
+            const uint32_t plane = planes ? (uint32_t)a.slab_bytes / (uint32_t)a.stem_rows : 0u;
+            const uint32_t pos_u = planes ? 1u : (uint32_t)(S::ROW_BYTES >> 4);
+            const uint32_t k_u = planes ? 2u * (plane >> 4) : 2u;
+            const uint64_t adesc0 = planes ? make_smem_desc_planes(sSlab, plane)
+                                           : make_smem_desc(S::SLAB ? sSlab : sA, S::ROW_BYTES);
             const uint64_t bdesc0 = make_smem_desc(sB, S::ROW_BYTES);
             int stage = 0, slot0 = 0;
             uint32_t phase = 0;
@@ -410,6 +459,9 @@ __global__ void __maxnreg__(168)
             int ss = 0;        // resident weights: slab slot and its phase
             uint32_t sph = 0;
             bool ok = true;
+            // pair units: the second half's rows start slab_t padded rows
+            // further into the slab; its accumulator BN columns further on
+            const uint64_t hoff = PAIR ? (uint64_t)((uint32_t)(a.slab_t * a.wp) * pos_u) : 0;
             if constexpr (S::WRES) {  // the resident weights, once per CTA
                 ok = wait(bars, 0u);
                 tc_fence_after();
@@ -431,11 +483,12 @@ __global__ void __maxnreg__(168)
                     break;
                 }
                 tc_fence_after();
-                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+                const uint32_t d_tmem = tmem_base + (uint32_t)(buf * S::ACC_COLS);
                 uint32_t acc = 0u;
+                bool two = false;  // pair unit with both halves present
+                if constexpr (PAIR) two = slab_unit<true>(a, unit / a.tiles_n).nh == 2;
                 if constexpr (S::WRES) {
                     // k-block of filter tap t and chunk cc sits at t * chunks + cc
-                    const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
                     const uint64_t bstep = (uint64_t)((uint32_t)(a.chunks * S::B_BYTES) >> 4);
                     for (int cc = 0; ok && cc < a.chunks; ++cc) {
                         if (!wait(sfull + 8u * ss, sph)) {
@@ -445,20 +498,25 @@ __global__ void __maxnreg__(168)
                         tc_fence_after();
                         const uint64_t slab_desc =
                             adesc0 + (uint64_t)((uint32_t)(ss * a.slab_pitch) >> 4);
-                        uint32_t roff = 0;  // r * wp * ROW_BYTES of the current tap (r, sx)
+                        uint32_t rpos = 0;  // r * wp: first slab position of filter row r
                         int sx = 0;
                         uint64_t bd = bdesc0 + (uint64_t)((uint32_t)(cc * S::B_BYTES) >> 4);
                         for (int tap = 0; tap < a.taps; ++tap, bd += bstep) {
-                            const uint64_t ad =
-                                slab_desc + (uint64_t)((roff + (uint32_t)sx * S::ROW_BYTES) >> 4);
+                            const uint64_t ad = slab_desc + (uint64_t)((rpos + (uint32_t)sx) * pos_u);
 #pragma unroll
                             for (int k = 0; k < BK / 16; ++k)
-                                mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                mma_bf16_ss(d_tmem, ad + (uint64_t)(k * k_u), bd + (uint64_t)(2 * k), idesc,
                                             acc | (uint32_t)k);
+                            if (PAIR && two) {
+#pragma unroll
+                                for (int k = 0; k < BK / 16; ++k)
+                                    mma_bf16_ss(d_tmem + (uint32_t)BN, ad + hoff + (uint64_t)(k * k_u),
+                                                bd + (uint64_t)(2 * k), idesc, acc | (uint32_t)k);
+                            }
                             acc = 1u;
                             if (++sx == a.kw) {
                                 sx = 0;
-                                roff += row_step;
+                                rpos += (uint32_t)a.wp;
                             }
                         }
                         mma_commit(sempty + 8u * ss);  // frees the slab
@@ -467,8 +525,7 @@ __global__ void __maxnreg__(168)
                             sph ^= 1u;
                         }
                     }
-                } else if constexpr (AMODE == kAModeSlab) {
-                    const uint32_t row_step = (uint32_t)a.wp * S::ROW_BYTES;  // one filter row
+                } else if constexpr (S::SLAB) {
                     for (int cc = 0; ok && cc < a.chunks; ++cc, ++sl) {
                         const int ss = sl & 1;
                         if (!wait(sfull + 8u * ss, (uint32_t)(sl >> 1) & 1u)) {
@@ -476,7 +533,7 @@ __global__ void __maxnreg__(168)
                             break;
                         }
                         const uint64_t slab_desc = adesc0 + (uint64_t)((ss * S::SLAB_BYTES) >> 4);
-                        uint32_t roff = 0;  // r * wp * ROW_BYTES of the current tap (r, sx)
+                        uint32_t rpos = 0;  // r * wp: first slab position of filter row r
                         int sx = 0;
                         for (int tap = 0; tap < a.taps; tap += G) {
                             const int gn = a.taps - tap < G ? a.taps - tap : G;
@@ -487,16 +544,15 @@ __global__ void __maxnreg__(168)
                             tc_fence_after();
                             uint64_t bd = bdesc0 + (uint64_t)((slot0 * S::B_BYTES) >> 4);
                             for (int g = 0; g < gn; ++g, bd += (uint64_t)(S::B_BYTES >> 4)) {
-                                const uint64_t ad =
-                                    slab_desc + (uint64_t)((roff + (uint32_t)sx * S::ROW_BYTES) >> 4);
+                                const uint64_t ad = slab_desc + (uint64_t)((rpos + (uint32_t)sx) * pos_u);
 #pragma unroll
                                 for (int k = 0; k < BK / 16; ++k)
-                                    mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k),
+                                    mma_bf16_ss(d_tmem, ad + (uint64_t)(k * k_u), bd + (uint64_t)(2 * k),
                                                 idesc, acc | (uint32_t)k);
                                 acc = 1u;
                                 if (++sx == a.kw) {
                                     sx = 0;
-                                    roff += row_step;
+                                    rpos += (uint32_t)a.wp;
                                 }
                             }
                             mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
@@ -545,8 +601,9 @@ __global__ void __maxnreg__(168)
         // BN <= 64: the two groups take alternate tiles (accumulator t % 2), all
         // chunks each.  BN >= 128: both groups take every tile, group `grp`
         // the chunks ci with ci % 2 == grp, so that a tile's accumulator is
-        // read, and released to the MMAs, twice as fast.
-        constexpr bool ALT = BN <= 64;
+        // read, and released to the MMAs, twice as fast.  Pair units: group
+        // `grp` takes half `grp` of every unit, all chunks.
+        constexpr bool ALT = BN <= 64 && !PAIR;
         const int grp = e >> 2;
         const uint32_t stg = sEpi + (uint32_t)e * S::EPI_TILE;
         const int trow = quarter * 32 + lane;  // this thread's row within the tile
@@ -556,7 +613,8 @@ __global__ void __maxnreg__(168)
         const uint32_t sw_own = ((uint32_t)lane >> 1) & 3u;
         const int cl_row = lane >> 2, cl_piece = lane & 3;  // coalesced: rows 8k + lane/4
         const int t_first = ALT ? grp : 0, t_step = ALT ? 2 : 1;
-        const int c_first = ALT ? 0 : grp, c_step = ALT ? 1 : 2;
+        const int c_first = ALT || PAIR ? 0 : grp, c_step = ALT || PAIR ? 1 : 2;
+        const int half = PAIR ? grp : 0;
         for (int unit = blockIdx.x + t_first * (int)gridDim.x, t = t_first; unit < num_units;
              unit += t_step * (int)gridDim.x, t += t_step) {
             const int tile = unit / SPL;
@@ -570,25 +628,41 @@ __global__ void __maxnreg__(168)
             tc_fence_after();
             const int mt = tile / a.tiles_n;
             const int n0 = (tile % a.tiles_n) * BN;
+            int img = 0, p0 = 0;
+            if constexpr (S::SLAB) {
+                const SlabUnit su = slab_unit<PAIR>(a, mt);
+                if (PAIR && half >= su.nh) {
+                    // single tile at the end of an image: nothing for this
+                    // group; its arrivals still count the unit in
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) {
+                        mbar_arrive(tempty + 8u * buf);
+                        mbar_arrive(oempty + 8u * ob);
+                    }
+                    continue;
+                }
+                img = su.img;
+                p0 = su.p0 + half * a.slab_t;
+            }
             // output pixel (row of out / residual) of the 4 rows this lane stores, or -1
             int orow[4];
 #pragma unroll
             for (int k = 0; k < 4; ++k) {
                 const int v = quarter * 32 + 8 * k + cl_row;
                 if constexpr (S::SLAB) {
-                    const int img = mt / a.tiles_per_img;
-                    const int p0 = (mt - img * a.tiles_per_img) * a.slab_t;
                     const int y = v / a.wp;
                     const int x = v - y * a.wp;
-                    const bool ok = y < a.slab_t && x < a.Wo && p0 + y < a.Ho;
-                    orow[k] = ok ? (img * a.Ho + p0 + y) * a.Wo + x : -1;
+                    const int row = (img * a.Ho + p0 + y) * a.Wo + x;
+                    const bool ok = y < a.slab_t && x < a.Wo && p0 + y < a.Ho && row < a.M;
+                    orow[k] = ok ? row : -1;
                 } else {
                     const int row = mt * S::BM + v;
                     orow[k] = row < a.M ? row : -1;
                 }
             }
-            const uint32_t tbase =
-                tmem_base + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(buf * BN);
+            const uint32_t tbase = tmem_base + ((uint32_t)(quarter * 32) << 16) +
+                                   (uint32_t)(buf * S::ACC_COLS + half * BN);
             const uint32_t bias_s = sBias + (uint32_t)(ob * S::BIAS_BYTES);
             const uint32_t res_s = sRes + (uint32_t)(ob * S::RES_TILE);
             // split-K: every split writes its fp32 partial of this warp's rows
@@ -808,7 +882,10 @@ static cudaError_t prepare_t() {
     X(64, 64, kAModeSlabRes, false)   \
     X(128, 64, kAModeSlabRes, false)  \
     X(64, 16, kAModeSlabRes, false)   \
-    X(64, 32, kAModeSlabRes, false)
+    X(64, 32, kAModeSlabRes, false)   \
+    X(64, 64, kAModeSlabRes2, false)  \
+    X(128, 64, kAModeSlabRes2, false) \
+    X(64, 32, kAModeSlabRes2, false)
 
 bool gemm_config_supported(const GemmConfig &c) {
 #define X(BN_, BK_, AM_, RES_) \
@@ -833,12 +910,12 @@ bool gemm_slab_res_fits(const GemmConfig &c, int num_kb, int slab_bytes) {
     int pool, bbytes;
     slab_pool_shape(c, pool, bbytes);
     const int pitch = (slab_bytes + 1023) / 1024 * 1024;
-    return c.amode == kAModeSlabRes && pool > 0 && num_kb * bbytes + 2 * pitch <= pool;
+    return amode_wres(c.amode) && pool > 0 && num_kb * bbytes + 2 * pitch <= pool;
 }
 
 void gemm_slab_pool(const GemmConfig &c, GemmArgs &a) {
     a.slab_off = a.slab_pitch = a.slab_slots = 0;
-    if (c.amode != kAModeSlabRes) return;
+    if (!amode_wres(c.amode)) return;
     int pool, bbytes;
     slab_pool_shape(c, pool, bbytes);
     a.slab_pitch = (a.slab_bytes + 1023) / 1024 * 1024;

@@ -54,7 +54,9 @@ struct GemmArgs {
     int num_tiles;  // tiles_m * tiles_n
     // slab mode (stride-1 convolution): a tile is slab_t output rows of one
     // image; tile row v = y * wp + x indexes the padded width wp, and filter
-    // tap (r, s) reads the slab from row r * wp + s on
+    // tap (r, s) reads the slab from row r * wp + s on.  Pair modes: a unit
+    // is tiles 2u and 2u + 1 of an image (the second one absent at the end of
+    // an image with an odd tiles_per_img), and num_tiles counts units
     int wp;             // padded input width (W + pad_l + pad_r)
     int slab_t;         // output rows per tile
     int tiles_per_img;  // ceil(Ho / slab_t)
@@ -83,6 +85,12 @@ struct GemmArgs {
     const __nv_bfloat16 *residual;    // [M, N] or null
     __nv_bfloat16 *out;               // [M, N]
     int *err;                         // device error word
+    // > 0: the slab comes from a stem layout (StemArgs) through a 5-D map,
+    // box {8 values, wp positions, slab rows, stem_rows image rows, 1} at
+    // (0, 0, first output row, 0, image), unswizzled: in shared memory
+    // stem_rows planes of slab_bytes / stem_rows, one 16-byte piece per
+    // slab position (the MMA reads them as no-swizzle core matrices)
+    int stem_rows;
 };
 
 enum AMode : int {
@@ -90,8 +98,16 @@ enum AMode : int {
     kAModeIm2col = 1,  // A through an im2col TMA map: one load per filter tap and chunk
     kAModeSlab = 2,    // stride-1 conv: one 4-D tiled slab per chunk, taps by row shift
     kAModeSlabRes = 3,  // slab mode, one column tile, all weights resident in shared memory
-    kAModeTileSplit = 4  // tile mode with the k-blocks of every tile split over `splits` CTAs
+    kAModeTileSplit = 4,  // tile mode with the k-blocks of every tile split over `splits` CTAs
+    // kAModeSlabRes in pair units: two vertically adjacent slab tiles of one
+    // image (2 x 128 MMA rows, two accumulators) share one slab load and the
+    // per-unit waits and commits
+    kAModeSlabRes2 = 5
 };
+
+constexpr bool amode_slab(int m) { return m == kAModeSlab || m == kAModeSlabRes || m == kAModeSlabRes2; }
+constexpr bool amode_pair(int m) { return m == kAModeSlabRes2; }
+constexpr bool amode_wres(int m) { return m == kAModeSlabRes || m == kAModeSlabRes2; }
 
 struct GemmConfig {
     int bn;      // tile width in output channels: 32, 64, 128, 256
@@ -100,8 +116,11 @@ struct GemmConfig {
     bool res;    // epilogue adds a residual tile (bn 64 or 128)
 };
 
-// Largest slab (one channel chunk) the slab mode holds, per buffer.
-constexpr int slab_max_bytes(int bk) { return bk == 64 ? 48 * 1024 : 24 * 1024; }
+// Largest slab (one channel chunk) the slab mode holds, per buffer; a pair
+// unit's slab covers both tiles' rows.
+constexpr int slab_max_bytes(int bk, bool pair = false) {
+    return pair ? (bk == 64 ? 56 * 1024 : 28 * 1024) : (bk == 64 ? 48 * 1024 : 24 * 1024);
+}
 constexpr int kMaxSlabSlots = 8;
 
 constexpr int kGemmBM = 128;
@@ -169,27 +188,24 @@ size_t dw_smem_bytes(const DwArgs &a);
 cudaError_t dw_prepare(const DwArgs &a);
 cudaError_t launch_dwconv(const CUtensorMap &tmX, const DwArgs &a, int grid, cudaStream_t st);
 
-// Boundary layout transform for a stride-2 stem with few input channels
-// (space-to-depth with zero padding, vertical filter taps stacked):
-//   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
-// for a < taps, zero outside the image and in channels a*16 + [4C, 16).
-// Space-to-depth of a stride-2 stem (C <= 4 channels) with the `taps`
-// vertical filter taps stacked into the channel dimension:
-//   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
-// zero outside x and in channels 4C..15 of each 16-channel group.
-struct S2dArgs {
-    const __nv_bfloat16 *x;  // [N, H, W, C]
-    __nv_bfloat16 *z;        // [N, Hz, Wz, 16 * taps]
+// Layout transform at the region boundary for a stride-2 stem with few
+// input channels (Section 3.2): the image with 4 channels and `pad` zero rows
+// and columns before it (zero after it up to Hq x Wq),
+//   xq[n, u, v, c] = x[n, u - pad, v - pad, c]   (c < C, inside x), else 0,
+// so that a pair of pixels is one aligned 16-byte piece.  The stem's GEMM
+// reads it through a 5-D tensor map (runtime.cu, encode_stem_slab).
+struct StemArgs {
+    const __nv_bfloat16 *x;  // [N, H, W, C], C <= 4
+    __nv_bfloat16 *xq;       // [N, Hq, Wq, 4]
     int N, H, W, C;
-    int Hz, Wz;              // N, Hz <= 65535
-    int taps;
+    int Hq, Wq;              // N * Hq <= 2^31 - 1; Wq even
     int pad;
 };
-// The transform stages 2 * taps input rows (W * C elements each) in shared
-// memory; the planner rejects stems whose rows need more than kS2dMaxSmem.
-constexpr size_t kS2dMaxSmem = 200 * 1024;
-size_t s2d_smem_bytes(const S2dArgs &a);
-cudaError_t launch_s2d(const S2dArgs &a, cudaStream_t st);
+// The transform stages kStemRows input rows (W * C bf16 each) in shared
+// memory; the planner rejects stems whose rows need more than this.
+constexpr size_t kStemLayoutMaxSmem = 48 * 1024;
+size_t stem_layout_smem_bytes(const StemArgs &a);
+cudaError_t launch_stem_layout(const StemArgs &a, cudaStream_t st);
 
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            int k, int s, int p, cudaStream_t st);

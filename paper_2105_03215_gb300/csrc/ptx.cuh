@@ -125,6 +125,15 @@ __device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap *tm,
         : "memory");
 }
 
+__device__ __forceinline__ void tma_load_5d(uint32_t dst, const CUtensorMap *tm, uint32_t bar,
+                                            int32_t c0, int32_t c1, int32_t c2, int32_t c3, int32_t c4) {
+    asm volatile(
+        "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%3, %4, %5, %6, %7}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(bar), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4)
+        : "memory");
+}
+
 // 4-D im2col load of an NHWC tensor: coordinates {c, w, h, n} of the first
 // pixel's filter origin, plus the filter-tap offsets {off_w, off_h}.  Loads
 // `pixelsPerColumn` pixels (traversing w, then h, then n inside the tensor
@@ -230,6 +239,22 @@ __device__ __forceinline__ uint64_t make_smem_desc(uint32_t saddr, uint32_t row_
     d |= static_cast<uint64_t>(1u) << 46;
     d |= static_cast<uint64_t>(layout) << 61;
     return d;
+}
+
+// Descriptor for a K-major operand without swizzle stored as row planes:
+// plane q holds the 8 K-values 8q .. 8q+7 of every operand row, 16 bytes per
+// row, rows consecutive; planes `plane_bytes` apart.  In the canonical
+// no-swizzle layout an 8-row x 16-byte core matrix is 128 contiguous bytes:
+// here the leading byte offset (between core matrices along K) is the plane
+// size and the stride byte offset (between 8-row groups) 128 bytes.  The
+// start may be any 16-byte-aligned row.
+__device__ __forceinline__ uint64_t make_smem_desc_planes(uint32_t saddr, uint32_t plane_bytes) {
+    uint64_t d = 0;
+    d |= static_cast<uint64_t>((saddr >> 4) & 0x3FFFu);
+    d |= static_cast<uint64_t>((plane_bytes >> 4) & 0x3FFFu) << 16;
+    d |= static_cast<uint64_t>(128u >> 4) << 32;
+    d |= static_cast<uint64_t>(1u) << 46;
+    return d;  // layout 0: no swizzle
 }
 
 // The same descriptor for an operand whose first row starts at an arbitrary

@@ -135,6 +135,29 @@ CUresult encode_slab(CUtensorMap *m, const void *ptr, int N, int H, int W, int C
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// Stem slab over the pixel-pair layout xq [N, Hq, Wq, 4] (StemArgs): dims
+// {8 G values (G pixel pairs), wp / G pair groups, E position rows, R image
+// rows, N} with E = (Hq - R) / 2 + 1.  A position row is two image rows on,
+// so the position-row and image-row dimensions overlap, and every in-range
+// element stays inside its image's Hq rows.  Box {8 G, wp / G, rows, R, 1}
+// at (0, 0, p, 0, n), without swizzle, lands in shared memory as R planes
+// [image row r][slab position (p + y, j)][16 bytes]; position rows past E
+// read as zeros.  (A 16-byte-wide operand row cannot be swizzled in place:
+// a 16-byte inner box under 128-byte swizzle is laid out at the 128-byte
+// span per row, hence the unswizzled planes.)
+CUresult encode_stem_slab(CUtensorMap *m, const void *ptr, int N, int Hq, int Wq, int R, int wp, int rows,
+                          int G) {
+    const cuuint64_t row = (cuuint64_t)Wq * 4 * 2;
+    const cuuint64_t E = (cuuint64_t)(Hq - R) / 2 + 1;
+    cuuint64_t dims[5] = {(cuuint64_t)8 * G, (cuuint64_t)(wp / G), E, (cuuint64_t)R, (cuuint64_t)N};
+    cuuint64_t strides[4] = {(cuuint64_t)16 * G, 2 * row, row, (cuuint64_t)Hq * row};
+    cuuint32_t box[5] = {(cuuint32_t)(8 * G), (cuuint32_t)(wp / G), (cuuint32_t)rows, (cuuint32_t)R, 1};
+    cuuint32_t es[5] = {1, 1, 1, 1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 5, const_cast<void *>(ptr), dims,
+                          strides, box, es, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 // Depthwise input box: in_rows x in_cols pixels x cc channels, no swizzle
 // (the kernel reads it with plain 16-byte shared-memory loads).
 CUresult encode_dw(CUtensorMap *m, const void *ptr, const byoc::DwArgs &a) {
@@ -208,7 +231,9 @@ struct LaunchPlan {
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
     // depthwise / space-to-depth / fused depthwise -> 1x1
     byoc::DwArgs dw{};
-    byoc::S2dArgs s2d{};
+    byoc::StemArgs stem{};
+    int stem_R = 0;  // stem GEMM: row taps per slab position (StemArgs layout), else 0
+    int stem_G = 0;  // stem GEMM: pixel pairs per innermost tensor-map box row
     byoc::DwPwArgs dp{};
     size_t w2_off = 0, w2_bytes = 0, b2_off = 0, b2_bytes = 0;  // fused: the 1x1 conv's constants
     double flops = 0, bytes = 0;
@@ -452,6 +477,35 @@ bool slab_geometry(int H, int W, int Ho, int Wo, int kh, int kw, int pt, int pl,
     return g.rows <= 256 && g.bytes <= byoc::slab_max_bytes(bk);
 }
 
+// Pair-unit slab (kAModeSlab2 / kAModeSlabRes2): the rows under two
+// vertically adjacent tiles of t output rows each.  The second tile's MMA
+// rows start t * wp slab rows in.
+bool slab_pair_geometry(int kh, int kw, int bk, const SlabGeom &g, SlabGeom &pg) {
+    pg = g;
+    const int dmax = (kh - 1) * g.wp + (kw - 1);
+    pg.rows = (g.t * g.wp + 128 + dmax + g.wp - 1) / g.wp;
+    pg.bytes = pg.rows * g.wp * bk * 2;
+    return pg.rows <= 256 && pg.bytes <= byoc::slab_max_bytes(bk, true);
+}
+
+// Makespan estimate (SM cycles) of a slab-mode launch: `units` m-units of
+// `halves` tiles each, times tiles_n column tiles, over the persistent grid.
+// A k-block costs the larger of its MMA time (halves x bk/16 MMAs of
+// M=128, N=bn: 40 / 48 / 64 / 128 cycles for bn = 32 / 64 / 128 / 256) and
+// the time to bring in its operand bytes (ring weights + its share of the
+// slab) at ~40 B/cycle per SM -- what the GB300 traces of the 28x28 and
+// 14x14 ResNet-50 3x3 layers deliver; plus ~300 cycles per unit.
+double slab_makespan(int64_t units, int64_t tiles_n, int64_t kblocks, int taps, int bn, int bk, int halves,
+                     bool wres, int slab_bytes, int num_sms) {
+    const double mma = bn <= 32 ? 40.0 : bn <= 64 ? 48.0 : bn <= 128 ? 64.0 : 128.0;
+    const double kb_bytes = (wres ? 0.0 : (double)bn * bk * 2) + (double)slab_bytes / std::max(1, taps);
+    const double per_kb = std::max(halves * (bk / 16) * mma, kb_bytes / 40.0);
+    const int64_t u = units * tiles_n;
+    const int64_t grid = std::max<int64_t>(1, std::min<int64_t>(u, num_sms));
+    const int64_t rounds = (u + grid - 1) / grid;
+    return (double)rounds * (300.0 + (double)kblocks * per_kb);
+}
+
 struct Affine {
     std::vector<double> scale, shift;
 };
@@ -660,8 +714,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
 
         // ---------------- GEMM (conv2d groups=1, or dense)
         int64_t M, Kreal;
-        int64_t stem_k = 0;     // > 0: the stem conv's reduction length before space-to-depth
-        int64_t stem_imgs = 0;  // stem: images per (space-to-depth, GEMM) launch pair
+        int64_t stem_k = 0;     // > 0: the stem conv's reduction length (before the pixel-pair layout)
         int kh = 1, kw = 1, taps = 1, chunks, bk;
         int64_t C;
         std::vector<double> wsrc;  // weights as [Cout][kh][kw][C] (channel innermost)
@@ -686,83 +739,114 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                                 op.dilation[0] == op.dilation[1] && op.pad[0] == op.pad[1] &&
                                 op.pad[2] == op.pad[3];
             if (C % 8) {
-                // Few-channel stride-2 stem.  A space-to-depth boundary transform
-                // turns the k x k stride-2 conv over C channels into a k2 x k2
-                // stride-1 conv over 4C (<= 16) channels, k2 = (k+1)/2, and also
-                // stacks the k2 vertical taps into the channel dimension, so the
-                // GEMM is a 1 x k2 conv over 16*k2 channels (128-byte operand rows
-                // for k2 = 4):
-                //   z[n, p, j, a*16 + (dy*2+dx)*C + c] = x[n, 2(p+a)+dy-pad, 2j+dx-pad, c]
-                //   w''[k][b][a*16 + (dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx]
-                // The stacked tensor is k2 times larger than the image, so the
-                // pair of launches runs over chunks of images whose z fits in
-                // L2 (about 32 MiB): z is written and read back without a DRAM
-                // round trip.
-                if (!(square && op.stride[0] == 2 && op.dilation[0] == 1 && C <= 4 && (kh % 2) == 1))
+                // Few-channel stride-2 stem (k x k, k odd <= 7, C <= 4), run
+                // as a stride-1 convolution over pixel pairs.  Output pixel
+                // (p, q), filter tap (r, s = 2b + dx) reads input pixel
+                // (2p + r - pad, 2q + 2b + dx - pad): with R >= k row taps
+                // (4 or 8) and k2 = (k + 1) / 2 column taps b, the operand
+                // row of slab position (p, j) is the R pixel pairs
+                //   xq[2p + r][2j], xq[2p + r][2j + 1]   (r = 0 .. R-1)
+                // of the boundary layout xq (4 channels, `pad` zero rows and
+                // columns in front; StemArgs): 8R values in the order
+                // r*8 + dx*4 + c, and tap b is that row read b positions on.
+                // The GEMM loads it with a 5-D tensor map {8 values, R rows,
+                // wp pairs, position rows (2 image rows apart), images}, so
+                // the layout is the image's size (no stacked copy), and
+                //   w'[k][b][r*8 + dx*4 + c] = w[k][c][r][2b + dx]   (0 outside the filter).
+                if (!(square && op.stride[0] == 2 && op.dilation[0] == 1 && C <= 4 && (kh % 2) == 1 &&
+                      kh <= 7))
                     return fail(BYOC_ERR_UNSUPPORTED,
-                                "op %d: %lld input channels: only a stride-2 odd square stem with "
+                                "op %d: %lld input channels: only a stride-2 odd square stem (k <= 7) with "
                                 "<= 4 channels is supported",
                                 o, (long long)C);
                 const int k2 = (kh + 1) / 2;
-                const int Cz = 16 * k2;
-                if (X.shape[0] > 65535 || Y.shape[1] > 65535)
-                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem batch or height above 65535", o);
-                const int64_t z_img = Y.shape[1] * (Y.shape[2] + k2 - 1) * Cz * 2;
-                // chunks of at most 128 MB of stacked tensor, which L2 (129 MB)
-                // mostly holds until the GEMM reads it (measured on the N=64
-                // ResNet-50 stem: one 105 MB chunk 75 us, two 79 us, four 86 us)
-                int64_t nck = (X.shape[0] * z_img + (128ll << 20) - 1) / (128ll << 20);
-                const int64_t room = (BYOC_PLAN_MAX_LAUNCHES - 1 - (int64_t)P.launches.size()) / 2;
-                nck = std::max<int64_t>(1, std::min<int64_t>({nck, room, X.shape[0]}));
-                stem_imgs = (X.shape[0] + nck - 1) / nck;
+                const int R = kh <= 3 ? 4 : 8;
+                const int Cz = 8 * R;
+                if (X.shape[0] > 65535)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem batch above 65535", o);
+                // slab positions per output row: at least Wo + k2 - 1, and a
+                // multiple of a group of G <= 32 pairs (G >= 16 where one
+                // fits), so that the tensor map's innermost box dimension is
+                // G contiguous pairs (16 G bytes), not one
+                int64_t wpz = Y.shape[2] + k2 - 1;
+                int G = (int)std::min<int64_t>(wpz, 32);
+                if (wpz > 32) {
+                    G = 0;
+                    for (int64_t w = wpz; G == 0 && w <= wpz + 16; ++w)
+                        for (int d = 32; d >= 16; --d)
+                            if (w % d == 0) {
+                                G = d;
+                                wpz = w;
+                                break;
+                            }
+                }
+                if (wpz > 128)
+                    return fail(BYOC_ERR_UNSUPPORTED,
+                                "op %d: stem output %lld wide: a slab tile covers at most 128 positions "
+                                "of one output row",
+                                o, (long long)Y.shape[2]);
+                // position rows the tensor map spans: the output rows and one
+                // more, or a whole slab (single or pair) if that is more
+                const int64_t tz = std::max<int64_t>(1, std::min<int64_t>(128 / wpz, Y.shape[1]));
+                const int64_t pos_rows = std::max<int64_t>(
+                    Y.shape[1] + 1, (tz * wpz + 128 + k2 - 1 + wpz - 1) / wpz);
+                const int64_t Hq = 2 * (pos_rows - 1) + R;  // image rows they reach
+                const int64_t Wq = 2 * wpz;
+                if ((int64_t)X.shape[0] * Hq > INT32_MAX)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem layout too large", o);
                 TensorInfo Z;
                 Z.ndim = 4;
-                Z.shape[0] = stem_imgs;
-                Z.shape[1] = Y.shape[1];
-                Z.shape[2] = Y.shape[2] + k2 - 1;
-                Z.shape[3] = Cz;
+                Z.shape[0] = X.shape[0];
+                Z.shape[1] = Hq;
+                Z.shape[2] = Wq;
+                Z.shape[3] = 4;
                 const int zid = (int)P.tensors.size();
                 P.tensors.push_back(Z);
                 LaunchPlan S;
                 S.kind = BYOC_LAUNCH_S2D;
                 S.x = op.in[0];
                 S.y = zid;
-                S.s2d.N = (int)X.shape[0];
-                S.s2d.H = (int)X.shape[1];
-                S.s2d.W = (int)X.shape[2];
-                S.s2d.C = (int)C;
-                S.s2d.Hz = (int)Z.shape[1];
-                S.s2d.Wz = (int)Z.shape[2];
-                S.s2d.taps = k2;
-                S.s2d.pad = op.pad[0];
-                S.bytes = (double)X.bytes();  // z is internal: not algorithmic traffic
-                if (byoc::s2d_smem_bytes(S.s2d) > byoc::kS2dMaxSmem)
+                S.stem.N = (int)X.shape[0];
+                S.stem.H = (int)X.shape[1];
+                S.stem.W = (int)X.shape[2];
+                S.stem.C = (int)C;
+                S.stem.Hq = (int)Hq;
+                S.stem.Wq = (int)Wq;
+                S.stem.pad = op.pad[0];
+                S.bytes = (double)X.bytes();  // xq is internal: not algorithmic traffic
+                if (byoc::stem_layout_smem_bytes(S.stem) > byoc::kStemLayoutMaxSmem)
                     return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem rows too wide (%lld x %lld)", o,
                                 (long long)X.shape[2], (long long)C);
                 P.launches.push_back(S);
                 wsrc.assign((size_t)Cout * k2 * Cz, 0.0);
                 for (int64_t k = 0; k < Cout; ++k)
-                    for (int a = 0; a < k2; ++a)
-                        for (int b = 0; b < k2; ++b)
-                            for (int dy = 0; dy < 2; ++dy)
-                                for (int dx = 0; dx < 2; ++dx)
-                                    for (int64_t c = 0; c < C; ++c) {
-                                        const int r = 2 * a + dy, s = 2 * b + dx;
-                                        if (r >= kh || s >= kw) continue;
-                                        wsrc[((size_t)k * k2 + b) * Cz + a * 16 + (dy * 2 + dx) * C + c] =
-                                            op.consts[0][((k * C + c) * kh + r) * kw + s];
-                                    }
+                    for (int b = 0; b < k2; ++b)
+                        for (int r = 0; r < kh; ++r)
+                            for (int dx = 0; dx < 2; ++dx)
+                                for (int64_t c = 0; c < C; ++c) {
+                                    const int sx = 2 * b + dx;
+                                    if (sx >= kw) continue;
+                                    wsrc[((size_t)k * k2 + b) * Cz + r * 8 + dx * 4 + c] =
+                                        op.consts[0][((k * C + c) * kh + r) * kw + sx];
+                                }
                 stem_k = (int64_t)kh * kw * C;  // the conv's own reduction length
                 L.x = zid;
+                L.stem_R = R;
+                L.stem_G = G;
                 C = Cz;
                 kh = 1;
                 kw = k2;
                 im2col = true;
-                // the 1 x k2 stride-1 conv over the stacked tensor reads well as slabs
-                slab = slab_geometry((int)Z.shape[1], (int)Z.shape[2], (int)Y.shape[1],
-                                     (int)Y.shape[2], 1, k2, 0, 0, 0, pick_bk(Cz), sgeo);
-                L.geo = Im2colGeom{(int)Z.shape[0], (int)Z.shape[1], (int)Z.shape[2], Cz,
-                                   1, k2, 1, 1, 0, 0, 0, 0, 1, 1};
+                // a 1 x k2 stride-1 conv over rows of wpz positions: tiles of
+                // t output rows, slabs of `rows` position rows
+                sgeo.wp = (int)wpz;
+                sgeo.t = (int)tz;
+                sgeo.rows = (int)((128 + k2 - 1 + wpz - 1) / wpz);
+                sgeo.bytes = sgeo.rows * sgeo.wp * Cz * 2;
+                slab = true;
+                if (sgeo.bytes > byoc::slab_max_bytes(Cz))
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem slab of %d bytes", o, sgeo.bytes);
+                L.geo = Im2colGeom{(int)X.shape[0], (int)Hq, (int)Wq, 4, 1, k2, 1, 1, 0, 0, 0, 0, 1, 1};
                 L.args.stride_h = L.args.stride_w = 1;
                 L.args.pad_t = L.args.pad_l = 0;
                 L.args.dil_h = L.args.dil_w = 1;
@@ -827,6 +911,34 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
             if (byoc::gemm_config_supported(rc) && byoc::gemm_slab_res_fits(rc, taps * chunks, sgeo.bytes))
                 L.cfg = rc;
         }
+        int64_t units_m = tiles_m;  // m-units of the launch: tiles, or pairs of tiles
+        if (slab && L.cfg.amode == byoc::kAModeSlabRes && (int64_t)taps * chunks * (bk / 16) <= 16) {
+            // Pair units (two adjacent tiles sharing each weight k-block and
+            // one slab) for resident-weight slabs with few MMAs per tile (the
+            // stem's 16): they halve the per-unit cost of waits, commits and
+            // descriptor set-up, which is a large part of such a tile.  With
+            // more MMAs per tile the MMA rate is bound by the shared-memory
+            // reads of its operands (A and B are read for every MMA), which
+            // pairs do not reduce: measured on GB300, the 56x56 / 28x28 /
+            // 14x14 ResNet-50 3x3 layers ran as fast or slower in pairs.
+            // The estimate still rules out pairs that leave SMs idle.
+            SlabGeom pg;
+            const int64_t tn = (Cout + bn - 1) / bn;
+            const int64_t pair_m = X.shape[0] * ((tiles_per_img + 1) / 2);
+            if (slab_pair_geometry(kh, kw, bk, sgeo, pg)) {
+                const GemmConfig pc{bn, bk, byoc::kAModeSlabRes2, false};
+                const double single = slab_makespan(tiles_m, tn, (int64_t)taps * chunks, taps, bn, bk, 1, true,
+                                                    sgeo.bytes, P.num_sms);
+                const double pair = slab_makespan(pair_m, tn, (int64_t)taps * chunks, taps, bn, bk, 2, true,
+                                                  pg.bytes, P.num_sms);
+                if (byoc::gemm_config_supported(pc) && byoc::gemm_slab_res_fits(pc, taps * chunks, pg.bytes) &&
+                    pair < single) {
+                    L.cfg = pc;
+                    units_m = pair_m;
+                    sgeo = pg;
+                }
+            }
+        }
         if (slab) {
             L.slab_rows = sgeo.rows;
             L.args.wp = sgeo.wp;
@@ -866,9 +978,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         A.Ho = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[1];
         A.Wo = op.kind == BYOC_OP_DENSE ? 1 : (int)Y.shape[2];
         A.tiles_n = L.n_pad / bn;
-        A.num_tiles = (int)(tiles_m * A.tiles_n);
+        A.num_tiles = (int)(units_m * A.tiles_n);
         A.taps = taps;
-        A.group = byoc::gemm_group(bn, bk, amode == byoc::kAModeSlab ? taps : (A.num_kb + splits - 1) / splits);
+        A.stem_rows = L.stem_R;
+        // a pair unit's k-block is twice the MMA work of a tile's
+        A.group = byoc::gemm_group(byoc::amode_pair(L.cfg.amode) ? 2 * bn : bn, bk,
+                                   amode == byoc::kAModeSlab ? taps : (A.num_kb + splits - 1) / splits);
         byoc::gemm_slab_pool(L.cfg, A);
         A.splits = splits;
         A.m_pad = (int)(tiles_m * byoc::kGemmBM);
@@ -880,38 +995,12 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
         L.grid = std::min(A.num_tiles * splits, P.num_sms);
         A.act = act;
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
-        const double in_bytes = stem_k > 0 ? 0.0  // z: counted as x by the transform
+        const double in_bytes = stem_k > 0 ? 0.0  // xq: the image is counted by the layout transform
                                 : L.x < P.n_region_tensors ? (double)X.bytes()
                                                            : (double)P.tensors[L.x].bytes();
         L.bytes = in_bytes + (double)Y.bytes() + (double)Cout * Kreal * 2 + (double)Cout * 4 +
                   (res >= 0 ? (double)P.tensors[res].bytes() : 0.0);
         P.launches.push_back(L);
-        if (stem_k > 0) {
-            // one (space-to-depth, GEMM) pair per chunk of stem_imgs images
-            const LaunchPlan S0 = P.launches[P.launches.size() - 2];
-            const LaunchPlan G0 = L;
-            P.launches.resize(P.launches.size() - 2);
-            const int64_t N = X.shape[0];
-            const int64_t hw = Y.shape[1] * Y.shape[2];
-            for (int64_t n0 = 0; n0 < N; n0 += stem_imgs) {
-                const int64_t nc = std::min(stem_imgs, N - n0);
-                const double frac = (double)nc / (double)N;
-                LaunchPlan S = S0;
-                S.s2d.N = (int)nc;
-                S.x_off = (size_t)(n0 * X.shape[1] * X.shape[2] * X.shape[3] * 2);
-                S.bytes = S0.bytes * frac;
-                P.launches.push_back(S);
-                LaunchPlan G = G0;
-                G.geo.N = (int)nc;
-                G.args.M = (int)(nc * hw);
-                G.args.num_tiles = (int)(nc * G.args.tiles_per_img * G.args.tiles_n);
-                G.grid = std::min(G.args.num_tiles, P.num_sms);
-                G.y_off = (size_t)(n0 * hw * Cout * 2);
-                G.flops = G0.flops * frac;
-                G.bytes = G0.bytes * frac;
-                P.launches.push_back(G);
-            }
-        }
         o = j;
     }
     // Workspace: every tensor that is neither a region input nor output.
@@ -963,11 +1052,12 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
                            : std::min(L.cfg.amode, (int)byoc::kAModeSlab);
         r->splits[i] = L.kind == BYOC_LAUNCH_GEMM ? std::max(1, L.args.splits) : 0;
         r->grid[i] = L.grid;
-        r->resident_b[i] = L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeSlabRes ? 1 : 0;
-        r->slab_slots[i] = L.kind != BYOC_LAUNCH_GEMM ? 0
-                           : L.cfg.amode == byoc::kAModeSlabRes ? L.args.slab_slots
-                           : L.cfg.amode == byoc::kAModeSlab    ? 2
-                                                                : 0;
+        const bool gm = L.kind == BYOC_LAUNCH_GEMM;
+        r->resident_b[i] = gm && byoc::amode_wres(L.cfg.amode) ? 1 : 0;
+        r->slab_slots[i] = !gm || !byoc::amode_slab(L.cfg.amode) ? 0
+                           : byoc::amode_wres(L.cfg.amode)      ? L.args.slab_slots
+                                                                : 2;
+        r->pair_units[i] = gm && byoc::amode_pair(L.cfg.amode) ? 1 : 0;
     }
     r->flops = P.flops;
     r->bytes = P.bytes;
@@ -1188,7 +1278,7 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
 static_assert(std::is_trivially_copyable<LaunchPlan>::value && std::is_trivially_copyable<TensorInfo>::value,
               "launch records are stored byte for byte");
 constexpr char kPlanMagic[8] = {'B', 'Y', 'O', 'C', 'P', 'L', 'N', '1'};
-constexpr uint32_t kPlanFormat = 1;
+constexpr uint32_t kPlanFormat = 2;
 
 uint64_t fnv1a(const uint8_t *p, size_t n, uint64_t h = 1469598103934665603ull) {
     for (size_t i = 0; i < n; ++i) {
@@ -1200,7 +1290,7 @@ uint64_t fnv1a(const uint8_t *p, size_t n, uint64_t h = 1469598103934665603ull) 
 
 uint64_t layout_tag() {
     const uint64_t sizes[] = {sizeof(TensorInfo), sizeof(LaunchPlan), sizeof(GemmArgs),
-                              sizeof(byoc::DwArgs), sizeof(byoc::S2dArgs), sizeof(Im2colGeom),
+                              sizeof(byoc::DwArgs), sizeof(byoc::StemArgs), sizeof(Im2colGeom),
                               kPlanFormat, BYOC_ABI_VERSION};
     return fnv1a(reinterpret_cast<const uint8_t *>(sizes), sizeof(sizes));
 }
@@ -1432,7 +1522,10 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
                 CUresult r;
-                if (L.cfg.amode == byoc::kAModeSlab || L.cfg.amode == byoc::kAModeSlabRes)
+                if (byoc::amode_slab(L.cfg.amode) && L.stem_R > 0)
+                    r = encode_stem_slab(&h->tmA[i], xa, L.geo.N, L.geo.H, L.geo.W, L.stem_R, L.args.wp,
+                                         L.slab_rows, L.stem_G);
+                else if (byoc::amode_slab(L.cfg.amode))
                     r = encode_slab(&h->tmA[i], xa, L.geo.N, L.geo.H, L.geo.W, L.geo.C, L.args.wp,
                                     L.slab_rows, L.cfg.bk);
                 else if (L.cfg.amode == byoc::kAModeIm2col)
@@ -1485,11 +1578,11 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
             e = byoc::launch_dwpw(h->tmA[i], h->tmB[i], a, L.grid, st);
         } else {
-            byoc::S2dArgs a = L.s2d;
+            byoc::StemArgs a = L.stem;
             a.x = reinterpret_cast<const __nv_bfloat16 *>(static_cast<const char *>(h->ptrs[L.x]) +
                                                            L.x_off);
-            a.z = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
-            e = byoc::launch_s2d(a, st);
+            a.xq = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
+            e = byoc::launch_stem_layout(a, st);
         }
         if (e != cudaSuccess) return cuda_fail(e, "kernel launch");
     }

@@ -12,6 +12,7 @@ import pytest
 
 from paper_2105_03215_gb300 import abi
 from paper_2105_03215_gb300 import inputs as I
+from paper_2105_03215_gb300 import partition as P
 from paper_2105_03215_gb300 import region as R
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -69,17 +70,21 @@ def test_plan_fuses_depthwise_into_the_pointwise_when_asked(monkeypatch):
     assert rep.act[0] == 2
 
 
-def test_plan_stem_inserts_space_to_depth():
+def test_plan_stem_inserts_the_pixel_pair_layout():
     g, _ = I.resnet50(N=1, H=32, W=32)
     rep = R.Region(g, [n.name for n in g.nodes[:3]], "stem").plan()
     assert rep.n_launches == 2
     assert rep.kind[0] == abi.LAUNCH_S2D and rep.kind[1] == abi.LAUNCH_GEMM
-    # 7x7/2 over 3 channels -> 1x4 stride-1 conv over 4 stacked taps x 16 channels (slab mode)
+    # 7x7/2 over 3 channels -> 1x4 stride-1 conv over 8 rows x 2 pixels x 4 channels (slab mode)
     assert rep.gemm_k[1] == 4 * 64 and rep.tile_k[1] == 64 and rep.im2col[1] == 2
+    # 3x3/2 -> 1x2 over 4 rows x 2 pixels x 4 channels (32-element k-blocks)
+    g, _ = I.stem(N=1, H=32, W=32, k=3, cout=32, C=3)
+    rep = R.whole_graph_region(g).plan()
+    assert rep.gemm_k[1] == 2 * 32 and rep.tile_k[1] == 32 and rep.im2col[1] == 2
 
 
-def test_stem_weights_follow_the_space_to_depth_definition():
-    # w''[k][b][a*16 + (dy*2+dx)*C + c] = w[k][c][2a+dy][2b+dx], zero where 2a+dy or 2b+dx >= 7
+def test_stem_weights_follow_the_pixel_pair_definition():
+    # w'[k][b][r*8 + dx*4 + c] = w[k][c][r][2b+dx], zero where r or 2b+dx >= 7 or c >= 3
     g, _ = I.resnet50(N=1, H=32, W=32)
     reg = R.Region(g, [n.name for n in g.nodes[:3]], "stem")
     rep = reg.plan()
@@ -88,34 +93,30 @@ def test_stem_weights_follow_the_space_to_depth_definition():
     scale = bn.consts["gamma"].astype(np.float64) / np.sqrt(
         bn.consts["moving_var"].astype(np.float64) + 1e-5)
     packed = np.frombuffer(reg.plan_constants(1, 0), dtype=np.uint16).reshape(-1, rep.gemm_k[1])
-    expect = np.zeros((64, 4, 4, 16), dtype=np.float64)            # [k][b][a][group]
-    for a in range(4):
-        for b in range(4):
-            for dy in range(2):
-                for dx in range(2):
-                    r, s_ = 2 * a + dy, 2 * b + dx
-                    if r < 7 and s_ < 7:
-                        expect[:, b, a, (dy * 2 + dx) * 3:(dy * 2 + dx) * 3 + 3] = w[:, :, r, s_]
-    expect *= scale[:, None, None, None]
+    expect = np.zeros((64, 4, 8, 2, 4), dtype=np.float64)          # [k][b][r][dx][c]
+    for b in range(4):
+        for r in range(7):
+            for dx in range(2):
+                if 2 * b + dx < 7:
+                    expect[:, b, r, dx, :3] = w[:, :, r, 2 * b + dx]
+    expect *= scale[:, None, None, None, None]
     want = I.bf16_bits(expect.reshape(64, -1).astype(np.float32))
     assert np.array_equal(packed[:64], want)
     # the flop count is the 7x7x3 convolution's, not the padded GEMM's
     assert rep.flops == pytest.approx(2.0 * 64 * 16 * 16 * 7 * 7 * 3, rel=1e-12)
 
 
-def test_stem_runs_in_image_chunks_that_fit_l2():
-    # stacked z: 112 x 115 x 64 bf16 = 1.65 MB per image; chunks of <= 128 MB
-    g, _ = I.stem(N=64, H=224, W=224)
-    rep = R.whole_graph_region(g).plan()
-    assert rep.n_launches == 2 and rep.gemm_m[1] == 64 * 112 * 112
-    assert rep.flops == pytest.approx(2.0 * 64 * 112 * 112 * 64 * 7 * 7 * 3, rel=1e-12)
-    g, _ = I.stem(N=170, H=224, W=224)
-    rep = R.whole_graph_region(g).plan()
-    # 170 x 1,648,640 bytes = 2.09 x 128 MiB -> 3 chunks of 57, 57, 56 images
-    assert rep.n_launches == 6
-    assert [rep.kind[i] for i in range(6)] == [abi.LAUNCH_S2D, abi.LAUNCH_GEMM] * 3
-    assert [rep.gemm_m[i] for i in (1, 3, 5)] == [57 * 12544, 57 * 12544, 56 * 12544]
-    assert rep.workspace_bytes <= 256 + 57 * 112 * 115 * 64 * 2 + 256
+def test_stem_layout_is_the_image_size_at_any_batch():
+    # xq: 232 rows x 230 columns x 4 channels of bf16 per image (2 Ho + 8 rows,
+    # 2 (Wo + 3) columns), read by one GEMM launch whatever the batch
+    for N in (64, 170):
+        g, _ = I.stem(N=N, H=224, W=224)
+        rep = R.whole_graph_region(g).plan()
+        assert rep.n_launches == 2 and rep.gemm_m[1] == N * 112 * 112
+        assert [rep.kind[i] for i in range(2)] == [abi.LAUNCH_S2D, abi.LAUNCH_GEMM]
+        assert rep.flops == pytest.approx(2.0 * N * 112 * 112 * 64 * 7 * 7 * 3, rel=1e-12)
+        assert rep.workspace_bytes <= 256 + N * 232 * 230 * 4 * 2 + 256
+        assert rep.resident_b[1] == 1 and rep.pair_units[1] == 1
 
 
 def test_plan_flops_match_mac_count():
@@ -312,3 +313,29 @@ def test_split_k_for_deep_reductions_with_few_tiles():
     # a shallow reduction is not split
     rep = R.whole_graph_region(I.conv_bias_relu(N=2, H=56, W=56, C=64, K=64)[0]).plan(152)
     assert rep.splits[0] == 1
+
+
+def test_pair_units_only_where_a_tile_has_few_mmas():
+    # Pair units (two adjacent tiles per unit, resident weights) for slabs
+    # with at most 16 MMAs per tile: the ResNet-50 stem's 1x4 GEMM at N=64.
+    # The stride-1 3x3 layers (36+ MMAs per tile) stay single, and so does
+    # the stem at N=1, where pairs would leave SMs idle.
+    for N, want in ((64, 1), (1, 0)):
+        g, _ = I.resnet50(N=N, H=224, W=224)
+        part = P.partition(g, P.PATTERN_TABLE, target=P.TARGET, max_ops=1)
+        slabs = 0
+        for ri in range(len(part.region_objects())):
+            rep = R.Region(g, part.region_nodes(ri), f"r{ri}").plan(152)
+            for i in range(rep.n_launches):
+                if rep.kind[i] != abi.LAUNCH_GEMM:
+                    continue
+                if rep.im2col[i] == 2:
+                    slabs += 1
+                stem = rep.n_launches == 2 and i == 1
+                assert rep.pair_units[i] == (want if stem else 0), (N, ri)
+        assert slabs == 12
+    # a 1x4 conv over 64 channels (the stem GEMM's shape) pairs as well
+    g, _ = I.conv_general(kernel=(1, 4), strides=(1, 1), padding=(0, 0, 0, 0), dilation=(1, 1),
+                          N=32, H=24, W=100, C=64, K=64)
+    rep = _plan(g)
+    assert rep.pair_units[0] == 1 and rep.resident_b[0] == 1 and rep.slab_slots[0] >= 2

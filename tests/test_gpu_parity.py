@@ -9,6 +9,7 @@ import numpy as np
 import pytest
 
 from oracle import graph as ograph
+from paper_2105_03215_gb300 import abi
 from paper_2105_03215_gb300 import inputs as I
 from paper_2105_03215_gb300 import region as R
 
@@ -61,6 +62,20 @@ def test_conv_small_int_bit_exact(N, H, W, C, K, k, stride, pad):
 def test_conv_general_small_int_bit_exact(kernel, strides, padding, dilation):
     g, inp = I.conv_general(kernel=kernel, strides=strides, padding=padding, dilation=dilation,
                             small_int=True)
+    _check_graph(g, inp, bit_exact=True)
+
+
+@pytest.mark.parametrize("N,H,W,C,K", [
+    (32, 24, 100, 64, 64),    # 1x4 conv over 64 channels (the stem GEMM's shape), 24 tiles per image
+    (32, 25, 100, 64, 48),    # 25 tiles per image: a single tile ends each image; 48 of 64 columns
+])
+def test_slab_pair_units_small_int_bit_exact(N, H, W, C, K):
+    # resident-weight slabs the planner runs as pair units: two adjacent
+    # tiles of an image share one slab load and the per-unit waits
+    g, inp = I.conv_general(kernel=(1, 4), strides=(1, 1), padding=(0, 0, 0, 0), dilation=(1, 1),
+                            N=N, H=H, W=W, C=C, K=K, small_int=True)
+    rep = R.whole_graph_region(g).plan(152)
+    assert rep.pair_units[0] == 1 and rep.im2col[0] == 2 and rep.resident_b[0] == 1
     _check_graph(g, inp, bit_exact=True)
 
 
@@ -148,23 +163,41 @@ def test_stem_variants(k, cout, C):
     _check_graph(g, inp, what=f"stem{k}x{k}")
 
 
-def test_stem_in_image_chunks_with_a_ragged_last_chunk():
-    # 83 images of 224 x 224: the stacked space-to-depth tensor (1.65 MB per
-    # image, 137 MB) runs as two launch pairs, of 42 and 41 images; the oracle
-    # checks 3000 sampled outputs, half of them in the second chunk
-    import torch
+@pytest.mark.parametrize("N,H,W,C,K,k,pair", [
+    (3, 30, 30, 3, 64, 7, 0),     # the ResNet-50 stem's filter on a small image
+    (2, 17, 23, 4, 32, 3, 0),     # odd sizes, 4 channels, 4 row taps (32-element k-blocks)
+    (2, 20, 24, 1, 48, 5, 0),     # one channel, 6 of 8 row taps used
+    (40, 64, 64, 2, 64, 7, 0),    # 11 tiles of 3 output rows per image
+    (64, 112, 112, 3, 64, 7, 1),  # pair units, 28 tiles of 2 output rows per image
+    (48, 90, 118, 3, 64, 7, 1),   # pair units, 23 tiles per image: a single tile ends each image
+])
+def test_stem_small_int_bit_exact(N, H, W, C, K, k, pair):
+    # stride-2 few-channel stems through the pixel-pair layout (every filter
+    # tap lands in one (r, dx, c) slot of its column tap b)
+    g, inp = I.conv_general(kernel=(k, k), strides=(2, 2), padding=(k // 2,) * 4, dilation=(1, 1),
+                            N=N, H=H, W=W, C=C, K=K, small_int=True)
+    rep = R.whole_graph_region(g).plan(152)
+    assert rep.kind[0] == abi.LAUNCH_S2D and rep.im2col[1] == 2 and rep.pair_units[1] == pair
+    _check_graph(g, inp, bit_exact=True)
+
+
+def test_stem_at_full_size_sampled():
+    # 83 images of 224 x 224 through the pixel-pair layout and one GEMM in
+    # pair units (5-D tensor-map slabs); the oracle checks 3000 sampled
+    # outputs, half of them in the last 20 images and the image borders
     from oracle import ops
-    from .parity import to_dev
     g, inp = I.stem(N=83, H=224, W=224, seed=17)
     reg = R.whole_graph_region(g)
-    rep = reg.plan()
-    assert rep.n_launches == 4 and rep.gemm_m[1] == 42 * 112 * 112 and rep.gemm_m[3] == 41 * 112 * 112
+    rep = reg.plan(152)
+    assert rep.n_launches == 2 and rep.gemm_m[1] == 83 * 112 * 112 and rep.pair_units[1] == 1
     got, cr = run_region(reg, inp)
     y = got[g.outputs[0]].reshape(-1, 64)
     rng = np.random.default_rng(3)
-    half = 42 * 112 * 112
-    pix = np.concatenate([rng.integers(0, half, 1500), rng.integers(half, 83 * 112 * 112, 1500)])
-    ks = rng.integers(0, 64, 3000)
+    border = np.array([(n * 112 + p) * 112 + q for n in (0, 82) for p in (0, 1, 110, 111)
+                       for q in (0, 1, 55, 110, 111)])
+    pix = np.concatenate([rng.integers(0, 63 * 112 * 112, 1460), rng.integers(63 * 112 * 112, 83 * 112 * 112, 1500),
+                          border])
+    ks = rng.integers(0, 64, pix.size)
     conv, bn = g.nodes[0], g.nodes[1]
     a = conv.attrs
     v = ops.conv2d_nhwc_sampled(inp["data"], conv.consts["weight"], pix, ks, a["strides"], a["padding"],
