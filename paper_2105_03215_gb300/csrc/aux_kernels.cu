@@ -500,8 +500,75 @@ __global__ void maxpool3_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N,
     if (two) *reinterpret_cast<uint4 *>(yo + C) = m1;
 }
 
+// 3x3 stride-2 windows, a 2 x 2 block of outputs per thread: rows
+// 2pp-p .. 2pp-p+4 and columns 2q0-p .. 2q0-p+4 of the input cover all four
+// windows (25 loads of 8 channels instead of 36).  Out-of-image positions
+// are clamped to the nearest in-window pixel, as in maxpool3_kernel.
+__global__ void maxpool3s2_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C, int p,
+                                  int Ho, int Wo) {
+    pdl_launch_dependents();
+    pdl_wait();
+    const int CV = C >> 3;
+    const int Wq = (Wo + 1) >> 1, Hq = (Ho + 1) >> 1;  // output column / row pairs
+    const int total = N * Hq * Wq * CV;
+    const int idx = (int)(blockIdx.x * blockDim.x + threadIdx.x);
+    if (idx >= total) return;
+    const int cv = idx % CV;
+    int t = idx / CV;
+    const int qp = t % Wq;
+    t /= Wq;
+    const int ph = t % Hq;
+    const int n = t / Hq;
+    const int q0 = 2 * qp, p0 = 2 * ph;
+    const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
+    // window (i, j) covers input rows 2(p0+i)-p + {0,1,2}, columns 2(q0+j)-p + {0,1,2}; a
+    // second row / column of windows past the output clamps onto the first
+    const int qj = q0 + 1 < Wo ? 1 : 0, pi = p0 + 1 < Ho ? 1 : 0;
+    int col[5];
+#pragma unroll
+    for (int c = 0; c < 5; ++c) {
+        const int cc = c < 3 ? c : 2 * qj + (c - 2);  // 3, 4 -> window 1's columns 1, 2 (or window 0's)
+        col[c] = min(max(2 * q0 - p + cc, 0), W - 1);
+    }
+    uint4 m00 = make_uint4(0, 0, 0, 0), m01 = m00, m10 = m00, m11 = m00;
+#pragma unroll
+    for (int r = 0; r < 5; ++r) {
+        const int rr = r < 3 ? r : 2 * pi + (r - 2);
+        const int h = min(max(2 * p0 - p + rr, 0), H - 1);
+        const __nv_bfloat16 *row = xn + (size_t)h * W * C;
+        uint4 v[5];
+#pragma unroll
+        for (int c = 0; c < 5; ++c) v[c] = ldg_v4(row + (size_t)col[c] * C);
+        const uint4 a = max8(max8(v[0], v[1]), v[2]);  // window column 0
+        const uint4 b = max8(max8(v[2], v[3]), v[4]);  // window column 1
+        if (r < 3) {
+            m00 = r == 0 ? a : max8(m00, a);
+            m01 = r == 0 ? b : max8(m01, b);
+        }
+        if (r >= 2) {
+            m10 = r == 2 ? a : max8(m10, a);
+            m11 = r == 2 ? b : max8(m11, b);
+        }
+    }
+    __nv_bfloat16 *yo = y + (((size_t)n * Ho + p0) * Wo + q0) * C + cv * 8;
+    *reinterpret_cast<uint4 *>(yo) = m00;
+    if (qj) *reinterpret_cast<uint4 *>(yo + C) = m01;
+    if (pi) {
+        *reinterpret_cast<uint4 *>(yo + (size_t)Wo * C) = m10;
+        if (qj) *reinterpret_cast<uint4 *>(yo + (size_t)Wo * C + C) = m11;
+    }
+}
+
 cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            int k, int s, int p, cudaStream_t st) {
+    if (k == 3 && s == 2) {
+        const int Ho = (H + 2 * p - 3) / 2 + 1;
+        const int Wo = (W + 2 * p - 3) / 2 + 1;
+        const long long total = (long long)N * ((Ho + 1) / 2) * ((Wo + 1) / 2) * (C / 8);
+        if (total < (1ll << 31))
+            return launch_pdl(maxpool3s2_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y,
+                              N, H, W, C, p, Ho, Wo);
+    }
     if (k == 3) {
         const int Ho = (H + 2 * p - 3) / s + 1;
         const int Wo = (W + 2 * p - 3) / s + 1;
