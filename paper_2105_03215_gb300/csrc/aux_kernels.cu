@@ -585,36 +585,56 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
 }
 
 // ------------------------------------------------------------ global average pool
-__global__ void avgpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W,
-                               int C) {
+// Block (channel block, image): 32 groups of 8 channels x 8 pixel slices.
+// Thread (g, sl) sums pixels sl, sl + 8, ... of its group in fp32 (a warp
+// reads 512 contiguous bytes per pixel); the slices are then added in slice
+// order through shared memory (deterministic), scaled by 1 / (H W) and
+// rounded to bf16 once.  64 x 7 x 7 x 2048 (ResNet-50): 512 blocks of 256
+// threads, about six loads in flight per thread.
+constexpr int kAvgGroups = 32, kAvgSlices = 8;
+
+__global__ void __launch_bounds__(kAvgGroups * kAvgSlices)
+    avgpool_kernel(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C) {
     pdl_launch_dependents();
     pdl_wait();
+    __shared__ float red[kAvgSlices][kAvgGroups][8];
     const int CV = C >> 3;
-    const long long total = (long long)N * CV;
-    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= total) return;
-    const int cv = (int)(idx % CV);
-    const int n = (int)(idx / CV);
+    const int cblocks = (CV + kAvgGroups - 1) / kAvgGroups;
+    const int n = blockIdx.x / cblocks;
+    const int cv = (blockIdx.x - n * cblocks) * kAvgGroups + (int)(threadIdx.x % kAvgGroups);
+    const int sl = (int)(threadIdx.x / kAvgGroups);
     float acc[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) acc[j] = 0.0f;
-    const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
-    for (int i = 0; i < H * W; ++i) {
-        float f[8];
-        unpack8(ldg_v4(xn + (size_t)i * C), f);
+    if (cv < CV) {
+        const __nv_bfloat16 *xn = x + (size_t)n * H * W * C + cv * 8;
+        for (int i = sl; i < H * W; i += kAvgSlices) {
+            float f[8];
+            unpack8(ldg_v4(xn + (size_t)i * C), f);
 #pragma unroll
-        for (int j = 0; j < 8; ++j) acc[j] += f[j];
+            for (int j = 0; j < 8; ++j) acc[j] += f[j];
+        }
     }
-    const float inv = 1.0f / (float)(H * W);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) acc[j] *= inv;
-    *reinterpret_cast<uint4 *>(y + (size_t)n * C + cv * 8) = pack8(acc);
+    for (int j = 0; j < 8; ++j) red[sl][threadIdx.x % kAvgGroups][j] = acc[j];
+    __syncthreads();
+    if (sl == 0 && cv < CV) {
+        const int g = (int)threadIdx.x;
+        for (int k = 1; k < kAvgSlices; ++k)
+#pragma unroll
+            for (int j = 0; j < 8; ++j) acc[j] += red[k][g][j];
+        const float inv = 1.0f / (float)(H * W);
+#pragma unroll
+        for (int j = 0; j < 8; ++j) acc[j] *= inv;
+        *reinterpret_cast<uint4 *>(y + (size_t)n * C + cv * 8) = pack8(acc);
+    }
 }
 
 cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int H, int W, int C,
                            cudaStream_t st) {
-    const long long total = (long long)N * (C / 8);
-    return launch_pdl(avgpool_kernel, dim3((unsigned)((total + 255) / 256)), dim3(256), 0, st, x, y, N,
+    const long long blocks = (long long)N * ((C / 8 + kAvgGroups - 1) / kAvgGroups);
+    if (blocks >= (1ll << 31)) return cudaErrorInvalidValue;
+    return launch_pdl(avgpool_kernel, dim3((unsigned)blocks), dim3(kAvgGroups * kAvgSlices), 0, st, x, y, N,
                       H, W, C);
 }
 

@@ -427,3 +427,21 @@ def test_max_pool_3x3_host_operator_bit_exact(N, H, W, C, s):
     torch.cuda.synchronize()
     ref = ops.max_pool2d_nhwc(x, (3, 3), (s, s), (1, 1, 1, 1))
     assert_bit_exact(y.float().cpu().numpy(), ref, f"maxpool {N}x{H}x{W}x{C} s{s}")
+
+
+@pytest.mark.parametrize("N,H,W,C", [(64, 7, 7, 2048), (3, 5, 9, 24), (2, 1, 1, 8), (5, 14, 14, 264)])
+def test_global_avg_pool_host_operator(N, H, W, C):
+    # the host average pool: fp32 sums of pixel slices added in a fixed order,
+    # one bf16 rounding -- within one bf16 rounding of the exact mean
+    import torch
+    from oracle import ops
+    from .parity import to_dev
+    rng = np.random.default_rng(N * 7 + C)
+    x = I.bf16_round(rng.standard_normal((N, H, W, C)).astype(np.float32))
+    y = torch.full((N, C), float("nan"), dtype=torch.bfloat16, device="cuda")
+    abi.check(abi.lib().byoc_global_avg_pool_nhwc(to_dev(x).data_ptr(), y.data_ptr(), N, H, W, C, None))
+    torch.cuda.synchronize()
+    ref = ops.global_avg_pool_nhwc(x)
+    got = y.float().cpu().numpy().astype(np.float64)
+    # bf16 keeps 8 significant bits: |got - ref| <= 2^-8 |ref| + fp32 summation error
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5), f"avgpool {N}x{H}x{W}x{C}"
