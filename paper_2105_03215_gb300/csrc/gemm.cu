@@ -712,11 +712,20 @@ __global__ void __maxnreg__(168)
                 __threadfence();  // the other splits' partials are read after the count
             }
 #pragma unroll 1
-            for (int ci = c_first, kk = 0; ci < NCH; ci += c_step, ++kk) {
+            // chunks holding output columns: the 32-column chunks of a ragged
+            // last column tile that lie wholly past N are neither read nor
+            // stored (split-K partials cover every chunk)
+            const int nch = SPLITK ? NCH : min(NCH, (a.N - n0 + 31) >> 5);
+            if (c_first >= nch) {  // nothing of this tile for this warp
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(tempty + 8u * buf);
+            }
+            for (int ci = c_first, kk = 0; ci < nch; ci += c_step, ++kk) {
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);  // includes tcgen05.wait::ld
-                if (ci + c_step >= NCH) {  // this warp's last read of the accumulator
+                if (ci + c_step >= nch) {  // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty + 8u * buf);
