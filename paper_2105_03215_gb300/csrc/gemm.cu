@@ -36,7 +36,7 @@
 //              stores.
 //   warp 10    producer of the epilogue operands: per tile, the tile's bias
 //              slice (bulk copy) and, when the region adds a residual, the
-//              128 x BN residual tile (TMA) into one of two buffers.
+//              128 x BN residual tile (TMA) into a ring of OPB buffers.
 #include "internal.h"
 #include "ptx.cuh"
 
@@ -66,8 +66,9 @@ struct GemmShape {
     static constexpr int RES_BOX = BM * 64 * 2;
     static constexpr int RES_TILE = RES ? BM * BN * 2 : 0;
     // epilogue-operand buffers (bias slice, residual tile): residual regions
-    // are HBM-bound and keep more residual tiles in flight
-    static constexpr int OPB = RES ? (BN >= 128 ? 3 : 4) : 2;
+    // are HBM-bound and keep more residual tiles in flight; bias-only slices
+    // are small, and eight in flight keep their L2 latency off short tiles
+    static constexpr int OPB = RES ? (BN >= 128 ? 3 : 4) : 8;
     static constexpr int BIAS_BYTES = BN * 4;
     static constexpr int BIAS_REGION = (OPB * BIAS_BYTES + 1023) / 1024 * 1024;
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
