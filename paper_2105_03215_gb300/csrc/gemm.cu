@@ -135,10 +135,17 @@ __global__ void __maxnreg__(168)
                         const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
     using S = GemmShape<BN, BK, AMODE, RES>;
     constexpr bool PAIR = S::PAIR;
-    // epilogue warps that read each accumulator: one group of four for
-    // narrow single tiles (groups alternate tiles), both groups otherwise
-    // (wide tiles: alternate 32-column chunks; pair units: one half each)
-    constexpr int kEpiArrivals = BN <= 64 && !PAIR ? kGemmEpiWarps / 2 : kGemmEpiWarps;
+    // The two epilogue warp groups take alternate tiles (all chunks each) for
+    // narrow tiles, and for launches of one column tile whose tiles hold an
+    // odd number of 32-column chunks (a 2 + 1 chunk split would leave one
+    // group idle half the time); otherwise both take every tile, splitting
+    // its chunks (pair units: one half each).  Epilogue warps that read each
+    // accumulator: four when alternating, else eight.
+    // (the run-time choice only where it occurs: 128-wide plain tiles)
+    constexpr bool ALT_RT = BN == 128 && AMODE == kAModeTile && !RES;
+    const bool alt = (BN <= 64 && !PAIR) ||
+                     (ALT_RT && a.tiles_n == 1 && ((min(BN / 32, (a.N + 31) >> 5)) & 1));
+    const int epi_arrivals = alt ? kGemmEpiWarps / 2 : kGemmEpiWarps;
     // split-K: a work unit is (tile, split); split sp covers k-blocks
     // [sp * num_kb / SPL, (sp + 1) * num_kb / SPL)
     constexpr bool SPLITK = AMODE == kAModeTileSplit;
@@ -178,7 +185,7 @@ __global__ void __maxnreg__(168)
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull + 8u * b, 1);                 // MMA commit
-            mbar_init(tempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
+            mbar_init(tempty + 8u * b, epi_arrivals);     // one arrive per epilogue warp of the tile
         }
         for (int b = 0; b < S::SLOTS_MAX; ++b) {
             mbar_init(sfull + 8u * b, 1);                 // producer + slab bytes
@@ -186,7 +193,7 @@ __global__ void __maxnreg__(168)
         }
         for (int b = 0; b < S::OPB; ++b) {
             mbar_init(ofull + 8u * b, 1);                 // operand producer + bytes
-            mbar_init(oempty + 8u * b, kEpiArrivals);     // one arrive per epilogue warp of the tile
+            mbar_init(oempty + 8u * b, epi_arrivals);     // one arrive per epilogue warp of the tile
         }
         mbar_init(drain, 1);
         *abort_flag = 0;
@@ -599,11 +606,12 @@ __global__ void __maxnreg__(168)
         const int e = warp - 2;            // 0..7
         const int quarter = warp & 3;      // TMEM lanes (= tile rows) this warp may access
         constexpr int NCH = BN / 32;       // 32-column chunks per tile
-        // BN <= 64: the two groups take alternate tiles (accumulator t % 2), all
-        // chunks each.  BN >= 128: both groups take every tile, group `grp`
+        // alt: the two groups take alternate tiles (accumulator t % 2), all
+        // chunks each.  Otherwise both groups take every tile, group `grp`
         // the chunks ci with ci % 2 == grp, so that a tile's accumulator is
         // read, and released to the MMAs, twice as fast.  Pair units: group
-        // `grp` takes half `grp` of every unit, all chunks.
+        // `grp` takes half `grp` of every unit, all chunks.  (Split-K keeps
+        // the compile-time choice ALT: its partial layout depends on it.)
         constexpr bool ALT = BN <= 64 && !PAIR;
         const int grp = e >> 2;
         const uint32_t stg = sEpi + (uint32_t)e * S::EPI_TILE;
@@ -613,8 +621,8 @@ __global__ void __maxnreg__(168)
         // writes and the coalesced reads below are free of bank conflicts.
         const uint32_t sw_own = ((uint32_t)lane >> 1) & 3u;
         const int cl_row = lane >> 2, cl_piece = lane & 3;  // coalesced: rows 8k + lane/4
-        const int t_first = ALT ? grp : 0, t_step = ALT ? 2 : 1;
-        const int c_first = ALT || PAIR ? 0 : grp, c_step = ALT || PAIR ? 1 : 2;
+        const int t_first = alt ? grp : 0, t_step = alt ? 2 : 1;
+        const int c_first = alt || PAIR ? 0 : grp, c_step = alt || PAIR ? 1 : 2;
         const int half = PAIR ? grp : 0;
         for (int unit = blockIdx.x + t_first * (int)gridDim.x, t = t_first; unit < num_units;
              unit += t_step * (int)gridDim.x, t += t_step) {
