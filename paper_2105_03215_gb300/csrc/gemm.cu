@@ -73,10 +73,18 @@ struct GemmShape {
     static constexpr int BIAS_REGION = (OPB * BIAS_BYTES + 1023) / 1024 * 1024;
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
-    static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE;
+    // plain tile mode stores its output with TMA from each warp's staging
+    // tile; the others read the staging tile back for coalesced stores
+    static constexpr bool TSTORE = AMODE == kAModeTile && !RES;
     static constexpr int CTRL_BYTES = 1024;
-    static constexpr int FIXED =
-        1024 + 2 * SLAB_BYTES + OPB * RES_TILE + EPI_BYTES + BIAS_REGION + CTRL_BYTES;
+    // TMA-store mode keeps a second staging tile per warp (one store in
+    // flight while the next chunk is staged) where the weight ring still
+    // has 8 stages with it: short-k-block configs (BK 16 / 32)
+    static constexpr int FIXED1 = 1024 + 2 * SLAB_BYTES + OPB * RES_TILE + BIAS_REGION + CTRL_BYTES;
+    static constexpr int EPI_BUFS =
+        TSTORE && (232448 - FIXED1 - 2 * kGemmEpiWarps * EPI_TILE) / STAGE_BYTES >= 8 ? 2 : 1;
+    static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE * EPI_BUFS;
+    static constexpr int FIXED = FIXED1 + EPI_BYTES;
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 32 ? 32 : STAGES_RAW;  // ring slots (k-blocks)
     static constexpr int POOL_BYTES = STAGES * STAGE_BYTES + 2 * SLAB_BYTES;
@@ -202,7 +210,7 @@ __global__ void __maxnreg__(168)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
-        if (RES) tma_prefetch_desc(&tmR);
+        if (RES || S::TSTORE) tma_prefetch_desc(&tmR);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), S::TMEM_COLS);
@@ -614,7 +622,8 @@ __global__ void __maxnreg__(168)
         // the compile-time choice ALT: its partial layout depends on it.)
         constexpr bool ALT = BN <= 64 && !PAIR;
         const int grp = e >> 2;
-        const uint32_t stg = sEpi + (uint32_t)e * S::EPI_TILE;
+        const uint32_t stg0 = sEpi + (uint32_t)(e * S::EPI_BUFS) * S::EPI_TILE;
+        int sb = 0;  // staging tile of the next chunk (TMA-store mode with two)
         const int trow = quarter * 32 + lane;  // this thread's row within the tile
         // 64-byte swizzle of the 32x32 bf16 staging tile: 16-byte piece c of
         // row r sits at piece c ^ ((r >> 1) & 3), so both the row-per-thread
@@ -806,6 +815,13 @@ __global__ void __maxnreg__(168)
                     for (int j = 0; j < 32; ++j) f[j] = apply_act(f[j], a.act);
                 }
                 // this thread's row -> swizzled staging -> coalesced global stores
+                // (TMA-store mode: one bulk tensor store of the 32 x 32 tile;
+                // the staging layout is the 64-byte swizzle TMA reads)
+                const uint32_t stg = stg0 + (uint32_t)(sb * S::EPI_TILE);
+                if constexpr (S::TSTORE) {
+                    // the store that last used this staging tile has read it
+                    if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
+                }
                 __syncwarp();
 #pragma unroll
                 for (int q = 0; q < 4; ++q) {
@@ -817,6 +833,17 @@ __global__ void __maxnreg__(168)
                     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0),
                                  "r"(w1), "r"(w2), "r"(w3)
                                  : "memory");
+                }
+                if constexpr (S::TSTORE) {
+                    // rows past M and columns past N are not written by TMA
+                    fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        tma_store_2d(&tmR, stg, col0, mt * S::BM + quarter * 32);
+                        bulk_commit_group();
+                    }
+                    if (S::EPI_BUFS == 2) sb ^= 1;
+                    continue;
                 }
                 __syncwarp();
                 const int gcol = col0 + cl_piece * 8;
@@ -837,6 +864,12 @@ __global__ void __maxnreg__(168)
             // bias / residual reads of this tile are done (ordered by __syncwarp)
             __syncwarp();
             if (lane == 0) mbar_arrive(oempty + 8u * ob);
+        }
+        if constexpr (S::TSTORE) {
+            // the output is written before the CTA exits (and its staging
+            // tiles stay valid until TMA has read them)
+            if (lane == 0) bulk_wait_group<0>();
+            __syncwarp();
         }
     }
 

@@ -75,6 +75,18 @@ CUresult encode(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, u
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// Output [rows, cols] bf16 in 32 x 32 boxes, 64-byte swizzle: the map the
+// GEMM's plain tile mode stores its output through.
+CUresult encode_out(CUtensorMap *m, void *ptr, uint64_t rows, uint64_t cols) {
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols * 2};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t es[2] = {1, 1};
+    return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, ptr, dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 bool misaligned(const void *p) { return !p || (reinterpret_cast<uintptr_t>(p) & 15u); }
 
 }  // namespace
@@ -118,11 +130,13 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     if ((e = cudaMemsetAsync(err_word, 0, sizeof(int), st)) != cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: clearing the error word");
 
-    CUtensorMap a1, b1m, a2, b2m;
+    CUtensorMap a1, b1m, a2, b2m, o1, o2;
     if (encode(&a1, x, (uint64_t)M, (uint64_t)D, byoc::kGemmBM) != CUDA_SUCCESS ||
         encode(&b1m, w1, (uint64_t)F, (uint64_t)D, kTileN) != CUDA_SUCCESS ||
         encode(&a2, hidden, (uint64_t)M, (uint64_t)F, byoc::kGemmBM) != CUDA_SUCCESS ||
-        encode(&b2m, w2, (uint64_t)D, (uint64_t)F, kTileN) != CUDA_SUCCESS)
+        encode(&b2m, w2, (uint64_t)D, (uint64_t)F, kTileN) != CUDA_SUCCESS ||
+        encode_out(&o1, hidden, (uint64_t)M, (uint64_t)F) != CUDA_SUCCESS ||
+        encode_out(&o2, y, (uint64_t)M, (uint64_t)D) != CUDA_SUCCESS)
         return fail(BYOC_ERR_CUDA, "byoc_ffn_noalloc: encoding a TMA descriptor failed");
 
     const byoc::GemmConfig cfg{kTileN, 64, byoc::kAModeTile, false};
@@ -144,7 +158,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.residual = nullptr;
     g.out = hidden;
     g.err = err_word;
-    if ((e = byoc::launch_gemm(cfg, a1, b1m, a1, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a1, b1m, o1, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: first GEMM launch");
     g.N = D;
@@ -156,7 +170,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.act = byoc::kActNone;
     g.bias = b2;
     g.out = static_cast<__nv_bfloat16 *>(y);
-    if ((e = byoc::launch_gemm(cfg, a2, b2m, a2, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a2, b2m, o2, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: second GEMM launch");
     return BYOC_OK;

@@ -1550,8 +1550,19 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                                 i, (int)r);
                 h->tmR_ptr[i] = a.residual;
             }
-            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a.residual ? h->tmR[i] : h->tmA[i], a,
-                                  L.grid, st);
+            // plain tile mode stores its output with TMA: [M, N] in 32 x 32 boxes,
+            // 64-byte swizzle (the layout of the epilogue's staging tiles); it
+            // travels in the residual map's slot, which that mode leaves unused
+            const bool tstore = L.cfg.amode == byoc::kAModeTile && !L.cfg.res;
+            if (tstore && h->tmR_ptr[i] != a.out) {
+                CUresult r = encode_2d(&h->tmR[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 32);
+                if (r != CUDA_SUCCESS)
+                    return fail(BYOC_ERR_CUDA, "launch %zu: encoding the output TMA map failed (%d)", i,
+                                (int)r);
+                h->tmR_ptr[i] = a.out;
+            }
+            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], (a.residual || tstore) ? h->tmR[i] : h->tmA[i],
+                                  a, L.grid, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
