@@ -73,9 +73,9 @@ struct GemmShape {
     static constexpr int BIAS_REGION = (OPB * BIAS_BYTES + 1023) / 1024 * 1024;
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
-    // plain tile mode stores its output with TMA from each warp's staging
-    // tile; the others read the staging tile back for coalesced stores
-    static constexpr bool TSTORE = AMODE == kAModeTile && !RES;
+    // tile mode stores its output with TMA from each warp's staging tile;
+    // the others read the staging tile back for coalesced stores
+    static constexpr bool TSTORE = AMODE == kAModeTile;
     static constexpr int CTRL_BYTES = 1024;
     // TMA-store mode keeps a second staging tile per warp (one store in
     // flight while the next chunk is staged) where the weight ring still
@@ -140,7 +140,8 @@ template <int BN, int BK, int AMODE, bool RES>
 __global__ void __maxnreg__(168)
     gemm_tcgen05_kernel(const __grid_constant__ CUtensorMap tmA,
                         const __grid_constant__ CUtensorMap tmB,
-                        const __grid_constant__ CUtensorMap tmR, const GemmArgs a) {
+                        const __grid_constant__ CUtensorMap tmR,
+                        const __grid_constant__ CUtensorMap tmO, const GemmArgs a) {
     using S = GemmShape<BN, BK, AMODE, RES>;
     constexpr bool PAIR = S::PAIR;
     // The two epilogue warp groups take alternate tiles (all chunks each) for
@@ -210,7 +211,8 @@ __global__ void __maxnreg__(168)
     if (warp == 0 && lane == 0) {
         tma_prefetch_desc(&tmA);
         tma_prefetch_desc(&tmB);
-        if (RES || S::TSTORE) tma_prefetch_desc(&tmR);
+        if (RES) tma_prefetch_desc(&tmR);
+        if (S::TSTORE) tma_prefetch_desc(&tmO);
     }
     if (warp == 1) {
         tmem_alloc(smem_u32(tmem_slot), S::TMEM_COLS);
@@ -839,7 +841,7 @@ __global__ void __maxnreg__(168)
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_2d(&tmR, stg, col0, mt * S::BM + quarter * 32);
+                        tma_store_2d(&tmO, stg, col0, mt * S::BM + quarter * 32);
                         bulk_commit_group();
                     }
                     if (S::EPI_BUFS == 2) sb ^= 1;
@@ -886,10 +888,10 @@ __global__ void __maxnreg__(168)
 
 template <int BN, int BK, int AMODE, bool RES>
 static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap &tmR,
-                            const GemmArgs &a, int grid, cudaStream_t st) {
+                            const CUtensorMap &tmO, const GemmArgs &a, int grid, cudaStream_t st) {
     using S = GemmShape<BN, BK, AMODE, RES>;
     return launch_pdl(gemm_tcgen05_kernel<BN, BK, AMODE, RES>, dim3(grid), dim3(kGemmThreads),
-                      (size_t)S::SMEM_BYTES, st, tmA, tmB, tmR, a);
+                      (size_t)S::SMEM_BYTES, st, tmA, tmB, tmR, tmO, a);
 }
 
 template <int BN, int BK, int AMODE, bool RES>
@@ -1003,10 +1005,11 @@ cudaError_t gemm_prepare(const GemmConfig &c) {
 }
 
 cudaError_t launch_gemm(const GemmConfig &c, const CUtensorMap &tmA, const CUtensorMap &tmB,
-                        const CUtensorMap &tmR, const GemmArgs &a, int grid, cudaStream_t st) {
+                        const CUtensorMap &tmR, const CUtensorMap &tmO, const GemmArgs &a, int grid,
+                        cudaStream_t st) {
 #define X(BN_, BK_, AM_, RES_)                                             \
     if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
-        return launch_t<BN_, BK_, AM_, RES_>(tmA, tmB, tmR, a, grid, st);
+        return launch_t<BN_, BK_, AM_, RES_>(tmA, tmB, tmR, tmO, a, grid, st);
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;

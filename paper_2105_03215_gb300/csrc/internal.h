@@ -150,13 +150,14 @@ int gemm_stages(const GemmConfig &cfg);
 bool gemm_slab_res_fits(const GemmConfig &cfg, int num_kb, int slab_bytes);
 void gemm_slab_pool(const GemmConfig &cfg, GemmArgs &a);
 cudaError_t gemm_prepare(const GemmConfig &cfg);  // raises the dynamic smem limit
-// tmR: with cfg.res, the residual [M, N] bf16 in 64-column x 128-row boxes,
-// 128-byte swizzle; in plain tile mode (kAModeTile, no residual), the OUTPUT
-// a.out [M, N] bf16 in 32-column x 32-row boxes, 64-byte swizzle, which the
-// epilogue stores through (required: any other map is written through);
-// otherwise unused.  a.bias must cover tiles_n * bn floats.
+// tmR: the residual [M, N] bf16 in 64-column x 128-row boxes, 128-byte
+// swizzle (read only when cfg.res).  tmO: in tile mode (kAModeTile), the
+// OUTPUT a.out [M, N] bf16 in 32-column x 32-row boxes, 64-byte swizzle,
+// which the epilogue stores through (required: any other map is written
+// through); unused in the other modes.  a.bias must cover tiles_n * bn floats.
 cudaError_t launch_gemm(const GemmConfig &cfg, const CUtensorMap &tmA, const CUtensorMap &tmB,
-                        const CUtensorMap &tmR, const GemmArgs &a, int grid, cudaStream_t st);
+                        const CUtensorMap &tmR, const CUtensorMap &tmO, const GemmArgs &a, int grid,
+                        cudaStream_t st);
 
 // Depthwise conv (groups = C), square kernel k in {3}, NHWC bf16, folded
 // weights fp32 [k*k][C] (tap-major), bias fp32 [C], fused activation.

@@ -158,7 +158,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.residual = nullptr;
     g.out = hidden;
     g.err = err_word;
-    if ((e = byoc::launch_gemm(cfg, a1, b1m, o1, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a1, b1m, a1, o1, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: first GEMM launch");
     g.N = D;
@@ -170,7 +170,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     g.act = byoc::kActNone;
     g.bias = b2;
     g.out = static_cast<__nv_bfloat16 *>(y);
-    if ((e = byoc::launch_gemm(cfg, a2, b2m, o2, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
+    if ((e = byoc::launch_gemm(cfg, a2, b2m, a2, o2, g, g.num_tiles < d.num_sms ? g.num_tiles : d.num_sms, st)) !=
         cudaSuccess)
         return cuda_fail(e, "byoc_ffn_noalloc: second GEMM launch");
     return BYOC_OK;

@@ -1084,6 +1084,8 @@ struct byoc_handle {
     std::vector<const void *> tmA_ptr;    // pointer each cached A map encodes
     std::vector<CUtensorMap> tmR;         // per launch: residual map, cached
     std::vector<const void *> tmR_ptr;
+    std::vector<CUtensorMap> tmO;         // per launch: output map (tile mode), cached
+    std::vector<const void *> tmO_ptr;
     std::vector<void *> ptrs;             // scratch: resolved tensor pointers
 };
 
@@ -1204,6 +1206,8 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
     h->tmA_ptr.assign(nl, nullptr);
     h->tmR.resize(nl);
     h->tmR_ptr.assign(nl, nullptr);
+    h->tmO.resize(nl);
+    h->tmO_ptr.assign(nl, nullptr);
     h->ptrs.assign(P.tensors.size(), nullptr);
     for (size_t i = 0; i < nl; ++i) {
         LaunchPlan &L = P.launches[i];
@@ -1550,19 +1554,18 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                                 i, (int)r);
                 h->tmR_ptr[i] = a.residual;
             }
-            // plain tile mode stores its output with TMA: [M, N] in 32 x 32 boxes,
-            // 64-byte swizzle (the layout of the epilogue's staging tiles); it
-            // travels in the residual map's slot, which that mode leaves unused
-            const bool tstore = L.cfg.amode == byoc::kAModeTile && !L.cfg.res;
-            if (tstore && h->tmR_ptr[i] != a.out) {
-                CUresult r = encode_2d(&h->tmR[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 32);
+            // tile mode stores its output with TMA: [M, N] in 32 x 32 boxes,
+            // 64-byte swizzle (the layout of the epilogue's staging tiles)
+            const bool tstore = L.cfg.amode == byoc::kAModeTile;
+            if (tstore && h->tmO_ptr[i] != a.out) {
+                CUresult r = encode_2d(&h->tmO[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 32);
                 if (r != CUDA_SUCCESS)
                     return fail(BYOC_ERR_CUDA, "launch %zu: encoding the output TMA map failed (%d)", i,
                                 (int)r);
-                h->tmR_ptr[i] = a.out;
+                h->tmO_ptr[i] = a.out;
             }
-            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], (a.residual || tstore) ? h->tmR[i] : h->tmA[i],
-                                  a, L.grid, st);
+            e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a.residual ? h->tmR[i] : h->tmA[i],
+                                  tstore ? h->tmO[i] : h->tmA[i], a, L.grid, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
