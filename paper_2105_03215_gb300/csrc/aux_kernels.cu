@@ -1,8 +1,9 @@
 // aux_kernels.cu -- the bandwidth-bound kernels of the offloaded path:
 //   * depthwise 3x3 conv + folded BN + activation (MobileNetV2 composite),
-//   * the space-to-depth boundary transform that turns a stride-2 stem over
-//     3 channels into a stride-1 convolution over 16 channels (a layout
-//     transformation node inserted at a region boundary, Section 3.2),
+//   * the layout transform of a stride-2 stem over <= 4 channels: the image
+//     with 4 channels and zero padding, read by the stem's GEMM as pixel
+//     pairs (a layout transformation node inserted at a region boundary,
+//     Section 3.2), and the NCHW fp32 -> NHWC bf16 boundary transform,
 //   * the host-graph operators of ResNet-50 (max pool, global average pool),
 //     which the paper leaves on the host (Section 3.4, CUDA as the host).
 // All tensors are bf16 NHWC; every thread moves 8 channels (16 bytes) at a

@@ -229,7 +229,7 @@ struct LaunchPlan {
     size_t part_off = 0, part_bytes = 0, cnt_off = 0, cnt_bytes = 0;
     // constants: byte offsets into the constant blob
     size_t w_off = 0, w_bytes = 0, b_off = 0, b_bytes = 0;
-    // depthwise / space-to-depth / fused depthwise -> 1x1
+    // depthwise / stem layout transform / fused depthwise -> 1x1
     byoc::DwArgs dw{};
     byoc::StemArgs stem{};
     int stem_R = 0;  // stem GEMM: row taps per slab position (StemArgs layout), else 0
