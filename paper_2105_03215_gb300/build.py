@@ -41,7 +41,10 @@ def _digest() -> str:
             h.update(n.encode())
             with open(p, "rb") as f:
                 h.update(f.read())
-    h.update(" ".join(ARCH + FLAGS).encode())
+    # the flags without the checkout's absolute paths, so that a copy of the
+    # same sources elsewhere has the same digest
+    flags = [{INCLUDE: "<include>", CSRC: "<csrc>"}.get(f, f) for f in ARCH + FLAGS]
+    h.update(" ".join(flags).encode())
     h.update(os.uname().machine.encode())
     return h.hexdigest()
 
