@@ -147,7 +147,7 @@ def test_bottleneck_full():
     _check_graph(g, inp)
 
 
-def test_stem_space_to_depth():
+def test_resnet50_stem_region():
     g, inp = I.resnet50(N=2, H=64, W=48, seed=4)
     stem = [n.name for n in g.nodes[:3]]  # conv 7x7/2 + bn + relu
     reg = R.Region(g, stem, "stem")
