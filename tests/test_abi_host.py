@@ -339,3 +339,23 @@ def test_pair_units_only_where_a_tile_has_few_mmas():
                           N=32, H=24, W=100, C=64, K=64)
     rep = _plan(g)
     assert rep.pair_units[0] == 1 and rep.resident_b[0] == 1 and rep.slab_slots[0] >= 2
+
+
+def test_source_digest_is_independent_of_the_checkout_path(tmp_path, monkeypatch):
+    # bench.py reports the profiled DRAM traffic only while the sources hash
+    # to the digest stored beside it: a copy of the same sources elsewhere
+    # must hash the same, and any change of a source must not
+    import shutil
+    from paper_2105_03215_gb300 import build as B
+    want = B._digest()
+    root = tmp_path / "copy"
+    shutil.copytree(B.CSRC, root / "pkg" / "csrc")
+    shutil.copytree(B.INCLUDE, root / "include")
+    csrc, inc = str(root / "pkg" / "csrc"), str(root / "include")
+    monkeypatch.setattr(B, "FLAGS", [{B.INCLUDE: inc, B.CSRC: csrc}.get(f, f) for f in B.FLAGS])
+    monkeypatch.setattr(B, "CSRC", csrc)
+    monkeypatch.setattr(B, "INCLUDE", inc)
+    assert B._digest() == want
+    with open(os.path.join(csrc, "ptx.cuh"), "a") as f:
+        f.write("\n")
+    assert B._digest() != want
