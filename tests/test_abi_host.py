@@ -359,3 +359,28 @@ def test_source_digest_is_independent_of_the_checkout_path(tmp_path, monkeypatch
     with open(os.path.join(csrc, "ptx.cuh"), "a") as f:
         f.write("\n")
     assert B._digest() != want
+
+
+@pytest.mark.parametrize("k,C,cout", [(3, 3, 32), (5, 4, 48), (7, 1, 64)])
+def test_stem_weights_for_every_filter_size(k, C, cout):
+    # w'[k][b][r*8 + dx*4 + c] = w[k][c][r][2b+dx] with R = 4 row taps (k = 3)
+    # or 8 (k = 5, 7) and zero where r >= k, 2b + dx >= k or c >= C
+    g, _ = I.stem(N=1, H=32, W=30, k=k, cout=cout, C=C)
+    reg = R.whole_graph_region(g)
+    rep = reg.plan()
+    k2, Rr = (k + 1) // 2, (4 if k <= 3 else 8)
+    assert rep.gemm_k[1] == k2 * 8 * Rr and rep.tile_k[1] == 8 * Rr
+    w = g.nodes[0].consts["weight"].astype(np.float64)            # [cout, C, k, k]
+    bn = g.nodes[1]
+    scale = bn.consts["gamma"].astype(np.float64) / np.sqrt(
+        bn.consts["moving_var"].astype(np.float64) + bn.attrs.get("epsilon", 1e-5))
+    packed = np.frombuffer(reg.plan_constants(1, 0), dtype=np.uint16).reshape(-1, rep.gemm_k[1])
+    expect = np.zeros((cout, k2, Rr, 2, 4), dtype=np.float64)     # [k][b][r][dx][c]
+    for b in range(k2):
+        for r in range(k):
+            for dx in range(2):
+                if 2 * b + dx < k:
+                    expect[:, b, r, dx, :C] = w[:, :, r, 2 * b + dx]
+    expect *= scale[:, None, None, None, None]
+    want = I.bf16_bits(expect.reshape(cout, -1).astype(np.float32))
+    assert np.array_equal(packed[:cout], want)
