@@ -205,6 +205,7 @@ def time_region(cr, ins, outs, flush, reps=20):
 def region_figures(flush, peaks):
     """Configs 1-4 of the workload list, each as one region (cold L2)."""
     import torch
+    from paper_2105_03215_gb300 import abi
     from paper_2105_03215_gb300 import inputs as I
     from paper_2105_03215_gb300 import region as R
     out = {}
@@ -227,9 +228,7 @@ def region_figures(flush, peaks):
                      "hbm_frac_of_measured": gb / peaks["hbm_gbs"]}
         if name.startswith("mbv2"):
             # the same region as one fused kernel (depthwise output kept on chip)
-            os.environ["BYOC_FUSE_DW_PW"] = "1"
-            fcr = reg.compile()
-            os.environ.pop("BYOC_FUSE_DW_PW")
+            fcr = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW).compile()
             tfz = time_region(fcr, ins, outs, flush)
             out[name + "_fused"] = {"us": tfz * 1e6, "gbps": fcr.bytes / tfz / 1e9, "launches": fcr.n_launches,
                                     "hbm_frac_of_measured": fcr.bytes / tfz / 1e9 / peaks["hbm_gbs"]}
@@ -254,10 +253,7 @@ def region_figures(flush, peaks):
     st = torch.cuda.current_stream()
     for tag, mo in (("", 1), ("_fused", None)):
         mres, minp = E.build_mobilenet_v2(N=BATCH, H=IMG, W=IMG, max_ops=mo)
-        if tag:
-            os.environ["BYOC_FUSE_DW_PW"] = "1"
-        mex = E.Executor(mres)
-        os.environ.pop("BYOC_FUSE_DW_PW", None)
+        mex = E.Executor(mres, options=abi.OPT_FUSE_DW_PW if tag else 0)
         mex.set_input("data", torch.from_numpy(minp["data"]).to(torch.bfloat16).cuda())
         mex.capture()
         for _ in range(3):
@@ -279,7 +275,6 @@ def region_figures(flush, peaks):
         mex.release()
     # the boundary layout transformation (Section 3.2) of the ResNet-50 input:
     # NCHW fp32 [64,3,224,224] -> NHWC bf16, one launch, HBM-bound
-    from paper_2105_03215_gb300 import abi
     xs = torch.randn(BATCH, 3, IMG, IMG, device="cuda")
     ys = torch.empty(BATCH, IMG, IMG, 3, dtype=torch.bfloat16, device="cuda")
     tb = []

@@ -47,7 +47,7 @@
 extern "C" {
 #endif
 
-#define BYOC_ABI_VERSION 1u
+#define BYOC_ABI_VERSION 2u
 
 typedef struct byoc_handle byoc_handle; /* opaque: packed constants, workspace, plans */
 
@@ -115,7 +115,19 @@ typedef struct {
     const int32_t *input_ids;     /* order of byoc_run's inputs[] */
     int32_t n_outputs;
     const int32_t *output_ids;    /* order of byoc_run's outputs[] */
+    uint32_t options;             /* BYOC_OPT_* bits: code-generation choices for this region */
 } byoc_region_desc;
+
+/* Code-generation options of one region (byoc_region_desc.options).  They
+ * choose between kernel plans that compute the same values; the choice is
+ * made at compile time and kept in the compiled (and serialised) plan.
+ *   BYOC_OPT_FUSE_DW_PW: a depthwise composite and the 1x1 composite that
+ *     consumes it run as one kernel whose depthwise output stays in shared
+ *     memory (the data-transfer saving that motivates merging operators into
+ *     one region, Section 3.1.2).  Off by default: on GB300 the depthwise
+ *     arithmetic, not HBM, bounds that kernel, and two launches are faster
+ *     on the MobileNetV2 shapes.  Results are bit-identical either way. */
+#define BYOC_OPT_FUSE_DW_PW 0x1u
 
 /* Figures describing a compiled region. */
 typedef struct {

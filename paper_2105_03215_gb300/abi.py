@@ -11,7 +11,10 @@ import os
 import threading
 from ctypes import POINTER, c_char_p, c_double, c_float, c_int32, c_int64, c_size_t, c_uint32, c_void_p
 
-ABI_VERSION = 1
+ABI_VERSION = 2
+
+# byoc_region_desc.options
+OPT_FUSE_DW_PW = 0x1
 
 # byoc_status
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
@@ -47,7 +50,7 @@ class RegionDesc(ctypes.Structure):
     _fields_ = [("abi_version", c_uint32), ("name", c_char_p), ("n_tensors", c_int32),
                 ("tensors", POINTER(Tensor)), ("n_ops", c_int32), ("ops", POINTER(Op)),
                 ("n_inputs", c_int32), ("input_ids", POINTER(c_int32)), ("n_outputs", c_int32),
-                ("output_ids", POINTER(c_int32))]
+                ("output_ids", POINTER(c_int32)), ("options", c_uint32)]
 
 
 class Info(ctypes.Structure):

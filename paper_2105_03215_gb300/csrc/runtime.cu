@@ -510,17 +510,6 @@ struct Affine {
     std::vector<double> scale, shift;
 };
 
-// Whether a depthwise composite and the 1x1 composite that consumes it, in
-// one region, are planned as one fused launch (dwpw.cu) rather than two.
-// Off unless BYOC_FUSE_DW_PW=1: on GB300 the fused kernel moves a third of
-// the bytes but its depthwise arithmetic, not HBM, bounds it, and the two
-// launches measure faster on the MobileNetV2 shapes.  Read at planning time,
-// so a compiled (or serialised) region keeps the choice it was made with.
-bool fuse_dw_pw() {
-    const char *f = std::getenv("BYOC_FUSE_DW_PW");
-    return f && f[0] == '1';
-}
-
 // Builds the launch list (no device work).
 byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
     P = Plan();
@@ -629,7 +618,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
             // is the depthwise output's only consumer: the intermediate stays
             // in shared memory (the gain of merging the two composites into
             // one region).
-            if (fuse_dw_pw() && j < d->n_ops && consumers[cur] == 1 && !is_output[cur] &&
+            if ((d->options & BYOC_OPT_FUSE_DW_PW) && j < d->n_ops && consumers[cur] == 1 && !is_output[cur] &&
                 act != byoc::kActGelu) {
                 const byoc_op &pw = d->ops[j];
                 if (pw.kind == BYOC_OP_CONV2D && pw.in[0] == cur && pw.groups == 1 && pw.kernel[0] == 1 &&

@@ -24,8 +24,10 @@ HOST_OPS = ("nn.max_pool2d", "nn.global_avg_pool2d", "nn.batch_flatten")
 
 
 class Executor:
-    def __init__(self, result: PartitionResult, serialized: Optional[List[bytes]] = None):
-        """Compile every region of ``result`` -- or, given ``serialized`` (one
+    def __init__(self, result: PartitionResult, serialized: Optional[List[bytes]] = None,
+                 options: int = 0):
+        """Compile every region of ``result`` with the code-generation
+        ``options`` (abi.OPT_* bits) -- or, given ``serialized`` (one
         ``CompiledRegion.serialize()`` blob per region, from ``serialize()``),
         load them without compiling (Section 3.3, option 3).  ``init_s`` is
         the wall time of that step (the engine initialisation of Section 4.1)."""
@@ -38,6 +40,8 @@ class Executor:
         self.by_name = {n.name: n for n in g.nodes}
         # steps: ("region", index) or ("host", node name), in a topological order
         self.regions = result.region_objects()
+        for r in self.regions:
+            r.options = int(options)
         t0 = time.perf_counter()
         if serialized is None:
             self.compiled = [r.compile() for r in self.regions]

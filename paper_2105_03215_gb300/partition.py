@@ -3,7 +3,7 @@ annotation of supported operators, greedy merging into regions, cost-based
 splitting and host fallback, and encapsulation of each region as a function
 with a target attribute.
 
-Readings of points the paper leaves open (each one is listed in the design doc):
+Readings of points the paper leaves open:
   * ``optional`` matches the sequence with and without the optional node; at
     one root the longer match is taken.
   * The pattern table is applied in order; each pattern is tried at every

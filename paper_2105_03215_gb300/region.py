@@ -46,8 +46,12 @@ class Region:
     """A set of nodes of ``graph`` encapsulated as one offloaded function."""
 
     def __init__(self, graph: Graph, node_names: Sequence[str], name: str = "region",
-                 outputs: Optional[Sequence[str]] = None):
+                 outputs: Optional[Sequence[str]] = None, options: int = 0):
+        """``options``: abi.OPT_* bits passed to the code generator
+        (byoc_region_desc.options); they pick among kernel plans that compute
+        the same values."""
         self.graph = graph
+        self.options = int(options)
         members = set(node_names)
         # ops keep the given order (the descriptor's op order, which decides
         # what the engine fuses); it must be topological within the region
@@ -130,7 +134,7 @@ class Region:
         cname = self.name.encode()
         keep += [in_ids, out_ids, cname]
         desc = abi.RegionDesc(abi.ABI_VERSION, cname, len(names), tensors, len(self.nodes), ops,
-                              len(self.inputs), in_ids, len(self.outputs), out_ids)
+                              len(self.inputs), in_ids, len(self.outputs), out_ids, self.options)
         return desc, keep
 
     # -------------------------------------------------------------- planning / compile
@@ -239,7 +243,7 @@ class CompiledRegion:
             pass
 
 
-def whole_graph_region(graph: Graph, name: Optional[str] = None) -> Region:
+def whole_graph_region(graph: Graph, name: Optional[str] = None, options: int = 0) -> Region:
     """All nodes of ``graph`` as one region (the offload-everything case)."""
     return Region(graph, [n.name for n in graph.nodes], name or graph.name or "region",
-                  outputs=graph.outputs)
+                  outputs=graph.outputs, options=options)

@@ -1,7 +1,7 @@
 """Run one offloaded region repeatedly, for profilers (ncu) and quick timing.
 
-  python -m paper_2105_03215_gb300.profile_region --workload resnet50 --batch 64 --region 5
-  python -m paper_2105_03215_gb300.profile_region --workload mbv2_dw_pw --reps 5 --time
+  python profile_region.py --workload resnet50 --batch 64 --region 5
+  python profile_region.py --workload mbv2_dw_pw --reps 5 --time
 
 ``--region i`` picks the i-th region of ResNet-50 partitioned one composite
 per region; the other workloads run as a single region.  Inputs are random
@@ -12,7 +12,13 @@ algorithmic TFLOP/s and GB/s are printed.
 from __future__ import annotations
 
 import argparse
+import os
 import statistics
+import sys
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
 
 
 def main():
@@ -27,13 +33,16 @@ def main():
     ap.add_argument("--warmup", type=int, default=2)
     ap.add_argument("--time", action="store_true")
     ap.add_argument("--list", action="store_true", help="list ResNet-50 regions and exit")
+    ap.add_argument("--fuse-dw-pw", action="store_true",
+                    help="compile with the fused depthwise -> 1x1 kernel (region option)")
     args = ap.parse_args()
 
     import torch
 
-    from . import inputs as I
-    from . import partition as P
-    from . import region as R
+    from paper_2105_03215_gb300 import abi
+    from paper_2105_03215_gb300 import inputs as I
+    from paper_2105_03215_gb300 import partition as P
+    from paper_2105_03215_gb300 import region as R
 
     if args.workload == "resnet50":
         g, _ = I.resnet50(N=args.batch, draw=False)
@@ -71,7 +80,7 @@ def main():
         if args.workload == "mbv2_dw":
             reg = R.Region(g, [n.name for n in g.nodes[:3]], "mbv2_dw")
         else:
-            reg = R.whole_graph_region(g)
+            reg = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW if args.fuse_dw_pw else 0)
     cr = reg.compile()
     ins = [torch.randn(g.shape_of(n), device="cuda").to(torch.bfloat16) for n in reg.inputs]
     outs = [torch.empty(g.shape_of(n), dtype=torch.bfloat16, device="cuda") for n in reg.outputs]

@@ -37,8 +37,8 @@ def test_library_exports_every_declared_function():
     assert set(abi.declared_symbols()) == declared
 
 
-def _plan(g, **kw):
-    return R.whole_graph_region(g).plan(**kw)
+def _plan(g, options=0, **kw):
+    return R.whole_graph_region(g, options=options).plan(**kw)
 
 
 def test_plan_fuses_composites_into_launches():
@@ -55,16 +55,17 @@ def test_plan_fuses_composites_into_launches():
     assert rep.act[0] == 2
 
 
-def test_plan_fuses_depthwise_into_the_pointwise_when_asked(monkeypatch):
+def test_plan_fuses_depthwise_into_the_pointwise_when_asked():
     # depthwise + BN + ReLU6 -> 1x1 + BN: one fused launch (the depthwise output stays on chip)
-    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
-    rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0])
+    assert _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0]).n_launches == 2  # the default: two launches
+    rep = _plan(I.mbv2_dw_pw(N=1, H=8, W=8)[0], options=abi.OPT_FUSE_DW_PW)
     assert rep.n_launches == 1 and rep.kind[0] == abi.LAUNCH_DWPW
     assert rep.n_ops[0] == 5 and rep.act[0] == 0
     assert (rep.gemm_m[0], rep.gemm_n[0], rep.gemm_k[0], rep.tile_n[0]) == (64, 24, 144, 32)
     # a depthwise whose output is also a region output stays a launch of its own
     g, _ = I.mbv2_dw_pw(N=1, H=8, W=8)
-    reg = R.Region(g, [n.name for n in g.nodes], "both", outputs=[g.nodes[2].name, g.outputs[0]])
+    reg = R.Region(g, [n.name for n in g.nodes], "both", outputs=[g.nodes[2].name, g.outputs[0]],
+                   options=abi.OPT_FUSE_DW_PW)
     rep = reg.plan()
     assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_DEPTHWISE, abi.LAUNCH_GEMM]
     assert rep.act[0] == 2
@@ -124,12 +125,11 @@ def test_plan_flops_match_mac_count():
         assert _plan(g).flops == pytest.approx(I.region_flops(g), rel=1e-12)
 
 
-def test_packed_weights_are_folded_rounded_and_k_major(monkeypatch):
-    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
+def test_packed_weights_are_folded_rounded_and_k_major():
     g, _ = I.conv_bias_relu(N=1, H=8, W=8, C=64, K=32, seed=3)
     g2, _ = I.mbv2_dw_pw(N=1, H=8, W=8, C=64, Cout=32)
     # conv -> bn (from the pointwise part of g2) : fold checked on the GEMM launch
-    reg = R.whole_graph_region(g2)
+    reg = R.whole_graph_region(g2, options=abi.OPT_FUSE_DW_PW)
     rep = reg.plan()
     pw = g2.nodes[3]
     bn = g2.nodes[4]

@@ -57,16 +57,16 @@ def test_mobilenet_v2_graph_replay_equals_eager():
     ex.release()
 
 
-def test_mobilenet_v2_fused_regions_match_one_composite_per_region_bit_for_bit(monkeypatch):
+def test_mobilenet_v2_fused_regions_match_one_composite_per_region_bit_for_bit():
     # the whole network as one region (+ the classifier): 11 of the 17
     # depthwise -> 1x1 pairs run as fused kernels, and the logits are the same
     # bits as with every composite in a region of its own
     import torch
-    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
+    from paper_2105_03215_gb300 import abi
     outs = []
     for mo in (1, None):
         res, inp = E.build_mobilenet_v2(N=2, H=96, W=96, max_ops=mo)
-        ex = E.Executor(res)
+        ex = E.Executor(res, options=abi.OPT_FUSE_DW_PW)
         ex.set_input("data", torch.from_numpy(inp["data"]).to(torch.bfloat16).cuda())
         ex.run_steps()
         torch.cuda.synchronize()

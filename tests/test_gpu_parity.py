@@ -18,8 +18,8 @@ from .parity import assert_bit_exact, assert_close, run_region
 pytestmark = pytest.mark.gpu
 
 
-def _check_graph(g, inp, bit_exact=False, what=""):
-    reg = R.whole_graph_region(g)
+def _check_graph(g, inp, bit_exact=False, what="", options=0):
+    reg = R.whole_graph_region(g, options=options)
     got, cr = run_region(reg, inp)
     ref = ograph.evaluate(g, inp)
     for name in g.outputs:
@@ -349,18 +349,18 @@ def _dw_pw_graph(N, H, W, C, Cout, stride, residual, seed, small_int=False):
     (2, 28, 28, 192, 64, 2, False),   # stride 2 at 28x28 (MobileNetV2 block 3 shape)
     (2, 14, 14, 384, 64, 1, True),    # 6 chunks, 64 outputs, residual
 ])
-def test_fused_depthwise_pointwise(N, H, W, C, Cout, stride, residual, monkeypatch):
+def test_fused_depthwise_pointwise(N, H, W, C, Cout, stride, residual):
     # depthwise + BN + ReLU6 -> 1x1 + BN (+ residual) in one kernel against the
     # oracle of the unfused chain
     from paper_2105_03215_gb300 import abi
-    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
     g, inp = _dw_pw_graph(N, H, W, C, Cout, stride, residual, seed=N + C + Cout)
-    rep = R.whole_graph_region(g).plan(152)
+    rep = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW).plan(152)
     assert rep.n_launches == 1 and rep.kind[0] == abi.LAUNCH_DWPW
-    _check_graph(g, inp, what=f"dw_pw {N}x{H}x{W}x{C}->{Cout} s{stride} res{residual}")
+    _check_graph(g, inp, what=f"dw_pw {N}x{H}x{W}x{C}->{Cout} s{stride} res{residual}",
+                 options=abi.OPT_FUSE_DW_PW)
 
 
-def test_fused_depthwise_pointwise_equals_the_two_launches_bit_for_bit(monkeypatch):
+def test_fused_depthwise_pointwise_equals_the_two_launches_bit_for_bit():
     # the fused kernel rounds the depthwise output to bf16 and accumulates the
     # 1x1 conv's K steps in the same order as the two separate launches, so the
     # outputs agree bit for bit (separate launches: the depthwise output is
@@ -368,9 +368,9 @@ def test_fused_depthwise_pointwise_equals_the_two_launches_bit_for_bit(monkeypat
     import torch
     from .parity import to_dev
     g, inp = I.mbv2_dw_pw(N=4, H=28, W=28, C=144, Cout=24, seed=12)
-    monkeypatch.setenv("BYOC_FUSE_DW_PW", "1")
-    fused = R.whole_graph_region(g)
-    split = R.Region(g, [n.name for n in g.nodes], "split", outputs=[g.nodes[2].name, g.outputs[0]])
+    fused = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW)
+    split = R.Region(g, [n.name for n in g.nodes], "split", outputs=[g.nodes[2].name, g.outputs[0]],
+                     options=abi.OPT_FUSE_DW_PW)
     got_f, cf = run_region(fused, inp)
     got_s, cs = run_region(split, inp)
     assert cf.n_launches == 1 and cs.n_launches == 2

@@ -202,3 +202,67 @@ def test_random_dags_match_reference_and_are_convex(seed):
         assert covered == sorted(nd.name for nd in g.nodes if nd.op == "nn.relu")
         for r in regs:
             assert ref.is_convex(g, r)
+
+
+# ------------------------------------------------------------ brute-force maximality
+
+def _dense_dag(seed, n=10):
+    """Random DAG with one- to three-input nodes, about three quarters of
+    them supported."""
+    rnd = random.Random(1000 + seed)
+    nodes, names = [], ["in"]
+    for i in range(n):
+        k = 1 if rnd.random() < 0.45 or len(names) < 2 else min(len(names), rnd.choice([2, 3]))
+        ins = rnd.sample(names, k)
+        op = "nn.relu" if rnd.random() < 0.75 else "host_op"
+        nodes.append(Node(f"n{i}", op, ins, shape=(1, 2, 2, 8)))
+        names.append(f"n{i}")
+    users = {nm: 0 for nm in names}
+    for nd in nodes:
+        for i in nd.inputs:
+            users[i] += 1
+    outs = [nd.name for nd in nodes if users[nd.name] == 0]
+    return Graph({"in": (1, 2, 2, 8)}, nodes, outs, "rand")
+
+
+def _weakly_connected(g, names):
+    s = set(names)
+    adj = {m: set() for m in s}
+    for nd in g.nodes:
+        if nd.name in s:
+            for i in nd.inputs:
+                if i in s:
+                    adj[nd.name].add(i)
+                    adj[i].add(nd.name)
+    start = next(iter(s))
+    seen, stack = {start}, [start]
+    while stack:
+        for w in adj[stack.pop()]:
+            if w not in seen:
+                seen.add(w)
+                stack.append(w)
+    return seen == s
+
+
+@pytest.mark.parametrize("seed", range(150))
+def test_greedy_merge_leaves_no_convex_union_of_regions(seed):
+    """Section 3.1.2 merges consecutive supported operators greedily to make
+    regions as large as possible.  Checked by brute force on <= 10-node DAGs:
+    every supported node is in exactly one region, every region is convex and
+    connected, and no union of two or more regions (every subset is tried) is
+    both connected -- its operators consecutive -- and convex, i.e. no region
+    could still grow by absorbing others."""
+    import itertools
+    g = _random_dag(seed) if seed % 2 else _dense_dag(seed)
+    res = P.partition(g, [], annotators={"nn.relu": lambda n: True}, fallback_no_mac=False)
+    regs = _regions(res)
+    assert regs == ref.partition(g, {"nn.relu"}, fallback_no_mac=False, patterns=[])
+    covered = sorted(m for r in regs for m in r)
+    assert covered == sorted(nd.name for nd in g.nodes if nd.op == "nn.relu")
+    for r in regs:
+        assert ref.is_convex(g, r) and _weakly_connected(g, r)
+    for size in range(2, len(regs) + 1):
+        for sub in itertools.combinations(range(len(regs)), size):
+            union = [m for i in sub for m in regs[i]]
+            assert not (_weakly_connected(g, union) and ref.is_convex(g, union)), \
+                f"regions {[regs[i] for i in sub]} could be merged into one convex region"
