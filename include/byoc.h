@@ -168,6 +168,8 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
 /* Read and clear the handle's device error word.  Call after the stream that
  * ran the handle has been synchronised; returns BYOC_ERR_TIMEOUT if a kernel
  * gave up on a bounded wait since the previous check, else BYOC_OK.
+ * With h == NULL it does the same for the error word of byoc_ffn_noalloc on
+ * the current device (BYOC_OK before the first such call there).
  * Synchronous (one 4-byte device-to-host copy). */
 byoc_status byoc_check(byoc_handle *h);
 
@@ -256,8 +258,12 @@ byoc_status byoc_nchw_to_nhwc_bf16(const void *x, void *y, int32_t N, int32_t C,
  * that first call before any stream capture.  Every call shares the array,
  * so calls that overlap on the GPU (for example on two streams) race; order
  * them on one stream.  The call enqueues work on cuda_stream and returns; a
- * bounded-wait timeout inside the kernels is recorded in the array but not
- * reported.  It calls no cudaMalloc, cudaFree or other allocating routine.
+ * bounded-wait timeout inside its kernels is recorded in the array and
+ * reported by byoc_check(NULL) once the stream has been synchronised (the
+ * next call clears it).  A set-up that fails is retried by the next call; a
+ * successful one is kept for the life of the process and is not valid after
+ * cudaDeviceReset of that device.  It calls no cudaMalloc, cudaFree or other
+ * allocating routine.
  * Errors: INVALID_ARG, UNSUPPORTED, CUDA. */
 byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int32_t F, const void *w1,
                              const float *b1, const void *w2, const float *b2, void *y,

@@ -9,11 +9,24 @@ which is the "partial quantization" cast at the offload boundary
 """
 from __future__ import annotations
 
-from typing import Dict, Iterable, Optional
+from typing import Dict, Iterable, Optional, Tuple
 
 import numpy as np
 
 from . import ops
+
+# Rounding-error model of an implementation that stores activations and
+# weights in bf16 and accumulates in fp32 (the arithmetic the method's
+# offloaded regions run in; Section 3.2 casts to the accelerator's type at the
+# region boundary).  Each rounding of a value v is v (1 + d) with d in
+# [-u, u]; the probabilistic model of rounding-error analysis takes the d of
+# different roundings as independent with mean zero, so that an error
+# sum_j a_j d_j has, by Hoeffding's inequality (1963),
+#   P(|sum_j a_j d_j| >= lam * sqrt(sum_j a_j^2 u_j^2)) <= 2 exp(-lam^2 / 2).
+# evaluate_with_error_scale propagates s^2 = sum_j a_j^2 u_j^2 per element.
+U_BF16 = 2.0 ** -9   # |bf16_rne(v) - v| <= U_BF16 |v|   (8 significant bits)
+U_FP32 = 2.0 ** -24  # |fp32_rne(v) - v| <= U_FP32 |v|
+GELU_LIPSCHITZ = 1.13  # max |d/dx x Phi(x)| = 1.1289 (at x = sqrt 2)
 
 
 def eval_node(node, args):
@@ -44,6 +57,98 @@ def eval_node(node, args):
     if op == "nn.global_avg_pool2d":
         return ops.global_avg_pool_nhwc(args[0])
     raise NotImplementedError(op)
+
+
+def _spread_node(node, args, sq):
+    """s^2 of ``node``'s output (before it is rounded for storage), given the
+    inputs' values ``args`` and their s^2 ``sq``:
+
+      conv2d / dense   sum_i sq_i w_i^2 + U_BF16^2 sum_i (x_i w_i)^2
+                       + (sqrt(K) U_FP32 sum_i |x_i w_i|)^2
+                       (input errors carried through the weights; each
+                       weight rounded to bf16 once -- after any batch norm is
+                       folded into it, which scales w_i and s alike; a K-term
+                       fp32 sum, in the sqrt(K) form of the probabilistic
+                       analysis of recursive summation)
+      batch_norm       sq (gamma / sqrt(var + eps))^2
+      bias_add, relu, clip   sq   (1-Lipschitz)
+      gelu             1.13^2 sq
+      add              sq_a + sq_b
+      max_pool         the window's largest sq
+      global_avg_pool  the window's mean sq
+    """
+    op, a, c = node.op, node.attrs, node.consts
+    if op in ("nn.conv2d", "nn.dense"):
+        w = np.asarray(c["weight"], dtype=np.float64)
+        x = args[0]
+        if op == "nn.conv2d":
+            K = w.shape[1] * w.shape[2] * w.shape[3]
+            lin = lambda t, ww: ops.conv2d_nhwc(t, ww, tuple(a["strides"]), tuple(a["padding"]),
+                                                tuple(a["dilation"]), int(a["groups"]))
+        else:
+            K = w.shape[1]
+            lin = ops.dense
+        acc = np.sqrt(K) * U_FP32 * lin(np.abs(x), np.abs(w))
+        return lin(sq[0], w * w) + U_BF16 ** 2 * lin(x * x, w * w) + acc * acc
+    if op == "nn.batch_norm":
+        sc = np.asarray(c["gamma"], np.float64) ** 2 / (
+            np.asarray(c["moving_var"], np.float64) + float(a.get("epsilon", 1e-5)))
+        return sq[0] * sc
+    if op in ("nn.bias_add", "nn.relu", "clip"):
+        return sq[0]
+    if op == "nn.gelu":
+        return GELU_LIPSCHITZ ** 2 * sq[0]
+    if op == "add":
+        return sq[0] + sq[1]
+    if op == "nn.max_pool2d":
+        return ops.max_pool2d_nhwc(sq[0], tuple(a["pool_size"]), tuple(a["strides"]),
+                                   tuple(a["padding"]))
+    if op == "nn.global_avg_pool2d":
+        return ops.global_avg_pool_nhwc(sq[0])
+    raise NotImplementedError(op)
+
+
+_GEMM_OR_POOL = ("nn.conv2d", "nn.dense", "nn.max_pool2d", "nn.global_avg_pool2d")
+
+
+def evaluate_with_error_scale(graph, inputs: Dict[str, np.ndarray], nodes: Optional[Iterable[str]] = None,
+                              keep: Optional[Iterable[str]] = None
+                              ) -> Tuple[Dict[str, np.ndarray], Dict[str, np.ndarray]]:
+    """``evaluate`` plus, for every kept tensor, the per-element error scale
+    s = sqrt(sum_j a_j^2 u_j^2) of an implementation with bf16 storage and
+    fp32 accumulation under the probabilistic rounding model (module
+    comment): its error exceeds lam * s with probability at most
+    2 exp(-lam^2 / 2).  Inputs count as exact (they arrive bf16-rounded).  A
+    tensor is stored in bf16 -- adding (U_BF16 v)^2 to its s^2 -- where such
+    an implementation must materialise it: when it is read by a conv2d,
+    dense or pool, by more than one operator, by an operator outside
+    ``nodes``, or is kept / a graph output.  The elementwise chains in
+    between (bias, batch norm, residual add, activation) are fused and not
+    rounded.  Returns (values, scales)."""
+    env = {k: np.asarray(v, dtype=np.float64) for k, v in inputs.items()}
+    sq = {k: np.zeros_like(v) for k, v in env.items()}
+    wanted = set(nodes) if nodes is not None else None
+    names = list(keep) if keep is not None else None
+    kept = set(names) if names is not None else set(graph.outputs)
+    readers: Dict[str, list] = {}
+    for n in graph.nodes:
+        for i in n.inputs:
+            readers.setdefault(i, []).append(n)
+    for n in graph.nodes:
+        if wanted is not None and n.name not in wanted:
+            continue
+        args = [env[i] for i in n.inputs]
+        v = eval_node(n, args)
+        q = _spread_node(n, args, [sq[i] for i in n.inputs])
+        rd = readers.get(n.name, [])
+        stored = (n.name in kept or len(rd) != 1 or rd[0].op in _GEMM_OR_POOL
+                  or (wanted is not None and rd[0].name not in wanted))
+        if stored:
+            q = q + (U_BF16 * v) ** 2
+        env[n.name], sq[n.name] = v, q
+    if names is None:
+        names = [o for o in graph.outputs if o in env]
+    return {k: env[k] for k in names}, {k: np.sqrt(sq[k]) for k in names}
 
 
 def evaluate(graph, inputs: Dict[str, np.ndarray], nodes: Optional[Iterable[str]] = None,

@@ -215,6 +215,9 @@ cudaError_t launch_maxpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
                            int k, int s, int p, cudaStream_t st);
 // Sets the thread-local message byoc_last_error() returns.
 void set_last_error(const char *msg);
+// The allocation-free entry point's error word on the current device: read,
+// clear, BYOC_ERR_TIMEOUT if a wait expired (noalloc.cu).
+int noalloc_check();
 
 // Depthwise 3x3 (pad 1, stride 1|2) + folded BN + activation fused with the
 // 1x1 conv + folded BN (+ residual) (+ activation) that consumes it (dwpw.cu).

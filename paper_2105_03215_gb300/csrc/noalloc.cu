@@ -13,7 +13,9 @@
 // array's name as a device address (it is a host-side stand-in), so the first
 // call on each device, with that device current, looks the address up with
 // cudaGetSymbolAddress and caches it; that first call also raises the GEMM
-// kernel's shared-memory limit and loads the TMA descriptor encoder.
+// kernel's shared-memory limit and loads the TMA descriptor encoder.  A set-up
+// that fails is retried by the next call; one that succeeded is kept for the
+// life of the process (it does not survive cudaDeviceReset of that device).
 #include <cuda.h>
 #include <cuda_runtime.h>
 #include <cudaTypedefs.h>
@@ -35,12 +37,12 @@ constexpr int kTileN = 128;
 static __device__ __align__(256) unsigned char g_ffn_scratch[kHeaderBytes + kHiddenMaxElems * 2];
 
 struct DeviceState {
-    std::once_flag once;
-    cudaError_t err = cudaSuccess;
+    bool ready = false;                // set only by a set-up that succeeded
     unsigned char *scratch = nullptr;  // device address of g_ffn_scratch
     int num_sms = 0;
 };
 DeviceState g_devices[kMaxDevices];
+std::mutex g_devices_mutex;
 
 PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
 std::once_flag g_encode_once;
@@ -58,11 +60,21 @@ byoc_status cuda_fail(cudaError_t e, const char *what) {
     return BYOC_ERR_CUDA;
 }
 
-void setup_device(DeviceState &d, int dev) {
-    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&d.scratch), g_ffn_scratch);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev);
+// Per-device set-up, with that device current.  Returns the first failing
+// call's error; the state is marked ready only when every step succeeded.
+cudaError_t setup_device(DeviceState &d, int dev) {
+    std::lock_guard<std::mutex> lock(g_devices_mutex);
+    if (d.ready) return cudaSuccess;
+    unsigned char *p = nullptr;
+    int sms = 0;
+    cudaError_t e = cudaGetSymbolAddress(reinterpret_cast<void **>(&p), g_ffn_scratch);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess) e = byoc::gemm_prepare(byoc::GemmConfig{kTileN, 64, byoc::kAModeTile, false});
-    d.err = e;
+    if (e != cudaSuccess) return e;
+    d.scratch = p;
+    d.num_sms = sms;
+    d.ready = true;
+    return cudaSuccess;
 }
 
 CUresult encode(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows) {
@@ -119,8 +131,7 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
     });
     if (g_encode_err != cudaSuccess) return cuda_fail(g_encode_err, "byoc_ffn_noalloc: TMA encoder");
     DeviceState &d = g_devices[dev];
-    std::call_once(d.once, [&d, dev] { setup_device(d, dev); });
-    if (d.err != cudaSuccess) return cuda_fail(d.err, "byoc_ffn_noalloc: per-device set-up");
+    if ((e = setup_device(d, dev)) != cudaSuccess) return cuda_fail(e, "byoc_ffn_noalloc: per-device set-up");
 
     cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
     int *err_word = reinterpret_cast<int *>(d.scratch);
@@ -175,3 +186,33 @@ extern "C" byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int
         return cuda_fail(e, "byoc_ffn_noalloc: second GEMM launch");
     return BYOC_OK;
 }
+
+namespace byoc {
+
+// byoc_check(NULL): read and clear the allocation-free entry point's error
+// word on the current device (the first word of g_ffn_scratch).  Before any
+// call on this device there is nothing to report.
+int noalloc_check() {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return cuda_fail(e, "byoc_check: cudaGetDevice");
+    if (dev < 0 || dev >= kMaxDevices) return fail(BYOC_ERR_UNSUPPORTED, "byoc_check: device ordinal");
+    DeviceState &d = g_devices[dev];
+    {
+        std::lock_guard<std::mutex> lock(g_devices_mutex);
+        if (!d.ready) return BYOC_OK;
+    }
+    int v = 0;
+    if ((e = cudaMemcpy(&v, d.scratch, sizeof v, cudaMemcpyDeviceToHost)) != cudaSuccess)
+        return cuda_fail(e, "byoc_check: reading the allocation-free error word");
+    if (v != 0) {
+        if ((e = cudaMemset(d.scratch, 0, sizeof v)) != cudaSuccess)
+            return cuda_fail(e, "byoc_check: clearing the allocation-free error word");
+        char buf[128];
+        snprintf(buf, sizeof buf, "byoc_ffn_noalloc: a kernel's bounded wait expired (code %d)", v);
+        return fail(BYOC_ERR_TIMEOUT, buf);
+    }
+    return BYOC_OK;
+}
+
+}  // namespace byoc

@@ -1593,7 +1593,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
 }
 
 byoc_status byoc_check(byoc_handle *h) {
-    if (!h) return fail(BYOC_ERR_INVALID_ARG, "null handle");
+    if (!h) return static_cast<byoc_status>(byoc::noalloc_check());
     int v = 0;
     cudaError_t e = cudaMemcpy(&v, h->d_err, sizeof v, cudaMemcpyDeviceToHost);
     if (e != cudaSuccess) return cuda_fail(e, "reading the error word");

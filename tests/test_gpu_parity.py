@@ -13,7 +13,7 @@ from paper_2105_03215_gb300 import abi
 from paper_2105_03215_gb300 import inputs as I
 from paper_2105_03215_gb300 import region as R
 
-from .parity import assert_bit_exact, assert_close, run_region
+from .parity import assert_bit_exact, assert_close, oracle, run_region, sampled_conv_scale
 
 pytestmark = pytest.mark.gpu
 
@@ -21,12 +21,12 @@ pytestmark = pytest.mark.gpu
 def _check_graph(g, inp, bit_exact=False, what="", options=0):
     reg = R.whole_graph_region(g, options=options)
     got, cr = run_region(reg, inp)
-    ref = ograph.evaluate(g, inp)
+    ref, sc = oracle(g, inp)
     for name in g.outputs:
         if bit_exact:
             assert_bit_exact(got[name], ref[name], what or g.name)
         else:
-            assert_close(got[name], ref[name], what or g.name)
+            assert_close(got[name], ref[name], sc[name], what or g.name)
     cr.release()
     return got, ref
 
@@ -152,8 +152,8 @@ def test_resnet50_stem_region():
     stem = [n.name for n in g.nodes[:3]]  # conv 7x7/2 + bn + relu
     reg = R.Region(g, stem, "stem")
     got, cr = run_region(reg, inp)
-    ref = ograph.evaluate(g, inp, nodes=stem, keep=reg.outputs)
-    assert_close(got[reg.outputs[0]], ref[reg.outputs[0]], "stem")
+    ref, sc = oracle(g, inp, nodes=stem, keep=reg.outputs)
+    assert_close(got[reg.outputs[0]], ref[reg.outputs[0]], sc[reg.outputs[0]], "stem")
     cr.release()
 
 
@@ -205,7 +205,9 @@ def test_stem_at_full_size_sampled():
     v = ops.batch_norm(v, bn.consts["gamma"][ks], bn.consts["beta"][ks], bn.consts["moving_mean"][ks],
                        bn.consts["moving_var"][ks], bn.attrs.get("epsilon", 1e-5))
     ref = ops.relu(v).ravel()
-    assert_close(y[pix, ks], ref, "stem chunks (sampled)")
+    bscale = np.abs(bn.consts["gamma"][ks]) / np.sqrt(bn.consts["moving_var"][ks].astype(np.float64) + 1e-5)
+    sc = sampled_conv_scale(inp["data"], conv.consts["weight"], pix, ks, a, bscale, ref)
+    assert_close(y[pix, ks], ref, sc, "stem chunks (sampled)")
     cr.release()
 
 
@@ -244,14 +246,15 @@ def test_region_can_run_twice_with_new_pointers():
     g, inp = I.conv_bias_relu(N=1, H=16, W=16, C=64, K=64, seed=11)
     reg = R.whole_graph_region(g)
     cr = reg.compile()
-    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    ref, sc = oracle(g, inp)
+    ref, sc = ref[g.outputs[0]], sc[g.outputs[0]]
     for _ in range(2):
         x = to_dev(inp["x"])
         y = torch.full(g.shape_of(g.outputs[0]), float("nan"), dtype=torch.bfloat16, device="cuda")
         cr.run([x], [y])
         torch.cuda.synchronize()
         cr.check()
-        assert_close(y.float().cpu().numpy(), ref, "rerun")
+        assert_close(y.float().cpu().numpy(), ref, sc, "rerun")
     cr.release()
 
 
@@ -271,7 +274,8 @@ def test_depthwise_regions_sharing_a_kernel_run_in_any_compile_order():
         cr.run([x], [y])
         torch.cuda.synchronize()
         cr.check()
-        assert_close(y.float().cpu().numpy(), ograph.evaluate(g, inp)[g.outputs[0]], g.name)
+        ref, sc = oracle(g, inp)
+        assert_close(y.float().cpu().numpy(), ref[g.outputs[0]], sc[g.outputs[0]], g.name)
     big.release()
     small.release()
 
@@ -294,7 +298,8 @@ def test_deserialized_region_runs_bit_identically(make):
     got2, _ = run_region(reg, inp, compiled=cr2)
     for name in g.outputs:
         assert np.array_equal(got[name].view(np.uint32), got2[name].view(np.uint32)), name
-    assert_close(got2[g.outputs[0]], ograph.evaluate(g, inp)[g.outputs[0]], g.name)
+    ref, sc = oracle(g, inp)
+    assert_close(got2[g.outputs[0]], ref[g.outputs[0]], sc[g.outputs[0]], g.name)
     cr2.release()
 
 
@@ -394,7 +399,8 @@ def test_split_k_dense_matches_and_is_deterministic(M, Iw, U):
     reg = R.whole_graph_region(g)
     rep = reg.plan(152)
     got, cr = run_region(reg, inp)
-    assert_close(got[g.outputs[0]], ograph.evaluate(g, inp)[g.outputs[0]], f"dense {M}x{Iw}->{U}")
+    ref, sc = oracle(g, inp)
+    assert_close(got[g.outputs[0]], ref[g.outputs[0]], sc[g.outputs[0]], f"dense {M}x{Iw}->{U}")
     out = torch.empty(g.shape_of(g.outputs[0]), dtype=torch.bfloat16, device="cuda")
     xs = [to_dev(inp["x"])]
     ref_bits = None
