@@ -269,6 +269,29 @@ byoc_status byoc_ffn_noalloc(const void *x, int32_t M, int32_t D, int32_t F, con
                              const float *b1, const void *w2, const float *b2, void *y,
                              void *cuda_stream);
 
+/* ---------------------------------------------------------------------------
+ * Kernel trace, for measurement.  Not part of the paper's flow: it lets a
+ * benchmark see how long the tensor-core GEMM kernel runs inside a forward
+ * pass without putting events between the launches (which would stop each
+ * kernel from overlapping its set-up with the previous kernel's tail).
+ *
+ * byoc_trace_begin(buf, capacity): until byoc_trace_end, every GEMM launch
+ * that byoc_run enqueues (also into a CUDA graph being captured) gets the
+ * next slot k of buf, a device array of capacity x 2 uint64:
+ *   buf[2k]     earliest %globaltimer (ns) at which a CTA of the launch had
+ *               finished waiting for the previous kernel (atomic min),
+ *   buf[2k + 1] latest %globaltimer at which a CTA of it exited (atomic max).
+ * The caller sets buf[2k] = UINT64_MAX and buf[2k + 1] = 0 before each run
+ * of the traced launches.  Launches past capacity are not traced.  The trace
+ * state is process-wide: begin and end on one thread, with no other thread
+ * calling byoc_run meanwhile.
+ * byoc_trace_end() returns the number of slots handed out (>= 0) and stops
+ * tracing; launches enqueued afterwards (and graphs captured afterwards) are
+ * not traced.  Errors (begin): INVALID_ARG for a null or misaligned buf or a
+ * capacity < 1. */
+byoc_status byoc_trace_begin(void *buf, int32_t capacity);
+int32_t byoc_trace_end(void);
+
 /* Number of SMs and the device's compute capability, for host-side planning
  * (current device).  Errors: CUDA. */
 byoc_status byoc_device_info(int32_t *num_sms, int32_t *cc_major, int32_t *cc_minor);

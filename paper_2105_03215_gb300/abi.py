@@ -84,6 +84,8 @@ _SIGNATURES = {
     "byoc_max_pool2d_nhwc": (c_int32, [c_void_p, c_void_p] + [c_int32] * 7 + [c_void_p]),
     "byoc_global_avg_pool_nhwc": (c_int32, [c_void_p, c_void_p] + [c_int32] * 4 + [c_void_p]),
     "byoc_device_info": (c_int32, [POINTER(c_int32), POINTER(c_int32), POINTER(c_int32)]),
+    "byoc_trace_begin": (c_int32, [c_void_p, c_int32]),
+    "byoc_trace_end": (c_int32, []),
     "byoc_ffn_noalloc": (c_int32, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_void_p,
                                    c_void_p, c_void_p, c_void_p, c_void_p]),
     "byoc_plan": (c_int32, [POINTER(RegionDesc), c_int32, POINTER(PlanReport)]),

@@ -242,6 +242,7 @@ __global__ void __maxnreg__(168)
         __syncwarp();
     }
     if (warp != 0) pdl_wait();
+    if (a.trace != nullptr && threadIdx.x == 32) atomicMin(a.trace, globaltimer_ns());
     // Ring stages of G k-blocks each; at least two stages.
     const int G = a.group < 1 ? 1 : (a.group > S::STAGES / 2 ? S::STAGES / 2 : a.group);
     const int nst = S::STAGES / G;
@@ -878,6 +879,7 @@ __global__ void __maxnreg__(168)
     __syncwarp();
     tc_fence_before();
     __syncthreads();
+    if (a.trace != nullptr && threadIdx.x == 0) atomicMax(a.trace + 1, globaltimer_ns());
     if (warp == 1) {
         tc_fence_after();
         tmem_dealloc(tmem_base, S::TMEM_COLS);

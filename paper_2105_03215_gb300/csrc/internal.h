@@ -85,6 +85,10 @@ struct GemmArgs {
     const __nv_bfloat16 *residual;    // [M, N] or null
     __nv_bfloat16 *out;               // [M, N]
     int *err;                         // device error word
+    // measurement only (byoc_trace_begin), else null: [0] earliest CTA's
+    // %globaltimer once its wait for the previous kernel returned (atomic
+    // min), [1] latest CTA's at exit (atomic max)
+    unsigned long long *trace;
     // > 0: the slab comes from a stem layout (StemArgs) through a 5-D map,
     // box {8 values, wp positions, slab rows, stem_rows image rows, 1} at
     // (0, 0, first output row, 0, image), unswizzled: in shared memory

@@ -1487,6 +1487,29 @@ byoc_status byoc_plan_deserialize(const void *src, size_t src_bytes, byoc_plan_r
     return BYOC_OK;
 }
 
+// Kernel trace (byoc_trace_begin): the buffer, its capacity in slots and the
+// next free slot.
+namespace {
+unsigned long long *g_trace = nullptr;
+int g_trace_cap = 0, g_trace_next = 0;
+}  // namespace
+
+byoc_status byoc_trace_begin(void *buf, int32_t capacity) {
+    if (!buf || (reinterpret_cast<uintptr_t>(buf) & 15u) || capacity < 1)
+        return fail(BYOC_ERR_INVALID_ARG, "trace: null or misaligned buffer, or capacity < 1");
+    g_trace = static_cast<unsigned long long *>(buf);
+    g_trace_cap = capacity;
+    g_trace_next = 0;
+    return BYOC_OK;
+}
+
+int32_t byoc_trace_end(void) {
+    const int n = g_trace_next;
+    g_trace = nullptr;
+    g_trace_cap = g_trace_next = 0;
+    return n;
+}
+
 byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *outputs,
                      void *cuda_stream) {
     if (!h) return fail(BYOC_ERR_INVALID_ARG, "null handle");
@@ -1532,6 +1555,7 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                 h->tmA_ptr[i] = xa;
             }
             GemmArgs a = L.args;
+            a.trace = g_trace && g_trace_next < g_trace_cap ? g_trace + 2 * g_trace_next++ : nullptr;
             a.out = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(h->ptrs[L.y]) + L.y_off);
             a.residual = L.res >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.res]) : nullptr;
             if (a.residual && h->tmR_ptr[i] != a.residual) {
