@@ -226,6 +226,17 @@ def region_figures(flush, peaks):
         out[name] = {"us": t * 1e6, "tflops": tf, "gbps": gb, "launches": cr.n_launches,
                      "tensor_frac_of_measured": tf / peaks["bf16_tflops"],
                      "hbm_frac_of_measured": gb / peaks["hbm_gbs"]}
+        if name.startswith(("bert", "resnet50_bottleneck")):
+            # the same region as one region kernel (every composite in one
+            # persistent launch; intermediates through L2)
+            kcr = R.whole_graph_region(g, options=abi.OPT_REGION_KERNEL).compile()
+            tk = time_region(kcr, ins, outs, flush)
+            tfk = kcr.flops / tk / 1e12
+            out[name + "_region_kernel"] = {
+                "us": tk * 1e6, "tflops": tfk, "gbps": kcr.bytes / tk / 1e9, "launches": kcr.n_launches,
+                "tensor_frac_of_measured": tfk / peaks["bf16_tflops"],
+                "hbm_frac_of_measured": kcr.bytes / tk / 1e9 / peaks["hbm_gbs"]}
+            kcr.release()
         if name.startswith("mbv2"):
             # the same region as one fused kernel (depthwise output kept on chip)
             fcr = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW).compile()
@@ -304,14 +315,17 @@ def partition_study(graph, data, flush, reps=10):
     changes is how many external calls (byoc_run) the host makes.  Per K:
     regions, kernel launches, compile time, the forward pass replayed as one
     CUDA graph, and enqueued eagerly from Python (host work per call
-    included); logits must be bit-identical to K=1."""
+    included); logits must be bit-identical to K=1 -- except with region
+    kernels (K=4, one launch per bottleneck), which run other kernels: their
+    largest logit difference is reported."""
     import torch
+    from paper_2105_03215_gb300 import abi
     from paper_2105_03215_gb300 import executor as E
     x = torch.from_numpy(data).to(torch.bfloat16).cuda()
     out, ref = {}, None
-    for mo in (1, 4, 16, None):
+    for mo, opt in ((1, 0), (4, 0), (4, abi.OPT_REGION_KERNEL), (16, 0), (None, 0)):
         res, _ = E.build_resnet50(max_ops=mo, graph=graph)
-        ex = E.Executor(res)
+        ex = E.Executor(res, options=opt)
         ex.set_input("data", x)
         ex.run_steps()
         torch.cuda.synchronize()
@@ -338,10 +352,12 @@ def partition_study(graph, data, flush, reps=10):
         eager_ms, host_ms = timed(ex.run_steps)
         ex.capture()
         graph_ms, _ = timed(ex.replay)
-        out["all" if mo is None else str(mo)] = {
+        key = ("all" if mo is None else str(mo)) + ("_region_kernels" if opt else "")
+        out[key] = {
             "regions": len(ex.regions), "launches": ex.n_launches, "compile_ms": ex.init_s * 1e3,
             "graph_ms": graph_ms, "eager_ms": eager_ms, "eager_host_enqueue_ms": host_ms,
-            "logits_bit_identical": bool(torch.equal(logits, ref))}
+            "logits_bit_identical": bool(torch.equal(logits, ref)),
+            "logits_max_abs_diff": float((logits.float() - ref.float()).abs().max())}
         ex.release()
     return out
 
@@ -426,7 +442,8 @@ def main():
     for i, (kind, x) in enumerate(ex.steps):
         if kind == "region":
             rep = ex.regions[x].plan(sms)
-            gemm_slots.append((i, x, sum(1 for k in range(rep.n_launches) if rep.kind[k] == abi.LAUNCH_GEMM)))
+            gemm_slots.append((i, x, sum(1 for k in range(rep.n_launches)
+                                         if rep.kind[k] in (abi.LAUNCH_GEMM, abi.LAUNCH_CHAIN))))
     cap = sum(n for _, _, n in gemm_slots)
     tbuf = torch.empty((cap, 2), dtype=torch.int64, device="cuda")
     gi = torch.cuda.CUDAGraph()

@@ -128,6 +128,13 @@ typedef struct {
  *     arithmetic, not HBM, bounds that kernel, and two launches are faster
  *     on the MobileNetV2 shapes.  Results are bit-identical either way. */
 #define BYOC_OPT_FUSE_DW_PW 0x1u
+/*   BYOC_OPT_REGION_KERNEL: a region whose composites are all conv2d / dense
+ *     (1x1 or k x k, no stem layout) and number two to four runs as one
+ *     persistent kernel: the intermediates are written once and read back
+ *     from L2, and a composite's output tiles start as soon as the tiles of
+ *     the earlier composites they read are done (no launch boundary between
+ *     composites).  Regions that do not qualify get the per-composite plan. */
+#define BYOC_OPT_REGION_KERNEL 0x2u
 
 /* Figures describing a compiled region. */
 typedef struct {

@@ -25,7 +25,8 @@ typedef enum {
     BYOC_LAUNCH_GEMM = 0,      /* tcgen05 implicit-GEMM conv2d / dense + fused epilogue */
     BYOC_LAUNCH_DEPTHWISE = 1, /* depthwise 3x3 conv + fused epilogue */
     BYOC_LAUNCH_S2D = 2,       /* layout transform of a stride-2 few-channel stem (4-channel, zero-padded pixel pairs) */
-    BYOC_LAUNCH_DWPW = 3       /* depthwise 3x3 + epilogue fused with the 1x1 conv + epilogue after it */
+    BYOC_LAUNCH_DWPW = 3,      /* depthwise 3x3 + epilogue fused with the 1x1 conv + epilogue after it */
+    BYOC_LAUNCH_CHAIN = 4      /* region kernel: 2-4 conv2d / dense composites in one persistent launch */
 } byoc_launch_kind;
 
 typedef struct {
@@ -47,6 +48,9 @@ typedef struct {
     int32_t splits[BYOC_PLAN_MAX_LAUNCHES];     /* GEMM: CTAs sharing each tile's k-blocks (split-K), else 0 */
     int32_t pair_units[BYOC_PLAN_MAX_LAUNCHES]; /* 1: slab-mode units of two adjacent 128-row tiles
                                                    sharing each weight k-block, else 0 */
+    int32_t stages[BYOC_PLAN_MAX_LAUNCHES];     /* region kernel: composites it runs (gemm_* fields
+                                                   describe the first), else 1 */
+    int32_t units[BYOC_PLAN_MAX_LAUNCHES];      /* region kernel: output tiles over all its composites */
     double flops;
     double bytes;
     size_t const_bytes;

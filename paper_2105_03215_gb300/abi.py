@@ -15,6 +15,7 @@ ABI_VERSION = 2
 
 # byoc_region_desc.options
 OPT_FUSE_DW_PW = 0x1
+OPT_REGION_KERNEL = 0x2
 
 # byoc_status
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
@@ -25,7 +26,7 @@ LAYOUT_NHWC, LAYOUT_NC = 0, 1
 
 OP_CONV2D, OP_DENSE, OP_BIAS_ADD, OP_BATCH_NORM, OP_RELU, OP_RELU6, OP_GELU, OP_ADD = range(8)
 
-LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D, LAUNCH_DWPW = range(4)
+LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D, LAUNCH_DWPW, LAUNCH_CHAIN = range(5)
 PLAN_MAX_LAUNCHES = 128
 
 
@@ -68,7 +69,8 @@ class PlanReport(ctypes.Structure):
                 ("gemm_m", c_int32 * _L), ("gemm_n", c_int32 * _L), ("gemm_k", c_int32 * _L),
                 ("tile_n", c_int32 * _L), ("tile_k", c_int32 * _L), ("im2col", c_int32 * _L),
                 ("grid", c_int32 * _L), ("resident_b", c_int32 * _L), ("slab_slots", c_int32 * _L),
-                ("splits", c_int32 * _L), ("pair_units", c_int32 * _L),
+                ("splits", c_int32 * _L), ("pair_units", c_int32 * _L), ("stages", c_int32 * _L),
+                ("units", c_int32 * _L),
                 ("flops", c_double), ("bytes", c_double),
                 ("const_bytes", c_size_t), ("workspace_bytes", c_size_t)]
 

@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libbyoc.so")
 
-SOURCES = ["gemm.cu", "aux_kernels.cu", "dwpw.cu", "runtime.cu", "noalloc.cu"]
+SOURCES = ["gemm.cu", "chain.cu", "aux_kernels.cu", "dwpw.cu", "runtime.cu", "noalloc.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC,-O2", "-I", INCLUDE, "-I", CSRC]
 
@@ -45,6 +45,7 @@ def _digest() -> str:
     # same sources elsewhere has the same digest
     flags = [{INCLUDE: "<include>", CSRC: "<csrc>"}.get(f, f) for f in ARCH + FLAGS]
     h.update(" ".join(flags).encode())
+    h.update(" ".join(SOURCES).encode())
     h.update(os.uname().machine.encode())
     return h.hexdigest()
 

@@ -254,6 +254,58 @@ cudaError_t dwpw_prepare(const DwPwArgs &a);
 cudaError_t launch_dwpw(const CUtensorMap &tmX, const CUtensorMap &tmB, const DwPwArgs &a, int grid,
                         cudaStream_t st);
 
+// Region kernel (chain.cu): a region's chain of conv2d / dense composites in
+// one persistent launch.  Stage s computes out_s[M, N] = act(A_s . B_s^T +
+// bias_s [+ residual_s]); A_s is a row-major matrix (tile mode: dense, 1x1
+// stride-1 conv) or the im2col matrix of an NHWC tensor, read through maps.A[s];
+// B_s through maps.B[s] (BN x 64 boxes); out_s is stored through maps.O[s]
+// (32 x 32 boxes, 64-byte swizzle).  A unit is one 128 x BN output tile of one
+// stage; order[u] = (stage << 24) | tile gives the u-th unit handed out, tile
+// = m-tile * tiles_n + n-tile.  Every 128-row m-tile of a stage has a
+// completion counter (counters[cbase + m-tile]) to which each of the 8
+// epilogue warps of each of its units adds 1 per launch.
+constexpr int kChainMaxStages = 4;
+enum : int { kChainTile = 0, kChainIm2col = 1 };
+// (Both structs are laid out without implicit padding: plans are serialised
+// byte for byte.)
+struct ChainStage {
+    const float *bias;       // [tiles_n * BN], zero padded
+    const __nv_bfloat16 *residual;  // [M, N] or null (a region input or an earlier stage's output)
+    int mode;                // kChainTile | kChainIm2col
+    int M, N;                // output rows; output channels (row stride of out and residual)
+    int num_kb, chunks, kw;  // k-blocks of 64 (im2col: taps x chunks), chunks per tap, filter width
+    int dil_h, dil_w, Ho, Wo, stride_h, stride_w, pad_t, pad_l;  // im2col geometry
+    int tiles_n, num_tiles;
+    int unit0;               // first unit of this stage in stage-major numbering (host bookkeeping)
+    int cbase;               // first completion counter of this stage (one per m-tile)
+    int act;
+    int consumed;            // a later stage reads this stage's output: its units count into the counters
+    int res_dep;             // the residual is an earlier stage's output (the epilogue acquires it too)
+    int reserved;
+};
+struct ChainArgs {
+    ChainStage st[kChainMaxStages];
+    const int *order;        // [total_units]: (stage << 24) | tile of the u-th unit
+    const int *cta_off;      // [grid + 1]: CTA b runs units cta_list[cta_off[b] .. cta_off[b+1]), in order
+    const int *cta_list;
+    const int *dep_off;      // [total_units + 1]: unit u's dependencies are the pairs
+    const int *dep_list;     //   (counter, count per launch) at dep_list[2 j], j in [dep_off[u], dep_off[u+1])
+    unsigned *flags;         // [n_counters] completion counters, zeroed at compile
+    unsigned *ctl;           // [4]: unused, CTAs finished, launches completed, unused
+    int *err;
+    unsigned long long *trace;  // as GemmArgs::trace
+    int n_stages, total_units, n_counters, reserved;
+};
+static_assert(sizeof(ChainStage) == 2 * 8 + 22 * 4 && sizeof(ChainArgs) == kChainMaxStages * sizeof(ChainStage) + 9 * 8 + 16,
+              "region kernel arguments without padding");
+struct ChainMaps {
+    CUtensorMap A[kChainMaxStages], B[kChainMaxStages], O[kChainMaxStages];
+};
+size_t chain_smem_bytes(int bn);
+int chain_stages(int bn);
+cudaError_t chain_prepare(int bn);  // bn: 128 or 256
+cudaError_t launch_chain(int bn, const ChainMaps &maps, const ChainArgs &a, int grid, cudaStream_t st);
+
 // NCHW fp32 -> NHWC bf16 (channels zero-padded to Cp) at a region boundary.
 // Requires W * Cp <= kNchwStageElems; y 16-byte aligned when its rows are.
 constexpr int kNchwStageElems = 16384;

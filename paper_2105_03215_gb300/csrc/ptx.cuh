@@ -23,6 +23,7 @@ enum : int {
     kErrTimeoutMma = 2,
     kErrTimeoutEpilogue = 3,
     kErrTimeoutDrain = 4,
+    kErrTimeoutDependency = 5,  // a region kernel's wait for an earlier stage's rows
 };
 
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;  // 2 s

@@ -236,6 +236,17 @@ struct LaunchPlan {
     int stem_G = 0;  // stem GEMM: pixel pairs per innermost tensor-map box row
     byoc::DwPwArgs dp{};
     size_t w2_off = 0, w2_bytes = 0, b2_off = 0, b2_bytes = 0;  // fused: the 1x1 conv's constants
+    // region kernel (BYOC_LAUNCH_CHAIN): per stage, the GEMM launch it replaces
+    int chain_bn = 0;
+    int cx[byoc::kChainMaxStages] = {}, cy[byoc::kChainMaxStages] = {}, cres[byoc::kChainMaxStages] = {};
+    Im2colGeom cgeo[byoc::kChainMaxStages] = {};
+    int64_t caM[byoc::kChainMaxStages] = {}, caK[byoc::kChainMaxStages] = {};
+    int c_npad[byoc::kChainMaxStages] = {}, c_kpack[byoc::kChainMaxStages] = {};
+    size_t cw_off[byoc::kChainMaxStages] = {}, cb_off[byoc::kChainMaxStages] = {};
+    size_t order_off = 0, dep_off_off = 0, dep_list_off = 0;  // constant blob: int32 unit order, dependencies
+    size_t cta_off_off = 0, cta_list_off = 0;                 // constant blob: int32 per-CTA unit lists
+    size_t flags_off = 0, flags_bytes = 0;     // workspace: unit flags + control words
+    byoc::ChainArgs chain{};
     double flops = 0, bytes = 0;
 };
 
@@ -510,8 +521,10 @@ struct Affine {
     std::vector<double> scale, shift;
 };
 
-// Builds the launch list (no device work).
-byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
+// Builds the launch list (no device work).  chain_bn > 0: plan every GEMM
+// composite for the region kernel (tile or im2col mode, 64-wide k-blocks,
+// BN = chain_bn, no split-K); plan_region then collapses them (make_chain).
+byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, int chain_bn) {
     P = Plan();
     P.num_sms = num_sms > 0 ? num_sms : 148;
     byoc_status st = validate(d, P);
@@ -866,7 +879,7 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
                     L.geo = Im2colGeom{(int)X.shape[0], (int)X.shape[1], (int)X.shape[2], (int)C,
                                        kh, kw, op.stride[0], op.stride[1], op.pad[0], op.pad[1],
                                        op.pad[2], op.pad[3], op.dilation[0], op.dilation[1]};
-                    slab = op.stride[0] == 1 && op.stride[1] == 1 && op.dilation[0] == 1 &&
+                    slab = chain_bn == 0 && op.stride[0] == 1 && op.stride[1] == 1 && op.dilation[0] == 1 &&
                            op.dilation[1] == 1 && res < 0 &&
                            slab_geometry((int)X.shape[1], (int)X.shape[2], (int)Y.shape[1],
                                          (int)Y.shape[2], kh, kw, op.pad[0], op.pad[1], op.pad[3],
@@ -881,14 +894,16 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
             }
         }
         taps = kh * kw;
-        bk = op.kind == BYOC_OP_DENSE ? 64 : pick_bk(C);
+        bk = op.kind == BYOC_OP_DENSE || chain_bn > 0 ? 64 : pick_bk(C);
         chunks = (int)((C + bk - 1) / bk);
         const bool has_res = res >= 0;
         const int amode = slab ? byoc::kAModeSlab : (im2col ? byoc::kAModeIm2col : byoc::kAModeTile);
         const int64_t tiles_per_img = slab ? (Y.shape[1] + sgeo.t - 1) / sgeo.t : 0;
         const int64_t tiles_m = slab ? X.shape[0] * tiles_per_img : (M + 127) / 128;
         int splits = 1;
-        const int bn = pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms, &splits);
+        const int bn = chain_bn > 0 ? chain_bn
+                                    : pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms,
+                                              &splits);
         if (bn < 0)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
                         o, bk, amode, (int)has_res);
@@ -1020,6 +1035,251 @@ byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
     return BYOC_OK;
 }
 
+// Region kernel: collapse a plan of 2 .. kChainMaxStages GEMM launches, made
+// by plan_region_impl with chain_bn = bn, into one BYOC_LAUNCH_CHAIN launch.
+// Returns false, leaving P unchanged, when the region does not qualify.
+//
+// Dependencies of a unit (stage s, m-tile mt) on the stage p that wrote its A
+// operand: tile mode reads rows [m0, m1] of p's output, the same pixels p
+// computed as its rows [m0, m1]; im2col mode reads, for output pixels
+// (n0, oh0) .. (n1, oh1), input rows oh0 * sh - pt .. oh1 * sh - pt + (kh - 1)
+// * dh of images n0 .. n1 (clamped to the image), which lie in the contiguous
+// range of p's rows from (n0, first row, 0) to (n1, last row, W - 1).  On the
+// stage that wrote its residual: rows [m0, m1].  Either way the unit waits
+// for the completion counters of p's m-tiles over those rows (every column
+// tile of p).
+bool make_chain(Plan &P, int bn) {
+    const int ns = (int)P.launches.size();
+    if (ns < 2 || ns > byoc::kChainMaxStages) return false;
+    for (const LaunchPlan &L : P.launches) {
+        if (L.kind != BYOC_LAUNCH_GEMM || L.cfg.bk != 64 || L.cfg.bn != bn || L.stem_R != 0 || L.x_off ||
+            L.y_off)
+            return false;
+        if (L.cfg.amode != byoc::kAModeTile && L.cfg.amode != byoc::kAModeIm2col) return false;
+        if ((L.cfg.amode == byoc::kAModeTile ? L.aK : (int64_t)L.geo.C) % 64) return false;
+        if (L.args.N % 32) return false;  // the epilogue reads residual rows in 32-column pieces
+        if (L.args.num_tiles != (L.args.M + byoc::kGemmBM - 1) / byoc::kGemmBM * L.args.tiles_n) return false;
+    }
+    LaunchPlan C;
+    C.kind = BYOC_LAUNCH_CHAIN;
+    C.chain_bn = bn;
+    C.first_op = P.launches[0].first_op;
+    C.x = P.launches[0].x;
+    C.y = P.launches.back().y;
+    C.res = P.launches.back().res;
+    C.act = P.launches.back().act;
+    byoc::ChainArgs &A = C.chain;
+    A.n_stages = ns;
+    int units = 0;
+    double wbytes = 0;
+    for (int s = 0; s < ns; ++s) {
+        const LaunchPlan &L = P.launches[s];
+        byoc::ChainStage &cs = A.st[s];
+        cs.mode = L.cfg.amode == byoc::kAModeIm2col ? byoc::kChainIm2col : byoc::kChainTile;
+        cs.M = L.args.M;
+        cs.N = L.args.N;
+        cs.num_kb = L.args.num_kb;
+        cs.chunks = L.args.chunks;
+        cs.kw = L.args.kw;
+        cs.dil_h = L.args.dil_h;
+        cs.dil_w = L.args.dil_w;
+        cs.Ho = L.args.Ho;
+        cs.Wo = L.args.Wo;
+        cs.stride_h = L.args.stride_h;
+        cs.stride_w = L.args.stride_w;
+        cs.pad_t = L.args.pad_t;
+        cs.pad_l = L.args.pad_l;
+        cs.tiles_n = L.args.tiles_n;
+        cs.num_tiles = L.args.num_tiles;
+        cs.unit0 = units;
+        units += cs.num_tiles;
+        cs.act = L.act;
+        C.n_ops += L.n_ops;
+        C.cx[s] = L.x;
+        C.cy[s] = L.y;
+        C.cres[s] = L.res;
+        C.cgeo[s] = L.geo;
+        C.caM[s] = L.aM;
+        C.caK[s] = L.aK;
+        C.c_npad[s] = L.n_pad;
+        C.c_kpack[s] = L.k_pack;
+        C.cw_off[s] = L.w_off;
+        C.cb_off[s] = L.b_off;
+        C.flops += L.flops;
+        // weights once: 2 M N K flops -> N K bf16 weights, N fp32 biases
+        wbytes += L.flops / (2.0 * cs.M) * 2.0 + (double)cs.N * 4.0;
+    }
+    A.total_units = units;
+    int ncnt = 0;
+    for (int s = 0; s < ns; ++s) {
+        A.st[s].cbase = ncnt;
+        ncnt += (A.st[s].M + byoc::kGemmBM - 1) / byoc::kGemmBM;
+    }
+    A.n_counters = ncnt;
+    auto producer = [&](int tensor, int before) -> int {
+        for (int p = 0; p < before; ++p)
+            if (C.cy[p] == tensor) return p;
+        return -1;
+    };
+    // Dependencies in the stages' own numbering (unit = unit0 + tile), as
+    // (counter, count per launch).
+    std::vector<std::vector<std::pair<int32_t, int32_t>>> udeps(units);
+    std::vector<int> ustage(units), utile(units);
+    for (int s = 0; s < ns; ++s) {
+        byoc::ChainStage &cs = A.st[s];
+        const int pa = producer(C.cx[s], s), pr = C.cres[s] >= 0 ? producer(C.cres[s], s) : -1;
+        if (pa >= 0) A.st[pa].consumed = 1;
+        if (pr >= 0) A.st[pr].consumed = 1;
+        cs.res_dep = pr >= 0 ? 1 : 0;
+        for (int tile = 0; tile < cs.num_tiles; ++tile) {
+            const int u = cs.unit0 + tile;
+            ustage[u] = s;
+            utile[u] = tile;
+            const int mt = tile / cs.tiles_n, nt = tile % cs.tiles_n;
+            const int64_t m0 = (int64_t)mt * byoc::kGemmBM;
+            const int64_t m1 = std::min<int64_t>(m0 + byoc::kGemmBM, cs.M) - 1;
+            std::vector<std::pair<int32_t, int32_t>> &d = udeps[u];
+            auto add_rows = [&](int p, int64_t lo, int64_t hi) {
+                const byoc::ChainStage &ps = A.st[p];
+                hi = std::min<int64_t>(hi, (int64_t)ps.M - 1);
+                for (int64_t pm = lo / byoc::kGemmBM; pm <= hi / byoc::kGemmBM; ++pm)
+                    d.emplace_back(ps.cbase + (int)pm, byoc::kGemmEpiWarps * ps.tiles_n);
+            };
+            if (pa >= 0) {
+                int64_t lo = m0, hi = m1;
+                if (cs.mode == byoc::kChainIm2col) {
+                    const Im2colGeom &g = C.cgeo[s];
+                    const int64_t hw = (int64_t)cs.Ho * cs.Wo;
+                    const int64_t n0 = m0 / hw, oh0 = (m0 % hw) / cs.Wo;
+                    const int64_t n1 = m1 / hw, oh1 = (m1 % hw) / cs.Wo;
+                    const int64_t ih0 = std::max<int64_t>(0, oh0 * g.sh - g.pt);
+                    const int64_t ih1 =
+                        std::max<int64_t>(0, std::min<int64_t>(g.H - 1, oh1 * g.sh - g.pt + (int64_t)(g.kh - 1) * g.dh));
+                    lo = n0 * g.H * g.W + ih0 * g.W;
+                    hi = std::max(lo, n1 * g.H * g.W + ih1 * g.W + g.W - 1);
+                }
+                add_rows(pa, lo, hi);
+            }
+            if (pr >= 0) {
+                if (A.st[pr].M != cs.M) return false;
+                add_rows(pr, m0, m1);
+            }
+            std::sort(d.begin(), d.end());
+            d.erase(std::unique(d.begin(), d.end()), d.end());
+        }
+    }
+    // The order units are handed out in: a list schedule of the launch on
+    // the grid's CTAs with estimated durations (SM cycles).  A unit's
+    // mainloop costs per k-block the larger of its MMA time (4 x 64 cycles
+    // at BN = 128, 4 x 128 at BN = 256) and its operand bytes at ~60 B per
+    // cycle into the SM; its epilogue ~400 cycles per two 32-column chunks
+    // (+ 300 with a residual).  Repeatedly, the CTA that frees first takes
+    // the unit that can start earliest among those whose dependencies are all
+    // scheduled (ties: stage-major order); it frees again when the unit's
+    // loads are issued (the epilogue overlaps the next unit).
+    const int grid = std::min(units, P.num_sms);
+    std::vector<double> main_c(ns), epi_c(ns);
+    for (int s = 0; s < ns; ++s) {
+        const double mma = 4.0 * (bn == 256 ? 128.0 : 64.0);
+        const double ingest = (double)(byoc::kGemmBM * 64 * 2 + bn * 64 * 2) / 60.0;
+        main_c[s] = 300.0 + A.st[s].num_kb * std::max(mma, ingest);
+        epi_c[s] = 400.0 * (double)((bn / 32 + 1) / 2) + (C.cres[s] >= 0 ? 300.0 : 0.0);
+    }
+    std::vector<int> remaining(ncnt, 0);
+    std::vector<double> cnt_done(ncnt, 0.0);
+    for (int u = 0; u < units; ++u) {
+        const byoc::ChainStage &cs = A.st[ustage[u]];
+        remaining[cs.cbase + utile[u] / cs.tiles_n]++;
+    }
+    std::vector<double> cta_free(grid, 0.0);
+    std::vector<char> taken(units, 0);
+    std::vector<int> ord, ord_cta;
+    ord.reserve(units);
+    ord_cta.reserve(units);
+    for (int i = 0; i < units; ++i) {
+        const int c = (int)(std::min_element(cta_free.begin(), cta_free.end()) - cta_free.begin());
+        const double f = cta_free[c];
+        int best = -1;
+        double best_start = 0;
+        for (int u = 0; u < units; ++u) {
+            if (taken[u]) continue;
+            double ready = 0;
+            bool ok = true;
+            for (const auto &dp : udeps[u]) {
+                if (remaining[dp.first] > 0) {
+                    ok = false;
+                    break;
+                }
+                ready = std::max(ready, cnt_done[dp.first]);
+            }
+            if (!ok) continue;
+            const double st0 = std::max(f, ready);
+            if (best < 0 || st0 < best_start - 1e-9) {
+                best = u;
+                best_start = st0;
+            }
+            if (st0 <= f) break;  // cannot start any earlier: keep stage-major order
+        }
+        taken[best] = 1;
+        ord.push_back(best);
+        ord_cta.push_back(c);
+        const int sb = ustage[best];
+        const int cnt = A.st[sb].cbase + utile[best] / A.st[sb].tiles_n;
+        remaining[cnt]--;
+        cnt_done[cnt] = std::max(cnt_done[cnt], best_start + main_c[sb] + epi_c[sb]);
+        cta_free[c] = best_start + main_c[sb];
+    }
+    std::vector<int32_t> order(units), off(1, 0), list;
+    for (int i = 0; i < units; ++i) {
+        const int u = ord[i];
+        order[i] = (ustage[u] << 24) | utile[u];
+        for (const auto &c : udeps[u]) {
+            list.push_back(c.first);
+            list.push_back(c.second);
+        }
+        off.push_back((int32_t)(list.size() / 2));
+    }
+    if (list.empty()) list.assign(2, 0);  // keeps the blob offset valid; never read
+    // each CTA's units, in the global order
+    std::vector<int32_t> cta_off(grid + 1, 0), cta_list(units);
+    for (int i = 0; i < units; ++i) cta_off[ord_cta[i] + 1]++;
+    for (int b = 0; b < grid; ++b) cta_off[b + 1] += cta_off[b];
+    {
+        std::vector<int32_t> fill(cta_off.begin(), cta_off.end() - 1);
+        for (int i = 0; i < units; ++i) cta_list[fill[ord_cta[i]]++] = i;
+    }
+    C.cta_off_off = blob_append(P.blob, cta_off.data(), cta_off.size() * 4);
+    C.cta_list_off = blob_append(P.blob, cta_list.data(), cta_list.size() * 4);
+    C.order_off = blob_append(P.blob, order.data(), order.size() * 4);
+    C.dep_off_off = blob_append(P.blob, off.data(), off.size() * 4);
+    C.dep_list_off = blob_append(P.blob, list.data(), list.size() * 4);
+    // algorithmic bytes: the region's inputs and outputs once, the weights once
+    double io = 0;
+    for (int t : P.inputs) io += (double)P.tensors[t].bytes();
+    for (int t : P.outputs) io += (double)P.tensors[t].bytes();
+    C.bytes = io + wbytes;
+    C.grid = grid;
+    // workspace: 4 control words, then one completion counter per m-tile
+    C.flags_off = P.ws_bytes;
+    C.flags_bytes = align_up(16 + 4 * (size_t)ncnt, 256);
+    P.ws_bytes += C.flags_bytes;
+    P.launches.assign(1, C);
+    P.flops = C.flops;
+    P.bytes = C.bytes;
+    return true;
+}
+
+byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
+    if (d && d->abi_version == BYOC_ABI_VERSION && (d->options & BYOC_OPT_REGION_KERNEL)) {
+        Plan C;
+        if (plan_region_impl(d, num_sms, C, 128) == BYOC_OK && make_chain(C, 128)) {
+            P = std::move(C);
+            return BYOC_OK;
+        }
+    }
+    return plan_region_impl(d, num_sms, P, 0);
+}
+
 void fill_report(const Plan &P, byoc_plan_report *r) {
     std::memset(r, 0, sizeof *r);
     r->n_launches = (int32_t)P.launches.size();
@@ -1047,6 +1307,19 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
                            : byoc::amode_wres(L.cfg.amode)      ? L.args.slab_slots
                                                                 : 2;
         r->pair_units[i] = gm && byoc::amode_pair(L.cfg.amode) ? 1 : 0;
+        r->stages[i] = 1;
+        if (L.kind == BYOC_LAUNCH_CHAIN) {
+            const byoc::ChainStage &s0 = L.chain.st[0];
+            r->stages[i] = L.chain.n_stages;
+            r->units[i] = L.chain.total_units;
+            r->gemm_m[i] = s0.M;
+            r->gemm_n[i] = s0.N;
+            r->gemm_k[i] = L.c_kpack[0];
+            r->tile_n[i] = L.chain_bn;
+            r->tile_k[i] = 64;
+            r->im2col[i] = s0.mode == byoc::kChainIm2col ? 1 : 0;
+            r->splits[i] = 1;
+        }
     }
     r->flops = P.flops;
     r->bytes = P.bytes;
@@ -1064,6 +1337,7 @@ void set_last_error(const char *msg) { g_err = msg ? msg : ""; }
 
 struct byoc_handle {
     Plan P;
+    int sms = 0;  // SMs of the device the handle was instantiated on
     uint8_t *d_const = nullptr;
     uint8_t *d_ws = nullptr;
     int *d_err = nullptr;
@@ -1075,6 +1349,8 @@ struct byoc_handle {
     std::vector<const void *> tmR_ptr;
     std::vector<CUtensorMap> tmO;         // per launch: output map (tile mode), cached
     std::vector<const void *> tmO_ptr;
+    std::vector<byoc::ChainMaps> cmaps;   // per launch: region kernel maps (A, O cached; B fixed)
+    std::vector<std::vector<const void *>> cptr;  // per launch: pointers the A [0, 4) and O [4, 8) maps encode
     std::vector<void *> ptrs;             // scratch: resolved tensor pointers
 };
 
@@ -1099,7 +1375,8 @@ byoc_status byoc_plan_constants(const byoc_region_desc *desc, int32_t num_sms, i
     if (launch < 0 || launch >= (int)P.launches.size())
         return fail(BYOC_ERR_INVALID_ARG, "launch %d out of range", launch);
     const LaunchPlan &L = P.launches[launch];
-    if (L.kind == BYOC_LAUNCH_S2D) return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants", launch);
+    if (L.kind == BYOC_LAUNCH_S2D || L.kind == BYOC_LAUNCH_CHAIN)
+        return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants of its own", launch);
     if ((what < 0 || what > 3) || (what > 1 && L.kind != BYOC_LAUNCH_DWPW))
         return fail(BYOC_ERR_INVALID_ARG, "launch %d has no constants of kind %d", launch, what);
     const size_t off = what == 0 ? L.w_off : what == 1 ? L.b_off : what == 2 ? L.w2_off : L.b2_off;
@@ -1168,6 +1445,10 @@ byoc_status check_device(int32_t *sms) {
 byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
     cudaError_t e;
     cudaGetDevice(&h->device);
+    if ((e = cudaDeviceGetAttribute(&h->sms, cudaDevAttrMultiProcessorCount, h->device)) != cudaSuccess) {
+        byoc_release(h);
+        return cuda_fail(e, "cudaDeviceGetAttribute");
+    }
     Plan &P = h->P;
     if (!P.blob.empty()) {
         if ((e = cudaMalloc(&h->d_const, P.blob.size())) != cudaSuccess) {
@@ -1197,6 +1478,8 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
     h->tmR_ptr.assign(nl, nullptr);
     h->tmO.resize(nl);
     h->tmO_ptr.assign(nl, nullptr);
+    h->cmaps.resize(nl);
+    h->cptr.assign(nl, std::vector<const void *>(2 * byoc::kChainMaxStages, nullptr));
     h->ptrs.assign(P.tensors.size(), nullptr);
     for (size_t i = 0; i < nl; ++i) {
         LaunchPlan &L = P.launches[i];
@@ -1237,6 +1520,40 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
                 return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(1x1 weights) = %d", i, (int)r);
             }
             if ((e = byoc::dwpw_prepare(L.dp)) != cudaSuccess) {
+                byoc_release(h);
+                return cuda_fail(e, "cudaFuncSetAttribute");
+            }
+        } else if (L.kind == BYOC_LAUNCH_CHAIN) {
+            byoc::ChainArgs &A = L.chain;
+            for (int st = 0; st < A.n_stages; ++st) {
+                A.st[st].bias = reinterpret_cast<const float *>(h->d_const + L.cb_off[st]);
+                CUresult r = encode_2d(&h->cmaps[i].B[st], h->d_const + L.cw_off[st], (uint64_t)L.c_npad[st],
+                                       (uint64_t)L.c_kpack[st], (uint32_t)L.chain_bn, 64, 64);
+                if (r != CUDA_SUCCESS) {
+                    byoc_release(h);
+                    return fail(BYOC_ERR_CUDA, "launch %zu stage %d: cuTensorMapEncodeTiled(weights) = %d", i,
+                                st, (int)r);
+                }
+            }
+            // every CTA of a region kernel must be resident at once (one per SM)
+            if (L.grid > h->sms) {
+                byoc_release(h);
+                return fail(BYOC_ERR_UNSUPPORTED, "region kernel of %d CTAs planned for more SMs than the device has",
+                            L.grid);
+            }
+            A.order = reinterpret_cast<const int *>(h->d_const + L.order_off);
+            A.cta_off = reinterpret_cast<const int *>(h->d_const + L.cta_off_off);
+            A.cta_list = reinterpret_cast<const int *>(h->d_const + L.cta_list_off);
+            A.dep_off = reinterpret_cast<const int *>(h->d_const + L.dep_off_off);
+            A.dep_list = reinterpret_cast<const int *>(h->d_const + L.dep_list_off);
+            A.ctl = reinterpret_cast<unsigned *>(h->d_ws + L.flags_off);
+            A.flags = A.ctl + 4;
+            A.err = h->d_err;
+            if ((e = cudaMemset(h->d_ws + L.flags_off, 0, L.flags_bytes)) != cudaSuccess) {
+                byoc_release(h);
+                return cuda_fail(e, "cudaMemset(region kernel flags)");
+            }
+            if ((e = byoc::chain_prepare(L.chain_bn)) != cudaSuccess) {
                 byoc_release(h);
                 return cuda_fail(e, "cudaFuncSetAttribute");
             }
@@ -1339,6 +1656,84 @@ void serialize_plan(const Plan &P, std::vector<uint8_t> &out) {
     put(out, &sum, 1);
 }
 
+// A deserialised region-kernel launch stays within the plan: stage tensors,
+// constants, dependency lists (each unit waits only for units before it, so
+// every wait of the kernel can end) and workspace flags.
+int g_chain_bad = 0;  // which consistency check failed (for the error message)
+bool chain_plan_ok(const Plan &P, const LaunchPlan &L) {
+    const byoc::ChainArgs &A = L.chain;
+    const int nt = (int)P.tensors.size();
+    if ((L.chain_bn != 128 && L.chain_bn != 256) || A.n_stages < 2 || A.n_stages > byoc::kChainMaxStages)
+        { g_chain_bad = 1; return false; }
+    int units = 0, ncnt = 0;
+    for (int s = 0; s < A.n_stages; ++s) {
+        const byoc::ChainStage &cs = A.st[s];
+        if (L.cx[s] < 0 || L.cx[s] >= nt || L.cy[s] < 0 || L.cy[s] >= nt || L.cres[s] >= nt) { g_chain_bad = 2; return false; }
+        if (cs.M < 1 || cs.N < 32 || cs.N % 32) { g_chain_bad = 3; return false; }
+        if (cs.tiles_n != L.c_npad[s] / L.chain_bn || L.c_npad[s] % L.chain_bn) { g_chain_bad = 13; return false; }
+        if (cs.num_tiles != (cs.M + byoc::kGemmBM - 1) / byoc::kGemmBM * cs.tiles_n || cs.num_tiles >= (1 << 24))
+            { g_chain_bad = 14; return false; }
+        if (cs.cbase != ncnt || cs.unit0 != units) { g_chain_bad = 15; return false; }
+        if (cs.num_kb < 1 || (size_t)cs.num_kb * 64 > (size_t)L.c_kpack[s]) { g_chain_bad = 16; return false; }
+        if (P.tensors[L.cy[s]].elems() != (size_t)cs.M * cs.N) { g_chain_bad = 4; return false; }
+        if (L.cw_off[s] + (size_t)L.c_npad[s] * L.c_kpack[s] * 2 > P.blob.size() ||
+            L.cb_off[s] + (size_t)L.c_npad[s] * 4 > P.blob.size())
+            { g_chain_bad = 5; return false; }
+        units += cs.num_tiles;
+        ncnt += (cs.M + byoc::kGemmBM - 1) / byoc::kGemmBM;
+    }
+    if (units != A.total_units || ncnt != A.n_counters || L.flags_off + 16 + 4 * (size_t)ncnt > P.ws_bytes ||
+        L.order_off + 4 * (size_t)units > P.blob.size() || L.dep_off_off + 4 * ((size_t)units + 1) > P.blob.size())
+        { g_chain_bad = 6; return false; }
+    const int32_t *order = reinterpret_cast<const int32_t *>(P.blob.data() + L.order_off);
+    const int32_t *off = reinterpret_cast<const int32_t *>(P.blob.data() + L.dep_off_off);
+    const int32_t *list = reinterpret_cast<const int32_t *>(P.blob.data() + L.dep_list_off);
+    const size_t pairs = L.dep_list_off < P.blob.size() ? (P.blob.size() - L.dep_list_off) / 8 : 0;
+    // the order is a permutation of the units; every counter a unit waits
+    // for is completed by units earlier in the order only
+    std::vector<char> seen(units, 0);
+    if (off[0] != 0) { g_chain_bad = 7; return false; }
+    for (int i = 0; i < units; ++i) {
+        const int s = order[i] >> 24, tile = order[i] & 0xFFFFFF;
+        if (s < 0 || s >= A.n_stages || tile >= A.st[s].num_tiles) { g_chain_bad = 8; return false; }
+        const int nat = A.st[s].unit0 + tile;
+        if (seen[nat]) { g_chain_bad = 9; return false; }
+        seen[nat] = 1;
+        if (off[i + 1] < off[i] || (size_t)off[i + 1] > pairs) { g_chain_bad = 10; return false; }
+        for (int j = off[i]; j < off[i + 1]; ++j) {
+            const int c = list[2 * j];
+            if (c < 0 || c >= ncnt || list[2 * j + 1] <= 0) { g_chain_bad = 11; return false; }
+        }
+    }
+    // a counter may only be waited for once all its units are before the waiter
+    std::vector<int> done_at(ncnt, -1);
+    for (int i = 0; i < units; ++i) {
+        const int s = order[i] >> 24;
+        const int c = A.st[s].cbase + (order[i] & 0xFFFFFF) / A.st[s].tiles_n;
+        done_at[c] = std::max(done_at[c], i);
+    }
+    for (int i = 0; i < units; ++i)
+        for (int j = off[i]; j < off[i + 1]; ++j)
+            if (done_at[list[2 * j]] >= i) { g_chain_bad = 12; return false; }
+    // per-CTA lists: a partition of the units, each list in the global order
+    if (L.grid < 1 || L.grid > units || L.cta_off_off + 4 * ((size_t)L.grid + 1) > P.blob.size() ||
+        L.cta_list_off + 4 * (size_t)units > P.blob.size())
+        { g_chain_bad = 17; return false; }
+    const int32_t *coff = reinterpret_cast<const int32_t *>(P.blob.data() + L.cta_off_off);
+    const int32_t *clist = reinterpret_cast<const int32_t *>(P.blob.data() + L.cta_list_off);
+    if (coff[0] != 0 || coff[L.grid] != units) { g_chain_bad = 18; return false; }
+    std::fill(seen.begin(), seen.end(), 0);
+    for (int b = 0; b < L.grid; ++b) {
+        if (coff[b + 1] < coff[b]) { g_chain_bad = 19; return false; }
+        for (int k = coff[b]; k < coff[b + 1]; ++k) {
+            const int i = clist[k];
+            if (i < 0 || i >= units || seen[i] || (k > coff[b] && clist[k - 1] >= i)) { g_chain_bad = 20; return false; }
+            seen[i] = 1;
+        }
+    }
+    return true;
+}
+
 byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
     if (!src) return fail(BYOC_ERR_INVALID_ARG, "null serialised plan");
     const uint8_t *b = static_cast<const uint8_t *>(src);
@@ -1399,8 +1794,10 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: workspace layout out of range");
     for (const LaunchPlan &L : P.launches) {
         if (L.kind != BYOC_LAUNCH_GEMM && L.kind != BYOC_LAUNCH_DEPTHWISE && L.kind != BYOC_LAUNCH_S2D &&
-            L.kind != BYOC_LAUNCH_DWPW)
+            L.kind != BYOC_LAUNCH_DWPW && L.kind != BYOC_LAUNCH_CHAIN)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad launch kind");
+        if (L.kind == BYOC_LAUNCH_CHAIN && !chain_plan_ok(P, L))
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent region kernel (check %d)", g_chain_bad);
         if (L.x < 0 || L.x >= nt || L.y < 0 || L.y >= nt || L.res >= nt)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad tensor id in a launch");
         if (L.w_off + L.w_bytes > P.blob.size() || L.b_off + L.b_bytes > P.blob.size() ||
@@ -1579,6 +1976,35 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             }
             e = byoc::launch_gemm(L.cfg, h->tmA[i], h->tmB[i], a.residual ? h->tmR[i] : h->tmA[i],
                                   tstore ? h->tmO[i] : h->tmA[i], a, L.grid, st);
+        } else if (L.kind == BYOC_LAUNCH_CHAIN) {
+            byoc::ChainArgs a = L.chain;
+            byoc::ChainMaps &mp = h->cmaps[i];
+            std::vector<const void *> &cp = h->cptr[i];
+            for (int sg = 0; sg < a.n_stages; ++sg) {
+                const void *xa = h->ptrs[L.cx[sg]];
+                if (cp[sg] != xa) {
+                    CUresult r = a.st[sg].mode == byoc::kChainIm2col
+                                     ? encode_im2col(&mp.A[sg], xa, L.cgeo[sg], 64)
+                                     : encode_2d(&mp.A[sg], xa, (uint64_t)L.caM[sg], (uint64_t)L.caK[sg],
+                                                 byoc::kGemmBM, 64, 64);
+                    if (r != CUDA_SUCCESS)
+                        return fail(BYOC_ERR_CUDA, "launch %zu stage %d: encoding the A map failed (%d)", i, sg,
+                                    (int)r);
+                    cp[sg] = xa;
+                }
+                void *ya = h->ptrs[L.cy[sg]];
+                if (cp[byoc::kChainMaxStages + sg] != ya) {
+                    CUresult r = encode_2d(&mp.O[sg], ya, (uint64_t)a.st[sg].M, (uint64_t)a.st[sg].N, 32, 32, 32);
+                    if (r != CUDA_SUCCESS)
+                        return fail(BYOC_ERR_CUDA, "launch %zu stage %d: encoding the output map failed (%d)", i,
+                                    sg, (int)r);
+                    cp[byoc::kChainMaxStages + sg] = ya;
+                }
+                a.st[sg].residual =
+                    L.cres[sg] >= 0 ? static_cast<const __nv_bfloat16 *>(h->ptrs[L.cres[sg]]) : nullptr;
+            }
+            a.trace = g_trace && g_trace_next < g_trace_cap ? g_trace + 2 * g_trace_next++ : nullptr;
+            e = byoc::launch_chain(L.chain_bn, mp, a, L.grid, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {
@@ -1623,6 +2049,10 @@ byoc_status byoc_check(byoc_handle *h) {
     if (e != cudaSuccess) return cuda_fail(e, "reading the error word");
     if (v != 0) {
         cudaMemset(h->d_err, 0, sizeof v);
+        // a region kernel that gave up left its unit counter and flags
+        // mid-launch: start them again from zero
+        for (const LaunchPlan &L : h->P.launches)
+            if (L.kind == BYOC_LAUNCH_CHAIN) cudaMemset(h->d_ws + L.flags_off, 0, L.flags_bytes);
         return fail(BYOC_ERR_TIMEOUT, "a kernel's bounded wait expired (code %d)", v);
     }
     return BYOC_OK;

@@ -35,6 +35,8 @@ def main():
     ap.add_argument("--list", action="store_true", help="list ResNet-50 regions and exit")
     ap.add_argument("--fuse-dw-pw", action="store_true",
                     help="compile with the fused depthwise -> 1x1 kernel (region option)")
+    ap.add_argument("--region-kernel", action="store_true",
+                    help="compile a chain of conv / dense composites as one region kernel (region option)")
     args = ap.parse_args()
 
     import torch
@@ -80,7 +82,8 @@ def main():
         if args.workload == "mbv2_dw":
             reg = R.Region(g, [n.name for n in g.nodes[:3]], "mbv2_dw")
         else:
-            reg = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW if args.fuse_dw_pw else 0)
+            reg = R.whole_graph_region(g, options=(abi.OPT_FUSE_DW_PW if args.fuse_dw_pw else 0) |
+                                       (abi.OPT_REGION_KERNEL if args.region_kernel else 0))
     cr = reg.compile()
     ins = [torch.randn(g.shape_of(n), device="cuda").to(torch.bfloat16) for n in reg.inputs]
     outs = [torch.empty(g.shape_of(n), dtype=torch.bfloat16, device="cuda") for n in reg.outputs]
