@@ -14,6 +14,7 @@ from typing import Dict, Iterable, Optional, Tuple
 import numpy as np
 
 from . import ops
+from . import quant
 
 # Rounding-error model of an implementation that stores activations and
 # weights in bf16 and accumulates in fp32 (the arithmetic the method's
@@ -29,13 +30,23 @@ U_FP32 = 2.0 ** -24  # |fp32_rne(v) - v| <= U_FP32 |v|
 GELU_LIPSCHITZ = 1.13  # max |d/dx x Phi(x)| = 1.1289 (at x = sqrt 2)
 
 
-def eval_node(node, args):
+def eval_node(node, args, weight=None):
+    """Value of ``node`` from its inputs' values.  ``weight`` replaces the
+    node's weight (the effective weights of an FP8 layer, fp8_weights)."""
     op, a, c = node.op, node.attrs, node.consts
+    w = c.get("weight") if weight is None else weight
     if op == "nn.conv2d":
-        return ops.conv2d_nhwc(args[0], c["weight"], tuple(a["strides"]), tuple(a["padding"]),
+        return ops.conv2d_nhwc(args[0], w, tuple(a["strides"]), tuple(a["padding"]),
                                tuple(a["dilation"]), int(a["groups"]))
     if op == "nn.dense":
-        return ops.dense(args[0], c["weight"])
+        return ops.dense(args[0], w)
+    if op == "qnn.quantize":
+        # Section 3.2 Q node: the value the next operator reads is the
+        # quantized tensor's real value (code x scale)
+        if a.get("dtype", "e4m3") == "e4m3":
+            return quant.dequantize_e4m3(quant.quantize_e4m3(args[0], float(a["scale"])), float(a["scale"]))
+        zp = int(a.get("zero_point", 0))
+        return quant.dequantize_int8(quant.quantize_int8(args[0], float(a["scale"]), zp), float(a["scale"]), zp)
     if op == "nn.bias_add":
         return ops.bias_add(args[0], c["bias"])
     if op == "nn.batch_norm":
@@ -59,7 +70,44 @@ def eval_node(node, args):
     raise NotImplementedError(op)
 
 
-def _spread_node(node, args, sq):
+def fp8_weights(graph, nodes=None):
+    """Effective weights of the FP8 layers: a conv2d / dense whose input is an
+    E4M3 Q node's output computes with its weights quantized per output
+    channel after folding the batch norms of its epilogue chain into them
+    (oracle.quant.quantize_weights_e4m3): w_eff = w_q S_w / s, so that the
+    unfolded chain conv(w_eff) -> batch norm (x s) computes with w_q S_w."""
+    by = {n.name: n for n in graph.nodes}
+    readers: Dict[str, list] = {}
+    for n in graph.nodes:
+        for i in n.inputs:
+            readers.setdefault(i, []).append(n)
+    out = {}
+    wanted = set(nodes) if nodes is not None else None
+    for n in graph.nodes:
+        if n.op not in ("nn.conv2d", "nn.dense") or (wanted is not None and n.name not in wanted):
+            continue
+        src = by.get(n.inputs[0])
+        if src is None or src.op != "qnn.quantize" or src.attrs.get("dtype", "e4m3") != "e4m3":
+            continue
+        w = np.asarray(n.consts["weight"], dtype=np.float64)
+        s = np.ones(w.shape[0])
+        cur = n.name
+        while len(readers.get(cur, [])) == 1 and readers[cur][0].op in ("nn.bias_add", "nn.batch_norm"):
+            nx = readers[cur][0]
+            if nx.op == "nn.batch_norm":
+                s = s * np.asarray(nx.consts["gamma"], np.float64) / np.sqrt(
+                    np.asarray(nx.consts["moving_var"], np.float64) + float(nx.attrs.get("epsilon", 1e-5)))
+            cur = nx.name
+        shape = (-1,) + (1,) * (w.ndim - 1)
+        wq, sw = quant.quantize_weights_e4m3(w * s.reshape(shape))
+        out[n.name] = wq * sw.reshape(shape) / s.reshape(shape)
+    return out
+
+
+U_E4M3 = 2.0 ** -3  # one E4M3 step, relative: the most a re-rounded code can move
+
+
+def _spread_node(node, args, sq, weight=None):
     """s^2 of ``node``'s output (before it is rounded for storage), given the
     inputs' values ``args`` and their s^2 ``sq``:
 
@@ -78,8 +126,14 @@ def _spread_node(node, args, sq):
       global_avg_pool  the window's mean sq
     """
     op, a, c = node.op, node.attrs, node.consts
+    if op == "qnn.quantize":
+        # an exact input is quantized identically on both sides (the same
+        # fp32 product decides the code); a computed one can land on the
+        # other side of a rounding boundary: one step
+        return np.where(sq[0] > 0, sq[0] + (U_E4M3 * args[0]) ** 2, 0.0)
     if op in ("nn.conv2d", "nn.dense"):
-        w = np.asarray(c["weight"], dtype=np.float64)
+        fp8 = weight is not None
+        w = np.asarray(c["weight"] if weight is None else weight, dtype=np.float64)
         x = args[0]
         if op == "nn.conv2d":
             K = w.shape[1] * w.shape[2] * w.shape[3]
@@ -89,6 +143,8 @@ def _spread_node(node, args, sq):
             K = w.shape[1]
             lin = ops.dense
         acc = np.sqrt(K) * U_FP32 * lin(np.abs(x), np.abs(w))
+        if fp8:  # the quantized weights are the same on both sides
+            return lin(sq[0], w * w) + acc * acc
         return lin(sq[0], w * w) + U_BF16 ** 2 * lin(x * x, w * w) + acc * acc
     if op == "nn.batch_norm":
         sc = np.asarray(c["gamma"], np.float64) ** 2 / (
@@ -134,15 +190,20 @@ def evaluate_with_error_scale(graph, inputs: Dict[str, np.ndarray], nodes: Optio
     for n in graph.nodes:
         for i in n.inputs:
             readers.setdefault(i, []).append(n)
+    w8 = fp8_weights(graph, nodes)
     for n in graph.nodes:
         if wanted is not None and n.name not in wanted:
             continue
         args = [env[i] for i in n.inputs]
-        v = eval_node(n, args)
-        q = _spread_node(n, args, [sq[i] for i in n.inputs])
+        v = eval_node(n, args, w8.get(n.name))
+        q = _spread_node(n, args, [sq[i] for i in n.inputs], w8.get(n.name))
         rd = readers.get(n.name, [])
         stored = (n.name in kept or len(rd) != 1 or rd[0].op in _GEMM_OR_POOL
                   or (wanted is not None and rd[0].name not in wanted))
+        # a quantizer's output is stored as its codes, exactly; a tensor a
+        # quantizer reads is never stored in bf16 (the quantizer takes it)
+        if n.op == "qnn.quantize" or (len(rd) == 1 and rd[0].op == "qnn.quantize" and n.name not in kept):
+            stored = False
         if stored:
             q = q + (U_BF16 * v) ** 2
         env[n.name], sq[n.name] = v, q
@@ -160,9 +221,10 @@ def evaluate(graph, inputs: Dict[str, np.ndarray], nodes: Optional[Iterable[str]
     (default: the graph outputs that were computed)."""
     env = {k: np.asarray(v, dtype=np.float64) for k, v in inputs.items()}
     wanted = set(nodes) if nodes is not None else None
+    w8 = fp8_weights(graph, nodes)
     for n in graph.nodes:
         if wanted is not None and n.name not in wanted:
             continue
-        env[n.name] = eval_node(n, [env[i] for i in n.inputs])
+        env[n.name] = eval_node(n, [env[i] for i in n.inputs], w8.get(n.name))
     names = list(keep) if keep is not None else [o for o in graph.outputs if o in env]
     return {k: env[k] for k in names}

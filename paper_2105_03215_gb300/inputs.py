@@ -158,6 +158,11 @@ class _Builder:
         assert self.g.shape_of(a) == self.g.shape_of(b)
         return self._add("add", [a, b], self.g.shape_of(a))
 
+    def quantize(self, x, scale, dtype="e4m3", zero_point=0):
+        """A Q node of Section 3.2 (scale S, zero point Z fixed at compile time)."""
+        return self._add("qnn.quantize", [x], self.g.shape_of(x),
+                         dict(scale=float(scale), zero_point=int(zero_point), dtype=dtype))
+
     def max_pool2d(self, x, k, stride, pad):
         N, H, W, C = self.g.shape_of(x)
         return self._add("nn.max_pool2d", [x], (N, conv_out(H, k, stride, pad, pad),
@@ -389,6 +394,45 @@ def conv_general(N=2, H=11, W=13, C=64, K=32, kernel=(1, 3), strides=(1, 1), pad
         g.nodes[0].consts["weight"] = rng.integers(-2, 3, size=(K, C, kh, kw)).astype(np.float32)
         g.nodes[1].consts["bias"] = rng.integers(-8, 9, size=K).astype(np.float32)
     return g, inp
+
+
+# Scales of the FP8 workloads, fixed from the known distributions of the
+# synthetic data (a stand-in for the calibration data of Section 3.2): region
+# inputs ~N(0, 1) are quantized over +-8 (8 standard deviations); the
+# intermediates after batch norm + ReLU (gamma ~ U(0.5, 1.5), Kaiming weights,
+# unit-variance outputs) over +-16.
+FP8_SCALE_INPUT = 8.0 / 448.0
+FP8_SCALE_HIDDEN = 16.0 / 448.0
+
+
+def fp8_conv(N=2, H=14, W=14, C=256, K=256, k=3, seed=31, act="relu"):
+    """conv2d + BN + activation computed in FP8: Q(x) -> conv -> BN -> act."""
+    b = _Builder(f"fp8_conv{k}x{k}")
+    x = b.input("x", (N, H, W, C))
+    y = b.batch_norm(b.conv2d(b.quantize(x, FP8_SCALE_INPUT), K, k))
+    y = b.relu(y) if act == "relu" else y
+    return _finish(b, [y], seed)
+
+
+def fp8_dense(M=256, D=768, F=1024, seed=32):
+    """dense + bias + GELU computed in FP8: Q(x) -> dense -> bias -> GELU."""
+    b = _Builder("fp8_dense")
+    x = b.input("x", (M, D))
+    y = b.gelu(b.bias_add(b.dense(b.quantize(x, FP8_SCALE_INPUT), F)))
+    return _finish(b, [y], seed)
+
+
+def fp8_bottleneck(N=32, H=14, W=14, C=1024, width=256, seed=3):
+    """The ResNet-50 stage-3 bottleneck of resnet_bottleneck (same seed, same
+    constants) with partial quantization (Section 3.2): Q nodes before each
+    convolution, each convolution in FP8; the residual stays bf16."""
+    b = _Builder("fp8_bottleneck")
+    x = b.input("x", (N, H, W, C))
+    t = b.relu(b.batch_norm(b.conv2d(b.quantize(x, FP8_SCALE_INPUT), width, 1)))
+    t = b.relu(b.batch_norm(b.conv2d(b.quantize(t, FP8_SCALE_HIDDEN), width, 3)))
+    t = b.batch_norm(b.conv2d(b.quantize(t, FP8_SCALE_HIDDEN), 4 * width, 1))
+    y = b.relu(b.add(t, x))
+    return _finish(b, [y], seed)
 
 
 def stem(N=2, H=32, W=30, k=7, cout=64, seed=13, C=3):
