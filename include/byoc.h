@@ -60,7 +60,11 @@ typedef enum {
     BYOC_ERR_TIMEOUT = 5      /* a kernel's bounded wait expired (reported by byoc_check) */
 } byoc_status;
 
-typedef enum { BYOC_BF16 = 0, BYOC_FP32 = 1 } byoc_dtype;
+typedef enum {
+    BYOC_BF16 = 0,
+    BYOC_FP32 = 1,
+    BYOC_E4M3 = 2  /* FP8 E4M3 codes (1 byte): the output of a BYOC_OP_QUANTIZE */
+} byoc_dtype;
 
 typedef enum {
     BYOC_LAYOUT_NHWC = 0, /* 4-D activation [N, H, W, C] */
@@ -77,7 +81,21 @@ typedef enum {
     BYOC_OP_RELU = 4,
     BYOC_OP_RELU6 = 5,      /* clip(x, 0, 6) */
     BYOC_OP_GELU = 6,       /* 0.5 x (1 + erf(x / sqrt 2)) */
-    BYOC_OP_ADD = 7         /* in[0] + in[1], same shape */
+    BYOC_OP_ADD = 7,        /* in[0] + in[1], same shape */
+    BYOC_OP_QUANTIZE = 8    /* Section 3.2 Q node: in[0] bf16 -> out BYOC_E4M3,
+                               out = e4m3(in * fp32(1 / S)) rounded to nearest even,
+                               saturating at +-448; consts[0] = &S (1 float > 0),
+                               consts[1] = &Z (1 float, must be 0: E4M3 is symmetric).
+                               A conv2d / dense reading an E4M3 tensor runs in FP8
+                               (kind::f8f6f4 tensor cores, fp32 accumulation): its
+                               weights, folded with the batch norm that follows, are
+                               quantized per output channel with power-of-two scales
+                               S_w[k] = 2^ceil(log2(max |w'[k]| / 448)) at compile time,
+                               and its output is dequantized (x S S_w[k]) in the epilogue.
+                               A QUANTIZE right after a conv2d / dense epilogue chain is
+                               fused into that epilogue; one on a region input is its own
+                               launch.  FP8 layers run in the region kernel (see
+                               BYOC_OPT_REGION_KERNEL) and need C % 128 == 0. */
 } byoc_op_kind;
 
 typedef struct {

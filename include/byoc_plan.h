@@ -26,7 +26,8 @@ typedef enum {
     BYOC_LAUNCH_DEPTHWISE = 1, /* depthwise 3x3 conv + fused epilogue */
     BYOC_LAUNCH_S2D = 2,       /* layout transform of a stride-2 few-channel stem (4-channel, zero-padded pixel pairs) */
     BYOC_LAUNCH_DWPW = 3,      /* depthwise 3x3 + epilogue fused with the 1x1 conv + epilogue after it */
-    BYOC_LAUNCH_CHAIN = 4      /* region kernel: 2-4 conv2d / dense composites in one persistent launch */
+    BYOC_LAUNCH_CHAIN = 4,     /* region kernel: 1-4 conv2d / dense composites in one persistent launch */
+    BYOC_LAUNCH_QUANT = 5      /* bf16 -> FP8 E4M3 quantization of a region input (Section 3.2 Q node) */
 } byoc_launch_kind;
 
 typedef struct {
@@ -51,6 +52,7 @@ typedef struct {
     int32_t stages[BYOC_PLAN_MAX_LAUNCHES];     /* region kernel: composites it runs (gemm_* fields
                                                    describe the first), else 1 */
     int32_t units[BYOC_PLAN_MAX_LAUNCHES];      /* region kernel: output tiles over all its composites */
+    int32_t fp8[BYOC_PLAN_MAX_LAUNCHES];        /* region kernel: composites computed in FP8 */
     double flops;
     double bytes;
     size_t const_bytes;

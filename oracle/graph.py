@@ -95,8 +95,11 @@ def fp8_weights(graph, nodes=None):
         while len(readers.get(cur, [])) == 1 and readers[cur][0].op in ("nn.bias_add", "nn.batch_norm"):
             nx = readers[cur][0]
             if nx.op == "nn.batch_norm":
+                # epsilon as the compiled region carries it (fp32): the rounding
+                # decisions below are then taken on the same folded weights
+                eps = float(np.float32(nx.attrs.get("epsilon", 1e-5)))
                 s = s * np.asarray(nx.consts["gamma"], np.float64) / np.sqrt(
-                    np.asarray(nx.consts["moving_var"], np.float64) + float(nx.attrs.get("epsilon", 1e-5)))
+                    np.asarray(nx.consts["moving_var"], np.float64) + eps)
             cur = nx.name
         shape = (-1,) + (1,) * (w.ndim - 1)
         wq, sw = quant.quantize_weights_e4m3(w * s.reshape(shape))

@@ -21,12 +21,12 @@ OPT_REGION_KERNEL = 0x2
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
 STATUS_NAMES = {0: "OK", 1: "INVALID_ARG", 2: "UNSUPPORTED", 3: "CUDA", 4: "OOM", 5: "TIMEOUT"}
 
-BF16, FP32 = 0, 1
+BF16, FP32, E4M3 = 0, 1, 2
 LAYOUT_NHWC, LAYOUT_NC = 0, 1
 
-OP_CONV2D, OP_DENSE, OP_BIAS_ADD, OP_BATCH_NORM, OP_RELU, OP_RELU6, OP_GELU, OP_ADD = range(8)
+OP_CONV2D, OP_DENSE, OP_BIAS_ADD, OP_BATCH_NORM, OP_RELU, OP_RELU6, OP_GELU, OP_ADD, OP_QUANTIZE = range(9)
 
-LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D, LAUNCH_DWPW, LAUNCH_CHAIN = range(5)
+LAUNCH_GEMM, LAUNCH_DEPTHWISE, LAUNCH_S2D, LAUNCH_DWPW, LAUNCH_CHAIN, LAUNCH_QUANT = range(6)
 PLAN_MAX_LAUNCHES = 128
 
 
@@ -70,7 +70,7 @@ class PlanReport(ctypes.Structure):
                 ("tile_n", c_int32 * _L), ("tile_k", c_int32 * _L), ("im2col", c_int32 * _L),
                 ("grid", c_int32 * _L), ("resident_b", c_int32 * _L), ("slab_slots", c_int32 * _L),
                 ("splits", c_int32 * _L), ("pair_units", c_int32 * _L), ("stages", c_int32 * _L),
-                ("units", c_int32 * _L),
+                ("units", c_int32 * _L), ("fp8", c_int32 * _L),
                 ("flops", c_double), ("bytes", c_double),
                 ("const_bytes", c_size_t), ("workspace_bytes", c_size_t)]
 

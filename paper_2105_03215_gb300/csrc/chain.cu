@@ -234,6 +234,7 @@ __global__ void __maxnreg__(168)
                     w0 = q * cs.stride_w - cs.pad_l;
                 }
                 int cc = 0, r = 0, sx = 0;
+                const int kel = cs.fp8 ? 2 * S::BK : S::BK;  // elements per 128-byte k-block
                 for (int kb = 0; kb < cs.num_kb; ++kb) {
                     if (!wait(bars + 8u * (S::STAGES + stage), phase ^ 1u)) {
                         ok = false;
@@ -243,7 +244,7 @@ __global__ void __maxnreg__(168)
                     mbar_arrive_expect_tx(full, (uint32_t)S::STAGE_BYTES);
                     const uint32_t dA = sA + stage * S::A_BYTES;
                     if (cs.mode == kChainIm2col) {
-                        tma_load_im2col_4d(dA, &maps.A[si], full, cc * S::BK, w0, h0, img,
+                        tma_load_im2col_4d(dA, &maps.A[si], full, cc * kel, w0, h0, img,
                                            (uint16_t)(sx * cs.dil_w), (uint16_t)(r * cs.dil_h));
                         if (++cc == cs.chunks) {
                             cc = 0;
@@ -253,9 +254,9 @@ __global__ void __maxnreg__(168)
                             }
                         }
                     } else {
-                        tma_load_2d(dA, &maps.A[si], full, kb * S::BK, m0);
+                        tma_load_2d(dA, &maps.A[si], full, kb * kel, m0);
                     }
-                    tma_load_2d(sB + stage * S::B_BYTES, &maps.B[si], full, kb * S::BK, n0);
+                    tma_load_2d(sB + stage * S::B_BYTES, &maps.B[si], full, kb * kel, n0);
                     ++issued;
                     if (++stage == S::STAGES) {
                         stage = 0;
@@ -336,7 +337,8 @@ __global__ void __maxnreg__(168)
             auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
                 return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutMma);
             };
-            constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
+            constexpr uint32_t idesc16 = make_idesc_bf16(S::BM, BN);
+            constexpr uint32_t idesc8 = make_idesc_e4m3(S::BM, BN);
             const uint64_t adesc0 = make_smem_desc(sA, S::ROW_BYTES);
             const uint64_t bdesc0 = make_smem_desc(sB, S::ROW_BYTES);
             int stage = 0;
@@ -354,6 +356,7 @@ __global__ void __maxnreg__(168)
                 }
                 tc_fence_after();
                 const uint32_t d_tmem = tmem_base + (uint32_t)(buf * BN);
+                const bool f8 = cs.fp8 != 0;
                 uint32_t acc = 0u;
                 for (int kb = 0; kb < cs.num_kb; ++kb) {
                     if (!wait(bars + 8u * stage, phase)) {
@@ -363,9 +366,18 @@ __global__ void __maxnreg__(168)
                     tc_fence_after();
                     const uint64_t ad = adesc0 + (uint64_t)((stage * S::A_BYTES) >> 4);
                     const uint64_t bd = bdesc0 + (uint64_t)((stage * S::B_BYTES) >> 4);
+                    // four MMAs per 128-byte k-block: K = 16 bf16 or K = 32 E4M3
+                    // values, 32 bytes each either way
+                    if (f8) {
 #pragma unroll
-                    for (int k = 0; k < S::BK / 16; ++k)
-                        mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc, acc | (uint32_t)k);
+                        for (int k = 0; k < 4; ++k)
+                            mma_f8_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc8, acc | (uint32_t)k);
+                    } else {
+#pragma unroll
+                        for (int k = 0; k < 4; ++k)
+                            mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc16,
+                                        acc | (uint32_t)k);
+                    }
                     acc = 1u;
                     mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
                     if (++stage == S::STAGES) {
@@ -414,15 +426,7 @@ __global__ void __maxnreg__(168)
 #pragma unroll
                 for (int q = 0; q < 4; ++q) rn[q] = ld_cg_v4(rp + 8 * q);
             };
-            // the bias slice of the chunk: the same 128 bytes in every lane
-            float4 bn4[8];
-            auto load_bias = [&](int ci) {
-                const float4 *bp = reinterpret_cast<const float4 *>(cs.bias + n0 + ci * 32);
-#pragma unroll
-                for (int q = 0; q < 8; ++q) bn4[q] = __ldg(bp + q);
-            };
             if (has_res && grp < nch) load_res(grp);
-            if (grp < nch) load_bias(grp);
             if (!mbar_wait(tfull + 8u * buf, ((uint32_t)(t >> 1)) & 1u, abort_flag, a.err, kErrTimeoutEpilogue))
                 break;
             tc_fence_after();
@@ -435,13 +439,24 @@ __global__ void __maxnreg__(168)
             for (int ci = grp; ci < nch; ci += 2) {
                 const int col0 = n0 + ci * 32;
                 uint4 rr[4];
-                float4 b4[8];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) rr[q] = rn[q];
-#pragma unroll
-                for (int q = 0; q < 8; ++q) b4[q] = bn4[q];
                 if (has_res && ci + 2 < nch) load_res(ci + 2);
-                if (ci + 2 < nch) load_bias(ci + 2);
+                // the chunk's bias (and FP8 dequantization scales): the same 128
+                // bytes in every lane, loaded while the TMEM load is in flight
+                float4 b4[8];
+                {
+                    const float4 *bp = reinterpret_cast<const float4 *>(cs.bias + col0);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) b4[q] = __ldg(bp + q);
+                }
+                // FP8: the accumulator is in units of S_x S_w[n] (dequantization scales)
+                float4 d4[8];
+                if (cs.fp8) {
+                    const float4 *dp = reinterpret_cast<const float4 *>(cs.dq + col0);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) d4[q] = __ldg(dp + q);
+                }
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
                 if (ci + 2 >= nch) {  // this warp's last read of the accumulator
@@ -450,12 +465,22 @@ __global__ void __maxnreg__(168)
                     if (lane == 0) mbar_arrive(tempty + 8u * buf);
                 }
                 float f[32];
+                if (cs.fp8) {
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
-                    f[4 * j] = __uint_as_float(v[4 * j]) + b4[j].x;
-                    f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4[j].y;
-                    f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4[j].z;
-                    f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4[j].w;
+                    for (int j = 0; j < 8; ++j) {
+                        f[4 * j] = fmaf(__uint_as_float(v[4 * j]), d4[j].x, b4[j].x);
+                        f[4 * j + 1] = fmaf(__uint_as_float(v[4 * j + 1]), d4[j].y, b4[j].y);
+                        f[4 * j + 2] = fmaf(__uint_as_float(v[4 * j + 2]), d4[j].z, b4[j].z);
+                        f[4 * j + 3] = fmaf(__uint_as_float(v[4 * j + 3]), d4[j].w, b4[j].w);
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j) {
+                        f[4 * j] = __uint_as_float(v[4 * j]) + b4[j].x;
+                        f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4[j].y;
+                        f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4[j].z;
+                        f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4[j].w;
+                    }
                 }
                 if (has_res) {
 #pragma unroll
@@ -485,16 +510,35 @@ __global__ void __maxnreg__(168)
                 const uint32_t stg = stg0 + (uint32_t)(sb * S::EPI_TILE);
                 if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
                 __syncwarp();
+                if (cs.out8) {
+                    // a fused Q node: E4M3 codes of f x fp32(1/S), 32 bytes per
+                    // row, rows 32 bytes apart (the unswizzled box of the map)
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
-                    const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
-                    const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
-                    const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
-                    const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
-                    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0), "r"(w1),
-                                 "r"(w2), "r"(w3)
-                                 : "memory");
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const float *g = f + 16 * h + 4 * k;
+                            w[k] = cvt_e4m3x2(g[0] * cs.out_inv, g[1] * cs.out_inv) |
+                                   (cvt_e4m3x2(g[2] * cs.out_inv, g[3] * cs.out_inv) << 16);
+                        }
+                        const uint32_t addr = stg + (uint32_t)lane * 32u + (uint32_t)h * 16u;
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]), "r"(w[1]),
+                                     "r"(w[2]), "r"(w[3])
+                                     : "memory");
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
+                        const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
+                        const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
+                        const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
+                        const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0), "r"(w1),
+                                     "r"(w2), "r"(w3)
+                                     : "memory");
+                    }
                 }
                 fence_proxy_async_smem();
                 __syncwarp();

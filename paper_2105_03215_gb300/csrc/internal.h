@@ -271,17 +271,21 @@ enum : int { kChainTile = 0, kChainIm2col = 1 };
 struct ChainStage {
     const float *bias;       // [tiles_n * BN], zero padded
     const __nv_bfloat16 *residual;  // [M, N] or null (a region input or an earlier stage's output)
+    const float *dq;         // FP8 stage: [tiles_n * BN] dequantization scales S_x S_w[n], else null
     int mode;                // kChainTile | kChainIm2col
     int M, N;                // output rows; output channels (row stride of out and residual)
-    int num_kb, chunks, kw;  // k-blocks of 64 (im2col: taps x chunks), chunks per tap, filter width
+    int num_kb, chunks, kw;  // k-blocks of 128 bytes (im2col: taps x chunks), chunks per tap, filter width
     int dil_h, dil_w, Ho, Wo, stride_h, stride_w, pad_t, pad_l;  // im2col geometry
     int tiles_n, num_tiles;
     int unit0;               // first unit of this stage in stage-major numbering (host bookkeeping)
     int cbase;               // first completion counter of this stage (one per m-tile)
     int act;
     int consumed;            // a later stage reads this stage's output: its units count into the counters
-    int res_dep;             // the residual is an earlier stage's output (the epilogue acquires it too)
-    int reserved;
+    int res_dep;             // the residual is an earlier stage's output
+    int fp8;                 // A and B are E4M3 codes (kind::f8f6f4); a k-block is 128 elements, not 64
+    int out8;                // the output is quantized to E4M3 codes with out_inv (a fused Q node)
+    float out_inv;           // fp32(1 / S) of that Q node
+    int reserved[2];
 };
 struct ChainArgs {
     ChainStage st[kChainMaxStages];
@@ -296,7 +300,9 @@ struct ChainArgs {
     unsigned long long *trace;  // as GemmArgs::trace
     int n_stages, total_units, n_counters, reserved;
 };
-static_assert(sizeof(ChainStage) == 2 * 8 + 22 * 4 && sizeof(ChainArgs) == kChainMaxStages * sizeof(ChainStage) + 9 * 8 + 16,
+// every field counted: 3 pointers and 26 4-byte fields, so no padding byte
+static_assert(sizeof(ChainStage) == 3 * 8 + 26 * 4 && offsetof(ChainStage, reserved) + 8 == sizeof(ChainStage) &&
+                  sizeof(ChainArgs) == kChainMaxStages * sizeof(ChainStage) + 9 * 8 + 16,
               "region kernel arguments without padding");
 struct ChainMaps {
     CUtensorMap A[kChainMaxStages], B[kChainMaxStages], O[kChainMaxStages];
@@ -305,6 +311,12 @@ size_t chain_smem_bytes(int bn);
 int chain_stages(int bn);
 cudaError_t chain_prepare(int bn);  // bn: 128 or 256
 cudaError_t launch_chain(int bn, const ChainMaps &maps, const ChainArgs &a, int grid, cudaStream_t st);
+
+// Section 3.2 Q node on a region input: q[i] = e4m3(x[i] * inv_scale) (the
+// product in fp32, nearest even, saturating at +-448); n a multiple of 8,
+// both pointers 16-byte aligned.
+cudaError_t launch_quantize_e4m3(const __nv_bfloat16 *x, uint8_t *q, size_t n, float inv_scale, int num_sms,
+                                 cudaStream_t st);
 
 // NCHW fp32 -> NHWC bf16 (channels zero-padded to Cp) at a region boundary.
 // Requires W * Cp <= kNchwStageElems; y 16-byte aligned when its rows are.

@@ -99,6 +99,18 @@ CUresult encode_2d(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+// 2-D row-major E4M3 (1-byte) matrix [rows, cols]; box = [box_cols, box_rows].
+CUresult encode_2d_u8(CUtensorMap *m, const void *ptr, uint64_t rows, uint64_t cols, uint32_t box_rows,
+                      uint32_t box_cols, CUtensorMapSwizzle swz) {
+    cuuint64_t dims[2] = {cols, rows};
+    cuuint64_t strides[1] = {cols};
+    cuuint32_t box[2] = {box_cols, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    return p_encode_tiled(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<void *>(ptr), dims, strides, box, es,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                          CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
 // Geometry of an im2col-read convolution input.
 struct Im2colGeom {
     int N, H, W, C;
@@ -109,16 +121,18 @@ struct Im2colGeom {
 // The bounding box of filter origins runs, per spatial dimension, from -pad_before
 // to (dim - 1) + pad_after - (k - 1) * dilation; corner and offset arrays list
 // the spatial dimensions innermost first (W, then H), like the tensor's dims.
-CUresult encode_im2col(CUtensorMap *m, const void *ptr, const Im2colGeom &g, int bk) {
+CUresult encode_im2col(CUtensorMap *m, const void *ptr, const Im2colGeom &g, int bk, bool e4m3 = false) {
+    const cuuint64_t es_b = e4m3 ? 1 : 2;
     cuuint64_t dims[4] = {(cuuint64_t)g.C, (cuuint64_t)g.W, (cuuint64_t)g.H, (cuuint64_t)g.N};
-    cuuint64_t strides[3] = {(cuuint64_t)g.C * 2, (cuuint64_t)g.W * g.C * 2,
-                             (cuuint64_t)g.H * g.W * g.C * 2};
+    cuuint64_t strides[3] = {(cuuint64_t)g.C * es_b, (cuuint64_t)g.W * g.C * es_b,
+                             (cuuint64_t)g.H * g.W * g.C * es_b};
     int lower[2] = {-g.pl, -g.pt};
     int upper[2] = {g.pr - (g.kw - 1) * g.dw, g.pb - (g.kh - 1) * g.dh};
     cuuint32_t es[4] = {1, (cuuint32_t)g.sw, (cuuint32_t)g.sh, 1};
-    return p_encode_im2col(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims,
-                           strides, lower, upper, (cuuint32_t)bk, (cuuint32_t)byoc::kGemmBM, es,
-                           CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
+    // E4M3: 128 codes per pixel fill the same 128-byte swizzled row as 64 bf16
+    return p_encode_im2col(m, e4m3 ? CU_TENSOR_MAP_DATA_TYPE_UINT8 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4,
+                           const_cast<void *>(ptr), dims, strides, lower, upper, (cuuint32_t)(e4m3 ? 2 * bk : bk),
+                           (cuuint32_t)byoc::kGemmBM, es, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle_for(bk),
                            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
@@ -196,17 +210,49 @@ uint16_t f32_to_bf16_rne(float f) {
 
 size_t align_up(size_t v, size_t a) { return (v + a - 1) / a * a; }
 
+// Nearest FP8 E4M3 code of v: 1 sign bit, 4 exponent bits (bias 7), 3
+// mantissa bits; a value in [2^e, 2^(e+1)) with e >= -6 is a multiple of
+// 2^(e-3), below 2^-6 the values are the multiples of 2^-9 (exponent field
+// 0).  Ties to even (nearbyint in the default rounding mode); magnitudes past
+// 448, the largest finite value, saturate to it.
+uint8_t e4m3_code(double v) {
+    const uint8_t sign = std::signbit(v) ? 0x80 : 0x00;
+    const double a = std::fabs(v);
+    if (!(a == a)) return 0x7F;
+    int ex = 0;
+    std::frexp(a, &ex);  // a = m 2^ex, 1/2 <= m < 1
+    int e = std::max(ex - 1, -6);
+    double q = std::nearbyint(std::ldexp(a, 3 - e));  // a / 2^(e-3)
+    if (q >= 16.0) {  // rounded up into the next binade
+        q = 8.0;
+        e += 1;
+    }
+    if (q < 8.0) return sign | (uint8_t)q;                    // exponent field 0 (e == -6)
+    if (e > 8 || (e == 8 && q > 14.0)) return sign | 0x7E;   // saturate at 448 = 1.75 x 2^8
+    return sign | (uint8_t)((e + 7) << 3) | (uint8_t)(q - 8.0);
+}
+
+// Per-output-channel scale of FP8 weights: the smallest power of two S with
+// max |w'| / S <= 448 (1 for an all-zero channel).
+double e4m3_weight_scale(double maxabs) {
+    if (!(maxabs > 0.0)) return 1.0;
+    int ex = 0;
+    const double f = std::frexp(maxabs / 448.0, &ex);
+    return std::ldexp(1.0, f == 0.5 ? ex - 1 : ex);
+}
+
 // ------------------------------------------------------------ plan structures
 
 struct TensorInfo {
     int ndim = 0;
+    int dtype = BYOC_BF16;  // BYOC_BF16 or BYOC_E4M3
     int64_t shape[4] = {0, 0, 0, 0};
     size_t elems() const {
         size_t e = 1;
         for (int i = 0; i < ndim; ++i) e *= (size_t)shape[i];
         return e;
     }
-    size_t bytes() const { return elems() * 2; }
+    size_t bytes() const { return elems() * (dtype == BYOC_E4M3 ? 1 : 2); }
     int64_t channels() const { return shape[ndim - 1]; }
 };
 
@@ -245,6 +291,16 @@ struct LaunchPlan {
     size_t cw_off[byoc::kChainMaxStages] = {}, cb_off[byoc::kChainMaxStages] = {};
     size_t order_off = 0, dep_off_off = 0, dep_list_off = 0;  // constant blob: int32 unit order, dependencies
     size_t cta_off_off = 0, cta_list_off = 0;                 // constant blob: int32 per-CTA unit lists
+    size_t c_dq_off[byoc::kChainMaxStages] = {};
+    // FP8 GEMM (region kernel only): A and B are E4M3 codes; dq = [n_pad] fp32
+    // dequantization scales S_x S_w[n] in the constant blob
+    int fp8 = 0;
+    size_t dq_off = 0;
+    // a Q node fused into the epilogue: the output is E4M3 codes of x fp32(1/S)
+    int out8 = 0;
+    float out_inv = 0.0f;
+    // BYOC_LAUNCH_QUANT: y = e4m3(x fp32(1/S))
+    float q_inv = 0.0f;
     size_t flags_off = 0, flags_bytes = 0;     // workspace: unit flags + control words
     byoc::ChainArgs chain{};
     double flops = 0, bytes = 0;
@@ -290,9 +346,10 @@ byoc_status validate(const byoc_region_desc *d, Plan &P) {
         if ((t.ndim == 4) != (t.layout == BYOC_LAYOUT_NHWC))
             return fail(BYOC_ERR_INVALID_ARG, "tensor %d: layout %d does not match ndim %d", i,
                         t.layout, t.ndim);
-        if (t.dtype != BYOC_BF16)
-            return fail(BYOC_ERR_UNSUPPORTED, "tensor %d: activations must be bf16", i);
+        if (t.dtype != BYOC_BF16 && t.dtype != BYOC_E4M3)
+            return fail(BYOC_ERR_UNSUPPORTED, "tensor %d: activations must be bf16 or E4M3 codes", i);
         P.tensors[i].ndim = t.ndim;
+        P.tensors[i].dtype = t.dtype;
         for (int k = 0; k < t.ndim; ++k) {
             if (t.shape[k] <= 0 || t.shape[k] > (int64_t)1 << 31)
                 return fail(BYOC_ERR_INVALID_ARG, "tensor %d: bad extent %lld", i,
@@ -320,7 +377,7 @@ byoc_status validate(const byoc_region_desc *d, Plan &P) {
     }
     for (int o = 0; o < d->n_ops; ++o) {
         const byoc_op &op = d->ops[o];
-        if (op.kind < BYOC_OP_CONV2D || op.kind > BYOC_OP_ADD)
+        if (op.kind < BYOC_OP_CONV2D || op.kind > BYOC_OP_QUANTIZE)
             return fail(BYOC_ERR_INVALID_ARG, "op %d: unknown kind %d", o, op.kind);
         const int want_in = op.kind == BYOC_OP_ADD ? 2 : 1;
         if (op.n_in != want_in)
@@ -346,7 +403,30 @@ byoc_status validate(const byoc_region_desc *d, Plan &P) {
                 if (a.shape[k] != b.shape[k]) return false;
             return true;
         };
+        // E4M3 tensors come from Q nodes and feed conv2d / dense only
+        if ((Y.dtype == BYOC_E4M3) != (op.kind == BYOC_OP_QUANTIZE))
+            return fail(BYOC_ERR_INVALID_ARG, "op %d: only a quantize op writes an E4M3 tensor", o);
+        for (int k = 0; k < op.n_in; ++k)
+            if (P.tensors[op.in[k]].dtype == BYOC_E4M3 &&
+                !(k == 0 && (op.kind == BYOC_OP_CONV2D || op.kind == BYOC_OP_DENSE)))
+                return fail(BYOC_ERR_UNSUPPORTED, "op %d: E4M3 tensors feed conv2d / dense data inputs only", o);
+        if (op.kind == BYOC_OP_CONV2D && X.dtype == BYOC_E4M3 && op.groups != 1)
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: grouped conv2d on E4M3 codes", o);
         switch (op.kind) {
+            case BYOC_OP_QUANTIZE: {
+                if (X.dtype != BYOC_BF16 || !same_shape(X, Y))
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: quantize needs a bf16 input of its output's shape", o);
+                if (!op.consts[0] || !op.consts[1])
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: quantize needs its scale and zero point", o);
+                const float S = op.consts[0][0], Z = op.consts[1][0];
+                if (!(S > 0.0f) || !std::isfinite(S) || !std::isfinite(1.0 / (double)S))
+                    return fail(BYOC_ERR_INVALID_ARG, "op %d: quantize scale %g", o, (double)S);
+                if (Z != 0.0f)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: E4M3 is symmetric: zero point must be 0", o);
+                if (X.channels() % 8)
+                    return fail(BYOC_ERR_UNSUPPORTED, "op %d: quantize needs channels % 8 == 0", o);
+                break;
+            }
             case BYOC_OP_CONV2D: {
                 if (X.ndim != 4 || Y.ndim != 4)
                     return fail(BYOC_ERR_INVALID_ARG, "op %d: conv2d needs NHWC tensors", o);
@@ -405,6 +485,12 @@ byoc_status validate(const byoc_region_desc *d, Plan &P) {
     for (int id : P.outputs)
         if (producer[id] < 0)
             return fail(BYOC_ERR_INVALID_ARG, "output tensor %d is produced by no op", id);
+    for (int id : P.inputs)
+        if (P.tensors[id].dtype != BYOC_BF16)
+            return fail(BYOC_ERR_UNSUPPORTED, "input tensor %d: region inputs are bf16", id);
+    for (int id : P.outputs)
+        if (P.tensors[id].dtype != BYOC_BF16)
+            return fail(BYOC_ERR_UNSUPPORTED, "output tensor %d: region outputs are bf16", id);
     return BYOC_OK;
 }
 
@@ -539,6 +625,23 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
     int o = 0;
     while (o < d->n_ops) {
         const byoc_op &op = d->ops[o];
+        if (op.kind == BYOC_OP_QUANTIZE) {
+            // a Q node that no epilogue absorbed (it reads a region input or
+            // a tensor with other readers): its own launch
+            if ((int)P.launches.size() >= BYOC_PLAN_MAX_LAUNCHES - 1)
+                return fail(BYOC_ERR_UNSUPPORTED, "region needs more than %d launches", BYOC_PLAN_MAX_LAUNCHES - 1);
+            LaunchPlan Q;
+            Q.kind = BYOC_LAUNCH_QUANT;
+            Q.first_op = o;
+            Q.n_ops = 1;
+            Q.x = op.in[0];
+            Q.y = op.out;
+            Q.q_inv = (float)(1.0 / (double)op.consts[0][0]);
+            Q.bytes = (double)P.tensors[op.in[0]].bytes() + (double)P.tensors[op.out].bytes();
+            P.launches.push_back(Q);
+            ++o;
+            continue;
+        }
         if (op.kind != BYOC_OP_CONV2D && op.kind != BYOC_OP_DENSE)
             return fail(BYOC_ERR_UNSUPPORTED,
                         "op %d (kind %d) is not preceded by a conv2d/dense it can fuse into; "
@@ -555,6 +658,11 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         // norm (folded into af), residual add and activation ops that follow
         // it, each the single consumer of the previous one.  Returns the index
         // of the first op after the chain.
+        int out8 = 0;
+        float out_inv = 0.0f;
+        // (region kernel) a Q node right after the chain is fused: the
+        // epilogue writes E4M3 codes
+        const bool fuse_q = chain_bn > 0 && (op.kind == BYOC_OP_DENSE || op.groups == 1);
         auto walk_chain = [&](int first, Affine &af, int &cur, int &res, int &act) -> int {
             const int64_t Co = P.tensors[d->ops[first].out].channels();
             af.scale.assign(Co, 1.0);
@@ -581,6 +689,12 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
                     if (r2 == cur) break;  // x + x: not a residual pattern
                     res = r2;
                     stage = 1;
+                } else if (nx.kind == BYOC_OP_QUANTIZE && fuse_q && first == o) {
+                    out8 = 1;
+                    out_inv = (float)(1.0 / (double)nx.consts[0][0]);
+                    cur = nx.out;
+                    ++jj;
+                    break;
                 } else if ((nx.kind == BYOC_OP_RELU || nx.kind == BYOC_OP_RELU6 ||
                             nx.kind == BYOC_OP_GELU) && stage <= 1) {
                     act = nx.kind == BYOC_OP_RELU ? byoc::kActRelu
@@ -895,7 +1009,13 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         }
         taps = kh * kw;
         bk = op.kind == BYOC_OP_DENSE || chain_bn > 0 ? 64 : pick_bk(C);
-        chunks = (int)((C + bk - 1) / bk);
+        // an E4M3 input makes an FP8 layer (region kernel only); its k-blocks
+        // hold 128 codes (128 bytes, like 64 bf16 values)
+        const bool fp8 = X.dtype == BYOC_E4M3;
+        if (fp8 && chain_bn == 0)
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: FP8 layers run in the region kernel", o);
+        const int kel = fp8 ? 128 : bk;
+        chunks = (int)((C + kel - 1) / kel);
         const bool has_res = res >= 0;
         const int amode = slab ? byoc::kAModeSlab : (im2col ? byoc::kAModeIm2col : byoc::kAModeTile);
         const int64_t tiles_per_img = slab ? (Y.shape[1] + sgeo.t - 1) / sgeo.t : 0;
@@ -951,21 +1071,53 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
             L.args.slab_bytes = sgeo.bytes;
         }
         L.n_pad = (int)((Cout + bn - 1) / bn * bn);
-        L.k_pack = taps * chunks * bk;
+        L.k_pack = taps * chunks * kel;
         Kreal = stem_k > 0 ? stem_k : (int64_t)taps * C;
-        // Folded, bf16-rounded, K-major packed weights [n_pad][k_pack].
-        std::vector<uint16_t> wp((size_t)L.n_pad * L.k_pack, 0);
-        for (int64_t k = 0; k < Cout; ++k)
-            for (int t = 0; t < taps; ++t)
-                for (int64_t c = 0; c < C; ++c) {
-                    const double v = wsrc[((size_t)k * taps + t) * C + c] * af.scale[k];
-                    const size_t col = ((size_t)t * chunks + c / bk) * bk + c % bk;
-                    wp[(size_t)k * L.k_pack + col] = f32_to_bf16_rne((float)v);
-                }
+        if (fp8) {
+            // FP8: the folded weights of output channel k quantized with the
+            // power-of-two scale S_w[k] to E4M3 codes, K-major [n_pad][k_pack];
+            // the epilogue multiplies by dq[k] = fp32(S_x S_w[k]), S_x the scale
+            // of the Q node that wrote the input
+            double sx = 0.0;
+            for (int q = 0; q < o; ++q)
+                if (d->ops[q].kind == BYOC_OP_QUANTIZE && d->ops[q].out == op.in[0]) sx = d->ops[q].consts[0][0];
+            if (!(sx > 0.0)) return fail(BYOC_ERR_INVALID_ARG, "op %d: E4M3 input without a quantize op", o);
+            std::vector<uint8_t> w8((size_t)L.n_pad * L.k_pack, 0);
+            std::vector<float> dq((size_t)L.n_pad, 0.0f);
+            for (int64_t k = 0; k < Cout; ++k) {
+                double m = 0.0;
+                for (size_t i = 0; i < (size_t)taps * C; ++i)
+                    m = std::max(m, std::fabs(wsrc[(size_t)k * taps * C + i] * af.scale[k]));
+                const double sw = e4m3_weight_scale(m);
+                for (int t = 0; t < taps; ++t)
+                    for (int64_t c = 0; c < C; ++c) {
+                        const double v = wsrc[((size_t)k * taps + t) * C + c] * af.scale[k];
+                        const size_t col = ((size_t)t * chunks + c / kel) * kel + c % kel;
+                        w8[(size_t)k * L.k_pack + col] = e4m3_code(v / sw);
+                    }
+                dq[k] = (float)(sx * sw);
+            }
+            L.w_off = blob_append(P.blob, w8.data(), w8.size());
+            L.w_bytes = w8.size();
+            L.dq_off = blob_append(P.blob, dq.data(), dq.size() * 4);
+            L.fp8 = 1;
+        } else {
+            // Folded, bf16-rounded, K-major packed weights [n_pad][k_pack].
+            std::vector<uint16_t> wp((size_t)L.n_pad * L.k_pack, 0);
+            for (int64_t k = 0; k < Cout; ++k)
+                for (int t = 0; t < taps; ++t)
+                    for (int64_t c = 0; c < C; ++c) {
+                        const double v = wsrc[((size_t)k * taps + t) * C + c] * af.scale[k];
+                        const size_t col = ((size_t)t * chunks + c / bk) * bk + c % bk;
+                        wp[(size_t)k * L.k_pack + col] = f32_to_bf16_rne((float)v);
+                    }
+            L.w_off = blob_append(P.blob, wp.data(), wp.size() * 2);
+            L.w_bytes = wp.size() * 2;
+        }
+        L.out8 = out8;
+        L.out_inv = out_inv;
         std::vector<float> bias((size_t)L.n_pad, 0.0f);
         for (int64_t k = 0; k < Cout; ++k) bias[k] = (float)af.shift[k];
-        L.w_off = blob_append(P.blob, wp.data(), wp.size() * 2);
-        L.w_bytes = wp.size() * 2;
         L.b_off = blob_append(P.blob, bias.data(), bias.size() * 4);
         L.b_bytes = bias.size() * 4;
 
@@ -1002,7 +1154,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         const double in_bytes = stem_k > 0 ? 0.0  // xq: the image is counted by the layout transform
                                 : L.x < P.n_region_tensors ? (double)X.bytes()
                                                            : (double)P.tensors[L.x].bytes();
-        L.bytes = in_bytes + (double)Y.bytes() + (double)Cout * Kreal * 2 + (double)Cout * 4 +
+        L.bytes = in_bytes + (double)Y.bytes() + (double)Cout * Kreal * (fp8 ? 1 : 2) + (double)Cout * 4 +
                   (res >= 0 ? (double)P.tensors[res].bytes() : 0.0);
         P.launches.push_back(L);
         o = j;
@@ -1049,16 +1201,30 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
 // for the completion counters of p's m-tiles over those rows (every column
 // tile of p).
 bool make_chain(Plan &P, int bn) {
+    // leading Q nodes on region inputs stay launches of their own
+    int q0 = 0;
+    while (q0 < (int)P.launches.size() && P.launches[q0].kind == BYOC_LAUNCH_QUANT) ++q0;
+    std::vector<LaunchPlan> quants(P.launches.begin(), P.launches.begin() + q0);
+    P.launches.erase(P.launches.begin(), P.launches.begin() + q0);
     const int ns = (int)P.launches.size();
-    if (ns < 2 || ns > byoc::kChainMaxStages) return false;
+    bool any8 = false;
+    for (const LaunchPlan &L : P.launches) any8 |= L.fp8 != 0;
+    // a single bf16 GEMM stays with the per-composite kernel
+    auto undo = [&]() {
+        P.launches.insert(P.launches.begin(), quants.begin(), quants.end());
+        return false;
+    };
+    if (ns < (any8 ? 1 : 2) || ns > byoc::kChainMaxStages) return undo();
     for (const LaunchPlan &L : P.launches) {
         if (L.kind != BYOC_LAUNCH_GEMM || L.cfg.bk != 64 || L.cfg.bn != bn || L.stem_R != 0 || L.x_off ||
             L.y_off)
-            return false;
-        if (L.cfg.amode != byoc::kAModeTile && L.cfg.amode != byoc::kAModeIm2col) return false;
-        if ((L.cfg.amode == byoc::kAModeTile ? L.aK : (int64_t)L.geo.C) % 64) return false;
-        if (L.args.N % 32) return false;  // the epilogue reads residual rows in 32-column pieces
-        if (L.args.num_tiles != (L.args.M + byoc::kGemmBM - 1) / byoc::kGemmBM * L.args.tiles_n) return false;
+            return undo();
+        if (L.cfg.amode != byoc::kAModeTile && L.cfg.amode != byoc::kAModeIm2col) return undo();
+        // whole 128-byte k-blocks: 64 bf16 channels, or 128 E4M3 channels
+        if ((L.cfg.amode == byoc::kAModeTile ? L.aK : (int64_t)L.geo.C) % (L.fp8 ? 128 : 64)) return undo();
+        if (L.args.N % 32) return undo();  // the epilogue reads residual rows in 32-column pieces
+        if (L.res >= 0 && P.tensors[L.res].dtype != BYOC_BF16) return undo();
+        if (L.args.num_tiles != (L.args.M + byoc::kGemmBM - 1) / byoc::kGemmBM * L.args.tiles_n) return undo();
     }
     LaunchPlan C;
     C.kind = BYOC_LAUNCH_CHAIN;
@@ -1094,6 +1260,10 @@ bool make_chain(Plan &P, int bn) {
         cs.unit0 = units;
         units += cs.num_tiles;
         cs.act = L.act;
+        cs.fp8 = L.fp8;
+        cs.out8 = L.out8;
+        cs.out_inv = L.out_inv;
+        C.c_dq_off[s] = L.dq_off;
         C.n_ops += L.n_ops;
         C.cx[s] = L.x;
         C.cy[s] = L.y;
@@ -1106,8 +1276,8 @@ bool make_chain(Plan &P, int bn) {
         C.cw_off[s] = L.w_off;
         C.cb_off[s] = L.b_off;
         C.flops += L.flops;
-        // weights once: 2 M N K flops -> N K bf16 weights, N fp32 biases
-        wbytes += L.flops / (2.0 * cs.M) * 2.0 + (double)cs.N * 4.0;
+        // weights once: 2 M N K flops -> N K bf16 (E4M3) weights, N fp32 biases
+        wbytes += L.flops / (2.0 * cs.M) * (L.fp8 ? 1.0 : 2.0) + (double)cs.N * (L.fp8 ? 8.0 : 4.0);
     }
     A.total_units = units;
     int ncnt = 0;
@@ -1253,9 +1423,17 @@ bool make_chain(Plan &P, int bn) {
     C.order_off = blob_append(P.blob, order.data(), order.size() * 4);
     C.dep_off_off = blob_append(P.blob, off.data(), off.size() * 4);
     C.dep_list_off = blob_append(P.blob, list.data(), list.size() * 4);
-    // algorithmic bytes: the region's inputs and outputs once, the weights once
+    // algorithmic bytes: what the stages read from outside the chain (region
+    // inputs, quantized inputs) and the region's outputs once, the weights once
     double io = 0;
-    for (int t : P.inputs) io += (double)P.tensors[t].bytes();
+    std::vector<int> seen_in;
+    for (int s = 0; s < ns; ++s)
+        for (int t : {C.cx[s], C.cres[s]}) {
+            if (t < 0 || producer(t, ns) >= 0 || std::find(seen_in.begin(), seen_in.end(), t) != seen_in.end())
+                continue;
+            seen_in.push_back(t);
+            io += (double)P.tensors[t].bytes();
+        }
     for (int t : P.outputs) io += (double)P.tensors[t].bytes();
     C.bytes = io + wbytes;
     C.grid = grid;
@@ -1263,19 +1441,32 @@ bool make_chain(Plan &P, int bn) {
     C.flags_off = P.ws_bytes;
     C.flags_bytes = align_up(16 + 4 * (size_t)ncnt, 256);
     P.ws_bytes += C.flags_bytes;
-    P.launches.assign(1, C);
+    P.launches = quants;
+    P.launches.push_back(C);
     P.flops = C.flops;
     P.bytes = C.bytes;
+    for (const LaunchPlan &Q : quants) P.bytes += Q.bytes;
     return true;
 }
 
 byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
-    if (d && d->abi_version == BYOC_ABI_VERSION && (d->options & BYOC_OPT_REGION_KERNEL)) {
+    bool fp8 = false;
+    if (d && d->abi_version == BYOC_ABI_VERSION && d->tensors)
+        for (int i = 0; i < d->n_tensors; ++i) fp8 |= d->tensors[i].dtype == BYOC_E4M3;
+    if (d && d->abi_version == BYOC_ABI_VERSION && ((d->options & BYOC_OPT_REGION_KERNEL) || fp8)) {
         Plan C;
-        if (plan_region_impl(d, num_sms, C, 128) == BYOC_OK && make_chain(C, 128)) {
+        const byoc_status st = plan_region_impl(d, num_sms, C, 128);
+        if (st == BYOC_OK && make_chain(C, 128)) {
             P = std::move(C);
             return BYOC_OK;
         }
+        // FP8 layers run only in the region kernel
+        if (fp8)
+            return st != BYOC_OK ? st
+                                 : fail(BYOC_ERR_UNSUPPORTED,
+                                        "FP8 region: the region kernel takes 1 to %d conv2d / dense composites "
+                                        "(1x1 or k x k, C %% 128 == 0 on E4M3 inputs) after its Q nodes",
+                                        byoc::kChainMaxStages);
     }
     return plan_region_impl(d, num_sms, P, 0);
 }
@@ -1308,7 +1499,10 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
                                                                 : 2;
         r->pair_units[i] = gm && byoc::amode_pair(L.cfg.amode) ? 1 : 0;
         r->stages[i] = 1;
+        r->fp8[i] = L.kind == BYOC_LAUNCH_GEMM ? L.fp8 : 0;
         if (L.kind == BYOC_LAUNCH_CHAIN) {
+            r->fp8[i] = 0;
+            for (int k = 0; k < L.chain.n_stages; ++k) r->fp8[i] += L.chain.st[k].fp8;
             const byoc::ChainStage &s0 = L.chain.st[0];
             r->stages[i] = L.chain.n_stages;
             r->units[i] = L.chain.total_units;
@@ -1527,8 +1721,13 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
             byoc::ChainArgs &A = L.chain;
             for (int st = 0; st < A.n_stages; ++st) {
                 A.st[st].bias = reinterpret_cast<const float *>(h->d_const + L.cb_off[st]);
-                CUresult r = encode_2d(&h->cmaps[i].B[st], h->d_const + L.cw_off[st], (uint64_t)L.c_npad[st],
-                                       (uint64_t)L.c_kpack[st], (uint32_t)L.chain_bn, 64, 64);
+                A.st[st].dq = A.st[st].fp8 ? reinterpret_cast<const float *>(h->d_const + L.c_dq_off[st]) : nullptr;
+                CUresult r = A.st[st].fp8
+                                 ? encode_2d_u8(&h->cmaps[i].B[st], h->d_const + L.cw_off[st], (uint64_t)L.c_npad[st],
+                                                (uint64_t)L.c_kpack[st], (uint32_t)L.chain_bn, 128,
+                                                CU_TENSOR_MAP_SWIZZLE_128B)
+                                 : encode_2d(&h->cmaps[i].B[st], h->d_const + L.cw_off[st], (uint64_t)L.c_npad[st],
+                                             (uint64_t)L.c_kpack[st], (uint32_t)L.chain_bn, 64, 64);
                 if (r != CUDA_SUCCESS) {
                     byoc_release(h);
                     return fail(BYOC_ERR_CUDA, "launch %zu stage %d: cuTensorMapEncodeTiled(weights) = %d", i,
@@ -1663,7 +1862,8 @@ int g_chain_bad = 0;  // which consistency check failed (for the error message)
 bool chain_plan_ok(const Plan &P, const LaunchPlan &L) {
     const byoc::ChainArgs &A = L.chain;
     const int nt = (int)P.tensors.size();
-    if ((L.chain_bn != 128 && L.chain_bn != 256) || A.n_stages < 2 || A.n_stages > byoc::kChainMaxStages)
+    if ((L.chain_bn != 128 && L.chain_bn != 256) || A.n_stages < 1 || A.n_stages > byoc::kChainMaxStages ||
+        (A.n_stages == 1 && !A.st[0].fp8))
         { g_chain_bad = 1; return false; }
     int units = 0, ncnt = 0;
     for (int s = 0; s < A.n_stages; ++s) {
@@ -1674,10 +1874,14 @@ bool chain_plan_ok(const Plan &P, const LaunchPlan &L) {
         if (cs.num_tiles != (cs.M + byoc::kGemmBM - 1) / byoc::kGemmBM * cs.tiles_n || cs.num_tiles >= (1 << 24))
             { g_chain_bad = 14; return false; }
         if (cs.cbase != ncnt || cs.unit0 != units) { g_chain_bad = 15; return false; }
-        if (cs.num_kb < 1 || (size_t)cs.num_kb * 64 > (size_t)L.c_kpack[s]) { g_chain_bad = 16; return false; }
+        if (cs.num_kb < 1 || (size_t)cs.num_kb * (cs.fp8 ? 128 : 64) > (size_t)L.c_kpack[s]) { g_chain_bad = 16; return false; }
         if (P.tensors[L.cy[s]].elems() != (size_t)cs.M * cs.N) { g_chain_bad = 4; return false; }
-        if (L.cw_off[s] + (size_t)L.c_npad[s] * L.c_kpack[s] * 2 > P.blob.size() ||
-            L.cb_off[s] + (size_t)L.c_npad[s] * 4 > P.blob.size())
+        if ((P.tensors[L.cy[s]].dtype == BYOC_E4M3) != (cs.out8 != 0) ||
+            (P.tensors[L.cx[s]].dtype == BYOC_E4M3) != (cs.fp8 != 0))
+            { g_chain_bad = 21; return false; }
+        if (L.cw_off[s] + (size_t)L.c_npad[s] * L.c_kpack[s] * (cs.fp8 ? 1 : 2) > P.blob.size() ||
+            L.cb_off[s] + (size_t)L.c_npad[s] * 4 > P.blob.size() ||
+            (cs.fp8 && L.c_dq_off[s] + (size_t)L.c_npad[s] * 4 > P.blob.size()))
             { g_chain_bad = 5; return false; }
         units += cs.num_tiles;
         ncnt += (cs.M + byoc::kGemmBM - 1) / byoc::kGemmBM;
@@ -1794,7 +1998,7 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: workspace layout out of range");
     for (const LaunchPlan &L : P.launches) {
         if (L.kind != BYOC_LAUNCH_GEMM && L.kind != BYOC_LAUNCH_DEPTHWISE && L.kind != BYOC_LAUNCH_S2D &&
-            L.kind != BYOC_LAUNCH_DWPW && L.kind != BYOC_LAUNCH_CHAIN)
+            L.kind != BYOC_LAUNCH_DWPW && L.kind != BYOC_LAUNCH_CHAIN && L.kind != BYOC_LAUNCH_QUANT)
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: bad launch kind");
         if (L.kind == BYOC_LAUNCH_CHAIN && !chain_plan_ok(P, L))
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent region kernel (check %d)", g_chain_bad);
@@ -1983,10 +2187,13 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             for (int sg = 0; sg < a.n_stages; ++sg) {
                 const void *xa = h->ptrs[L.cx[sg]];
                 if (cp[sg] != xa) {
+                    const bool f8 = a.st[sg].fp8 != 0;
                     CUresult r = a.st[sg].mode == byoc::kChainIm2col
-                                     ? encode_im2col(&mp.A[sg], xa, L.cgeo[sg], 64)
-                                     : encode_2d(&mp.A[sg], xa, (uint64_t)L.caM[sg], (uint64_t)L.caK[sg],
-                                                 byoc::kGemmBM, 64, 64);
+                                     ? encode_im2col(&mp.A[sg], xa, L.cgeo[sg], 64, f8)
+                                     : f8 ? encode_2d_u8(&mp.A[sg], xa, (uint64_t)L.caM[sg], (uint64_t)L.caK[sg],
+                                                         byoc::kGemmBM, 128, CU_TENSOR_MAP_SWIZZLE_128B)
+                                          : encode_2d(&mp.A[sg], xa, (uint64_t)L.caM[sg], (uint64_t)L.caK[sg],
+                                                      byoc::kGemmBM, 64, 64);
                     if (r != CUDA_SUCCESS)
                         return fail(BYOC_ERR_CUDA, "launch %zu stage %d: encoding the A map failed (%d)", i, sg,
                                     (int)r);
@@ -1994,7 +2201,11 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                 }
                 void *ya = h->ptrs[L.cy[sg]];
                 if (cp[byoc::kChainMaxStages + sg] != ya) {
-                    CUresult r = encode_2d(&mp.O[sg], ya, (uint64_t)a.st[sg].M, (uint64_t)a.st[sg].N, 32, 32, 32);
+                    // bf16: 32 x 32 boxes, 64-byte swizzle; E4M3 codes: 32 x 32 bytes, unswizzled
+                    CUresult r = a.st[sg].out8
+                                     ? encode_2d_u8(&mp.O[sg], ya, (uint64_t)a.st[sg].M, (uint64_t)a.st[sg].N, 32, 32,
+                                                    CU_TENSOR_MAP_SWIZZLE_NONE)
+                                     : encode_2d(&mp.O[sg], ya, (uint64_t)a.st[sg].M, (uint64_t)a.st[sg].N, 32, 32, 32);
                     if (r != CUDA_SUCCESS)
                         return fail(BYOC_ERR_CUDA, "launch %zu stage %d: encoding the output map failed (%d)", i,
                                     sg, (int)r);
@@ -2005,6 +2216,10 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
             }
             a.trace = g_trace && g_trace_next < g_trace_cap ? g_trace + 2 * g_trace_next++ : nullptr;
             e = byoc::launch_chain(L.chain_bn, mp, a, L.grid, st);
+        } else if (L.kind == BYOC_LAUNCH_QUANT) {
+            e = byoc::launch_quantize_e4m3(static_cast<const __nv_bfloat16 *>(h->ptrs[L.x]),
+                                           static_cast<uint8_t *>(h->ptrs[L.y]), P.tensors[L.x].elems(), L.q_inv,
+                                           h->sms, st);
         } else if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             const void *xa = static_cast<const char *>(h->ptrs[L.x]) + L.x_off;
             if (h->tmA_ptr[i] != xa) {

@@ -160,8 +160,9 @@ class _Builder:
 
     def quantize(self, x, scale, dtype="e4m3", zero_point=0):
         """A Q node of Section 3.2 (scale S, zero point Z fixed at compile time)."""
+        # the scale as a float32 value: the compiled region carries it in fp32
         return self._add("qnn.quantize", [x], self.g.shape_of(x),
-                         dict(scale=float(scale), zero_point=int(zero_point), dtype=dtype))
+                         dict(scale=float(np.float32(scale)), zero_point=int(zero_point), dtype=dtype))
 
     def max_pool2d(self, x, k, stride, pad):
         N, H, W, C = self.g.shape_of(x)

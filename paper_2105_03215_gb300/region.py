@@ -26,6 +26,7 @@ _OP_KIND = {
     "nn.relu": abi.OP_RELU,
     "nn.gelu": abi.OP_GELU,
     "add": abi.OP_ADD,
+    "qnn.quantize": abi.OP_QUANTIZE,
 }
 
 OFFLOADABLE_OPS = frozenset(list(_OP_KIND) + ["clip"])
@@ -88,13 +89,15 @@ class Region:
         g = self.graph
         names = list(self.inputs) + [n.name for n in self.nodes]
         tid = {nm: i for i, nm in enumerate(names)}
+        by_name = {n.name for n in g.nodes}
         tensors = (abi.Tensor * len(names))()
         for i, nm in enumerate(names):
             shp = g.shape_of(nm)
             tensors[i].ndim = len(shp)
             for k, s in enumerate(shp):
                 tensors[i].shape[k] = int(s)
-            tensors[i].dtype = abi.BF16
+            src = g.node(nm) if nm in by_name else None
+            tensors[i].dtype = abi.E4M3 if src is not None and src.op == "qnn.quantize" else abi.BF16
             tensors[i].layout = abi.LAYOUT_NHWC if len(shp) == 4 else abi.LAYOUT_NC
         keep: list = [tensors]
         ops = (abi.Op * len(self.nodes))()
@@ -122,6 +125,11 @@ class Region:
                 consts = [n.consts["gamma"], n.consts["beta"], n.consts["moving_mean"],
                           n.consts["moving_var"]]
                 o.eps = float(n.attrs.get("epsilon", 1e-5))
+            elif n.op == "qnn.quantize":
+                if n.attrs.get("dtype", "e4m3") != "e4m3":
+                    raise abi.ByocError(abi.ERR_UNSUPPORTED, f"{n.name}: only E4M3 quantization runs here")
+                consts = [np.array([n.attrs["scale"]], np.float32),
+                          np.array([n.attrs.get("zero_point", 0)], np.float32)]
             else:
                 consts = []
             for k, c in enumerate(consts):

@@ -1,0 +1,115 @@
+"""Partial quantization (Section 3.2): regions with Q nodes run their
+convolutions / dense layers in FP8 (E4M3 codes on kind::f8f6f4 tensor cores,
+fp32 accumulation) in the region kernel, against the oracle's definition of
+the quantized chain (oracle/quant.py, oracle/graph.py)."""
+import numpy as np
+import pytest
+
+from oracle import graph as ograph
+from paper_2105_03215_gb300 import abi
+from paper_2105_03215_gb300 import inputs as I
+from paper_2105_03215_gb300 import region as R
+
+from .parity import assert_bit_exact, assert_close, oracle, run_region
+
+
+def _identity_fp8_conv(N=2, H=9, W=11, C=256, seed=5):
+    """FP8 1x1 conv with identity weights and a unit-scale batch norm: the
+    output is the dequantized input, code x S, rounded once to bf16."""
+    g, inp = I.fp8_conv(N=N, H=H, W=W, C=C, K=C, k=1, act="none", seed=seed)
+    conv, bn = g.nodes[1], g.nodes[2]
+    conv.consts["weight"] = np.eye(C, dtype=np.float32).reshape(C, C, 1, 1)
+    bn.consts.update(gamma=np.ones(C, np.float32), beta=np.zeros(C, np.float32),
+                     moving_mean=np.zeros(C, np.float32), moving_var=np.full(C, 1.0 - 1e-5, np.float32))
+    # a power-of-two scale: code x S is exact in fp32 and in bf16
+    g.nodes[0].attrs["scale"] = 1.0 / 32.0
+    rng = np.random.default_rng(seed)
+    # values over the whole E4M3 range of the scale, ties and saturation included
+    x = rng.standard_normal((N, H, W, C)).astype(np.float32) * np.float32(3.0)
+    x.reshape(-1)[:64] = np.float32(500.0 / 32.0)  # 500 / 32 quantizes to the saturated 448
+    inp["x"] = I.bf16_round(x)
+    return g, inp
+
+
+# ------------------------------------------------------------ plans (CPU)
+
+@pytest.mark.parametrize("make,stages", [(lambda: I.fp8_conv(N=1), 1), (lambda: I.fp8_dense(M=64), 1),
+                                         (lambda: I.fp8_bottleneck(N=2), 3)])
+def test_fp8_region_plans_a_quantize_launch_and_a_region_kernel(make, stages):
+    g, _ = make()
+    rep = R.whole_graph_region(g).plan(152)
+    kinds = [rep.kind[i] for i in range(rep.n_launches)]
+    assert kinds == [abi.LAUNCH_QUANT, abi.LAUNCH_CHAIN]
+    assert rep.stages[1] == stages and rep.fp8[1] == stages
+    blob = R.whole_graph_region(g).plan_serialized(152)
+    assert [R.load_plan_report(blob).kind[i] for i in range(2)] == kinds
+
+
+def test_fp8_regions_the_kernels_do_not_cover_are_rejected_on_the_host():
+    # a zero point on E4M3, and E4M3 codes read by an elementwise op
+    g, _ = I.fp8_conv(N=1, H=4, W=4, C=128, K=128)
+    g.nodes[0].attrs["zero_point"] = 3
+    with pytest.raises(abi.ByocError) as e:
+        R.whole_graph_region(g).plan(152)
+    assert e.value.status == abi.ERR_UNSUPPORTED
+    b = I._Builder("q_relu")
+    x = b.input("x", (1, 4, 4, 128))
+    y = b.relu(b.quantize(x, 0.1))
+    g2, _ = I._finish(b, [y], 1)
+    with pytest.raises(abi.ByocError) as e:
+        R.whole_graph_region(g2).plan(152)
+    assert e.value.status == abi.ERR_UNSUPPORTED
+    # FP8 on fewer than 128 channels per k-block
+    g3, _ = I.fp8_conv(N=1, H=4, W=4, C=64, K=64)
+    with pytest.raises(abi.ByocError):
+        R.whole_graph_region(g3).plan(152)
+
+
+# ------------------------------------------------------------ GPU parity
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("N,H,W,C", [(2, 9, 11, 256), (1, 7, 7, 128), (3, 14, 14, 512)])
+def test_fp8_identity_conv_reproduces_the_quantized_input_bit_for_bit(N, H, W, C):
+    g, inp = _identity_fp8_conv(N=N, H=H, W=W, C=C)
+    got, cr = run_region(R.whole_graph_region(g), inp)
+    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    assert_bit_exact(got[g.outputs[0]], ref, f"fp8 identity {N}x{H}x{W}x{C}")
+    cr.release()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("make", [
+    lambda: I.fp8_conv(N=2, H=14, W=14, C=256, K=256, k=3),
+    lambda: I.fp8_conv(N=3, H=9, W=10, C=128, K=96, k=1),
+    lambda: I.fp8_dense(M=200, D=768, F=1024),
+])
+def test_fp8_layer_matches_the_oracle(make):
+    g, inp = make()
+    got, cr = run_region(R.whole_graph_region(g), inp)
+    ref, sc = oracle(g, inp)
+    o = g.outputs[0]
+    assert_close(got[o], ref[o], sc[o], g.name)
+    cr.release()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("N", [2, 32])
+def test_fp8_bottleneck_matches_the_oracle(N):
+    # config 4 with Q nodes before each convolution: the intermediates t1, t2
+    # leave their epilogues as E4M3 codes (fused Q nodes)
+    g, inp = I.fp8_bottleneck(N=N)
+    got, cr = run_region(R.whole_graph_region(g), inp)
+    assert cr.n_launches == 2
+    ref, sc = oracle(g, inp)
+    o = g.outputs[0]
+    _, _, literal = assert_close(got[o], ref[o], sc[o], g.name)
+    # re-rounded codes rarely land on the other side of a rounding boundary:
+    # nearly every element also meets the stated bar alone
+    assert literal > 0.98, literal
+    # quantization error of the whole region against the bf16 model (reported)
+    gb, _ = I.resnet_bottleneck(N=N, seed=3)
+    full = ograph.evaluate(gb, inp)[gb.outputs[0]]
+    rel = np.linalg.norm(got[o] - full) / np.linalg.norm(full)
+    print(f"fp8 bottleneck N={N}: relative L2 error against the unquantized region {rel:.4f}")
+    assert rel < 0.1
+    cr.release()
