@@ -202,13 +202,148 @@ def time_region(cr, ins, outs, flush, reps=20):
     return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3  # seconds
 
 
+def time_region_stream(reg, make_inputs, out_shapes, per_call_bytes, flush, calls_min=24, max_sets=320, reps=5):
+    """Per-call device time of back-to-back calls of one region: one CUDA graph
+    of R calls rotating over S compiled handles (each with its own packed
+    weights and workspace), input sets and output sets, with S chosen so that
+    more than twice the L2 capacity of other data passes between two uses of
+    the same set -- inputs, weights and outputs come from / go to HBM, as in
+    a model's forward pass.  The graph is replayed between events (L2 flushed
+    before each replay) and the time divided by R, so the fixed cost of one
+    graph launch is spread over the R calls."""
+    import math
+
+    import torch
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    S = max(2, min(max_sets, math.ceil(2 * l2 / max(1, per_call_bytes)) + 1))
+    crs = [reg.compile() for _ in range(S)]
+    ins = [make_inputs() for _ in range(S)]
+    outs = [[torch.empty(sh, dtype=torch.bfloat16, device="cuda") for sh in out_shapes] for _ in range(S)]
+    R = S * math.ceil(calls_min / S)
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        for i in range(S):
+            crs[i].run(ins[i], outs[i], st)
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(graph, stream=st):
+        for r in range(R):
+            crs[r % S].run(ins[r % S], outs[r % S], st)
+    cur = torch.cuda.current_stream()
+    ts = []
+    for _ in range(reps):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(cur)
+        graph.replay()
+        b.record(cur)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b) * 1e-3 / R)
+    for c in crs:
+        c.check()
+    del graph
+    for c in crs:
+        c.release()
+    return statistics.median(ts), S, R
+
+
+def graph_floor(flush, reps=20):
+    """Event-timed replay of a graph holding one one-element kernel, L2
+    flushed before it: the fixed cost inside every single-call figure."""
+    import torch
+    x = torch.zeros(1, device="cuda")
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        x.add_(1)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=st):
+        x.add_(1)
+    cur = torch.cuda.current_stream()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(reps)]
+    for a, b in evs:
+        flush.zero_()
+        a.record(cur)
+        g.replay()
+        b.record(cur)
+    torch.cuda.synchronize()
+    return statistics.median(a.elapsed_time(b) for a, b in evs) * 1e-3
+
+
+def copy_reference(nbytes, flush):
+    """torch's device copy moving the same bytes (half read, half written):
+    single call as time_region times it, and back to back over buffers that
+    rotate through more than twice L2 -- what a plain copy reaches at this size."""
+    import math
+
+    import torch
+    nbytes = int(nbytes)
+    n = max(4096, nbytes // 4 // 4096 * 4096)  # bf16 elements per side (torch vectorizes whole multiples)
+    src = torch.empty(n, dtype=torch.bfloat16, device="cuda")
+    dst = torch.empty_like(src)
+
+    class _Copy:
+        def run(self, ins, outs, st=None):
+            outs[0].copy_(ins[0])
+
+        def check(self):
+            pass
+    single = time_region(_Copy(), [src], [dst], flush)
+    l2 = torch.cuda.get_device_properties(0).L2_cache_size
+    S = max(2, min(48, math.ceil(2 * l2 / nbytes) + 1))
+    srcs = [torch.empty_like(src) for _ in range(S)]
+    dsts = [torch.empty_like(src) for _ in range(S)]
+    R = S * math.ceil(24 / S)
+    st = torch.cuda.Stream()
+    with torch.cuda.stream(st):
+        dsts[0].copy_(srcs[0])
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=st):
+        for r in range(R):
+            dsts[r % S].copy_(srcs[r % S])
+    cur = torch.cuda.current_stream()
+    ts = []
+    for _ in range(5):
+        flush.zero_()
+        a = torch.cuda.Event(enable_timing=True)
+        b = torch.cuda.Event(enable_timing=True)
+        a.record(cur)
+        g.replay()
+        b.record(cur)
+        torch.cuda.synchronize()
+        ts.append(a.elapsed_time(b) * 1e-3 / R)
+    return single, statistics.median(ts)
+
+
+def _stream_fields(cr, t, S, R, peaks):
+    f = {"us_back_to_back": t * 1e6, "back_to_back_sets": S, "back_to_back_calls": R,
+         "gbps_back_to_back": cr.bytes / t / 1e9,
+         "hbm_frac_back_to_back": cr.bytes / t / 1e9 / peaks["hbm_gbs"]}
+    if cr.flops > 0:
+        f["tflops_back_to_back"] = cr.flops / t / 1e12
+        f["tensor_frac_back_to_back"] = cr.flops / t / 1e12 / peaks["bf16_tflops"]
+    return f
+
+
 def region_figures(flush, peaks):
-    """Configs 1-4 of the workload list, each as one region (cold L2)."""
+    """Configs 1-4 of the workload list, each as one region.  Per region:
+    ``us`` -- one call, L2 flushed before it, timed around a graph replay
+    (it includes the fixed cost of launching a graph, ``graph_replay_floor_us``);
+    ``us_back_to_back`` -- the per-call time of back-to-back calls whose data
+    and weights rotate through more than twice L2 (time_region_stream)."""
     import torch
     from paper_2105_03215_gb300 import abi
     from paper_2105_03215_gb300 import inputs as I
     from paper_2105_03215_gb300 import region as R
-    out = {}
+    out = {"graph_replay_floor_us": graph_floor(flush) * 1e6}
+
+    def stream(reg, g, cr):
+        def make():
+            return [torch.randn(g.shape_of(n), device="cuda").to(torch.bfloat16) for n in reg.inputs]
+        t, S, Rc = time_region_stream(reg, make, [g.shape_of(n) for n in reg.outputs], cr.bytes, flush)
+        return _stream_fields(cr, t, S, Rc, peaks)
     cases = {
         "conv3x3_bias_relu_1x56x56x64": I.conv_bias_relu(seed=0),
         "bert_ffn_1024x768x3072": I.bert_ffn(seed=1),
@@ -226,23 +361,27 @@ def region_figures(flush, peaks):
         out[name] = {"us": t * 1e6, "tflops": tf, "gbps": gb, "launches": cr.n_launches,
                      "tensor_frac_of_measured": tf / peaks["bf16_tflops"],
                      "hbm_frac_of_measured": gb / peaks["hbm_gbs"]}
+        out[name].update(stream(reg, g, cr))
         if name.startswith(("bert", "resnet50_bottleneck")):
             # the same region as one region kernel (every composite in one
             # persistent launch; intermediates through L2)
-            kcr = R.whole_graph_region(g, options=abi.OPT_REGION_KERNEL).compile()
+            kreg = R.whole_graph_region(g, options=abi.OPT_REGION_KERNEL)
+            kcr = kreg.compile()
             tk = time_region(kcr, ins, outs, flush)
             tfk = kcr.flops / tk / 1e12
             out[name + "_region_kernel"] = {
                 "us": tk * 1e6, "tflops": tfk, "gbps": kcr.bytes / tk / 1e9, "launches": kcr.n_launches,
                 "tensor_frac_of_measured": tfk / peaks["bf16_tflops"],
                 "hbm_frac_of_measured": kcr.bytes / tk / 1e9 / peaks["hbm_gbs"]}
+            out[name + "_region_kernel"].update(stream(kreg, g, kcr))
             kcr.release()
         if name.startswith("resnet50_bottleneck"):
             # partial quantization (Section 3.2): Q nodes before the three
             # convolutions, each computed in FP8 (E4M3, kind::f8f6f4); the
             # quantize launch of the input and one region kernel
             qg, _ = I.fp8_bottleneck(seed=3)
-            qcr = R.whole_graph_region(qg).compile()
+            qreg = R.whole_graph_region(qg)
+            qcr = qreg.compile()
             tq = time_region(qcr, ins, outs, flush)
             tfq = qcr.flops / tq / 1e12
             fp8_peak = 2.0 * peaks["bf16_tflops"]  # measured bf16 x the nominal fp8 / bf16 ratio (4.5 / 2.25)
@@ -251,13 +390,19 @@ def region_figures(flush, peaks):
                 "tensor_frac_of_fp8_peak": tfq / fp8_peak, "fp8_peak_tflops": fp8_peak,
                 "fp8_peak_source": "measured bf16 burst x 2 (nominal fp8 / bf16 ratio)",
                 "hbm_frac_of_measured": qcr.bytes / tq / 1e9 / peaks["hbm_gbs"]}
+            sq = stream(qreg, qg, qcr)
+            sq["tensor_frac_of_fp8_peak_back_to_back"] = qcr.flops / (sq["us_back_to_back"] * 1e-6) / 1e12 / fp8_peak
+            sq.pop("tensor_frac_back_to_back", None)
+            out[name + "_fp8"].update(sq)
             qcr.release()
         if name.startswith("mbv2"):
             # the same region as one fused kernel (depthwise output kept on chip)
-            fcr = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW).compile()
+            freg = R.whole_graph_region(g, options=abi.OPT_FUSE_DW_PW)
+            fcr = freg.compile()
             tfz = time_region(fcr, ins, outs, flush)
             out[name + "_fused"] = {"us": tfz * 1e6, "gbps": fcr.bytes / tfz / 1e9, "launches": fcr.n_launches,
                                     "hbm_frac_of_measured": fcr.bytes / tfz / 1e9 / peaks["hbm_gbs"]}
+            out[name + "_fused"].update(stream(freg, g, fcr))
             fcr.release()
             # the depthwise launch alone (the bandwidth-bound composite)
             dwg, dwi = I.mbv2_dw_pw(seed=2)
@@ -269,6 +414,11 @@ def region_figures(flush, peaks):
             out["depthwise3x3_bn_relu6_32x56x56x144"] = {
                 "us": td * 1e6, "gbps": dcr.bytes / td / 1e9,
                 "hbm_frac_of_measured": dcr.bytes / td / 1e9 / peaks["hbm_gbs"]}
+            out["depthwise3x3_bn_relu6_32x56x56x144"].update(stream(dreg, dwg, dcr))
+            # what torch's own device copy of the same bytes reaches, both ways
+            c1, cs = copy_reference(dcr.bytes, flush)
+            out["depthwise3x3_bn_relu6_32x56x56x144"].update(
+                {"same_bytes_copy_us": c1 * 1e6, "same_bytes_copy_us_back_to_back": cs * 1e6})
             dcr.release()
         cr.release()
     # MobileNetV2 1.0 end to end (53 regions, global average pool on the host):

@@ -153,6 +153,16 @@ typedef struct {
  *     the earlier composites they read are done (no launch boundary between
  *     composites).  Regions that do not qualify get the per-composite plan. */
 #define BYOC_OPT_REGION_KERNEL 0x2u
+/*   BYOC_OPT_MULTICAST: a GEMM launch whose weights are streamed through its
+ *     ring (tile, im2col or ringed slab mode, no split-K, at least two
+ *     m-tiles) runs in clusters of two CTAs that take adjacent m-tiles of one
+ *     column tile together and share each weight tile by TMA multicast,
+ *     halving the weight bytes each SM reads from L2.  Off by default:
+ *     measured on GB300 it is slower on every ResNet-50 / BERT layer here
+ *     (the tensor cores' shared-memory operand reads, not L2, bound these
+ *     layers, and the CTA pairs wait for each other at every ring stage).
+ *     Results are bit-identical either way. */
+#define BYOC_OPT_MULTICAST 0x4u
 
 /* Figures describing a compiled region. */
 typedef struct {

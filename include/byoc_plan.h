@@ -53,6 +53,8 @@ typedef struct {
                                                    describe the first), else 1 */
     int32_t units[BYOC_PLAN_MAX_LAUNCHES];      /* region kernel: output tiles over all its composites */
     int32_t fp8[BYOC_PLAN_MAX_LAUNCHES];        /* region kernel: composites computed in FP8 */
+    int32_t multicast[BYOC_PLAN_MAX_LAUNCHES];  /* GEMM: 1 if clusters of two CTAs share each
+                                                   weight tile by TMA multicast (grid even) */
     double flops;
     double bytes;
     size_t const_bytes;

@@ -16,6 +16,7 @@ ABI_VERSION = 2
 # byoc_region_desc.options
 OPT_FUSE_DW_PW = 0x1
 OPT_REGION_KERNEL = 0x2
+OPT_MULTICAST = 0x4
 
 # byoc_status
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)
@@ -70,7 +71,7 @@ class PlanReport(ctypes.Structure):
                 ("tile_n", c_int32 * _L), ("tile_k", c_int32 * _L), ("im2col", c_int32 * _L),
                 ("grid", c_int32 * _L), ("resident_b", c_int32 * _L), ("slab_slots", c_int32 * _L),
                 ("splits", c_int32 * _L), ("pair_units", c_int32 * _L), ("stages", c_int32 * _L),
-                ("units", c_int32 * _L), ("fp8", c_int32 * _L),
+                ("units", c_int32 * _L), ("fp8", c_int32 * _L), ("multicast", c_int32 * _L),
                 ("flops", c_double), ("bytes", c_double),
                 ("const_bytes", c_size_t), ("workspace_bytes", c_size_t)]
 

@@ -37,12 +37,24 @@
 //   warp 10    producer of the epilogue operands: per tile, the tile's bias
 //              slice (bulk copy) and, when the region adds a residual, the
 //              128 x BN residual tile (TMA) into a ring of OPB buffers.
+//
+// Cluster multicast (MC, on request: BYOC_OPT_MULTICAST): the kernel runs in
+// clusters of two CTAs that take
+// the m-tiles 2i and 2i + 1 of the same column tile together, k-block by
+// k-block.  Both need the same weight tile, so each CTA loads half of its
+// rows and multicasts them to both; a ring stage is refilled once both CTAs'
+// MMAs have read it (each MMA commit arrives on the stage's empty barrier in
+// both CTAs).  This halves the weight bytes each SM pulls from L2 -- the
+// operand traffic that bounds the layers whose weights are re-read by every
+// m-tile.  With an odd number of m-tiles the last cluster's second CTA runs a
+// phantom m-tile past the end: its loads fall outside the tensors and read
+// zeros, its stores are clipped or skipped.
 #include "internal.h"
 #include "ptx.cuh"
 
 namespace byoc {
 
-template <int BN, int BK, int AMODE, bool RES>
+template <int BN, int BK, int AMODE, bool RES, bool MC>
 struct GemmShape {
     static constexpr int BM = kGemmBM;
     static constexpr bool SLAB = amode_slab(AMODE);
@@ -100,6 +112,10 @@ struct GemmShape {
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
     static_assert(!(RES && SLAB), "slab tiles skip pad columns; no residual tile");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
+    static_assert(!MC || (!WRES && !PAIR && AMODE != kAModeTileSplit),
+                  "multicast: weights streamed through the ring, one tile per unit");
+    static constexpr int B_HALF = B_BYTES / 2;  // multicast: the rows one CTA loads
+    static_assert(!MC || B_HALF % 1024 == 0, "a multicast half keeps the swizzle's 1 KB alignment");
 };
 
 // Slab modes: image, first output row and tile count (halves) of m-unit mt.
@@ -134,7 +150,7 @@ __device__ __forceinline__ float apply_act(float v, int act) {
     }
 }
 
-template <int BN, int BK, int AMODE, bool RES>
+template <int BN, int BK, int AMODE, bool RES, bool MC>
 // 168 registers: 11 warps put three on some SM sub-partitions, and three
 // warps x 32 lanes x 168 fit a sub-partition's 16384 registers.
 __global__ void __maxnreg__(168)
@@ -142,7 +158,7 @@ __global__ void __maxnreg__(168)
                         const __grid_constant__ CUtensorMap tmB,
                         const __grid_constant__ CUtensorMap tmR,
                         const __grid_constant__ CUtensorMap tmO, const GemmArgs a) {
-    using S = GemmShape<BN, BK, AMODE, RES>;
+    using S = GemmShape<BN, BK, AMODE, RES, MC>;
     constexpr bool PAIR = S::PAIR;
     // The two epilogue warp groups take alternate tiles (all chunks each) for
     // narrow tiles, and for launches of one column tile whose tiles hold an
@@ -160,6 +176,22 @@ __global__ void __maxnreg__(168)
     constexpr bool SPLITK = AMODE == kAModeTileSplit;
     const int SPL = SPLITK ? a.splits : 1;
     const int num_units = a.num_tiles * SPL;
+    // The loop over work units, the same in every role: unit u_first,
+    // u_first + u_step, ... below num_loop.  MC: a unit is the pair of
+    // m-tiles (2i, 2i + 1) of one column tile, this CTA taking m-tile
+    // 2i + crank; tile_of() gives the tile (split-K: the unit's tile).
+    const int crank = MC ? (int)cluster_ctarank() : 0;
+    const int num_loop = MC ? ((a.num_tiles / a.tiles_n + 1) >> 1) * a.tiles_n : num_units;
+    const int u_first = MC ? (int)(blockIdx.x >> 1) : (int)blockIdx.x;
+    const int u_step = MC ? (int)(gridDim.x >> 1) : (int)gridDim.x;
+    auto tile_of = [&](int u) -> int {
+        if constexpr (MC) {
+            const int mp = u / a.tiles_n;
+            return (2 * mp + crank) * a.tiles_n + (u - mp * a.tiles_n);
+        } else {
+            return u / SPL;
+        }
+    };
     extern __shared__ __align__(1024) uint8_t smem_raw[];
     const uint32_t raw = smem_u32(smem_raw);
     const uint32_t base = (raw + 1023u) & ~1023u;
@@ -190,7 +222,7 @@ __global__ void __maxnreg__(168)
     if (threadIdx.x == 0) {
         for (int s = 0; s < S::STAGES; ++s) {
             mbar_init(bars + 8u * s, 1);                  // full[s]: producer + TMA bytes
-            mbar_init(bars + 8u * (S::STAGES + s), 1);    // empty[s]: MMA commit
+            mbar_init(bars + 8u * (S::STAGES + s), MC ? 2 : 1);  // empty[s]: MMA commit (MC: both CTAs')
         }
         for (int b = 0; b < 2; ++b) {
             mbar_init(tfull + 8u * b, 1);                 // MMA commit
@@ -221,21 +253,32 @@ __global__ void __maxnreg__(168)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    if constexpr (MC) cluster_sync();  // both CTAs' barriers initialised
     const uint32_t tmem_base = *tmem_slot;
     // Set-up done: the next kernel may be scheduled; global memory is touched
     // only after the previous kernel has completed -- except for the packed
     // weights, constant for the handle's lifetime: the operand warp
-    // prefetches this CTA's first tile's weight rows into L2, and the
+    // prefetches its share of its first tile's weight rows into L2, and the
     // producer loads the first ring stages' weights (resident-weight mode:
     // all of them) into shared memory, while the previous kernel finishes;
     // the producer waits for it only before its first activation load.
     pdl_launch_dependents();
-    if (!SPLITK && warp == kGemmOperandWarp && a.w != nullptr && (int)blockIdx.x < a.num_tiles) {
+    if (!SPLITK && warp == kGemmOperandWarp && a.w != nullptr && u_first < num_loop) {
         if (elect_one()) {
+            // The CTAs whose first unit is in column tile j (units j,
+            // j + tiles_n, ...) share its weight rows (MC: this CTA's half of
+            // them): each prefetches its own part, so L2 sees every byte
+            // requested once.
+            constexpr int PF_ROWS = MC ? BN / 2 : BN;
             const size_t row_bytes = (size_t)a.k_pack * 2;
-            const uint8_t *src =
-                static_cast<const uint8_t *>(a.w) + (size_t)((int)blockIdx.x % a.tiles_n) * BN * row_bytes;
-            const size_t bytes = (size_t)BN * row_bytes;
+            const int j = u_first % a.tiles_n, q = u_first / a.tiles_n;
+            const int users = (min(u_step, num_loop) - 1 - j) / a.tiles_n + 1;
+            const size_t slice = (size_t)PF_ROWS * row_bytes;
+            const size_t part = (slice / (size_t)users + 15) / 16 * 16;
+            const size_t lo = min(slice, (size_t)q * part);
+            const uint8_t *src = static_cast<const uint8_t *>(a.w) +
+                                 ((size_t)j * BN + (size_t)crank * PF_ROWS) * row_bytes + lo;
+            const size_t bytes = min(slice, lo + part) - lo;
             for (size_t off = 0; off < bytes; off += 32768)
                 bulk_prefetch_l2(src + off, (uint32_t)(bytes - off < 32768 ? bytes - off : 32768));
         }
@@ -276,6 +319,15 @@ __global__ void __maxnreg__(168)
             };
             int ss = 0;        // resident weights: slab slot of slab sl, and its phase
             uint32_t sph = 0;
+            // one weight tile (BN rows at n0, k-block column kx) into ring slot
+            // dst; MC: this CTA's half of the rows, to both CTAs
+            auto load_b = [&](uint32_t dst, uint32_t bar, int kx, int n0) {
+                if constexpr (MC)
+                    tma_load_2d_mc(dst + (uint32_t)(crank * S::B_HALF), &tmB, bar, kx, n0 + crank * (BN / 2),
+                                   (uint16_t)0x3);
+                else
+                    tma_load_2d(dst, &tmB, bar, kx, n0);
+            };
             if constexpr (S::WRES) {
                 // the whole weight matrix once, on ring stage 0
                 if (claim((uint32_t)(a.num_kb * S::B_BYTES))) {
@@ -293,9 +345,9 @@ __global__ void __maxnreg__(168)
             // ~2 us on the ResNet-50 step, so that mode waits first)
             int pre = 0;
             if constexpr (!S::SLAB) {
-                if ((int)blockIdx.x < num_units) {
-                    const int u0 = blockIdx.x;
-                    const int t0 = u0 / SPL, sp0 = u0 - (u0 / SPL) * SPL;
+                if (u_first < num_loop) {
+                    const int t0 = tile_of(u_first);
+                    const int sp0 = SPLITK ? u_first - t0 * SPL : 0;
                     const int n00 = (t0 % a.tiles_n) * BN;
                     const int lo = SPLITK ? sp0 * a.num_kb / SPL : 0;
                     const int hi = SPLITK ? (sp0 + 1) * a.num_kb / SPL : a.num_kb;
@@ -304,15 +356,14 @@ __global__ void __maxnreg__(168)
                         // fresh ring: stage pre is free; the full barrier expects A and B
                         mbar_arrive_expect_tx(bars + 8u * pre, (uint32_t)(gn * S::STAGE_BYTES));
                         for (int g = 0; g < gn; ++g)
-                            tma_load_2d(sB + (pre * G + g) * S::B_BYTES, &tmB, bars + 8u * pre, (kb + g) * BK,
-                                        n00);
+                            load_b(sB + (pre * G + g) * S::B_BYTES, bars + 8u * pre, (kb + g) * BK, n00);
                     }
                 }
             }
             pdl_wait();
-            for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x) {
-                const int tile = unit / SPL;
-                const int sp = unit - tile * SPL;
+            for (int unit = u_first; ok && unit < num_loop; unit += u_step) {
+                const int tile = tile_of(unit);
+                const int sp = SPLITK ? unit - tile * SPL : 0;
                 const int mt = tile / a.tiles_n;
                 const int n0 = (tile % a.tiles_n) * BN;
                 if constexpr (S::WRES) {
@@ -358,8 +409,8 @@ __global__ void __maxnreg__(168)
                                 break;
                             }
                             for (int g = 0; g < gn; ++g)
-                                tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, bars + 8u * stage,
-                                            (kb + g * a.chunks) * BK, n0);
+                                load_b(sB + (slot0 + g) * S::B_BYTES, bars + 8u * stage, (kb + g * a.chunks) * BK,
+                                       n0);
                             kb += gn * a.chunks;
                             advance();
                         }
@@ -404,8 +455,7 @@ __global__ void __maxnreg__(168)
                             } else {
                                 tma_load_2d(dA, &tmA, full, (kb + g) * BK, m0);
                             }
-                            if (!preloaded)
-                                tma_load_2d(sB + (slot0 + g) * S::B_BYTES, &tmB, full, (kb + g) * BK, n0);
+                            if (!preloaded) load_b(sB + (slot0 + g) * S::B_BYTES, full, (kb + g) * BK, n0);
                         }
                         advance();
                     }
@@ -425,8 +475,8 @@ __global__ void __maxnreg__(168)
         if (elect_one()) {
             // ------------------------------------------------ epilogue-operand producer
             int t = 0;
-            for (int unit = blockIdx.x; unit < num_units; unit += gridDim.x, ++t) {
-                const int tile = unit / SPL;
+            for (int unit = u_first; unit < num_loop; unit += u_step, ++t) {
+                const int tile = tile_of(unit);
                 const int ob = t % S::OPB;
                 const uint32_t oph = (uint32_t)(t / S::OPB) & 1u;
                 if (!mbar_wait(oempty + 8u * ob, oph ^ 1u, abort_flag, a.err, kErrTimeoutProducer))
@@ -493,8 +543,15 @@ __global__ void __maxnreg__(168)
                     phase ^= 1u;
                 }
             };
-            for (int unit = blockIdx.x; ok && unit < num_units; unit += gridDim.x, ++t) {
-                const int sp = unit - (unit / SPL) * SPL;
+            // a ring stage's MMAs are done (MC: in both CTAs' empty barriers)
+            auto free_stage = [&](int st) {
+                if constexpr (MC)
+                    mma_commit_mc(bars + 8u * (S::STAGES + st), (uint16_t)0x3);
+                else
+                    mma_commit(bars + 8u * (S::STAGES + st));
+            };
+            for (int unit = u_first; ok && unit < num_loop; unit += u_step, ++t) {
+                const int sp = SPLITK ? unit - (unit / SPL) * SPL : 0;
                 const int buf = t & 1;
                 const uint32_t aph = (uint32_t)(t >> 1) & 1u;
                 if (!wait(tempty + 8u * buf, aph ^ 1u)) {
@@ -574,7 +631,7 @@ __global__ void __maxnreg__(168)
                                     rpos += (uint32_t)a.wp;
                                 }
                             }
-                            mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
+                            free_stage(stage);
                             advance();
                         }
                         if (!ok) break;
@@ -600,7 +657,7 @@ __global__ void __maxnreg__(168)
                                             acc | (uint32_t)k);
                             acc = 1u;
                         }
-                        mma_commit(bars + 8u * (S::STAGES + stage));  // frees the stage
+                        free_stage(stage);
                         advance();
                     }
                 }
@@ -636,9 +693,9 @@ __global__ void __maxnreg__(168)
         const int t_first = alt ? grp : 0, t_step = alt ? 2 : 1;
         const int c_first = alt || PAIR ? 0 : grp, c_step = alt || PAIR ? 1 : 2;
         const int half = PAIR ? grp : 0;
-        for (int unit = blockIdx.x + t_first * (int)gridDim.x, t = t_first; unit < num_units;
-             unit += t_step * (int)gridDim.x, t += t_step) {
-            const int tile = unit / SPL;
+        for (int unit = u_first + t_first * u_step, t = t_first; unit < num_loop;
+             unit += t_step * u_step, t += t_step) {
+            const int tile = tile_of(unit);
             const int buf = t & 1;
             const uint32_t aph = (uint32_t)(t >> 1) & 1u;
             if (!mbar_wait(tfull + 8u * buf, aph, abort_flag, a.err, kErrTimeoutEpilogue)) break;
@@ -691,7 +748,7 @@ __global__ void __maxnreg__(168)
             // warp's slot; the split that completes the count sums all partials
             // in split order (the same bits whichever split finishes last) and
             // runs the epilogue.  No split waits for another.
-            const int sp = unit - tile * SPL;
+            const int sp = SPLITK ? unit - tile * SPL : 0;
             // Partials are laid out the way the warp reads TMEM, not as the
             // output matrix: per (tile, warp slot, chunk) 32 x 32 fp32 with
             // the 16-byte piece q of lane l at (q * 32 + l) * 16 bytes, so
@@ -732,7 +789,6 @@ __global__ void __maxnreg__(168)
                 }
                 __threadfence();  // the other splits' partials are read after the count
             }
-#pragma unroll 1
             // chunks holding output columns: the 32-column chunks of a ragged
             // last column tile that lie wholly past N are neither read nor
             // stored (split-K partials cover every chunk)
@@ -742,6 +798,7 @@ __global__ void __maxnreg__(168)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(tempty + 8u * buf);
             }
+#pragma unroll 1
             for (int ci = c_first, kk = 0; ci < nch; ci += c_step, ++kk) {
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
@@ -842,7 +899,8 @@ __global__ void __maxnreg__(168)
                     fence_proxy_async_smem();
                     __syncwarp();
                     if (lane == 0) {
-                        tma_store_2d(&tmO, stg, col0, mt * S::BM + quarter * 32);
+                        // (a box wholly past M -- the ragged or phantom m-tile's -- is skipped)
+                        if (mt * S::BM + quarter * 32 < a.M) tma_store_2d(&tmO, stg, col0, mt * S::BM + quarter * 32);
                         bulk_commit_group();
                     }
                     if (S::EPI_BUFS == 2) sb ^= 1;
@@ -879,6 +937,9 @@ __global__ void __maxnreg__(168)
     __syncwarp();
     tc_fence_before();
     __syncthreads();
+    // MC: the peer's multicast copies into this CTA and its MMA commits on
+    // this CTA's barriers are complete once it has passed its own waits
+    if constexpr (MC) cluster_sync();
     if (a.trace != nullptr && threadIdx.x == 0) atomicMax(a.trace + 1, globaltimer_ns());
     if (warp == 1) {
         tc_fence_after();
@@ -888,63 +949,78 @@ __global__ void __maxnreg__(168)
 
 // ---------------------------------------------------------------- dispatch
 
-template <int BN, int BK, int AMODE, bool RES>
+template <int BN, int BK, int AMODE, bool RES, bool MC>
 static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, const CUtensorMap &tmR,
                             const CUtensorMap &tmO, const GemmArgs &a, int grid, cudaStream_t st) {
-    using S = GemmShape<BN, BK, AMODE, RES>;
-    return launch_pdl(gemm_tcgen05_kernel<BN, BK, AMODE, RES>, dim3(grid), dim3(kGemmThreads),
-                      (size_t)S::SMEM_BYTES, st, tmA, tmB, tmR, tmO, a);
+    using S = GemmShape<BN, BK, AMODE, RES, MC>;
+    return launch_pdl_cluster(gemm_tcgen05_kernel<BN, BK, AMODE, RES, MC>, dim3(grid), dim3(kGemmThreads),
+                      (size_t)S::SMEM_BYTES, st, MC ? 2 : 1, tmA, tmB, tmR, tmO, a);
 }
 
-template <int BN, int BK, int AMODE, bool RES>
+template <int BN, int BK, int AMODE, bool RES, bool MC>
 static cudaError_t prepare_t() {
-    using S = GemmShape<BN, BK, AMODE, RES>;
-    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, AMODE, RES>,
+    using S = GemmShape<BN, BK, AMODE, RES, MC>;
+    return cudaFuncSetAttribute(gemm_tcgen05_kernel<BN, BK, AMODE, RES, MC>,
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, S::SMEM_BYTES);
 }
 
-// The instantiated (BN, BK, A mode, residual) combinations.
-#define BYOC_GEMM_CONFIGS(X)          \
-    X(32, 64, kAModeTile, false)      \
-    X(64, 64, kAModeTile, false)      \
-    X(128, 64, kAModeTile, false)     \
-    X(256, 64, kAModeTile, false)     \
-    X(64, 64, kAModeTile, true)       \
-    X(32, 16, kAModeTile, false)      \
-    X(64, 16, kAModeTile, false)      \
-    X(128, 16, kAModeTile, false)     \
-    X(32, 32, kAModeTile, false)      \
-    X(64, 32, kAModeTile, false)      \
-    X(128, 32, kAModeTile, false)     \
-    X(128, 64, kAModeTile, true)      \
-    X(32, 64, kAModeIm2col, false)    \
-    X(64, 64, kAModeIm2col, false)    \
-    X(128, 64, kAModeIm2col, false)   \
-    X(256, 64, kAModeIm2col, false)   \
-    X(64, 64, kAModeIm2col, true)     \
-    X(128, 64, kAModeIm2col, true)    \
-    X(64, 16, kAModeIm2col, false)    \
-    X(64, 32, kAModeIm2col, false)    \
-    X(128, 32, kAModeIm2col, false)   \
-    X(64, 64, kAModeSlab, false)      \
-    X(128, 64, kAModeSlab, false)     \
-    X(256, 64, kAModeSlab, false)     \
-    X(64, 16, kAModeSlab, false)      \
-    X(64, 32, kAModeSlab, false)      \
-    X(64, 64, kAModeTileSplit, false) \
-    X(128, 64, kAModeTileSplit, false) \
-    X(256, 64, kAModeTileSplit, false) \
-    X(64, 64, kAModeSlabRes, false)   \
-    X(128, 64, kAModeSlabRes, false)  \
-    X(64, 16, kAModeSlabRes, false)   \
-    X(64, 32, kAModeSlabRes, false)   \
-    X(64, 64, kAModeSlabRes2, false)  \
-    X(128, 64, kAModeSlabRes2, false) \
-    X(64, 32, kAModeSlabRes2, false)
+// The instantiated (BN, BK, A mode, residual, cluster multicast) combinations.
+#define BYOC_GEMM_CONFIGS(X)                 \
+    X(32, 64, kAModeTile, false, false)      \
+    X(64, 64, kAModeTile, false, false)      \
+    X(128, 64, kAModeTile, false, false)     \
+    X(256, 64, kAModeTile, false, false)     \
+    X(64, 64, kAModeTile, true, false)       \
+    X(32, 16, kAModeTile, false, false)      \
+    X(64, 16, kAModeTile, false, false)      \
+    X(128, 16, kAModeTile, false, false)     \
+    X(32, 32, kAModeTile, false, false)      \
+    X(64, 32, kAModeTile, false, false)      \
+    X(128, 32, kAModeTile, false, false)     \
+    X(128, 64, kAModeTile, true, false)      \
+    X(32, 64, kAModeIm2col, false, false)    \
+    X(64, 64, kAModeIm2col, false, false)    \
+    X(128, 64, kAModeIm2col, false, false)   \
+    X(256, 64, kAModeIm2col, false, false)   \
+    X(64, 64, kAModeIm2col, true, false)     \
+    X(128, 64, kAModeIm2col, true, false)    \
+    X(64, 16, kAModeIm2col, false, false)    \
+    X(64, 32, kAModeIm2col, false, false)    \
+    X(128, 32, kAModeIm2col, false, false)   \
+    X(64, 64, kAModeSlab, false, false)      \
+    X(128, 64, kAModeSlab, false, false)     \
+    X(256, 64, kAModeSlab, false, false)     \
+    X(64, 16, kAModeSlab, false, false)      \
+    X(64, 32, kAModeSlab, false, false)      \
+    X(64, 64, kAModeTileSplit, false, false) \
+    X(128, 64, kAModeTileSplit, false, false) \
+    X(256, 64, kAModeTileSplit, false, false) \
+    X(64, 64, kAModeSlabRes, false, false)   \
+    X(128, 64, kAModeSlabRes, false, false)  \
+    X(64, 16, kAModeSlabRes, false, false)   \
+    X(64, 32, kAModeSlabRes, false, false)   \
+    X(64, 64, kAModeSlabRes2, false, false)  \
+    X(128, 64, kAModeSlabRes2, false, false) \
+    X(64, 32, kAModeSlabRes2, false, false)  \
+    X(64, 64, kAModeTile, false, true)       \
+    X(128, 64, kAModeTile, false, true)      \
+    X(256, 64, kAModeTile, false, true)      \
+    X(64, 64, kAModeTile, true, true)        \
+    X(128, 64, kAModeTile, true, true)       \
+    X(64, 64, kAModeIm2col, false, true)     \
+    X(128, 64, kAModeIm2col, false, true)    \
+    X(256, 64, kAModeIm2col, false, true)    \
+    X(128, 64, kAModeIm2col, true, true)     \
+    X(64, 64, kAModeSlab, false, true)       \
+    X(128, 64, kAModeSlab, false, true)      \
+    X(256, 64, kAModeSlab, false, true)
+
+#define BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_) \
+    ((c).bn == BN_ && (c).bk == BK_ && (c).amode == AM_ && (c).res == RES_ && (c).mc == MC_)
 
 bool gemm_config_supported(const GemmConfig &c) {
-#define X(BN_, BK_, AM_, RES_) \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) return true;
+#define X(BN_, BK_, AM_, RES_, MC_) \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) return true;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return false;
@@ -952,10 +1028,10 @@ bool gemm_config_supported(const GemmConfig &c) {
 
 static void slab_pool_shape(const GemmConfig &c, int &pool, int &bbytes) {
     pool = bbytes = 0;
-#define X(BN_, BK_, AM_, RES_)                                            \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) { \
-        pool = GemmShape<BN_, BK_, AM_, RES_>::POOL_BYTES;                \
-        bbytes = GemmShape<BN_, BK_, AM_, RES_>::B_BYTES;                 \
+#define X(BN_, BK_, AM_, RES_, MC_)                                  \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) {              \
+        pool = GemmShape<BN_, BK_, AM_, RES_, MC_>::POOL_BYTES;      \
+        bbytes = GemmShape<BN_, BK_, AM_, RES_, MC_>::B_BYTES;       \
     }
     BYOC_GEMM_CONFIGS(X)
 #undef X
@@ -980,27 +1056,27 @@ void gemm_slab_pool(const GemmConfig &c, GemmArgs &a) {
 }
 
 size_t gemm_smem_bytes(const GemmConfig &c) {
-#define X(BN_, BK_, AM_, RES_)                                             \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
-        return (size_t)GemmShape<BN_, BK_, AM_, RES_>::SMEM_BYTES;
+#define X(BN_, BK_, AM_, RES_, MC_)                     \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) \
+        return (size_t)GemmShape<BN_, BK_, AM_, RES_, MC_>::SMEM_BYTES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 int gemm_stages(const GemmConfig &c) {
-#define X(BN_, BK_, AM_, RES_)                                             \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
-        return GemmShape<BN_, BK_, AM_, RES_>::STAGES;
+#define X(BN_, BK_, AM_, RES_, MC_)                     \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) \
+        return GemmShape<BN_, BK_, AM_, RES_, MC_>::STAGES;
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return 0;
 }
 
 cudaError_t gemm_prepare(const GemmConfig &c) {
-#define X(BN_, BK_, AM_, RES_)                                             \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
-        return prepare_t<BN_, BK_, AM_, RES_>();
+#define X(BN_, BK_, AM_, RES_, MC_)                     \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) \
+        return prepare_t<BN_, BK_, AM_, RES_, MC_>();
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;
@@ -1009,9 +1085,10 @@ cudaError_t gemm_prepare(const GemmConfig &c) {
 cudaError_t launch_gemm(const GemmConfig &c, const CUtensorMap &tmA, const CUtensorMap &tmB,
                         const CUtensorMap &tmR, const CUtensorMap &tmO, const GemmArgs &a, int grid,
                         cudaStream_t st) {
-#define X(BN_, BK_, AM_, RES_)                                             \
-    if (c.bn == BN_ && c.bk == BK_ && c.amode == AM_ && c.res == RES_) \
-        return launch_t<BN_, BK_, AM_, RES_>(tmA, tmB, tmR, tmO, a, grid, st);
+    if (c.mc && (grid < 2 || grid % 2)) return cudaErrorInvalidValue;  // whole clusters of two
+#define X(BN_, BK_, AM_, RES_, MC_)                     \
+    if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) \
+        return launch_t<BN_, BK_, AM_, RES_, MC_>(tmA, tmB, tmR, tmO, a, grid, st);
     BYOC_GEMM_CONFIGS(X)
 #undef X
     return cudaErrorInvalidValue;

@@ -20,19 +20,31 @@ enum Act : int { kActNone = 0, kActRelu = 1, kActRelu6 = 2, kActGelu = 3 };
 // access, so only set-up work (barrier init, TMEM allocation, descriptor
 // prefetch) overlaps the previous kernel's tail.
 template <typename... KArgs, typename... Args>
-inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                              cudaStream_t st, Args... args) {
+inline cudaError_t launch_pdl_cluster(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                      cudaStream_t st, int cluster_x, Args... args) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = grid;
     cfg.blockDim = block;
     cfg.dynamicSmemBytes = smem;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
+    if (cluster_x > 1) {  // thread-block clusters of cluster_x CTAs along x
+        attr[1].id = cudaLaunchAttributeClusterDimension;
+        attr[1].val.clusterDim.x = (unsigned)cluster_x;
+        attr[1].val.clusterDim.y = 1;
+        attr[1].val.clusterDim.z = 1;
+        cfg.numAttrs = 2;
+    }
     return cudaLaunchKernelEx(&cfg, kernel, args...);
+}
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t st, Args... args) {
+    return launch_pdl_cluster(kernel, grid, block, smem, st, 1, args...);
 }
 
 // Implicit-GEMM problem: out[M, N] = act(A[M, K] . B[N, K]^T + bias [+ residual]).
@@ -118,6 +130,10 @@ struct GemmConfig {
     int bk;      // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
     int amode;   // AMode
     bool res;    // epilogue adds a residual tile (bn 64 or 128)
+    // clusters of two CTAs sharing each weight tile by TMA multicast (tile,
+    // im2col and ringed slab modes); the launch grid is even and the weight
+    // map's box is bn / 2 rows
+    bool mc = false;
 };
 
 // Largest slab (one channel chunk) the slab mode holds, per buffer; a pair

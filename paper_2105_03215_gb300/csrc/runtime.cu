@@ -1035,6 +1035,15 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
             if (byoc::gemm_config_supported(rc) && byoc::gemm_slab_res_fits(rc, taps * chunks, sgeo.bytes))
                 L.cfg = rc;
         }
+        // Cluster multicast of the weight tiles, on request (tile, im2col and
+        // ringed slab modes without split-K; at least two m-tiles to pair)
+        if (chain_bn == 0 && (d->options & BYOC_OPT_MULTICAST) && tiles_m >= 2 && P.num_sms >= 2 &&
+            (L.cfg.amode == byoc::kAModeTile || L.cfg.amode == byoc::kAModeIm2col ||
+             L.cfg.amode == byoc::kAModeSlab)) {
+            GemmConfig mc = L.cfg;
+            mc.mc = true;
+            if (byoc::gemm_config_supported(mc)) L.cfg = mc;
+        }
         int64_t units_m = tiles_m;  // m-units of the launch: tiles, or pairs of tiles
         if (slab && L.cfg.amode == byoc::kAModeSlabRes && (int64_t)taps * chunks * (bk / 16) <= 16) {
             // Pair units (two adjacent tiles sharing each weight k-block and
@@ -1149,6 +1158,8 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
             L.cnt_bytes = (size_t)A.num_tiles * 8 * 4;
         }
         L.grid = std::min(A.num_tiles * splits, P.num_sms);
+        if (L.cfg.mc)  // whole clusters: one per pair of m-tiles of a column tile, at most num_sms / 2
+            L.grid = 2 * (int)std::min<int64_t>((units_m + 1) / 2 * A.tiles_n, P.num_sms / 2);
         A.act = act;
         L.flops = 2.0 * (double)M * (double)Kreal * (double)Cout;
         const double in_bytes = stem_k > 0 ? 0.0  // xq: the image is counted by the layout transform
@@ -1498,6 +1509,7 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
                            : byoc::amode_wres(L.cfg.amode)      ? L.args.slab_slots
                                                                 : 2;
         r->pair_units[i] = gm && byoc::amode_pair(L.cfg.amode) ? 1 : 0;
+        r->multicast[i] = gm && L.cfg.mc ? 1 : 0;
         r->stages[i] = 1;
         r->fp8[i] = L.kind == BYOC_LAUNCH_GEMM ? L.fp8 : 0;
         if (L.kind == BYOC_LAUNCH_CHAIN) {
@@ -1690,9 +1702,10 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
                     return cuda_fail(e, "cudaMemset(split-K counters)");
                 }
             }
+            // multicast: each CTA of a cluster loads half of a weight tile's rows
             CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
-                                   (uint64_t)L.k_pack, (uint32_t)L.cfg.bn, (uint32_t)L.cfg.bk,
-                                   L.cfg.bk);
+                                   (uint64_t)L.k_pack, (uint32_t)(L.cfg.mc ? L.cfg.bn / 2 : L.cfg.bn),
+                                   (uint32_t)L.cfg.bk, L.cfg.bk);
             if (r != CUDA_SUCCESS) {
                 byoc_release(h);
                 return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(weights) = %d", i, (int)r);
