@@ -503,15 +503,23 @@ int pick_bk(int64_t C) {
 }
 
 // Choose the output-channel tile among the compiled configurations by a
-// makespan estimate of the persistent grid, in SM cycles, calibrated on
-// GB300 traces of this kernel:
-//   mainloop per tile  = 300 + k-blocks x per-k-block cost: with A loaded per
-//                        k-block (tile, im2col) ~450 cycles of TMA delivery at
-//                        small bn, tensor-core bound (~2.5 bn) at bn = 256;
-//                        in slab mode A arrives once per channel chunk, so a
-//                        k-block costs the MMA time (~2.5 bn, at least 150);
-//   epilogue per tile  = ~600 cycles per pair of 32-column chunks (two warps
-//                        per accumulator row block work in parallel).
+// makespan estimate of the persistent grid, in SM cycles, fitted to GB300
+// traces of this kernel.  A k-block (bk channels of one filter tap) costs the
+// largest of
+//   * the tensor-core time of its bk / 16 MMAs (M = 128, N = bn: 40 / 48 /
+//     64 / 128 cycles at bn = 32 / 64 / 128 / 256);
+//   * its shared-memory traffic: every K16 MMA reads A (4 KB) and B (bn x 32
+//     bytes) from shared memory, and TMA writes the k-block's operands into
+//     it (A 128 x bk and B bn x bk; slab mode: B and the k-block's share of
+//     the slab).  Operand reads and TMA writes share the SM's shared-memory
+//     bandwidth, ~145 bytes/cycle in tile and im2col mode and ~118 in slab
+//     mode (traced per 64-wide k-block: 427 / 690 cycles at bn = 128 / 256 in
+//     tile mode, 316 / 420 at bn = 64 / 128 in slab mode; sharing each
+//     weight tile between two SMs by multicast, which halves L2 reads but not
+//     these bytes, measured no faster);
+//   * in tile and im2col mode, ~450 x bk / 64 cycles of TMA round trip.
+// epilogue per tile = ~600 cycles per pair of 32-column chunks (two warps per
+// accumulator row block work in parallel), ~3x that with GELU (traced).
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
 // time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
 //   split-K (tile mode, no residual, one wave of units only): S splits of
@@ -519,17 +527,23 @@ int pick_bk(int64_t C) {
 //                        fp32 partial (~26 bn cycles, traced) and the last one
 //                        reads the other S - 1 back (~10 bn cycles each)
 //                        before the epilogue.
+// slab_kb_bytes: slab mode, the bytes of one channel chunk's slab / taps.
 int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool res, int num_sms,
-            int *splits_out = nullptr) {
+            int *splits_out = nullptr, double slab_kb_bytes = 0.0, bool gelu = false) {
     int best = -1, best_s = 1;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
         GemmConfig c{bn, bk, amode, res};
         if (!byoc::gemm_config_supported(c)) continue;
         const int64_t tiles = tiles_m * ((N + bn - 1) / bn);
-        const double kb = amode == byoc::kAModeSlab ? std::max(2.5 * bn * bk / 64.0, 150.0)
-                                                    : std::max(2.5 * bn, 450.0);
-        const double epilogue = 600.0 * std::max(1, bn / 64);
+        const double steps = bk / 16.0;  // K16 MMAs per k-block
+        const double mma = steps * (bn <= 32 ? 40.0 : bn <= 64 ? 48.0 : bn <= 128 ? 64.0 : 128.0);
+        const double reads = steps * (4096.0 + 32.0 * bn);
+        const bool slab = amode == byoc::kAModeSlab;
+        const double writes = slab ? 2.0 * bk * bn + slab_kb_bytes : 2.0 * bk * (128.0 + bn);
+        const double kb = slab ? std::max(mma, (reads + writes) / 118.0)
+                               : std::max({mma, (reads + writes) / 145.0, 450.0 * bk / 64.0});
+        const double epilogue = 600.0 * std::max(1, bn / 64) * (gelu ? 3.0 : 1.0);
         for (int S = 1; S <= 4; ++S) {
             if (S > 1 && (!splits_out || amode != byoc::kAModeTile || res || kblocks < 4 * S ||
                           tiles * S > num_sms ||
@@ -1023,7 +1037,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         int splits = 1;
         const int bn = chain_bn > 0 ? chain_bn
                                     : pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms,
-                                              &splits);
+                                              &splits, slab ? (double)sgeo.bytes / taps : 0.0, act == byoc::kActGelu);
         if (bn < 0)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
                         o, bk, amode, (int)has_res);
