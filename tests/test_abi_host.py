@@ -303,10 +303,11 @@ def test_fusion_follows_the_composites_at_every_region_size():
 def test_split_k_for_deep_reductions_with_few_tiles():
     # BERT FFN's second dense (1024 x 3072 -> 768): 48 tiles of 128 x 128 would
     # leave most SMs idle for 48 k-blocks; three CTAs share each tile's
-    # k-blocks instead (144 CTAs); the first dense keeps one CTA per tile
+    # k-blocks instead (144 CTAs); the first dense (GELU epilogue) keeps one
+    # CTA per tile, 192 tiles of 128 x 128 on the 152 SMs
     rep = \
         R.whole_graph_region(I.bert_ffn()[0]).plan(152)
-    assert rep.splits[0] == 1 and rep.tile_n[0] == 256 and rep.grid[0] == 96
+    assert rep.splits[0] == 1 and rep.tile_n[0] == 128 and rep.grid[0] == 152
     assert rep.splits[1] == 3 and rep.tile_n[1] == 128 and rep.grid[1] == 144
     # fp32 partials [3][1024][768] + counters live in the handle's workspace
     assert rep.workspace_bytes >= 3 * 1024 * 768 * 4 + 1024 * 3072 * 2

@@ -66,10 +66,11 @@ def test_multicast_plans_pair_ctas_on_request(name):
 
 
 def test_multicast_grid_covers_the_tile_pairs():
-    # FFN first layer: 8 m-tiles x 12 column tiles of 256 -> 48 clusters
+    # FFN first layer: 8 m-tiles (4 pairs) x 3072 / BN column tiles, at most
+    # 76 clusters of two on 152 SMs
     g, _ = I.bert_ffn()
     rep = R.whole_graph_region(g, options=MC).plan(152)
-    assert rep.multicast[0] == 1 and rep.tile_n[0] == 256 and rep.grid[0] == 96
+    assert rep.multicast[0] == 1 and rep.grid[0] == 2 * min(4 * (3072 // rep.tile_n[0]), 76)
     # three m-tiles pair up as (0, 1) and (2, phantom): 2 pairs x 4 column tiles of 64
     g, _ = CASES["tile_1x1_odd_m"]()
     rep = R.whole_graph_region(g, options=MC).plan(152)
