@@ -163,6 +163,17 @@ typedef struct {
  *     layers, and the CTA pairs wait for each other at every ring stage).
  *     Results are bit-identical either way. */
 #define BYOC_OPT_MULTICAST 0x4u
+/*   BYOC_OPT_CLUSTER_SPLIT_K: a GEMM launch that splits each tile's k-blocks
+ *     over several CTAs (deep reductions over few tiles; tiles at most 128
+ *     wide, at most 4 splits) runs each tile's CTAs as one thread-block
+ *     cluster that exchanges the fp32 partial accumulators through
+ *     distributed shared memory, each CTA summing and storing its share of
+ *     the tile's 32-column chunks.  Off by default: the partials then go
+ *     through the handle's workspace in global memory, which measured as fast
+ *     or faster on GB300 (clusters of three CTAs are much slower).  The
+ *     partials are summed in split order either way: results are
+ *     bit-identical. */
+#define BYOC_OPT_CLUSTER_SPLIT_K 0x8u
 
 /* Figures describing a compiled region. */
 typedef struct {

@@ -17,6 +17,7 @@ ABI_VERSION = 2
 OPT_FUSE_DW_PW = 0x1
 OPT_REGION_KERNEL = 0x2
 OPT_MULTICAST = 0x4
+OPT_CLUSTER_SPLIT_K = 0x8
 
 # byoc_status
 OK, ERR_INVALID_ARG, ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM, ERR_TIMEOUT = range(6)

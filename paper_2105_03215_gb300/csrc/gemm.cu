@@ -89,10 +89,15 @@ struct GemmShape {
     // the others read the staging tile back for coalesced stores
     static constexpr bool TSTORE = AMODE == kAModeTile;
     static constexpr int CTRL_BYTES = 1024;
+    // cluster split-K: the blocks of partial sums the other CTAs send
+    static constexpr bool CLSPLIT = AMODE == kAModeTileSplitCl;
+    static constexpr int RECV_BLOCK = BM * 32 * 4;  // 128 rows x 32 fp32
+    static constexpr int RECV_BYTES = CLSPLIT ? kClRecvBlocks * RECV_BLOCK : 0;
+    static constexpr int RECV_BARS = CLSPLIT ? 2 : 0;  // one per chunk this CTA owns (BN <= 128)
     // TMA-store mode keeps a second staging tile per warp (one store in
     // flight while the next chunk is staged) where the weight ring still
     // has 8 stages with it: short-k-block configs (BK 16 / 32)
-    static constexpr int FIXED1 = 1024 + 2 * SLAB_BYTES + OPB * RES_TILE + BIAS_REGION + CTRL_BYTES;
+    static constexpr int FIXED1 = 1024 + 2 * SLAB_BYTES + RECV_BYTES + OPB * RES_TILE + BIAS_REGION + CTRL_BYTES;
     static constexpr int EPI_BUFS =
         TSTORE && (232448 - FIXED1 - 2 * kGemmEpiWarps * EPI_TILE) / STAGE_BYTES >= 8 ? 2 : 1;
     static constexpr int EPI_BYTES = kGemmEpiWarps * EPI_TILE * EPI_BUFS;
@@ -100,7 +105,7 @@ struct GemmShape {
     static constexpr int STAGES_RAW = (232448 - FIXED) / STAGE_BYTES;
     static constexpr int STAGES = STAGES_RAW > 32 ? 32 : STAGES_RAW;  // ring slots (k-blocks)
     static constexpr int POOL_BYTES = STAGES * STAGE_BYTES + 2 * SLAB_BYTES;
-    static constexpr int NUM_BARS = 2 * STAGES + 5 + 2 * SLOTS_MAX + 2 * OPB;
+    static constexpr int NUM_BARS = 2 * STAGES + 5 + 2 * SLOTS_MAX + 2 * OPB + RECV_BARS;
     static constexpr int SMEM_BYTES = FIXED + STAGES * STAGE_BYTES;
     static_assert(8 * NUM_BARS + 16 <= CTRL_BYTES, "control block");
     static_assert(STAGES >= 2, "ring depth");
@@ -112,7 +117,8 @@ struct GemmShape {
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
     static_assert(!(RES && SLAB), "slab tiles skip pad columns; no residual tile");
     static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
-    static_assert(!MC || (!WRES && !PAIR && AMODE != kAModeTileSplit),
+    static_assert(!CLSPLIT || (BN <= 128 && !RES), "cluster split-K: BN <= 128, no residual");
+    static_assert(!MC || (!WRES && !PAIR && !amode_split(AMODE)),
                   "multicast: weights streamed through the ring, one tile per unit");
     static constexpr int B_HALF = B_BYTES / 2;  // multicast: the rows one CTA loads
     static_assert(!MC || B_HALF % 1024 == 0, "a multicast half keeps the swizzle's 1 KB alignment");
@@ -173,7 +179,8 @@ __global__ void __maxnreg__(168)
     const int epi_arrivals = alt ? kGemmEpiWarps / 2 : kGemmEpiWarps;
     // split-K: a work unit is (tile, split); split sp covers k-blocks
     // [sp * num_kb / SPL, (sp + 1) * num_kb / SPL)
-    constexpr bool SPLITK = AMODE == kAModeTileSplit;
+    constexpr bool SPLITK = AMODE == kAModeTileSplit || AMODE == kAModeTileSplitCl;
+    constexpr bool CLSPLIT = S::CLSPLIT;  // a tile's splits form one cluster (rank = split)
     const int SPL = SPLITK ? a.splits : 1;
     const int num_units = a.num_tiles * SPL;
     // The loop over work units, the same in every role: unit u_first,
@@ -201,7 +208,8 @@ __global__ void __maxnreg__(168)
     const uint32_t sPoolEnd = sB + S::STAGES * S::B_BYTES + 2 * S::SLAB_BYTES;
     // slabs: 2 x SLAB_BYTES after the ring, or (resident weights) slab_slots x slab_pitch
     const uint32_t sSlab = S::WRES ? sB + (uint32_t)a.slab_off : sB + S::STAGES * S::B_BYTES;
-    const uint32_t sRes = sPoolEnd;                        // OPB x RES_TILE
+    const uint32_t sRecv = sPoolEnd;                       // RECV_BYTES (cluster split-K)
+    const uint32_t sRes = sRecv + S::RECV_BYTES;           // OPB x RES_TILE
     const uint32_t sEpi = sRes + S::OPB * S::RES_TILE;     // EPI_BYTES
     const uint32_t sBias = sEpi + S::EPI_BYTES;            // 2 x BIAS_BYTES
     const uint32_t ctrl = sBias + S::BIAS_REGION;
@@ -213,6 +221,7 @@ __global__ void __maxnreg__(168)
     const uint32_t sfull = oempty + 8u * S::OPB;           // SLOTS_MAX: slab loaded
     const uint32_t sempty = sfull + 8u * S::SLOTS_MAX;     // SLOTS_MAX: slab consumed
     const uint32_t drain = sempty + 8u * S::SLOTS_MAX;
+    const uint32_t recv_bar = drain + 8u;                  // RECV_BARS: a received chunk complete
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
 
@@ -237,6 +246,8 @@ __global__ void __maxnreg__(168)
             mbar_init(oempty + 8u * b, epi_arrivals);     // one arrive per epilogue warp of the tile
         }
         mbar_init(drain, 1);
+        // every lane of the four warps that read a chunk, in each other CTA
+        for (int b = 0; b < S::RECV_BARS; ++b) mbar_init(recv_bar + 8u * b, 128u * (uint32_t)(a.splits - 1));
         *abort_flag = 0;
         fence_barrier_init();
     }
@@ -253,7 +264,7 @@ __global__ void __maxnreg__(168)
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if constexpr (MC) cluster_sync();  // both CTAs' barriers initialised
+    if constexpr (MC || CLSPLIT) cluster_sync();  // the cluster's barriers initialised
     const uint32_t tmem_base = *tmem_slot;
     // Set-up done: the next kernel may be scheduled; global memory is touched
     // only after the previous kernel has completed -- except for the packed
@@ -761,7 +772,40 @@ __global__ void __maxnreg__(168)
                                               (size_t)lane * 4
                                         : 0;
             const size_t pstride = SPLITK ? (size_t)a.num_tiles * (size_t)(S::BM * BN) : 0;  // one split
-            if constexpr (SPLITK) {
+            if constexpr (CLSPLIT) {
+                // Cluster split-K (one tile per cluster, split = rank): chunk ci
+                // belongs to rank ci % splits.  Each chunk of this warp that
+                // another rank owns goes to that rank's receive block (block
+                // (ci / splits) * (splits - 1) + the sender's place among the
+                // other ranks; row r at r * 128 bytes, 16-byte piece q at
+                // q ^ (r & 7)), then each lane arrives on the owner's barrier
+                // for it, releasing its stores.  Every send comes before any
+                // wait, so no rank waits on a rank that is itself waiting.
+                int owned = 0;
+#pragma unroll 1
+                for (int ci = c_first; ci < NCH; ci += c_step) {
+                    const int owner = ci % SPL;
+                    if (owner == sp) {
+                        ++owned;
+                        continue;
+                    }
+                    uint32_t v[32];
+                    tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
+                    const int blk = (ci / SPL) * (SPL - 1) + (sp < owner ? sp : sp - 1);
+                    const uint32_t dst =
+                        mapa_shared(sRecv + (uint32_t)(blk * S::RECV_BLOCK) + (uint32_t)trow * 128u, (uint32_t)owner);
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        st_cluster_v4(dst + ((((uint32_t)q) ^ ((uint32_t)trow & 7u)) << 4), v[4 * q], v[4 * q + 1],
+                                      v[4 * q + 2], v[4 * q + 3]);
+                    mbar_arrive_remote(mapa_shared(recv_bar + 8u * (uint32_t)(ci / SPL), (uint32_t)owner));
+                }
+                if (owned == 0) {  // no more reads of the accumulator by this warp
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(tempty + 8u * buf);
+                }
+            } else if constexpr (SPLITK) {
 #pragma unroll 1
                 for (int ci = c_first, k = 0; ci < NCH; ci += c_step, ++k) {
                     uint32_t v[32];
@@ -800,15 +844,49 @@ __global__ void __maxnreg__(168)
             }
 #pragma unroll 1
             for (int ci = c_first, kk = 0; ci < nch; ci += c_step, ++kk) {
+                if (CLSPLIT && ci % SPL != sp) continue;  // sent to its owner above
                 const int col0 = n0 + ci * 32;
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);  // includes tcgen05.wait::ld
-                if (ci + c_step >= nch) {  // this warp's last read of the accumulator
+                int next = ci + c_step;  // this warp's next chunk (cluster split-K: that this rank owns)
+                if constexpr (CLSPLIT)
+                    while (next < nch && next % SPL != sp) next += c_step;
+                if (next >= nch) {  // this warp's last read of the accumulator
                     tc_fence_before();
                     __syncwarp();
                     if (lane == 0) mbar_arrive(tempty + 8u * buf);
                 }
-                if constexpr (SPLITK) {
+                if constexpr (CLSPLIT) {
+                    // the other ranks' blocks of this chunk, summed in split
+                    // order with this rank's own (the bits of the global split-K)
+                    mbar_wait_cluster(recv_bar + 8u * (uint32_t)(ci / SPL), 0u, abort_flag, a.err,
+                                      kErrTimeoutEpilogue);
+                    float sum[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) sum[j] = 0.0f;
+                    for (int s2 = 0; s2 < SPL; ++s2) {
+                        if (s2 == sp) {
+#pragma unroll
+                            for (int j = 0; j < 32; ++j) sum[j] += __uint_as_float(v[j]);
+                        } else {
+                            const int blk = (ci / SPL) * (SPL - 1) + (s2 < sp ? s2 : s2 - 1);
+                            const uint32_t src = sRecv + (uint32_t)(blk * S::RECV_BLOCK) + (uint32_t)trow * 128u;
+#pragma unroll
+                            for (int q = 0; q < 8; ++q) {
+                                float4 p4;
+                                asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                                             : "=f"(p4.x), "=f"(p4.y), "=f"(p4.z), "=f"(p4.w)
+                                             : "r"(src + ((((uint32_t)q) ^ ((uint32_t)trow & 7u)) << 4)));
+                                sum[4 * q] += p4.x;
+                                sum[4 * q + 1] += p4.y;
+                                sum[4 * q + 2] += p4.z;
+                                sum[4 * q + 3] += p4.w;
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) v[j] = __float_as_uint(sum[j]);
+                } else if constexpr (SPLITK) {
                     float sum[32];
 #pragma unroll
                     for (int j = 0; j < 32; ++j) sum[j] = 0.0f;
@@ -939,7 +1017,7 @@ __global__ void __maxnreg__(168)
     __syncthreads();
     // MC: the peer's multicast copies into this CTA and its MMA commits on
     // this CTA's barriers are complete once it has passed its own waits
-    if constexpr (MC) cluster_sync();
+    if constexpr (MC || CLSPLIT) cluster_sync();
     if (a.trace != nullptr && threadIdx.x == 0) atomicMax(a.trace + 1, globaltimer_ns());
     if (warp == 1) {
         tc_fence_after();
@@ -954,7 +1032,7 @@ static cudaError_t launch_t(const CUtensorMap &tmA, const CUtensorMap &tmB, cons
                             const CUtensorMap &tmO, const GemmArgs &a, int grid, cudaStream_t st) {
     using S = GemmShape<BN, BK, AMODE, RES, MC>;
     return launch_pdl_cluster(gemm_tcgen05_kernel<BN, BK, AMODE, RES, MC>, dim3(grid), dim3(kGemmThreads),
-                      (size_t)S::SMEM_BYTES, st, MC ? 2 : 1, tmA, tmB, tmR, tmO, a);
+                      (size_t)S::SMEM_BYTES, st, MC ? 2 : (S::CLSPLIT ? a.splits : 1), tmA, tmB, tmR, tmO, a);
 }
 
 template <int BN, int BK, int AMODE, bool RES, bool MC>
@@ -995,6 +1073,8 @@ static cudaError_t prepare_t() {
     X(64, 64, kAModeTileSplit, false, false) \
     X(128, 64, kAModeTileSplit, false, false) \
     X(256, 64, kAModeTileSplit, false, false) \
+    X(64, 64, kAModeTileSplitCl, false, false) \
+    X(128, 64, kAModeTileSplitCl, false, false) \
     X(64, 64, kAModeSlabRes, false, false)   \
     X(128, 64, kAModeSlabRes, false, false)  \
     X(64, 16, kAModeSlabRes, false, false)   \
@@ -1086,6 +1166,9 @@ cudaError_t launch_gemm(const GemmConfig &c, const CUtensorMap &tmA, const CUten
                         const CUtensorMap &tmR, const CUtensorMap &tmO, const GemmArgs &a, int grid,
                         cudaStream_t st) {
     if (c.mc && (grid < 2 || grid % 2)) return cudaErrorInvalidValue;  // whole clusters of two
+    // cluster split-K: one cluster of `splits` CTAs per tile, every tile in the grid
+    if (c.amode == kAModeTileSplitCl && (!cl_split_fits(c.bn, a.splits) || grid != a.num_tiles * a.splits))
+        return cudaErrorInvalidValue;
 #define X(BN_, BK_, AM_, RES_, MC_)                     \
     if (BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_)) \
         return launch_t<BN_, BK_, AM_, RES_, MC_>(tmA, tmB, tmR, tmO, a, grid, st);

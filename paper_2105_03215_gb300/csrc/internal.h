@@ -118,10 +118,24 @@ enum AMode : int {
     // kAModeSlabRes in pair units: two vertically adjacent slab tiles of one
     // image (2 x 128 MMA rows, two accumulators) share one slab load and the
     // per-unit waits and commits
-    kAModeSlabRes2 = 5
+    kAModeSlabRes2 = 5,
+    // kAModeTileSplit with the `splits` CTAs of a tile forming one thread-block
+    // cluster: the partial accumulators are summed through distributed shared
+    // memory (each CTA owns every splits-th 32-column chunk of the tile)
+    // instead of fp32 partials in global memory.  BN <= 128, splits <= 4,
+    // at most kClRecvBlocks received 128 x 32 blocks per CTA.
+    kAModeTileSplitCl = 6
 };
 
 constexpr bool amode_slab(int m) { return m == kAModeSlab || m == kAModeSlabRes || m == kAModeSlabRes2; }
+constexpr bool amode_split(int m) { return m == kAModeTileSplit || m == kAModeTileSplitCl; }
+constexpr int kClMaxSplits = 4;
+constexpr int kClRecvBlocks = 4;  // 128 x 32 fp32 blocks (16 KB each) a CTA receives
+// whether a cluster split of `splits` CTAs fits the receive buffer at tile width bn
+constexpr bool cl_split_fits(int bn, int splits) {
+    return splits >= 2 && splits <= kClMaxSplits && bn <= 128 &&
+           ((bn / 32 + splits - 1) / splits) * (splits - 1) <= kClRecvBlocks;
+}
 constexpr bool amode_pair(int m) { return m == kAModeSlabRes2; }
 constexpr bool amode_wres(int m) { return m == kAModeSlabRes || m == kAModeSlabRes2; }
 

@@ -523,14 +523,20 @@ int pick_bk(int64_t C) {
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
 // time is rounds x max(mainloop, epilogue) + min(mainloop, epilogue).
 //   split-K (tile mode, no residual, one wave of units only): S splits of
-//                        kblocks / S each; every split writes and fences its
-//                        fp32 partial (~26 bn cycles, traced) and the last one
-//                        reads the other S - 1 back (~10 bn cycles each)
-//                        before the epilogue.
+//                        kblocks / S each.  Through global memory: every
+//                        split writes and fences its fp32 partial (~26 bn
+//                        cycles, traced) and the last one reads the other
+//                        S - 1 back (~10 bn cycles each) before the epilogue.
+//                        As one cluster (BN <= 128, S <= 4): the partials move
+//                        through distributed shared memory (~2000 + 10 bn
+//                        cycles) and each CTA runs the epilogue of its 1 / S
+//                        of the tile's chunks.
 // slab_kb_bytes: slab mode, the bytes of one channel chunk's slab / taps.
+// *cluster_out: whether the chosen split is the cluster one.
 int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool res, int num_sms,
-            int *splits_out = nullptr, double slab_kb_bytes = 0.0, bool gelu = false) {
+            int *splits_out = nullptr, double slab_kb_bytes = 0.0, bool gelu = false, bool *cluster_out = nullptr) {
     int best = -1, best_s = 1;
+    bool best_cl = false;
     double best_cost = 1e300;
     for (int bn : {256, 128, 64, 32}) {
         GemmConfig c{bn, bk, amode, res};
@@ -545,25 +551,34 @@ int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool
                                : std::max({mma, (reads + writes) / 145.0, 450.0 * bk / 64.0});
         const double epilogue = 600.0 * std::max(1, bn / 64) * (gelu ? 3.0 : 1.0);
         for (int S = 1; S <= 4; ++S) {
+            const bool global_ok =
+                byoc::gemm_config_supported(GemmConfig{bn, bk, byoc::kAModeTileSplit, false});
+            const bool cl_ok = cluster_out && byoc::cl_split_fits(bn, S) &&
+                               byoc::gemm_config_supported(GemmConfig{bn, bk, byoc::kAModeTileSplitCl, false});
             if (S > 1 && (!splits_out || amode != byoc::kAModeTile || res || kblocks < 4 * S ||
-                          tiles * S > num_sms ||
-                          !byoc::gemm_config_supported(GemmConfig{bn, bk, byoc::kAModeTileSplit, false})))
+                          tiles * S > num_sms || !(global_ok || cl_ok)))
                 continue;
             const int64_t units = tiles * S;
             const int64_t grid = std::min<int64_t>(units, num_sms);
             const int64_t rounds = (units + grid - 1) / grid;
             const double mainloop = 300.0 + (double)((kblocks + S - 1) / S) * kb;
+            const int nch = bn / 32;
+            const double cost_global = mainloop + 26.0 * bn + 10.0 * bn * (S - 1) + epilogue;
+            const double cost_cl = mainloop + 2000.0 + 10.0 * bn + epilogue * ((nch + S - 1) / S) / nch;
+            const bool cl = S > 1 && cl_ok && (!global_ok || cost_cl < cost_global);
             const double cost =
                 S == 1 ? (double)rounds * std::max(mainloop, epilogue) + std::min(mainloop, epilogue)
-                       : mainloop + 26.0 * bn + 10.0 * bn * (S - 1) + epilogue;
+                       : (cl ? cost_cl : cost_global);
             if (cost < best_cost - 1e-9) {
                 best_cost = cost;
                 best = bn;
                 best_s = S;
+                best_cl = cl;
             }
         }
     }
     if (splits_out) *splits_out = best_s;
+    if (cluster_out) *cluster_out = best_cl;
     return best;
 }
 
@@ -1035,13 +1050,17 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         const int64_t tiles_per_img = slab ? (Y.shape[1] + sgeo.t - 1) / sgeo.t : 0;
         const int64_t tiles_m = slab ? X.shape[0] * tiles_per_img : (M + 127) / 128;
         int splits = 1;
+        bool cl_split = false;
         const int bn = chain_bn > 0 ? chain_bn
                                     : pick_bn(tiles_m, Cout, (int64_t)taps * chunks, bk, amode, has_res, P.num_sms,
-                                              &splits, slab ? (double)sgeo.bytes / taps : 0.0, act == byoc::kActGelu);
+                                              &splits, slab ? (double)sgeo.bytes / taps : 0.0, act == byoc::kActGelu,
+                                              (d->options & BYOC_OPT_CLUSTER_SPLIT_K) ? &cl_split : nullptr);
         if (bn < 0)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: no compiled tile for BK=%d mode=%d residual=%d",
                         o, bk, amode, (int)has_res);
-        L.cfg = GemmConfig{bn, bk, splits > 1 ? byoc::kAModeTileSplit : amode, has_res};
+        L.cfg = GemmConfig{bn, bk,
+                           splits > 1 ? (cl_split ? byoc::kAModeTileSplitCl : byoc::kAModeTileSplit) : amode,
+                           has_res};
         if (slab && Cout <= bn) {
             // one column tile: keep the whole weight matrix in shared memory
             // when it fits beside two slabs
@@ -1167,7 +1186,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         A.splits = splits;
         A.m_pad = (int)(tiles_m * byoc::kGemmBM);
         A.n_pad = L.n_pad;
-        if (splits > 1) {
+        if (splits > 1 && !cl_split) {  // global split-K: partials and counters in the workspace
             L.part_bytes = (size_t)splits * A.m_pad * A.n_pad * 4;
             L.cnt_bytes = (size_t)A.num_tiles * 8 * 4;
         }
@@ -1512,7 +1531,7 @@ void fill_report(const Plan &P, byoc_plan_report *r) {
         r->gemm_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.k_pack : (dp ? L.dp.C : 0);
         r->tile_n[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bn : (dp ? L.dp.n_pad : 0);
         r->tile_k[i] = L.kind == BYOC_LAUNCH_GEMM ? L.cfg.bk : (dp ? byoc::kDpChunk : 0);
-        r->im2col[i] = L.kind != BYOC_LAUNCH_GEMM || L.cfg.amode == byoc::kAModeTileSplit
+        r->im2col[i] = L.kind != BYOC_LAUNCH_GEMM || byoc::amode_split(L.cfg.amode)
                            ? 0
                            : std::min(L.cfg.amode, (int)byoc::kAModeSlab);
         r->splits[i] = L.kind == BYOC_LAUNCH_GEMM ? std::max(1, L.args.splits) : 0;
@@ -2038,6 +2057,16 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: split-K scratch out of range");
         if (L.kind == BYOC_LAUNCH_GEMM && !byoc::gemm_config_supported(L.cfg))
             return fail(BYOC_ERR_UNSUPPORTED, "serialised plan: tile configuration not in this build");
+        if (L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeTileSplit &&
+            (L.args.splits < 2 ||
+             L.part_bytes < (size_t)L.args.splits * (size_t)L.args.m_pad * (size_t)L.args.n_pad * 4 ||
+             L.cnt_bytes < (size_t)L.args.num_tiles * 8 * 4))
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: split-K scratch too small");
+        if (L.kind == BYOC_LAUNCH_GEMM && L.cfg.amode == byoc::kAModeTileSplitCl &&
+            (!byoc::cl_split_fits(L.cfg.bn, L.args.splits) || L.grid != L.args.num_tiles * L.args.splits))
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent cluster split-K");
+        if (L.kind == BYOC_LAUNCH_GEMM && L.cfg.mc && (L.grid < 2 || L.grid % 2))
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: multicast launch of an odd grid");
     }
     return BYOC_OK;
 }
