@@ -73,6 +73,7 @@ class Executor:
                 src = self.entries[node.inputs[0]]
                 self.entries[name] = src.view(node.shape)
         self._graph = None
+        self._pipe = None
         self.n_launches = sum(c.n_launches for c in self.compiled) + sum(
             1 for k, x in self.steps if k == "host" and self.by_name[x].op != "nn.batch_flatten")
 
@@ -201,6 +202,61 @@ class Executor:
             raise RuntimeError("capture() first")
         self._graph.replay()
 
+    def capture_double_buffered(self, name: str = "data") -> None:
+        """Record two CUDA graphs of the forward pass that read the input entry
+        ``name`` from two different device buffers, for run_from_host: while
+        one pass runs, the next pass's input is uploaded into the other."""
+        torch = self.torch
+        self.capture()  # warm-up and the first graph, on the entry's own buffer
+        first = self.entries[name]
+        second = torch.empty_like(first)
+        self.entries[name] = second
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            self.run_steps()
+        self.entries[name] = first
+        self._pipe = {"name": name, "bufs": [first, second], "graphs": [self._graph, g],
+                      "copy": torch.cuda.Stream(),
+                      "in_ready": [torch.cuda.Event(), torch.cuda.Event()],
+                      "in_free": [torch.cuda.Event(), torch.cuda.Event()]}
+
+    def run_from_host(self, host_inputs: Sequence, host_outputs: Sequence) -> None:
+        """Forward passes over a sequence of batches in (pinned) host memory:
+        pass i reads host_inputs[i] and writes its output to host_outputs[i].
+        Inputs are uploaded on a copy stream into alternating device buffers,
+        each as soon as the pass that last read that buffer has finished, so
+        pass i + 1's upload overlaps pass i; passes run in order on the current
+        stream, each followed by the read-back of its output.  Returns once
+        every output is in host memory."""
+        if getattr(self, "_pipe", None) is None:
+            raise RuntimeError("capture_double_buffered() first")
+        torch = self.torch
+        p = self._pipe
+        cs = torch.cuda.current_stream()
+        cp = p["copy"]
+        n = len(host_inputs)
+        if len(host_outputs) != n:
+            raise ValueError("one output buffer per input batch")
+
+        def upload(i):
+            b = i & 1
+            cp.wait_event(p["in_free"][b])  # the pass that last read buffer b is done
+            with torch.cuda.stream(cp):
+                p["bufs"][b].copy_(host_inputs[i], non_blocking=True)
+            p["in_ready"][b].record(cp)
+
+        if n:
+            upload(0)
+        for i in range(n):
+            if i + 1 < n:
+                upload(i + 1)
+            b = i & 1
+            cs.wait_event(p["in_ready"][b])
+            p["graphs"][b].replay()
+            p["in_free"][b].record(cs)
+            host_outputs[i].copy_(self.output(), non_blocking=True)
+        cs.synchronize()
+
     def check(self) -> None:
         for c in self.compiled:
             c.check()
@@ -210,6 +266,7 @@ class Executor:
             c.release()
         self.compiled = []
         self._graph = None
+        self._pipe = None
         self.entries = {}
 
 
