@@ -517,7 +517,9 @@ int pick_bk(int64_t C) {
 //     tile mode, 316 / 420 at bn = 64 / 128 in slab mode; sharing each
 //     weight tile between two SMs by multicast, which halves L2 reads but not
 //     these bytes, measured no faster);
-//   * in tile and im2col mode, ~450 x bk / 64 cycles of TMA round trip.
+//   * in tile and im2col mode, ~450 cycles of TMA round trip and per-k-block
+//     overhead, whatever bk (a k-block of 16 channels costs as much: the
+//     MobileNetV2 112x112 16 -> 96 layer, measured in the whole network).
 // epilogue per tile = ~600 cycles per pair of 32-column chunks (two warps per
 // accumulator row block work in parallel), ~3x that with GELU (traced).
 // A CTA overlaps one tile's epilogue with the next tile's mainloop, so its
@@ -548,7 +550,7 @@ int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool
         const bool slab = amode == byoc::kAModeSlab;
         const double writes = slab ? 2.0 * bk * bn + slab_kb_bytes : 2.0 * bk * (128.0 + bn);
         const double kb = slab ? std::max(mma, (reads + writes) / 118.0)
-                               : std::max({mma, (reads + writes) / 145.0, 450.0 * bk / 64.0});
+                               : std::max({mma, (reads + writes) / 145.0, 450.0});
         const double epilogue = 600.0 * std::max(1, bn / 64) * (gelu ? 3.0 : 1.0);
         for (int S = 1; S <= 4; ++S) {
             const bool global_ok =
