@@ -2069,6 +2069,13 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent cluster split-K");
         if (L.kind == BYOC_LAUNCH_GEMM && L.cfg.mc && (L.grid < 2 || L.grid % 2))
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: multicast launch of an odd grid");
+        if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
+            const byoc::DwArgs &w = L.dw;
+            const size_t box = (size_t)w.in_rows * w.in_cols * w.cc * 2;
+            if (w.cc < 8 || w.cc > 256 || w.in_rows < 1 || w.in_rows > 256 || w.in_cols < 1 || w.in_cols > 256 ||
+                (size_t)w.buf_bytes < box || (size_t)w.buf_bytes > byoc::kDwBufBudget)
+                return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent depthwise tiling");
+        }
     }
     return BYOC_OK;
 }
