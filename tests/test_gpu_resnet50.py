@@ -55,12 +55,15 @@ def test_resnet50_small_image_every_region_teacher_forced():
         for o in r.outputs:
             assert_close(_f64(ex.entries[o]), ref[o], sc[o], f"{r.name}:{o}")
     _check_host_steps(ex)
-    # end-to-end (not gated): fp64 oracle forward from the same input
+    # end to end: fp64 oracle forward from the same input.  A CPU emulation
+    # of bf16 storage with fp32-exact sums lands 0.6% (relative L2) from the
+    # oracle on this network (tests/test_tolerance.py); the GPU must stay
+    # within 5x that
     full = ograph.evaluate(g, inp)[g.outputs[0]]
     got = _f64(ex.output())
     rel = np.linalg.norm(got - full) / np.linalg.norm(full)
     print(f"resnet50 N=2 64x64 end-to-end logits relative L2 error {rel:.4f}")
-    assert rel < 0.2
+    assert rel < 0.03
     ex.release()
 
 

@@ -107,3 +107,18 @@ def test_planted_mistakes_fail_the_rule(kind):
     o = g.outputs[0]
     with pytest.raises(AssertionError):
         assert_close(bad[o], ref[o], sc[o], kind)
+
+
+def test_resnet50_end_to_end_bf16_storage_error_is_small():
+    # End to end through 54 regions the per-element error scale outgrows the
+    # values themselves (the random-init network amplifies every rounding), so
+    # the end-to-end logits are gated by relative L2 instead: bf16-storage
+    # arithmetic lands within 1.5% of the fp64 oracle here (measured 0.60%),
+    # the number the GPU end-to-end test's 3% gate is set from
+    from paper_2105_03215_gb300 import executor as E
+    res, inp = E.build_resnet50(N=2, H=64, W=64)
+    g = res.graph
+    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    em = _emulate(g, inp)[g.outputs[0]]
+    rel = np.linalg.norm(em - ref) / np.linalg.norm(ref)
+    assert 1e-4 < rel < 0.015, rel
