@@ -32,6 +32,8 @@ def test_mobilenet_v2_small_image_every_region_teacher_forced():
         ref, sc = oracle(g, feed, nodes=[n.name for n in r.nodes], keep=r.outputs)
         for o in r.outputs:
             assert_close(_f64(ex.entries[o]), ref[o], sc[o], f"{r.name}:{o}")
+    # end to end: a CPU emulation of bf16 storage lands 11.7% (relative L2)
+    # from the fp64 oracle on this random-init network (tests/test_tolerance.py)
     full = ograph.evaluate(g, inp)[g.outputs[0]]
     got = _f64(ex.output())
     rel = np.linalg.norm(got - full) / np.linalg.norm(full)

@@ -122,3 +122,17 @@ def test_resnet50_end_to_end_bf16_storage_error_is_small():
     em = _emulate(g, inp)[g.outputs[0]]
     rel = np.linalg.norm(em - ref) / np.linalg.norm(ref)
     assert 1e-4 < rel < 0.015, rel
+
+
+def test_mobilenet_v2_end_to_end_bf16_storage_error():
+    # The same for MobileNetV2 (N=2, 96x96): this random-init network
+    # amplifies rounding far more (ReLU6 clipping, depthwise layers) --
+    # bf16-storage arithmetic lands 11.7% from the fp64 oracle end to end,
+    # the figure the GPU end-to-end test's 20% gate is set from
+    from paper_2105_03215_gb300 import executor as E
+    res, inp = E.build_mobilenet_v2(N=2, H=96, W=96)
+    g = res.graph
+    ref = ograph.evaluate(g, inp)[g.outputs[0]]
+    em = _emulate(g, inp)[g.outputs[0]]
+    rel = np.linalg.norm(em - ref) / np.linalg.norm(ref)
+    assert 0.01 < rel < 0.15, rel
