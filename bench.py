@@ -470,6 +470,24 @@ def region_figures(flush, peaks):
     nbytes = xs.numel() * 4 + ys.numel() * 2
     out[f"boundary_nchw_f32_to_nhwc_bf16_{BATCH}x3x{IMG}x{IMG}"] = {
         "us": tb * 1e6, "gbps": nbytes / tb / 1e9, "hbm_frac_of_measured": nbytes / tb / 1e9 / peaks["hbm_gbs"]}
+    # every config's roofline fraction against its target in one place: conv /
+    # dense regions against 0.60 of the measured bf16 tensor peak, the
+    # depthwise launch against 0.70 of the measured HBM bandwidth; single call
+    # (graph-replay floor included) and back to back
+    targets = {}
+    for name, bound, target in (("conv3x3_bias_relu_1x56x56x64", "tensor", 0.60),
+                                ("bert_ffn_1024x768x3072", "tensor", 0.60),
+                                ("mbv2_dw_pw_32x56x56x144", "hbm", 0.70),
+                                ("depthwise3x3_bn_relu6_32x56x56x144", "hbm", 0.70),
+                                ("resnet50_bottleneck_32x14x14x1024", "tensor", 0.60)):
+        r = out.get(name)
+        if not r:
+            continue
+        key, key2 = (("tensor_frac_of_measured", "tensor_frac_back_to_back") if bound == "tensor"
+                     else ("hbm_frac_of_measured", "hbm_frac_back_to_back"))
+        targets[name] = {"bound": bound, "target": target, "single_call": r.get(key),
+                         "back_to_back": r.get(key2), "met": bool((r.get(key2) or 0.0) >= target)}
+    out["roofline_targets"] = targets
     return out
 
 
