@@ -349,15 +349,20 @@ __global__ void __maxnreg__(168)
                     ok = false;
                 }
             }
-            // One column tile (tiles_n == 1): every unit reads the same weight
-            // k-blocks, and where a unit's ring stages (spu of them) divide the
-            // ring, ring slot s holds the same k-blocks on every pass.  After
-            // the first pass over the ring the weights are in place and only A
-            // is loaded: one TMA copy per k-block instead of two (measured on
-            // MobileNetV2's short-K 1x1 layers: the 112x112 32 -> 16 layer
-            // 37.4 -> 29.2 us; their rate is set by the per-tile copy chain).
+            // Where all of this CTA's units are in one column tile (tiles_n == 1,
+            // or a grid that is a multiple of tiles_n: units u_first + k u_step
+            // share u_first % tiles_n) they read the same weight k-blocks, and
+            // where a unit's ring stages (spu of them) divide the ring, ring
+            // slot s holds the same k-blocks on every pass.  After the first
+            // pass over the ring the weights are in place and only A is loaded:
+            // one TMA copy per k-block instead of two (measured on MobileNetV2's
+            // short-K 1x1 layers: the 112x112 32 -> 16 layer 37.4 -> 29.2 us;
+            // their rate is set by the per-tile copy chain).
             const int spu = (a.num_kb + G - 1) / G;
-            const bool b_keep = !SPLITK && !MC && !S::SLAB && a.tiles_n == 1 && nst % spu == 0;
+            // (several column tiles: not with a residual, where the same-box
+            // A/B on ResNet-50's conv3 layers measured ~3 us slower per step)
+            const bool b_keep = !SPLITK && !MC && !S::SLAB &&
+                                (a.tiles_n == 1 || (!RES && u_step % a.tiles_n == 0)) && nst % spu == 0;
             // Tile / im2col / split modes: claim the first unit's first ring
             // stages and load their weights before waiting for the previous
             // kernel; their activations follow the wait (same stage barriers).

@@ -1193,6 +1193,13 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
             L.cnt_bytes = (size_t)A.num_tiles * 8 * 4;
         }
         L.grid = std::min(A.num_tiles * splits, P.num_sms);
+        // Short reductions over several rounds of tiles: a grid that is a
+        // multiple of the column tiles keeps every CTA in one column tile, so
+        // the kernel keeps its weight k-blocks in the ring (gemm.cu) -- at most
+        // tiles_n - 1 SMs idle (none for 2, 4 or 8 column tiles)
+        if (splits == 1 && !L.cfg.mc && !slab && !has_res && A.tiles_n > 1 && A.tiles_n <= 8 && A.num_kb <= 4 &&
+            A.num_tiles >= 3 * P.num_sms && P.num_sms >= A.tiles_n)
+            L.grid = P.num_sms / A.tiles_n * A.tiles_n;
         if (L.cfg.mc)  // whole clusters: one per pair of m-tiles of a column tile, at most num_sms / 2
             L.grid = 2 * (int)std::min<int64_t>((units_m + 1) / 2 * A.tiles_n, P.num_sms / 2);
         A.act = act;

@@ -12,8 +12,10 @@ from paper_2105_03215_gb300 import region as R
 
 from .parity import run_region
 
-# (K, N, tiles per CTA wanted): K = 64 / 128 / 192 / 320 channels, N <= the tile width
-CASES = [(64, 24, 20), (128, 64, 12), (192, 24, 8), (320, 32, 6)]
+# (K, N, tiles per CTA wanted): K = 64 / 128 / 192 / 320 channels, N <= the
+# tile width; and two or three column tiles with a grid that is a multiple of
+# them (every CTA stays in one column tile)
+CASES = [(64, 24, 20), (128, 64, 12), (192, 24, 8), (320, 32, 6), (64, 144, 24), (128, 256, 16)]
 
 
 def _dense_int(M, K, N, seed):
@@ -31,11 +33,12 @@ def _dense_int(M, K, N, seed):
 @pytest.mark.gpu
 @pytest.mark.parametrize("K,N,per_cta", CASES)
 def test_single_column_tile_launches_reuse_their_weights_bit_exact(K, N, per_cta):
-    M = 128 * 152 * per_cta + 77  # a ragged last tile
+    M = 128 * 152 * per_cta // max(1, -(-N // 64)) + 77  # a ragged last tile
     g, inp = _dense_int(M, K, N, seed=K + N)
     reg = R.whole_graph_region(g)
     rep = reg.plan(152)
-    assert rep.tile_n[0] >= N and rep.splits[0] == 1  # one column tile
+    tiles_n = -(-N // rep.tile_n[0])
+    assert rep.splits[0] == 1 and rep.grid[0] % tiles_n == 0  # every CTA in one column tile
     got, cr = run_region(reg, inp)
     exact = inp["x"] @ g.nodes[0].consts["weight"].T + g.nodes[1].consts["bias"]  # integers, exact in fp32
     want = I.bf16_round(exact.astype(np.float32))
