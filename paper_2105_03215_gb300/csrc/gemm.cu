@@ -38,6 +38,13 @@
 //              slice (bulk copy) and, when the region adds a residual, the
 //              128 x BN residual tile (TMA) into a ring of OPB buffers.
 //
+// FP8 (BK = kF8BK; Section 3.2's partial quantization): A holds the E4M3
+// codes a Q node wrote, B the weights quantized per output channel; a k-block
+// is 128 codes (128 bytes, the same swizzled rows as 64 bf16 values), one
+// kind::f8f6f4 MMA per 32 of them.  The epilogue dequantizes with one fma
+// (accumulator x S_x S_w[n] + bias[n]) and, when a Q node follows the
+// composite, writes E4M3 codes instead of bf16 (TMA store of 32 x 32 bytes).
+//
 // Cluster multicast (MC, on request: BYOC_OPT_MULTICAST): the kernel runs in
 // clusters of two CTAs that take
 // the m-tiles 2i and 2i + 1 of the same column tile together, k-block by
@@ -62,9 +69,11 @@ struct GemmShape {
     static constexpr bool PAIR = amode_pair(AMODE);  // two tiles (halves) per unit
     static constexpr int HALVES = PAIR ? 2 : 1;
     static_assert(!PAIR || WRES, "pair units keep their weights resident");
-    static constexpr int ROW_BYTES = BK * 2;  // one K-major operand row (= swizzle width)
-    static constexpr int A_BYTES = SLAB ? 0 : BM * BK * 2;
-    static constexpr int B_BYTES = BN * BK * 2;
+    // FP8: E4M3 operands, 128 codes per k-block (kind::f8f6f4, K = 32 per MMA)
+    static constexpr bool F8 = BK == kF8BK;
+    static constexpr int ROW_BYTES = F8 ? BK : BK * 2;  // one K-major operand row (= swizzle width)
+    static constexpr int A_BYTES = SLAB ? 0 : BM * ROW_BYTES;
+    static constexpr int B_BYTES = BN * ROW_BYTES;
     static constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
     static constexpr int SLAB_BYTES = SLAB ? slab_max_bytes(BK, PAIR) : 0;
     // slab barriers: two slots beside a weight ring; up to kMaxSlabSlots
@@ -81,13 +90,13 @@ struct GemmShape {
     // are HBM-bound and keep more residual tiles in flight; bias-only slices
     // are small, and eight in flight keep their L2 latency off short tiles
     static constexpr int OPB = RES ? (BN >= 128 ? 3 : 4) : 8;
-    static constexpr int BIAS_BYTES = BN * 4;
+    static constexpr int BIAS_BYTES = BN * 4 * (F8 ? 2 : 1);  // bias slice (FP8: then the dq slice)
     static constexpr int BIAS_REGION = (OPB * BIAS_BYTES + 1023) / 1024 * 1024;
     // epilogue staging: one 32x32 bf16 output tile per epilogue warp
     static constexpr int EPI_TILE = 32 * 32 * 2;
-    // tile mode stores its output with TMA from each warp's staging tile;
-    // the others read the staging tile back for coalesced stores
-    static constexpr bool TSTORE = AMODE == kAModeTile;
+    // tile mode (and FP8) stores its output with TMA from each warp's
+    // staging tile; the others read the staging tile back for coalesced stores
+    static constexpr bool TSTORE = gemm_tstore(AMODE, BK);
     static constexpr int CTRL_BYTES = 1024;
     // cluster split-K: the blocks of partial sums the other CTAs send
     static constexpr bool CLSPLIT = AMODE == kAModeTileSplitCl;
@@ -116,7 +125,9 @@ struct GemmShape {
     static_assert(TMEM_COLS <= 512, "TMEM: two accumulators of HALVES x BN columns");
     static_assert(!RES || BN % 64 == 0, "residual tiles are loaded in 64-column boxes");
     static_assert(!(RES && SLAB), "slab tiles skip pad columns; no residual tile");
-    static_assert(BK == 16 || BK == 32 || BK == 64, "BK");
+    static_assert(BK == 16 || BK == 32 || BK == 64 || F8, "BK");
+    static_assert(!F8 || (AMODE == kAModeTile || AMODE == kAModeIm2col || AMODE == kAModeTileSplit),
+                  "FP8: tile, im2col and split-K modes");
     static_assert(!CLSPLIT || (BN <= 128 && !RES), "cluster split-K: BN <= 128, no residual");
     static_assert(!MC || (!WRES && !PAIR && !amode_split(AMODE)),
                   "multicast: weights streamed through the ring, one tile per unit");
@@ -281,7 +292,7 @@ __global__ void __maxnreg__(168)
             // them): each prefetches its own part, so L2 sees every byte
             // requested once.
             constexpr int PF_ROWS = MC ? BN / 2 : BN;
-            const size_t row_bytes = (size_t)a.k_pack * 2;
+            const size_t row_bytes = (size_t)a.k_pack * (S::F8 ? 1 : 2);
             const int j = u_first % a.tiles_n, q = u_first / a.tiles_n;
             const int users = (min(u_step, num_loop) - 1 - j) / a.tiles_n + 1;
             const size_t slice = (size_t)PF_ROWS * row_bytes;
@@ -511,7 +522,12 @@ __global__ void __maxnreg__(168)
                 const int m0 = (tile / a.tiles_n) * S::BM;
                 const int n0 = (tile % a.tiles_n) * BN;
                 mbar_arrive_expect_tx(ofull + 8u * ob, S::BIAS_BYTES + S::RES_TILE);
-                bulk_load_1d(sBias + ob * S::BIAS_BYTES, a.bias + n0, S::BIAS_BYTES, ofull + 8u * ob);
+                if constexpr (S::F8) {  // bias slice, then the dequantization scales
+                    bulk_load_1d(sBias + ob * S::BIAS_BYTES, a.bias + n0, BN * 4, ofull + 8u * ob);
+                    bulk_load_1d(sBias + ob * S::BIAS_BYTES + BN * 4, a.dq + n0, BN * 4, ofull + 8u * ob);
+                } else {
+                    bulk_load_1d(sBias + ob * S::BIAS_BYTES, a.bias + n0, S::BIAS_BYTES, ofull + 8u * ob);
+                }
                 if constexpr (RES) {
 #pragma unroll
                     for (int j = 0; j < BN / 64; ++j)
@@ -537,7 +553,7 @@ __global__ void __maxnreg__(168)
             auto wait = [&](uint32_t bar, uint32_t parity) -> bool {
                 return mbar_wait(bar, parity, abort_flag, a.err, kErrTimeoutMma);
             };
-            constexpr uint32_t idesc = make_idesc_bf16(S::BM, BN);
+            constexpr uint32_t idesc = S::F8 ? make_idesc_e4m3(S::BM, BN) : make_idesc_bf16(S::BM, BN);
             // Slab operands, in descriptor units (16 bytes): pos_u per slab
             // position (= operand row) and k_u per K16 slice.  TMA-swizzled
             // slabs: rows of ROW_BYTES, a slice 32 bytes on.  Stem slabs (row
@@ -678,10 +694,17 @@ __global__ void __maxnreg__(168)
                         uint64_t bd = bdesc0 + (uint64_t)((slot0 * S::B_BYTES) >> 4);
                         for (int g = 0; g < gn; ++g, ad += (uint64_t)(S::A_BYTES >> 4),
                                  bd += (uint64_t)(S::B_BYTES >> 4)) {
+                            // one MMA per 32 bytes of the k-block row: K = 16
+                            // bf16 values or K = 32 E4M3 codes
 #pragma unroll
-                            for (int k = 0; k < BK / 16; ++k)
-                                mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
-                                            acc | (uint32_t)k);
+                            for (int k = 0; k < S::ROW_BYTES / 32; ++k) {
+                                if constexpr (S::F8)
+                                    mma_f8_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                              acc | (uint32_t)k);
+                                else
+                                    mma_bf16_ss(d_tmem, ad + (uint64_t)(2 * k), bd + (uint64_t)(2 * k), idesc,
+                                                acc | (uint32_t)k);
+                            }
                             acc = 1u;
                         }
                         free_stage(stage);
@@ -933,10 +956,23 @@ __global__ void __maxnreg__(168)
                     asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
                                  : "=f"(b4.x), "=f"(b4.y), "=f"(b4.z), "=f"(b4.w)
                                  : "r"(bias_s + (uint32_t)(ci * 32 + 4 * j) * 4u));
-                    f[4 * j] = __uint_as_float(v[4 * j]) + b4.x;
-                    f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4.y;
-                    f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4.z;
-                    f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4.w;
+                    if constexpr (S::F8) {
+                        // the accumulator is in units of S_x S_w[n]: one fma
+                        // dequantizes and adds the bias
+                        float4 d4;
+                        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                                     : "=f"(d4.x), "=f"(d4.y), "=f"(d4.z), "=f"(d4.w)
+                                     : "r"(bias_s + (uint32_t)(BN + ci * 32 + 4 * j) * 4u));
+                        f[4 * j] = fmaf(__uint_as_float(v[4 * j]), d4.x, b4.x);
+                        f[4 * j + 1] = fmaf(__uint_as_float(v[4 * j + 1]), d4.y, b4.y);
+                        f[4 * j + 2] = fmaf(__uint_as_float(v[4 * j + 2]), d4.z, b4.z);
+                        f[4 * j + 3] = fmaf(__uint_as_float(v[4 * j + 3]), d4.w, b4.w);
+                    } else {
+                        f[4 * j] = __uint_as_float(v[4 * j]) + b4.x;
+                        f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4.y;
+                        f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4.z;
+                        f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4.w;
+                    }
                 }
                 if constexpr (RES) {
                     // residual row `trow`, columns ci*32.. of the 128B-swizzled box ci/2
@@ -977,16 +1013,35 @@ __global__ void __maxnreg__(168)
                     if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
                 }
                 __syncwarp();
+                if (S::F8 && a.out8) {
+                    // a fused Q node: E4M3 codes of f x fp32(1/S), 32 bytes per
+                    // row, rows 32 bytes apart (the unswizzled box of the byte map)
 #pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
-                    const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
-                    const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
-                    const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
-                    const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
-                    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0),
-                                 "r"(w1), "r"(w2), "r"(w3)
-                                 : "memory");
+                    for (int h = 0; h < 2; ++h) {
+                        uint32_t w[4];
+#pragma unroll
+                        for (int k = 0; k < 4; ++k) {
+                            const float *g = f + 16 * h + 4 * k;
+                            w[k] = cvt_e4m3x2(g[0] * a.out_inv, g[1] * a.out_inv) |
+                                   (cvt_e4m3x2(g[2] * a.out_inv, g[3] * a.out_inv) << 16);
+                        }
+                        const uint32_t addr = stg + (uint32_t)lane * 32u + (uint32_t)h * 16u;
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]),
+                                     "r"(w[1]), "r"(w[2]), "r"(w[3])
+                                     : "memory");
+                    }
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
+                        const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
+                        const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
+                        const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
+                        const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
+                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0),
+                                     "r"(w1), "r"(w2), "r"(w3)
+                                     : "memory");
+                    }
                 }
                 if constexpr (S::TSTORE) {
                     // rows past M and columns past N are not written by TMA
@@ -1058,7 +1113,8 @@ static cudaError_t prepare_t() {
                                 cudaFuncAttributeMaxDynamicSharedMemorySize, S::SMEM_BYTES);
 }
 
-// The instantiated (BN, BK, A mode, residual, cluster multicast) combinations.
+// The instantiated (BN, BK, A mode, residual, cluster multicast)
+// combinations; BK = kF8BK (128) are the FP8 ones.
 #define BYOC_GEMM_CONFIGS(X)                 \
     X(32, 64, kAModeTile, false, false)      \
     X(64, 64, kAModeTile, false, false)      \
@@ -1109,7 +1165,19 @@ static cudaError_t prepare_t() {
     X(128, 64, kAModeIm2col, true, true)     \
     X(64, 64, kAModeSlab, false, true)       \
     X(128, 64, kAModeSlab, false, true)      \
-    X(256, 64, kAModeSlab, false, true)
+    X(256, 64, kAModeSlab, false, true)       \
+    X(64, 128, kAModeTile, false, false)      \
+    X(128, 128, kAModeTile, false, false)     \
+    X(256, 128, kAModeTile, false, false)     \
+    X(64, 128, kAModeTile, true, false)       \
+    X(128, 128, kAModeTile, true, false)      \
+    X(64, 128, kAModeIm2col, false, false)    \
+    X(128, 128, kAModeIm2col, false, false)   \
+    X(256, 128, kAModeIm2col, false, false)   \
+    X(128, 128, kAModeIm2col, true, false)    \
+    X(64, 128, kAModeTileSplit, false, false) \
+    X(128, 128, kAModeTileSplit, false, false) \
+    X(256, 128, kAModeTileSplit, false, false)
 
 #define BYOC_GEMM_MATCH(c, BN_, BK_, AM_, RES_, MC_) \
     ((c).bn == BN_ && (c).bk == BK_ && (c).amode == AM_ && (c).res == RES_ && (c).mc == MC_)

@@ -97,6 +97,13 @@ struct GemmArgs {
     const __nv_bfloat16 *residual;    // [M, N] or null
     __nv_bfloat16 *out;               // [M, N]
     int *err;                         // device error word
+    // FP8 GEMM (bk = kF8BK): the accumulator counts code products; column n
+    // is dequantized by dq[n] = S_x S_w[n] before the bias (dq [tiles_n * BN],
+    // zero padded).  out8: a fused Q node -- the output is E4M3 codes of
+    // value x out_inv, written through the byte output map.
+    const float *dq;
+    int out8;
+    float out_inv;
     // measurement only (byoc_trace_begin), else null: [0] earliest CTA's
     // %globaltimer once its wait for the previous kernel returned (atomic
     // min), [1] latest CTA's at exit (atomic max)
@@ -138,10 +145,20 @@ constexpr bool cl_split_fits(int bn, int splits) {
 }
 constexpr bool amode_pair(int m) { return m == kAModeSlabRes2; }
 constexpr bool amode_wres(int m) { return m == kAModeSlabRes || m == kAModeSlabRes2; }
+// FP8 GEMM (E4M3 A and B, kind::f8f6f4): a k-block of 128 codes (128 bytes,
+// the row of one 128-byte swizzle atom, like 64 bf16 values)
+constexpr int kF8BK = 128;
+// whether the epilogue stores its output with TMA (a map over [M, N] in
+// 32 x 32 boxes): tile mode, and every FP8 row-tiled mode (tile, im2col,
+// split-K), whose fused Q node writes E4M3 codes through a byte map
+constexpr bool gemm_tstore(int amode, int bk) {
+    return amode == kAModeTile || (bk == kF8BK && (amode == kAModeIm2col || amode == kAModeTileSplit));
+}
 
 struct GemmConfig {
     int bn;      // tile width in output channels: 32, 64, 128, 256
-    int bk;      // k-block width in elements: 16, 32, 64 (sets the swizzle: 32/64/128 B)
+    int bk;      // k-block width in elements: 16, 32, 64 bf16 (sets the swizzle: 32/64/128 B),
+                 // or kF8BK: an FP8 GEMM (E4M3 operands, 128-byte swizzle)
     int amode;   // AMode
     bool res;    // epilogue adds a residual tile (bn 64 or 128)
     // clusters of two CTAs sharing each weight tile by TMA multicast (tile,
@@ -185,10 +202,11 @@ bool gemm_slab_res_fits(const GemmConfig &cfg, int num_kb, int slab_bytes);
 void gemm_slab_pool(const GemmConfig &cfg, GemmArgs &a);
 cudaError_t gemm_prepare(const GemmConfig &cfg);  // raises the dynamic smem limit
 // tmR: the residual [M, N] bf16 in 64-column x 128-row boxes, 128-byte
-// swizzle (read only when cfg.res).  tmO: in tile mode (kAModeTile), the
-// OUTPUT a.out [M, N] bf16 in 32-column x 32-row boxes, 64-byte swizzle,
-// which the epilogue stores through (required: any other map is written
-// through); unused in the other modes.  a.bias must cover tiles_n * bn floats.
+// swizzle (read only when cfg.res).  tmO: where gemm_tstore(amode, bk), the
+// OUTPUT a.out [M, N] bf16 in 32-column x 32-row boxes, 64-byte swizzle
+// (a.out8: E4M3 codes in 32 x 32-byte boxes, unswizzled), which the epilogue
+// stores through (required: any other map is written through); unused in the
+// other modes.  a.bias (and, FP8, a.dq) must cover tiles_n * bn floats.
 cudaError_t launch_gemm(const GemmConfig &cfg, const CUtensorMap &tmA, const CUtensorMap &tmB,
                         const CUtensorMap &tmR, const CUtensorMap &tmO, const GemmArgs &a, int grid,
                         cudaStream_t st);

@@ -544,11 +544,15 @@ int pick_bn(int64_t tiles_m, int64_t N, int64_t kblocks, int bk, int amode, bool
         GemmConfig c{bn, bk, amode, res};
         if (!byoc::gemm_config_supported(c)) continue;
         const int64_t tiles = tiles_m * ((N + bn - 1) / bn);
-        const double steps = bk / 16.0;  // K16 MMAs per k-block
+        // bytes of one operand row of a k-block: an FP8 k-block (128 codes)
+        // is as many bytes, MMAs (K = 32 each, at twice the K16 rate) and
+        // cycles as a bf16 one of 64 values
+        const int kbytes = bk == byoc::kF8BK ? bk : 2 * bk;
+        const double steps = kbytes / 32.0;  // MMAs per k-block
         const double mma = steps * (bn <= 32 ? 40.0 : bn <= 64 ? 48.0 : bn <= 128 ? 64.0 : 128.0);
         const double reads = steps * (4096.0 + 32.0 * bn);
         const bool slab = amode == byoc::kAModeSlab;
-        const double writes = slab ? 2.0 * bk * bn + slab_kb_bytes : 2.0 * bk * (128.0 + bn);
+        const double writes = slab ? (double)kbytes * bn + slab_kb_bytes : (double)kbytes * (128.0 + bn);
         const double kb = slab ? std::max(mma, (reads + writes) / 118.0)
                                : std::max({mma, (reads + writes) / 145.0, 450.0});
         const double epilogue = 600.0 * std::max(1, bn / 64) * (gelu ? 3.0 : 1.0);
@@ -691,9 +695,11 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         // of the first op after the chain.
         int out8 = 0;
         float out_inv = 0.0f;
-        // (region kernel) a Q node right after the chain is fused: the
-        // epilogue writes E4M3 codes
-        const bool fuse_q = chain_bn > 0 && (op.kind == BYOC_OP_DENSE || op.groups == 1);
+        // a Q node right after the chain is fused: the epilogue writes E4M3
+        // codes (region kernel: after any conv2d / dense; per-composite
+        // kernel: after an FP8 one)
+        const bool fuse_q = chain_bn > 0 ? (op.kind == BYOC_OP_DENSE || op.groups == 1)
+                                         : X.dtype == BYOC_E4M3;
         auto walk_chain = [&](int first, Affine &af, int &cur, int &res, int &act) -> int {
             const int64_t Co = P.tensors[d->ops[first].out].channels();
             af.scale.assign(Co, 1.0);
@@ -753,6 +759,9 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         if (Cout % 8)
             return fail(BYOC_ERR_UNSUPPORTED, "op %d: %lld output channels (multiple of 8 needed)",
                         o, (long long)Cout);
+        if (X.dtype == BYOC_E4M3 && X.channels() % byoc::kF8BK)
+            return fail(BYOC_ERR_UNSUPPORTED, "op %d: FP8 on %lld input channels (whole k-blocks of %d codes)",
+                        o, (long long)X.channels(), byoc::kF8BK);
 
         if (op.kind == BYOC_OP_CONV2D && op.groups > 1) {
             // ---------------- depthwise
@@ -1024,7 +1033,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
                     L.geo = Im2colGeom{(int)X.shape[0], (int)X.shape[1], (int)X.shape[2], (int)C,
                                        kh, kw, op.stride[0], op.stride[1], op.pad[0], op.pad[1],
                                        op.pad[2], op.pad[3], op.dilation[0], op.dilation[1]};
-                    slab = chain_bn == 0 && op.stride[0] == 1 && op.stride[1] == 1 && op.dilation[0] == 1 &&
+                    slab = chain_bn == 0 && X.dtype != BYOC_E4M3 && op.stride[0] == 1 && op.stride[1] == 1 && op.dilation[0] == 1 &&
                            op.dilation[1] == 1 && res < 0 &&
                            slab_geometry((int)X.shape[1], (int)X.shape[2], (int)Y.shape[1],
                                          (int)Y.shape[2], kh, kw, op.pad[0], op.pad[1], op.pad[3],
@@ -1040,12 +1049,13 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         }
         taps = kh * kw;
         bk = op.kind == BYOC_OP_DENSE || chain_bn > 0 ? 64 : pick_bk(C);
-        // an E4M3 input makes an FP8 layer (region kernel only); its k-blocks
-        // hold 128 codes (128 bytes, like 64 bf16 values)
+        // an E4M3 input makes an FP8 layer; its k-blocks hold 128 codes (128
+        // bytes, like 64 bf16 values).  The per-composite kernel takes them
+        // as BK = kF8BK configurations (the region kernel keeps bk = 64 and
+        // switches per stage).
         const bool fp8 = X.dtype == BYOC_E4M3;
-        if (fp8 && chain_bn == 0)
-            return fail(BYOC_ERR_UNSUPPORTED, "op %d: FP8 layers run in the region kernel", o);
-        const int kel = fp8 ? 128 : bk;
+        if (fp8 && chain_bn == 0) bk = byoc::kF8BK;
+        const int kel = fp8 ? byoc::kF8BK : bk;
         chunks = (int)((C + kel - 1) / kel);
         const bool has_res = res >= 0;
         const int amode = slab ? byoc::kAModeSlab : (im2col ? byoc::kAModeIm2col : byoc::kAModeTile);
@@ -1072,7 +1082,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         }
         // Cluster multicast of the weight tiles, on request (tile, im2col and
         // ringed slab modes without split-K; at least two m-tiles to pair)
-        if (chain_bn == 0 && (d->options & BYOC_OPT_MULTICAST) && tiles_m >= 2 && P.num_sms >= 2 &&
+        if (chain_bn == 0 && !fp8 && (d->options & BYOC_OPT_MULTICAST) && tiles_m >= 2 && P.num_sms >= 2 &&
             (L.cfg.amode == byoc::kAModeTile || L.cfg.amode == byoc::kAModeIm2col ||
              L.cfg.amode == byoc::kAModeSlab)) {
             GemmConfig mc = L.cfg;
@@ -1182,7 +1192,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         A.taps = taps;
         A.stem_rows = L.stem_R;
         // a pair unit's k-block is twice the MMA work of a tile's
-        A.group = byoc::gemm_group(byoc::amode_pair(L.cfg.amode) ? 2 * bn : bn, bk,
+        A.group = byoc::gemm_group(byoc::amode_pair(L.cfg.amode) ? 2 * bn : bn, fp8 ? 64 : bk,
                                    amode == byoc::kAModeSlab ? taps : (A.num_kb + splits - 1) / splits);
         byoc::gemm_slab_pool(L.cfg, A);
         A.splits = splits;
@@ -1503,23 +1513,12 @@ bool make_chain(Plan &P, int bn) {
 }
 
 byoc_status plan_region(const byoc_region_desc *d, int num_sms, Plan &P) {
-    bool fp8 = false;
-    if (d && d->abi_version == BYOC_ABI_VERSION && d->tensors)
-        for (int i = 0; i < d->n_tensors; ++i) fp8 |= d->tensors[i].dtype == BYOC_E4M3;
-    if (d && d->abi_version == BYOC_ABI_VERSION && ((d->options & BYOC_OPT_REGION_KERNEL) || fp8)) {
+    if (d && d->abi_version == BYOC_ABI_VERSION && (d->options & BYOC_OPT_REGION_KERNEL)) {
         Plan C;
-        const byoc_status st = plan_region_impl(d, num_sms, C, 128);
-        if (st == BYOC_OK && make_chain(C, 128)) {
+        if (plan_region_impl(d, num_sms, C, 128) == BYOC_OK && make_chain(C, 128)) {
             P = std::move(C);
             return BYOC_OK;
         }
-        // FP8 layers run only in the region kernel
-        if (fp8)
-            return st != BYOC_OK ? st
-                                 : fail(BYOC_ERR_UNSUPPORTED,
-                                        "FP8 region: the region kernel takes 1 to %d conv2d / dense composites "
-                                        "(1x1 or k x k, C %% 128 == 0 on E4M3 inputs) after its Q nodes",
-                                        byoc::kChainMaxStages);
     }
     return plan_region_impl(d, num_sms, P, 0);
 }
@@ -1736,6 +1735,9 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
             L.args.err = h->d_err;
             L.args.w = h->d_const + L.w_off;
             L.args.k_pack = L.k_pack;
+            L.args.dq = L.fp8 ? reinterpret_cast<const float *>(h->d_const + L.dq_off) : nullptr;
+            L.args.out8 = L.out8;
+            L.args.out_inv = L.out_inv;
             if (L.part_bytes) {
                 L.args.partial = reinterpret_cast<float *>(h->d_ws + L.part_off);
                 L.args.counters = reinterpret_cast<unsigned *>(h->d_ws + L.cnt_off);
@@ -1744,10 +1746,14 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
                     return cuda_fail(e, "cudaMemset(split-K counters)");
                 }
             }
-            // multicast: each CTA of a cluster loads half of a weight tile's rows
-            CUresult r = encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
-                                   (uint64_t)L.k_pack, (uint32_t)(L.cfg.mc ? L.cfg.bn / 2 : L.cfg.bn),
-                                   (uint32_t)L.cfg.bk, L.cfg.bk);
+            // multicast: each CTA of a cluster loads half of a weight tile's
+            // rows; FP8: E4M3 codes, 128 per k-block row
+            CUresult r = L.fp8 ? encode_2d_u8(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
+                                              (uint64_t)L.k_pack, (uint32_t)L.cfg.bn, byoc::kF8BK,
+                                              CU_TENSOR_MAP_SWIZZLE_128B)
+                               : encode_2d(&h->tmB[i], h->d_const + L.w_off, (uint64_t)L.n_pad,
+                                           (uint64_t)L.k_pack, (uint32_t)(L.cfg.mc ? L.cfg.bn / 2 : L.cfg.bn),
+                                           (uint32_t)L.cfg.bk, L.cfg.bk);
             if (r != CUDA_SUCCESS) {
                 byoc_release(h);
                 return fail(BYOC_ERR_CUDA, "launch %zu: cuTensorMapEncodeTiled(weights) = %d", i, (int)r);
@@ -2076,6 +2082,14 @@ byoc_status deserialize_plan(const void *src, size_t n, Plan &P) {
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent cluster split-K");
         if (L.kind == BYOC_LAUNCH_GEMM && L.cfg.mc && (L.grid < 2 || L.grid % 2))
             return fail(BYOC_ERR_INVALID_ARG, "serialised plan: multicast launch of an odd grid");
+        if (L.kind == BYOC_LAUNCH_GEMM &&
+            ((L.fp8 != 0) != (L.cfg.bk == byoc::kF8BK) ||
+             (P.tensors[L.x].dtype == BYOC_E4M3) != (L.fp8 != 0) ||
+             (P.tensors[L.y].dtype == BYOC_E4M3) != (L.out8 != 0) ||
+             (L.out8 && !L.fp8) ||
+             (L.fp8 && (L.dq_off + (size_t)L.n_pad * 4 > P.blob.size() ||
+                        L.w_bytes < (size_t)L.n_pad * L.k_pack || L.k_pack % byoc::kF8BK))))
+            return fail(BYOC_ERR_INVALID_ARG, "serialised plan: inconsistent FP8 launch");
         if (L.kind == BYOC_LAUNCH_DEPTHWISE) {
             const byoc::DwArgs &w = L.dw;
             const size_t box = (size_t)w.in_rows * w.in_cols * w.cc * 2;
@@ -2218,7 +2232,11 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                     r = encode_slab(&h->tmA[i], xa, L.geo.N, L.geo.H, L.geo.W, L.geo.C, L.args.wp,
                                     L.slab_rows, L.cfg.bk);
                 else if (L.cfg.amode == byoc::kAModeIm2col)
-                    r = encode_im2col(&h->tmA[i], xa, L.geo, L.cfg.bk);
+                    r = L.fp8 ? encode_im2col(&h->tmA[i], xa, L.geo, 64, true)  // 128 codes per pixel
+                              : encode_im2col(&h->tmA[i], xa, L.geo, L.cfg.bk);
+                else if (L.fp8)
+                    r = encode_2d_u8(&h->tmA[i], xa, (uint64_t)L.aM, (uint64_t)L.aK, byoc::kGemmBM,
+                                     byoc::kF8BK, CU_TENSOR_MAP_SWIZZLE_128B);
                 else
                     r = encode_2d(&h->tmA[i], xa, (uint64_t)L.aM, (uint64_t)L.aK, byoc::kGemmBM,
                                   (uint32_t)L.cfg.bk, L.cfg.bk);
@@ -2240,11 +2258,14 @@ byoc_status byoc_run(byoc_handle *h, const void *const *inputs, void *const *out
                                 i, (int)r);
                 h->tmR_ptr[i] = a.residual;
             }
-            // tile mode stores its output with TMA: [M, N] in 32 x 32 boxes,
-            // 64-byte swizzle (the layout of the epilogue's staging tiles)
-            const bool tstore = L.cfg.amode == byoc::kAModeTile;
+            // tile mode (and FP8) stores its output with TMA: [M, N] in 32 x
+            // 32 boxes, 64-byte swizzle (the layout of the epilogue's staging
+            // tiles); E4M3 codes of a fused Q node: 32 x 32 bytes, unswizzled
+            const bool tstore = byoc::gemm_tstore(L.cfg.amode, L.cfg.bk);
             if (tstore && h->tmO_ptr[i] != a.out) {
-                CUresult r = encode_2d(&h->tmO[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 32);
+                CUresult r = a.out8 ? encode_2d_u8(&h->tmO[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32,
+                                                   CU_TENSOR_MAP_SWIZZLE_NONE)
+                                    : encode_2d(&h->tmO[i], a.out, (uint64_t)a.M, (uint64_t)a.N, 32, 32, 32);
                 if (r != CUDA_SUCCESS)
                     return fail(BYOC_ERR_CUDA, "launch %zu: encoding the output TMA map failed (%d)", i,
                                 (int)r);

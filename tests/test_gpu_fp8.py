@@ -1,6 +1,7 @@
 """Partial quantization (Section 3.2): regions with Q nodes run their
 convolutions / dense layers in FP8 (E4M3 codes on kind::f8f6f4 tensor cores,
-fp32 accumulation) in the region kernel, against the oracle's definition of
+fp32 accumulation), as per-composite GEMM launches (the default) or in the
+region kernel (BYOC_OPT_REGION_KERNEL), against the oracle's definition of
 the quantized chain (oracle/quant.py, oracle/graph.py)."""
 import numpy as np
 import pytest
@@ -31,18 +32,65 @@ def _identity_fp8_conv(N=2, H=9, W=11, C=256, seed=5):
     return g, inp
 
 
+RK = abi.OPT_REGION_KERNEL
+PLANS = {"per_composite": 0, "region_kernel": RK}
+
+
+def _int_fp8(g, seed):
+    """Small-integer weights and inputs, unit-scale batch norm and Q scales of
+    1/16: every code, code product and fp32 sum is exact (multiples of a power
+    of two far below 2^24 ulps), so any correct plan gives the same bits."""
+    rng = np.random.Generator(np.random.PCG64(seed))
+    for n in g.nodes:
+        if n.op in ("nn.conv2d", "nn.dense"):
+            n.consts["weight"] = rng.integers(-1, 2, size=n.attrs["weight_shape"]).astype(np.float32)
+        elif n.op == "nn.batch_norm":
+            C = n.shape[-1]
+            n.consts.update(gamma=np.ones(C, np.float32), beta=rng.integers(-4, 5, C).astype(np.float32),
+                            moving_mean=np.zeros(C, np.float32), moving_var=np.full(C, 1.0 - 1e-5, np.float32))
+        elif n.op == "nn.bias_add":
+            n.consts["bias"] = rng.integers(-4, 5, n.shape[-1]).astype(np.float32)
+        elif n.op == "qnn.quantize":
+            n.attrs["scale"] = 1.0 / 16.0
+    return {k: rng.integers(-2, 3, size=g.shape_of(k)).astype(np.float32) for k in g.inputs}
+
+
 # ------------------------------------------------------------ plans (CPU)
 
 @pytest.mark.parametrize("make,stages", [(lambda: I.fp8_conv(N=1), 1), (lambda: I.fp8_dense(M=64), 1),
                                          (lambda: I.fp8_bottleneck(N=2), 3)])
-def test_fp8_region_plans_a_quantize_launch_and_a_region_kernel(make, stages):
+def test_fp8_region_kernel_plan_is_a_quantize_launch_and_a_region_kernel(make, stages):
     g, _ = make()
-    rep = R.whole_graph_region(g).plan(152)
+    rep = R.whole_graph_region(g, options=RK).plan(152)
     kinds = [rep.kind[i] for i in range(rep.n_launches)]
     assert kinds == [abi.LAUNCH_QUANT, abi.LAUNCH_CHAIN]
     assert rep.stages[1] == stages and rep.fp8[1] == stages
-    blob = R.whole_graph_region(g).plan_serialized(152)
+    blob = R.whole_graph_region(g, options=RK).plan_serialized(152)
     assert [R.load_plan_report(blob).kind[i] for i in range(2)] == kinds
+
+
+@pytest.mark.parametrize("make,gemms", [(lambda: I.fp8_conv(N=1), 1), (lambda: I.fp8_dense(M=64), 1),
+                                        (lambda: I.fp8_bottleneck(N=2), 3)])
+def test_fp8_per_composite_plan_is_a_quantize_launch_and_fp8_gemms(make, gemms):
+    # the leading Q node on the region input is a launch of its own; the Q
+    # nodes after the first two bottleneck convolutions are fused into their
+    # epilogues (E4M3 outputs)
+    g, _ = make()
+    rep = R.whole_graph_region(g).plan(152)
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_QUANT] + [abi.LAUNCH_GEMM] * gemms
+    for i in range(1, rep.n_launches):
+        assert rep.fp8[i] == 1 and rep.tile_k[i] == 128 and rep.multicast[i] == 0
+    blob = R.whole_graph_region(g).plan_serialized(152)
+    back = R.load_plan_report(blob)
+    assert [back.fp8[i] for i in range(back.n_launches)] == [rep.fp8[i] for i in range(rep.n_launches)]
+
+
+def test_fp8_split_k_plans_for_few_tiles():
+    # 2 m-tiles x 12 column tiles of a 3072-deep reduction: the k-blocks are
+    # split over CTAs (global split-K on FP8 k-blocks)
+    g, _ = I.fp8_dense(M=256, D=3072, F=768)
+    rep = R.whole_graph_region(g).plan(152)
+    assert rep.kind[1] == abi.LAUNCH_GEMM and rep.fp8[1] == 1 and rep.splits[1] > 1
 
 
 def test_fp8_regions_the_kernels_do_not_cover_are_rejected_on_the_host():
@@ -68,24 +116,30 @@ def test_fp8_regions_the_kernels_do_not_cover_are_rejected_on_the_host():
 # ------------------------------------------------------------ GPU parity
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("plan", sorted(PLANS))
 @pytest.mark.parametrize("N,H,W,C", [(2, 9, 11, 256), (1, 7, 7, 128), (3, 14, 14, 512)])
-def test_fp8_identity_conv_reproduces_the_quantized_input_bit_for_bit(N, H, W, C):
+def test_fp8_identity_conv_reproduces_the_quantized_input_bit_for_bit(N, H, W, C, plan):
     g, inp = _identity_fp8_conv(N=N, H=H, W=W, C=C)
-    got, cr = run_region(R.whole_graph_region(g), inp)
+    got, cr = run_region(R.whole_graph_region(g, options=PLANS[plan]), inp)
     ref = ograph.evaluate(g, inp)[g.outputs[0]]
     assert_bit_exact(got[g.outputs[0]], ref, f"fp8 identity {N}x{H}x{W}x{C}")
     cr.release()
 
 
+FP8_LAYERS = {
+    "conv3x3": lambda: I.fp8_conv(N=2, H=14, W=14, C=256, K=256, k=3),
+    "conv1x1_ragged": lambda: I.fp8_conv(N=3, H=9, W=10, C=128, K=96, k=1),
+    "dense": lambda: I.fp8_dense(M=200, D=768, F=1024),
+    "dense_split_k": lambda: I.fp8_dense(M=256, D=3072, F=768),
+}
+
+
 @pytest.mark.gpu
-@pytest.mark.parametrize("make", [
-    lambda: I.fp8_conv(N=2, H=14, W=14, C=256, K=256, k=3),
-    lambda: I.fp8_conv(N=3, H=9, W=10, C=128, K=96, k=1),
-    lambda: I.fp8_dense(M=200, D=768, F=1024),
-])
-def test_fp8_layer_matches_the_oracle(make):
-    g, inp = make()
-    got, cr = run_region(R.whole_graph_region(g), inp)
+@pytest.mark.parametrize("plan", sorted(PLANS))
+@pytest.mark.parametrize("name", sorted(FP8_LAYERS))
+def test_fp8_layer_matches_the_oracle(name, plan):
+    g, inp = FP8_LAYERS[name]()
+    got, cr = run_region(R.whole_graph_region(g, options=PLANS[plan]), inp)
     ref, sc = oracle(g, inp)
     o = g.outputs[0]
     assert_close(got[o], ref[o], sc[o], g.name)
@@ -93,13 +147,14 @@ def test_fp8_layer_matches_the_oracle(make):
 
 
 @pytest.mark.gpu
+@pytest.mark.parametrize("plan", sorted(PLANS))
 @pytest.mark.parametrize("N", [2, 32])
-def test_fp8_bottleneck_matches_the_oracle(N):
+def test_fp8_bottleneck_matches_the_oracle(N, plan):
     # config 4 with Q nodes before each convolution: the intermediates t1, t2
     # leave their epilogues as E4M3 codes (fused Q nodes)
     g, inp = I.fp8_bottleneck(N=N)
-    got, cr = run_region(R.whole_graph_region(g), inp)
-    assert cr.n_launches == 2
+    got, cr = run_region(R.whole_graph_region(g, options=PLANS[plan]), inp)
+    assert cr.n_launches == (2 if plan == "region_kernel" else 4)
     ref, sc = oracle(g, inp)
     o = g.outputs[0]
     _, _, literal = assert_close(got[o], ref[o], sc[o], g.name)
@@ -113,3 +168,18 @@ def test_fp8_bottleneck_matches_the_oracle(N):
     print(f"fp8 bottleneck N={N}: relative L2 error against the unquantized region {rel:.4f}")
     assert rel < 0.1
     cr.release()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["bottleneck"] + sorted(FP8_LAYERS))
+def test_fp8_per_composite_equals_the_region_kernel_on_small_integers(name):
+    # the two kernels issue different tile shapes (and split-K) over the same
+    # codes; with exact sums and the same epilogue arithmetic the bits agree
+    g, _ = I.fp8_bottleneck(N=2) if name == "bottleneck" else FP8_LAYERS[name]()
+    inp = _int_fp8(g, seed=len(name))
+    pc, c1 = run_region(R.whole_graph_region(g), inp)
+    rk, c2 = run_region(R.whole_graph_region(g, options=RK), inp)
+    for o in g.outputs:
+        assert np.array_equal(pc[o].view(np.uint32), rk[o].view(np.uint32)), o
+    c1.release()
+    c2.release()
