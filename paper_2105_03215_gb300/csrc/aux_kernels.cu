@@ -644,29 +644,44 @@ cudaError_t launch_avgpool(const __nv_bfloat16 *x, __nv_bfloat16 *y, int N, int 
 namespace byoc {
 
 // ------------------------------------------------------------ Q node (Section 3.2)
-// Eight elements per thread per step: one 16-byte load of bf16, eight fp32
-// products with 1/S, four paired conversions to E4M3, one 8-byte store.
+// Eight elements per thread per 16-byte piece: one load of bf16, eight fp32
+// products with 1/S, four paired conversions to E4M3, one 8-byte store.  A
+// thread issues the loads of four pieces (a grid stride apart) before
+// converting any, so that each SM keeps enough bytes in flight to stream HBM.
 __global__ void __launch_bounds__(256) quantize_e4m3_kernel(const __nv_bfloat16 *__restrict__ x,
                                                             uint8_t *__restrict__ q, size_t n8, float inv) {
     pdl_launch_dependents();
     pdl_wait();
-    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n8; i += (size_t)gridDim.x * blockDim.x) {
-        const uint4 v = __ldg(reinterpret_cast<const uint4 *>(x) + i);
-        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-        uint32_t p[4];
+    constexpr int U = 4;
+    const size_t stride = (size_t)gridDim.x * blockDim.x;
+    for (size_t i0 = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i0 < n8; i0 += U * stride) {
+        uint4 v[U];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) p[k] = cvt_e4m3x2(bf16lo(w[k]) * inv, bf16hi(w[k]) * inv);
-        uint2 o;
-        o.x = p[0] | (p[1] << 16);
-        o.y = p[2] | (p[3] << 16);
-        reinterpret_cast<uint2 *>(q)[i] = o;
+        for (int u = 0; u < U; ++u) {
+            const size_t i = i0 + (size_t)u * stride;
+            v[u] = i < n8 ? __ldg(reinterpret_cast<const uint4 *>(x) + i) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const size_t i = i0 + (size_t)u * stride;
+            if (i >= n8) break;
+            const uint32_t w[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+            uint32_t p[4];
+#pragma unroll
+            for (int k = 0; k < 4; ++k) p[k] = cvt_e4m3x2(bf16lo(w[k]) * inv, bf16hi(w[k]) * inv);
+            uint2 o;
+            o.x = p[0] | (p[1] << 16);
+            o.y = p[2] | (p[3] << 16);
+            reinterpret_cast<uint2 *>(q)[i] = o;
+        }
     }
 }
 
+// One wave: up to 8 CTAs of 256 threads per SM, each thread 4 pieces per pass.
 cudaError_t launch_quantize_e4m3(const __nv_bfloat16 *x, uint8_t *q, size_t n, float inv_scale, int num_sms,
                                  cudaStream_t st) {
     const size_t n8 = n / 8;
-    const size_t blocks = (n8 + 255) / 256;
+    const size_t blocks = (n8 + 4 * 256 - 1) / (4 * 256);
     const int grid = (int)(blocks < (size_t)num_sms * 8 ? blocks : (size_t)num_sms * 8);
     return launch_pdl(quantize_e4m3_kernel, dim3(grid > 0 ? grid : 1), dim3(256), 0, st, x, q, n8, inv_scale);
 }
