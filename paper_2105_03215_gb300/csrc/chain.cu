@@ -62,7 +62,7 @@ struct ChainShape {
     static constexpr int USLOTS = 4;  // unit broadcast ring
     static constexpr int NUM_BARS = 2 * STAGES + 4 + 2 * USLOTS + 1;
     static constexpr int TMEM_COLS = 2 * BN;
-    static_assert(8 * NUM_BARS + 16 + 4 * USLOTS <= CTRL_BYTES, "control block");
+    static_assert(8 * NUM_BARS + 16 + 8 * USLOTS <= CTRL_BYTES && USLOTS <= 4, "control block");
     static_assert(STAGES >= 2, "ring depth");
     static_assert(SMEM_BYTES <= 232448, "shared memory budget");
     static_assert(BN == 128 || BN == 256, "BN");
@@ -155,7 +155,8 @@ __global__ void __maxnreg__(168)
     const uint32_t drain = uempty + 8u * S::USLOTS;
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + (ctrl - base) + 8 * S::NUM_BARS);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tmem_slot + 1);
-    volatile int *unit_ids = reinterpret_cast<volatile int *>(tmem_slot + 4);
+    volatile int *unit_ids = reinterpret_cast<volatile int *>(tmem_slot + 4);    // USLOTS
+    volatile int *unit_codes = reinterpret_cast<volatile int *>(tmem_slot + 8);  // USLOTS: order[u]
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -197,11 +198,14 @@ __global__ void __maxnreg__(168)
     if (a.trace != nullptr && threadIdx.x == 32) atomicMin(a.trace, globaltimer_ns());
 
     // Wait for a unit broadcast slot t and read its unit id (-1: no more
-    // units); every reader arrives on the slot's empty barrier once.
-    auto read_unit = [&](int t, int code, bool &ok) -> int {
+    // units) and code (stage << 24 | tile); every reader arrives on the
+    // slot's empty barrier once.
+    auto read_unit = [&](int t, int err_code, bool &ok, int &ucode) -> int {
         const int slot = t % S::USLOTS;
-        ok = mbar_wait(ufull + 8u * slot, (uint32_t)(t / S::USLOTS) & 1u, abort_flag, a.err, code);
-        return ok ? unit_ids[slot] : -1;
+        ok = mbar_wait(ufull + 8u * slot, (uint32_t)(t / S::USLOTS) & 1u, abort_flag, a.err, err_code);
+        if (!ok) return -1;
+        ucode = unit_codes[slot];
+        return unit_ids[slot];
     };
 
     if (warp == 0) {
@@ -214,10 +218,10 @@ __global__ void __maxnreg__(168)
             uint32_t phase = 0;
             bool ok = true;
             for (int t = 0; ok; ++t) {
-                const int u = read_unit(t, kErrTimeoutProducer, ok);
+                int code = 0;
+                const int u = read_unit(t, kErrTimeoutProducer, ok, code);
                 if (ok) mbar_arrive(uempty + 8u * (t % S::USLOTS));
                 if (u < 0) break;
-                const int code = a.order[u];
                 const int si = code >> 24;
                 const ChainStage &cs = a.st[si];
                 const int tile = code & 0xFFFFFF;
@@ -282,22 +286,49 @@ __global__ void __maxnreg__(168)
         // the publication (mbarrier release / acquire), so after the acquire.
         if (elect_one()) {
             const unsigned run = ld_acquire_gpu(a.ctl + 2);
-            // The next unit's counters are polled (loads issued) as soon as
-            // the current unit is published, so their latency overlaps the
-            // CTA's work instead of adding to every unit.
-            int idx = a.cta_off[blockIdx.x];
-            const int end = a.cta_off[blockIdx.x + 1];
-            constexpr int kPoll = 4;
-            unsigned pv[kPoll];
-            auto issue_polls = [&](int u) {
-                if (u < 0) return;
-                const int j0 = a.dep_off[u], n = min(a.dep_off[u + 1] - j0, kPoll);
+            // This CTA's unit records are read one ahead (the record after
+            // the current unit loads while the current one is handled), and
+            // a unit's dependency counters are polled (loads issued) as soon
+            // as the unit before it is published, so that neither latency
+            // adds to every unit.  Record: {u, code, n, dep_off[u]},
+            // {counter, count} x kChainRecDeps.
+            static_assert(kChainRecInts == 12 && kChainRecDeps == 4, "record layout");
+            const int r0 = a.cta_off[blockIdx.x], r1 = a.cta_off[blockIdx.x + 1];
+            const int4 *recs = reinterpret_cast<const int4 *>(a.cta_rec);
+            int4 cur[3], nxt[3];
+            auto load_rec = [&](int k, int4 (&r)[3]) {
+                if (r0 + k < r1) {
 #pragma unroll
-                for (int k = 0; k < kPoll; ++k)
-                    if (k < n) pv[k] = ld_relaxed_gpu(a.flags + a.dep_list[2 * (j0 + k)]);
+                    for (int q = 0; q < 3; ++q) r[q] = __ldg(recs + (size_t)(r0 + k) * 3 + q);
+                } else {
+                    r[0] = make_int4(-1, 0, 0, 0);
+                    r[1] = r[2] = make_int4(0, 0, 0, 0);
+                }
             };
-            int u = idx < end ? a.cta_list[idx] : -1;
-            issue_polls(u);
+            unsigned pv[kChainRecDeps];
+            auto issue_polls = [&](const int4 (&r)[3]) {
+                const int n = r[0].z;
+                if (r[0].x < 0 || n <= 0) return;
+                pv[0] = ld_relaxed_gpu(a.flags + r[1].x);
+                if (n > 1) pv[1] = ld_relaxed_gpu(a.flags + r[1].z);
+                if (n > 2) pv[2] = ld_relaxed_gpu(a.flags + r[2].x);
+                if (n > 3) pv[3] = ld_relaxed_gpu(a.flags + r[2].z);
+            };
+            // every polled counter has reached its count for this launch
+            // (units with more dependencies than a record holds: wait_deps)
+            auto polled_ready = [&](const int4 (&r)[3]) -> bool {
+                const int n = r[0].z;
+                if (n > kChainRecDeps) return false;
+                const unsigned k1 = run + 1u;
+                bool ready = (int)(pv[0] - (unsigned)r[1].y * k1) >= 0;
+                if (n > 1) ready = ready && (int)(pv[1] - (unsigned)r[1].w * k1) >= 0;
+                if (n > 2) ready = ready && (int)(pv[2] - (unsigned)r[2].y * k1) >= 0;
+                if (n > 3) ready = ready && (int)(pv[3] - (unsigned)r[2].w * k1) >= 0;
+                return ready;
+            };
+            load_rec(0, cur);
+            load_rec(1, nxt);
+            issue_polls(cur);
             int t = 0;
             bool ok = true;
             for (;; ++t) {
@@ -307,14 +338,9 @@ __global__ void __maxnreg__(168)
                     ok = false;
                     break;
                 }
-                if (u >= 0 && a.dep_off[u + 1] > a.dep_off[u]) {
-                    const int j0 = a.dep_off[u], n = a.dep_off[u + 1] - j0;
-                    bool ready = n <= kPoll;
-#pragma unroll
-                    for (int k = 0; k < kPoll; ++k)
-                        if (k < n && (int)(pv[k] - (unsigned)a.dep_list[2 * (j0 + k) + 1] * (run + 1u)) < 0)
-                            ready = false;
-                    if (!ready && !wait_deps(a, u, run, abort_flag)) {
+                const int u = cur[0].x;
+                if (u >= 0 && cur[0].z > 0) {
+                    if (!polled_ready(cur) && !wait_deps(a, u, run, abort_flag)) {
                         ok = false;
                         break;
                     }
@@ -322,11 +348,13 @@ __global__ void __maxnreg__(168)
                     fence_proxy_async_global();
                 }
                 unit_ids[slot] = u;
+                unit_codes[slot] = cur[0].y;
                 mbar_arrive(ufull + 8u * slot);
                 if (u < 0) break;
-                ++idx;
-                u = idx < end ? a.cta_list[idx] : -1;
-                issue_polls(u);
+#pragma unroll
+                for (int q = 0; q < 3; ++q) cur[q] = nxt[q];
+                issue_polls(cur);
+                load_rec(t + 2, nxt);
             }
             (void)ok;
         }
@@ -345,10 +373,11 @@ __global__ void __maxnreg__(168)
             uint32_t phase = 0;
             bool ok = true;
             for (int t = 0; ok; ++t) {
-                const int u = read_unit(t, kErrTimeoutMma, ok);
+                int code = 0;
+                const int u = read_unit(t, kErrTimeoutMma, ok, code);
                 if (ok) mbar_arrive(uempty + 8u * (t % S::USLOTS));
                 if (u < 0) break;
-                const ChainStage &cs = a.st[a.order[u] >> 24];
+                const ChainStage &cs = a.st[code >> 24];
                 const int buf = t & 1;
                 if (!wait(tempty + 8u * buf, (((uint32_t)(t >> 1)) & 1u) ^ 1u)) {
                     ok = false;
@@ -402,11 +431,11 @@ __global__ void __maxnreg__(168)
         const uint32_t sw_own = ((uint32_t)lane >> 1) & 3u;
         for (int t = 0;; ++t) {
             bool ok;
-            int u = read_unit(t, kErrTimeoutEpilogue, ok);
+            int code = 0;
+            int u = read_unit(t, kErrTimeoutEpilogue, ok, code);
             __syncwarp();
             if (ok && lane == 0) mbar_arrive(uempty + 8u * (t % S::USLOTS));
             if (u < 0) break;
-            const int code = a.order[u];
             const int si = code >> 24;
             const ChainStage &cs = a.st[si];
             const int tile = code & 0xFFFFFF;
@@ -427,6 +456,18 @@ __global__ void __maxnreg__(168)
                 for (int q = 0; q < 4; ++q) rn[q] = ld_cg_v4(rp + 8 * q);
             };
             if (has_res && grp < nch) load_res(grp);
+            // this warp's chunks' bias (and FP8 dequantization scales), one
+            // column per lane, loaded before the accumulator is ready; lane j
+            // hands column j to the others by shuffle (both arrays are zero
+            // padded to tiles_n x BN)
+            constexpr int KC = S::NCH / 2;  // chunks per warp
+            float bl[KC], dl[KC];
+#pragma unroll
+            for (int k = 0; k < KC; ++k) {
+                const int c = n0 + (grp + 2 * k) * 32 + lane;
+                bl[k] = __ldg(cs.bias + c);
+                dl[k] = cs.fp8 ? __ldg(cs.dq + c) : 0.0f;
+            }
             if (!mbar_wait(tfull + 8u * buf, ((uint32_t)(t >> 1)) & 1u, abort_flag, a.err, kErrTimeoutEpilogue))
                 break;
             tc_fence_after();
@@ -436,27 +477,15 @@ __global__ void __maxnreg__(168)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(tempty + 8u * buf);
             }
-            for (int ci = grp; ci < nch; ci += 2) {
+#pragma unroll
+            for (int k = 0; k < KC; ++k) {
+                const int ci = grp + 2 * k;
+                if (ci >= nch) break;
                 const int col0 = n0 + ci * 32;
                 uint4 rr[4];
 #pragma unroll
                 for (int q = 0; q < 4; ++q) rr[q] = rn[q];
                 if (has_res && ci + 2 < nch) load_res(ci + 2);
-                // the chunk's bias (and FP8 dequantization scales): the same 128
-                // bytes in every lane, loaded while the TMEM load is in flight
-                float4 b4[8];
-                {
-                    const float4 *bp = reinterpret_cast<const float4 *>(cs.bias + col0);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) b4[q] = __ldg(bp + q);
-                }
-                // FP8: the accumulator is in units of S_x S_w[n] (dequantization scales)
-                float4 d4[8];
-                if (cs.fp8) {
-                    const float4 *dp = reinterpret_cast<const float4 *>(cs.dq + col0);
-#pragma unroll
-                    for (int q = 0; q < 8; ++q) d4[q] = __ldg(dp + q);
-                }
                 uint32_t v[32];
                 tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
                 if (ci + 2 >= nch) {  // this warp's last read of the accumulator
@@ -466,21 +495,14 @@ __global__ void __maxnreg__(168)
                 }
                 float f[32];
                 if (cs.fp8) {
+                    // FP8: the accumulator is in units of S_x S_w[n]
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        f[4 * j] = fmaf(__uint_as_float(v[4 * j]), d4[j].x, b4[j].x);
-                        f[4 * j + 1] = fmaf(__uint_as_float(v[4 * j + 1]), d4[j].y, b4[j].y);
-                        f[4 * j + 2] = fmaf(__uint_as_float(v[4 * j + 2]), d4[j].z, b4[j].z);
-                        f[4 * j + 3] = fmaf(__uint_as_float(v[4 * j + 3]), d4[j].w, b4[j].w);
-                    }
+                    for (int j = 0; j < 32; ++j)
+                        f[j] = fmaf(__uint_as_float(v[j]), __shfl_sync(0xffffffffu, dl[k], j),
+                                    __shfl_sync(0xffffffffu, bl[k], j));
                 } else {
 #pragma unroll
-                    for (int j = 0; j < 8; ++j) {
-                        f[4 * j] = __uint_as_float(v[4 * j]) + b4[j].x;
-                        f[4 * j + 1] = __uint_as_float(v[4 * j + 1]) + b4[j].y;
-                        f[4 * j + 2] = __uint_as_float(v[4 * j + 2]) + b4[j].z;
-                        f[4 * j + 3] = __uint_as_float(v[4 * j + 3]) + b4[j].w;
-                    }
+                    for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]) + __shfl_sync(0xffffffffu, bl[k], j);
                 }
                 if (has_res) {
 #pragma unroll

@@ -314,6 +314,13 @@ cudaError_t launch_dwpw(const CUtensorMap &tmX, const CUtensorMap &tmB, const Dw
 // epilogue warps of each of its units adds 1 per launch.
 constexpr int kChainMaxStages = 4;
 enum : int { kChainTile = 0, kChainIm2col = 1 };
+// A CTA's schedule entry (cta_rec): kChainRecInts int32 -- the unit u, its
+// code order[u], its dependency count n, its first dependency pair
+// dep_off[u], then its first min(n, kChainRecDeps) (counter, count per
+// launch) pairs -- so that the scheduler reads one self-contained, 16-byte
+// aligned record per unit instead of a chain of dependent loads.
+constexpr int kChainRecDeps = 4;
+constexpr int kChainRecInts = 4 + 2 * kChainRecDeps;
 // (Both structs are laid out without implicit padding: plans are serialised
 // byte for byte.)
 struct ChainStage {
@@ -338,8 +345,8 @@ struct ChainStage {
 struct ChainArgs {
     ChainStage st[kChainMaxStages];
     const int *order;        // [total_units]: (stage << 24) | tile of the u-th unit
-    const int *cta_off;      // [grid + 1]: CTA b runs units cta_list[cta_off[b] .. cta_off[b+1]), in order
-    const int *cta_list;
+    const int *cta_off;      // [grid + 1]: CTA b runs the units of records cta_off[b] .. cta_off[b+1]), in order
+    const int *cta_rec;      // [total_units * kChainRecInts]: the records, CTA after CTA
     const int *dep_off;      // [total_units + 1]: unit u's dependencies are the pairs
     const int *dep_list;     //   (counter, count per launch) at dep_list[2 j], j in [dep_off[u], dep_off[u+1])
     unsigned *flags;         // [n_counters] completion counters, zeroed at compile

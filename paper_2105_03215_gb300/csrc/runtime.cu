@@ -290,7 +290,7 @@ struct LaunchPlan {
     int c_npad[byoc::kChainMaxStages] = {}, c_kpack[byoc::kChainMaxStages] = {};
     size_t cw_off[byoc::kChainMaxStages] = {}, cb_off[byoc::kChainMaxStages] = {};
     size_t order_off = 0, dep_off_off = 0, dep_list_off = 0;  // constant blob: int32 unit order, dependencies
-    size_t cta_off_off = 0, cta_list_off = 0;                 // constant blob: int32 per-CTA unit lists
+    size_t cta_off_off = 0, cta_rec_off = 0;                  // constant blob: int32 per-CTA unit records
     size_t c_dq_off[byoc::kChainMaxStages] = {};
     // FP8 GEMM (region kernel only): A and B are E4M3 codes; dq = [n_pad] fp32
     // dequantization scales S_x S_w[n] in the constant blob
@@ -1473,16 +1473,27 @@ bool make_chain(Plan &P, int bn) {
         off.push_back((int32_t)(list.size() / 2));
     }
     if (list.empty()) list.assign(2, 0);  // keeps the blob offset valid; never read
-    // each CTA's units, in the global order
-    std::vector<int32_t> cta_off(grid + 1, 0), cta_list(units);
+    // each CTA's units, in the global order, as records (unit, code,
+    // dependency count, first dependency, the first kChainRecDeps pairs)
+    std::vector<int32_t> cta_off(grid + 1, 0), cta_rec((size_t)units * byoc::kChainRecInts, 0);
     for (int i = 0; i < units; ++i) cta_off[ord_cta[i] + 1]++;
     for (int b = 0; b < grid; ++b) cta_off[b + 1] += cta_off[b];
     {
         std::vector<int32_t> fill(cta_off.begin(), cta_off.end() - 1);
-        for (int i = 0; i < units; ++i) cta_list[fill[ord_cta[i]]++] = i;
+        for (int i = 0; i < units; ++i) {
+            int32_t *r = &cta_rec[(size_t)fill[ord_cta[i]]++ * byoc::kChainRecInts];
+            r[0] = i;
+            r[1] = order[i];
+            r[2] = off[i + 1] - off[i];
+            r[3] = off[i];
+            for (int k = 0; k < std::min(r[2], byoc::kChainRecDeps); ++k) {
+                r[4 + 2 * k] = list[2 * (off[i] + k)];
+                r[5 + 2 * k] = list[2 * (off[i] + k) + 1];
+            }
+        }
     }
     C.cta_off_off = blob_append(P.blob, cta_off.data(), cta_off.size() * 4);
-    C.cta_list_off = blob_append(P.blob, cta_list.data(), cta_list.size() * 4);
+    C.cta_rec_off = blob_append(P.blob, cta_rec.data(), cta_rec.size() * 4);
     C.order_off = blob_append(P.blob, order.data(), order.size() * 4);
     C.dep_off_off = blob_append(P.blob, off.data(), off.size() * 4);
     C.dep_list_off = blob_append(P.blob, list.data(), list.size() * 4);
@@ -1803,7 +1814,7 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
             }
             A.order = reinterpret_cast<const int *>(h->d_const + L.order_off);
             A.cta_off = reinterpret_cast<const int *>(h->d_const + L.cta_off_off);
-            A.cta_list = reinterpret_cast<const int *>(h->d_const + L.cta_list_off);
+            A.cta_rec = reinterpret_cast<const int *>(h->d_const + L.cta_rec_off);
             A.dep_off = reinterpret_cast<const int *>(h->d_const + L.dep_off_off);
             A.dep_list = reinterpret_cast<const int *>(h->d_const + L.dep_list_off);
             A.ctl = reinterpret_cast<unsigned *>(h->d_ws + L.flags_off);
@@ -1848,7 +1859,7 @@ byoc_status instantiate(byoc_handle *h, byoc_handle **out) {
 static_assert(std::is_trivially_copyable<LaunchPlan>::value && std::is_trivially_copyable<TensorInfo>::value,
               "launch records are stored byte for byte");
 constexpr char kPlanMagic[8] = {'B', 'Y', 'O', 'C', 'P', 'L', 'N', '1'};
-constexpr uint32_t kPlanFormat = 2;
+constexpr uint32_t kPlanFormat = 3;
 
 uint64_t fnv1a(const uint8_t *p, size_t n, uint64_t h = 1469598103934665603ull) {
     for (size_t i = 0; i < n; ++i) {
@@ -1980,20 +1991,26 @@ bool chain_plan_ok(const Plan &P, const LaunchPlan &L) {
     for (int i = 0; i < units; ++i)
         for (int j = off[i]; j < off[i + 1]; ++j)
             if (done_at[list[2 * j]] >= i) { g_chain_bad = 12; return false; }
-    // per-CTA lists: a partition of the units, each list in the global order
+    // per-CTA records: a partition of the units, each CTA's in the global
+    // order, each record a copy of its unit's code and dependencies
     if (L.grid < 1 || L.grid > units || L.cta_off_off + 4 * ((size_t)L.grid + 1) > P.blob.size() ||
-        L.cta_list_off + 4 * (size_t)units > P.blob.size())
+        L.cta_rec_off % 16 || L.cta_rec_off + 4 * (size_t)units * byoc::kChainRecInts > P.blob.size())
         { g_chain_bad = 17; return false; }
     const int32_t *coff = reinterpret_cast<const int32_t *>(P.blob.data() + L.cta_off_off);
-    const int32_t *clist = reinterpret_cast<const int32_t *>(P.blob.data() + L.cta_list_off);
+    const int32_t *crec = reinterpret_cast<const int32_t *>(P.blob.data() + L.cta_rec_off);
     if (coff[0] != 0 || coff[L.grid] != units) { g_chain_bad = 18; return false; }
     std::fill(seen.begin(), seen.end(), 0);
     for (int b = 0; b < L.grid; ++b) {
         if (coff[b + 1] < coff[b]) { g_chain_bad = 19; return false; }
         for (int k = coff[b]; k < coff[b + 1]; ++k) {
-            const int i = clist[k];
-            if (i < 0 || i >= units || seen[i] || (k > coff[b] && clist[k - 1] >= i)) { g_chain_bad = 20; return false; }
+            const int32_t *r = crec + (size_t)k * byoc::kChainRecInts;
+            const int i = r[0];
+            if (i < 0 || i >= units || seen[i] || (k > coff[b] && r[-byoc::kChainRecInts] >= i)) { g_chain_bad = 20; return false; }
             seen[i] = 1;
+            if (r[1] != order[i] || r[2] != off[i + 1] - off[i] || r[3] != off[i]) { g_chain_bad = 22; return false; }
+            for (int q = 0; q < std::min(r[2], byoc::kChainRecDeps); ++q)
+                if (r[4 + 2 * q] != list[2 * (off[i] + q)] || r[5 + 2 * q] != list[2 * (off[i] + q) + 1])
+                    { g_chain_bad = 22; return false; }
         }
     }
     return true;
