@@ -2,6 +2,7 @@
 
   python profile_region.py --workload resnet50 --batch 64 --region 5
   python profile_region.py --workload mbv2_dw_pw --reps 5 --time
+  python profile_region.py --workload fp8_bottleneck --reps 5 --time
 
 ``--region i`` picks the i-th region of ResNet-50 partitioned one composite
 per region; the other workloads run as a single region.  Inputs are random
@@ -24,7 +25,8 @@ if ROOT not in sys.path:
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--workload", default="resnet50",
-                    choices=["resnet50", "conv3x3", "bert_ffn", "mbv2_dw_pw", "mbv2_dw", "bottleneck"])
+                    choices=["resnet50", "conv3x3", "bert_ffn", "mbv2_dw_pw", "mbv2_dw", "bottleneck",
+                             "fp8_bottleneck"])
     ap.add_argument("--batch", type=int, default=64)
     ap.add_argument("--n", type=int, default=None,
                     help="batch of the other workloads (default: the workload's own)")
@@ -78,7 +80,8 @@ def main():
                 "bert_ffn": lambda: I.bert_ffn(seed=1),
                 "mbv2_dw_pw": lambda: I.mbv2_dw_pw(seed=2, **nk),
                 "mbv2_dw": lambda: I.mbv2_dw_pw(seed=2, **nk),
-                "bottleneck": lambda: I.resnet_bottleneck(seed=3, **nk)}[args.workload]()
+                "bottleneck": lambda: I.resnet_bottleneck(seed=3, **nk),
+                "fp8_bottleneck": lambda: I.fp8_bottleneck(seed=3, **nk)}[args.workload]()
         if args.workload == "mbv2_dw":
             reg = R.Region(g, [n.name for n in g.nodes[:3]], "mbv2_dw")
         else:
