@@ -183,3 +183,86 @@ def test_fp8_per_composite_equals_the_region_kernel_on_small_integers(name):
         assert np.array_equal(pc[o].view(np.uint32), rk[o].view(np.uint32)), o
     c1.release()
     c2.release()
+
+
+# ------------------------------------------------------------ more FP8 shapes
+
+def _fp8_conv_residual(N=2, H=14, W=14, C=128, seed=41):
+    """Q(x) -> 3x3 conv -> BN -> + x -> ReLU: the im2col mode with a bf16 residual tile."""
+    b = I._Builder("fp8_conv3x3_residual")
+    x = b.input("x", (N, H, W, C))
+    y = b.relu(b.add(b.batch_norm(b.conv2d(b.quantize(x, I.FP8_SCALE_INPUT), C, 3)), x))
+    return I._finish(b, [y], seed)
+
+
+def _fp8_conv_stride2(N=2, H=15, W=15, C=256, K=128, seed=42):
+    """Q(x) -> 3x3 stride-2 conv -> BN -> ReLU (im2col with a stride, ragged last m-tile)."""
+    b = I._Builder("fp8_conv3x3_s2")
+    x = b.input("x", (N, H, W, C))
+    y = b.relu(b.batch_norm(b.conv2d(b.quantize(x, I.FP8_SCALE_INPUT), K, 3, stride=2)))
+    return I._finish(b, [y], seed)
+
+
+def _fp8_mlp(M=256, D=3072, F=768, U=256, seed=43):
+    """Q(x) -> dense (split-K) + bias + ReLU -> Q -> dense + bias: the first
+    layer's split-K epilogue writes the E4M3 codes the second one reads."""
+    b = I._Builder("fp8_mlp")
+    x = b.input("x", (M, D))
+    h = b.relu(b.bias_add(b.dense(b.quantize(x, I.FP8_SCALE_INPUT), F)))
+    y = b.bias_add(b.dense(b.quantize(h, I.FP8_SCALE_HIDDEN), U))
+    return I._finish(b, [y], seed)
+
+
+def _fp8_two_readers(N=2, H=9, W=11, C=128, seed=44):
+    """t = ReLU(BN(conv1x1(Q(x)))) is a region output and also feeds Q -> conv:
+    its Q node cannot be fused into the producing epilogue (a quantize launch)."""
+    b = I._Builder("fp8_two_readers")
+    x = b.input("x", (N, H, W, C))
+    t = b.relu(b.batch_norm(b.conv2d(b.quantize(x, I.FP8_SCALE_INPUT), C, 1)))
+    y = b.batch_norm(b.conv2d(b.quantize(t, I.FP8_SCALE_HIDDEN), C, 1))
+    return I._finish(b, [t, y], seed)
+
+
+MORE = {"conv3x3_residual": _fp8_conv_residual, "conv3x3_stride2": _fp8_conv_stride2,
+        "mlp_split_k_q": _fp8_mlp, "two_readers": _fp8_two_readers}
+
+
+def test_fp8_more_plans():
+    rep = R.whole_graph_region(_fp8_conv_residual()[0]).plan(152)
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_QUANT, abi.LAUNCH_GEMM]
+    assert rep.im2col[1] == 1 and rep.residual[1] >= 0 and rep.fp8[1] == 1
+    rep = R.whole_graph_region(_fp8_conv_stride2()[0]).plan(152)
+    assert rep.im2col[1] == 1 and rep.fp8[1] == 1
+    # the hidden Q node is fused into the split-K layer's epilogue: no second quantize launch
+    rep = R.whole_graph_region(_fp8_mlp()[0]).plan(152)
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_QUANT, abi.LAUNCH_GEMM, abi.LAUNCH_GEMM]
+    assert rep.splits[1] > 1 and rep.fp8[1] == 1 and rep.fp8[2] == 1
+    # t is an output: its Q node is a launch of its own
+    rep = R.whole_graph_region(_fp8_two_readers()[0]).plan(152)
+    assert [rep.kind[i] for i in range(rep.n_launches)] == [abi.LAUNCH_QUANT, abi.LAUNCH_GEMM, abi.LAUNCH_QUANT,
+                                                            abi.LAUNCH_GEMM]
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", sorted(MORE))
+def test_fp8_more_shapes_match_the_oracle(name):
+    g, inp = MORE[name]()
+    got, cr = run_region(R.whole_graph_region(g), inp)
+    ref, sc = oracle(g, inp)
+    for o in g.outputs:
+        assert_close(got[o], ref[o], sc[o], f"{name} {o}")
+    cr.release()
+
+
+@pytest.mark.gpu
+@pytest.mark.parametrize("name", ["conv3x3_residual", "conv3x3_stride2", "mlp_split_k_q"])
+def test_fp8_more_shapes_per_composite_equals_the_region_kernel_on_small_integers(name):
+    g, _ = MORE[name]()
+    inp = _int_fp8(g, seed=len(name))
+    pc, c1 = run_region(R.whole_graph_region(g), inp)
+    rk, c2 = run_region(R.whole_graph_region(g, options=RK), inp)
+    assert c2.n_launches == 2  # the quantize launch and one region kernel
+    for o in g.outputs:
+        assert np.array_equal(pc[o].view(np.uint32), rk[o].view(np.uint32)), o
+    c1.release()
+    c2.release()
