@@ -92,10 +92,12 @@ typedef enum {
                                quantized per output channel with power-of-two scales
                                S_w[k] = 2^ceil(log2(max |w'[k]| / 448)) at compile time,
                                and its output is dequantized (x S S_w[k]) in the epilogue.
-                               A QUANTIZE right after a conv2d / dense epilogue chain is
-                               fused into that epilogue; one on a region input is its own
-                               launch.  FP8 layers run in the region kernel (see
-                               BYOC_OPT_REGION_KERNEL) and need C % 128 == 0. */
+                               A QUANTIZE right after the epilogue chain of an FP8
+                               conv2d / dense (with BYOC_OPT_REGION_KERNEL: of any
+                               conv2d / dense) is fused into that epilogue, which then
+                               writes the E4M3 codes; one on a region input, or on a
+                               tensor with other readers, is its own launch.  FP8
+                               layers need C % 128 == 0. */
 } byoc_op_kind;
 
 typedef struct {

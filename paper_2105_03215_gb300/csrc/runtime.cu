@@ -292,7 +292,7 @@ struct LaunchPlan {
     size_t order_off = 0, dep_off_off = 0, dep_list_off = 0;  // constant blob: int32 unit order, dependencies
     size_t cta_off_off = 0, cta_rec_off = 0;                  // constant blob: int32 per-CTA unit records
     size_t c_dq_off[byoc::kChainMaxStages] = {};
-    // FP8 GEMM (region kernel only): A and B are E4M3 codes; dq = [n_pad] fp32
+    // FP8 GEMM (cfg.bk = kF8BK, or a region-kernel stage): A and B are E4M3 codes; dq = [n_pad] fp32
     // dequantization scales S_x S_w[n] in the constant blob
     int fp8 = 0;
     size_t dq_off = 0;
