@@ -149,11 +149,14 @@ typedef struct {
  *     on the MobileNetV2 shapes.  Results are bit-identical either way. */
 #define BYOC_OPT_FUSE_DW_PW 0x1u
 /*   BYOC_OPT_REGION_KERNEL: a region whose composites are all conv2d / dense
- *     (1x1 or k x k, no stem layout) and number two to four runs as one
- *     persistent kernel: the intermediates are written once and read back
- *     from L2, and a composite's output tiles start as soon as the tiles of
- *     the earlier composites they read are done (no launch boundary between
- *     composites).  Regions that do not qualify get the per-composite plan. */
+ *     (1x1 or k x k, no stem layout) and number two to four (one to four
+ *     when FP8) runs as one persistent kernel after its leading quantize
+ *     launches: the intermediates are written once and read back from L2,
+ *     and a composite's output tiles start as soon as the tiles of the
+ *     earlier composites they read are done (no launch boundary between
+ *     composites).  Regions that do not qualify get the per-composite plan.
+ *     Off by default: measured on GB300 it is slower than the per-composite
+ *     plan on the BERT FFN and the ResNet-50 bottleneck. */
 #define BYOC_OPT_REGION_KERNEL 0x2u
 /*   BYOC_OPT_MULTICAST: a GEMM launch whose weights are streamed through its
  *     ring (tile, im2col or ringed slab mode, no split-K, at least two
