@@ -68,6 +68,11 @@ struct ChainShape {
     static_assert(BN == 128 || BN == 256, "BN");
 };
 
+template <bool B>
+struct BoolTag {
+    static constexpr bool value = B;
+};
+
 // readers of a unit broadcast slot: the producer lane, the MMA lane, 8
 // epilogue warps
 constexpr uint32_t kChainUnitReaders = 1 + kGemmEpiWarps + 1;
@@ -442,18 +447,25 @@ __global__ void __maxnreg__(168)
             const int m0 = (tile / cs.tiles_n) * S::BM;
             const int n0 = (tile % cs.tiles_n) * BN;
             const int buf = t & 1;
-            const int row = m0 + quarter * 32 + lane;  // this thread's output row
             const int nch = min(S::NCH, (cs.N - n0 + 31) >> 5);
-            const bool has_res = cs.residual != nullptr && row < cs.M;
-            // The residual row segment of this warp's next chunk is loaded one
-            // chunk ahead, the first one before the accumulator is ready (a
-            // residual written by earlier stages was acquired before the unit
-            // was published).
+            const bool has_res = cs.residual != nullptr;
+            // The residual of this warp's 32 rows x 32 columns of its next
+            // chunk is loaded one chunk ahead, the first before the
+            // accumulator is ready (a residual written by earlier stages was
+            // acquired before the unit was published): coalesced, lane l
+            // reading 16-byte piece l % 4 of row 8k + l / 4, so that each load
+            // instruction covers eight 64-byte row segments rather than 32
+            // (measured: one row per lane left ~1.7 us of latency on a
+            // chunk); the chunk's staging tile turns it into one row per lane.
+            const int rrow = lane >> 2, rpiece = lane & 3;
             uint4 rn[4];
             auto load_res = [&](int ci) {
-                const __nv_bfloat16 *rp = cs.residual + (size_t)row * cs.N + (n0 + ci * 32);
 #pragma unroll
-                for (int q = 0; q < 4; ++q) rn[q] = ld_cg_v4(rp + 8 * q);
+                for (int k = 0; k < 4; ++k) {
+                    const int rw = m0 + quarter * 32 + 8 * k + rrow;
+                    rn[k] = rw < cs.M ? ld_cg_v4(cs.residual + (size_t)rw * cs.N + (n0 + ci * 32 + rpiece * 8))
+                                      : make_uint4(0u, 0u, 0u, 0u);
+                }
             };
             if (has_res && grp < nch) load_res(grp);
             // this warp's chunks' bias (and FP8 dequantization scales), one
@@ -477,99 +489,132 @@ __global__ void __maxnreg__(168)
                 __syncwarp();
                 if (lane == 0) mbar_arrive(tempty + 8u * buf);
             }
+            // the chunks, compiled once with and once without the residual
+            // (one copy for both measured ~1 us slower on the BERT FFN's GELU stage)
+            auto chunks = [&](auto res_tag) {
+                constexpr bool RESID = decltype(res_tag)::value;
 #pragma unroll
-            for (int k = 0; k < KC; ++k) {
-                const int ci = grp + 2 * k;
-                if (ci >= nch) break;
-                const int col0 = n0 + ci * 32;
-                uint4 rr[4];
+                for (int k = 0; k < KC; ++k) {
+                    const int ci = grp + 2 * k;
+                    if (ci >= nch) break;
+                    const int col0 = n0 + ci * 32;
+                    uint4 rc[4];  // this chunk's residual pieces (coalesced layout)
 #pragma unroll
-                for (int q = 0; q < 4; ++q) rr[q] = rn[q];
-                if (has_res && ci + 2 < nch) load_res(ci + 2);
-                uint32_t v[32];
-                tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
-                if (ci + 2 >= nch) {  // this warp's last read of the accumulator
-                    tc_fence_before();
+                    for (int q = 0; q < 4; ++q) rc[q] = rn[q];
+                    if (RESID && ci + 2 < nch) load_res(ci + 2);
+                    uint32_t v[32];
+                    tmem_ld_32cols(tbase + (uint32_t)(ci * 32), v);
+                    if (ci + 2 >= nch) {  // this warp's last read of the accumulator
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) mbar_arrive(tempty + 8u * buf);
+                    }
+                    float f[32];
+                    if (cs.fp8) {
+                        // FP8: the accumulator is in units of S_x S_w[n]
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            f[j] = fmaf(__uint_as_float(v[j]), __shfl_sync(0xffffffffu, dl[k], j),
+                                        __shfl_sync(0xffffffffu, bl[k], j));
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]) + __shfl_sync(0xffffffffu, bl[k], j);
+                    }
+                    const uint32_t stg = stg0 + (uint32_t)(sb * S::EPI_TILE);
+                    if constexpr (RESID) {
+                        // the store that last used this staging tile has read it
+                        if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
+                        __syncwarp();
+                        // residual pieces -> staging tile (64-byte swizzle, as the
+                        // output below) -> this lane's row
+#pragma unroll
+                        for (int p = 0; p < 4; ++p) {
+                            const uint32_t r = (uint32_t)(8 * p + rrow);
+                            const uint32_t addr = stg + r * 64u + ((((uint32_t)rpiece) ^ ((r >> 1) & 3u)) << 4);
+                            asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(rc[p].x),
+                                         "r"(rc[p].y), "r"(rc[p].z), "r"(rc[p].w)
+                                         : "memory");
+                        }
+                        __syncwarp();
+                        uint4 rr[4];
+#pragma unroll
+                        for (int q = 0; q < 4; ++q)
+                            asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                                         : "=r"(rr[q].x), "=r"(rr[q].y), "=r"(rr[q].z), "=r"(rr[q].w)
+                                         : "r"(stg + (uint32_t)lane * 64u + ((((uint32_t)q) ^ sw_own) << 4))
+                                         : "memory");
+                        __syncwarp();  // every row read before the output overwrites the tile
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const uint32_t w4[4] = {rr[q].x, rr[q].y, rr[q].z, rr[q].w};
+#pragma unroll
+                            for (int e2 = 0; e2 < 4; ++e2) {
+                                f[8 * q + 2 * e2] += bf16lo(w4[e2]);
+                                f[8 * q + 2 * e2 + 1] += bf16hi(w4[e2]);
+                            }
+                        }
+                    }
+                    if (cs.act == kActGelu) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const uint64_t g = gelu2(f32x2(f[2 * j], f[2 * j + 1]));
+                            f[2 * j] = lane0(g);
+                            f[2 * j + 1] = lane1(g);
+                        }
+                    } else if (cs.act == kActRelu) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) f[j] = fmaxf(f[j], 0.0f);
+                    } else if (cs.act == kActRelu6) {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j) f[j] = fminf(fmaxf(f[j], 0.0f), 6.0f);
+                    }
+                    if constexpr (!RESID) {  // (with a residual: waited for above)
+                        if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
+                        __syncwarp();
+                    }
+                    if (cs.out8) {
+                        // a fused Q node: E4M3 codes of f x fp32(1/S), 32 bytes per
+                        // row, rows 32 bytes apart (the unswizzled box of the map)
+#pragma unroll
+                        for (int h = 0; h < 2; ++h) {
+                            uint32_t w[4];
+#pragma unroll
+                            for (int k = 0; k < 4; ++k) {
+                                const float *g = f + 16 * h + 4 * k;
+                                w[k] = cvt_e4m3x2(g[0] * cs.out_inv, g[1] * cs.out_inv) |
+                                       (cvt_e4m3x2(g[2] * cs.out_inv, g[3] * cs.out_inv) << 16);
+                            }
+                            const uint32_t addr = stg + (uint32_t)lane * 32u + (uint32_t)h * 16u;
+                            asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]), "r"(w[1]),
+                                         "r"(w[2]), "r"(w[3])
+                                         : "memory");
+                        }
+                    } else {
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
+                            const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
+                            const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
+                            const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
+                            const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
+                            asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0), "r"(w1),
+                                         "r"(w2), "r"(w3)
+                                         : "memory");
+                        }
+                    }
+                    fence_proxy_async_smem();
                     __syncwarp();
-                    if (lane == 0) mbar_arrive(tempty + 8u * buf);
-                }
-                float f[32];
-                if (cs.fp8) {
-                    // FP8: the accumulator is in units of S_x S_w[n]
-#pragma unroll
-                    for (int j = 0; j < 32; ++j)
-                        f[j] = fmaf(__uint_as_float(v[j]), __shfl_sync(0xffffffffu, dl[k], j),
-                                    __shfl_sync(0xffffffffu, bl[k], j));
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) f[j] = __uint_as_float(v[j]) + __shfl_sync(0xffffffffu, bl[k], j);
-                }
-                if (has_res) {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint32_t w4[4] = {rr[q].x, rr[q].y, rr[q].z, rr[q].w};
-#pragma unroll
-                        for (int e2 = 0; e2 < 4; ++e2) {
-                            f[8 * q + 2 * e2] += bf16lo(w4[e2]);
-                            f[8 * q + 2 * e2 + 1] += bf16hi(w4[e2]);
-                        }
+                    if (lane == 0) {
+                        tma_store_2d(&maps.O[si], stg, col0, m0 + quarter * 32);
+                        bulk_commit_group();
                     }
+                    if (S::EPI_BUFS == 2) sb ^= 1;
                 }
-                if (cs.act == kActGelu) {
-#pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const uint64_t g = gelu2(f32x2(f[2 * j], f[2 * j + 1]));
-                        f[2 * j] = lane0(g);
-                        f[2 * j + 1] = lane1(g);
-                    }
-                } else if (cs.act == kActRelu) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) f[j] = fmaxf(f[j], 0.0f);
-                } else if (cs.act == kActRelu6) {
-#pragma unroll
-                    for (int j = 0; j < 32; ++j) f[j] = fminf(fmaxf(f[j], 0.0f), 6.0f);
-                }
-                const uint32_t stg = stg0 + (uint32_t)(sb * S::EPI_TILE);
-                if (lane == 0) bulk_wait_group_read<S::EPI_BUFS - 1>();
-                __syncwarp();
-                if (cs.out8) {
-                    // a fused Q node: E4M3 codes of f x fp32(1/S), 32 bytes per
-                    // row, rows 32 bytes apart (the unswizzled box of the map)
-#pragma unroll
-                    for (int h = 0; h < 2; ++h) {
-                        uint32_t w[4];
-#pragma unroll
-                        for (int k = 0; k < 4; ++k) {
-                            const float *g = f + 16 * h + 4 * k;
-                            w[k] = cvt_e4m3x2(g[0] * cs.out_inv, g[1] * cs.out_inv) |
-                                   (cvt_e4m3x2(g[2] * cs.out_inv, g[3] * cs.out_inv) << 16);
-                        }
-                        const uint32_t addr = stg + (uint32_t)lane * 32u + (uint32_t)h * 16u;
-                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w[0]), "r"(w[1]),
-                                     "r"(w[2]), "r"(w[3])
-                                     : "memory");
-                    }
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint32_t w0 = pack_bf16x2(f[8 * q + 0], f[8 * q + 1]);
-                        const uint32_t w1 = pack_bf16x2(f[8 * q + 2], f[8 * q + 3]);
-                        const uint32_t w2 = pack_bf16x2(f[8 * q + 4], f[8 * q + 5]);
-                        const uint32_t w3 = pack_bf16x2(f[8 * q + 6], f[8 * q + 7]);
-                        const uint32_t addr = stg + (uint32_t)lane * 64u + (((uint32_t)q ^ sw_own) << 4);
-                        asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(w0), "r"(w1),
-                                     "r"(w2), "r"(w3)
-                                     : "memory");
-                    }
-                }
-                fence_proxy_async_smem();
-                __syncwarp();
-                if (lane == 0) {
-                    tma_store_2d(&maps.O[si], stg, col0, m0 + quarter * 32);
-                    bulk_commit_group();
-                }
-                if (S::EPI_BUFS == 2) sb ^= 1;
-            }
+            };
+            if (has_res)
+                chunks(BoolTag<true>{});
+            else
+                chunks(BoolTag<false>{});
             __syncwarp();
             if (cs.consumed) {
                 // the unit's rows are read by later stages: count this warp's
