@@ -85,6 +85,12 @@ def test_fp8_per_composite_plan_is_a_quantize_launch_and_fp8_gemms(make, gemms):
     assert [back.fp8[i] for i in range(back.n_launches)] == [rep.fp8[i] for i in range(rep.n_launches)]
 
 
+def test_fp8_short_k_plans_a_grid_of_whole_column_tiles():
+    g, _ = I.fp8_dense(M=16384, D=256, F=512)
+    rep = R.whole_graph_region(g).plan(152)
+    assert rep.fp8[1] == 1 and rep.tile_n[1] == 64 and rep.grid[1] % (512 // 64) == 0
+
+
 def test_fp8_split_k_plans_for_few_tiles():
     # 2 m-tiles x 12 column tiles of a 3072-deep reduction: the k-blocks are
     # split over CTAs (global split-K on FP8 k-blocks)
@@ -131,6 +137,9 @@ FP8_LAYERS = {
     "conv1x1_ragged": lambda: I.fp8_conv(N=3, H=9, W=10, C=128, K=96, k=1),
     "dense": lambda: I.fp8_dense(M=200, D=768, F=1024),
     "dense_split_k": lambda: I.fp8_dense(M=256, D=3072, F=768),
+    # two k-blocks per tile, 1024 tiles over a grid that is a multiple of the
+    # 8 column tiles: every CTA keeps its weight k-blocks in the ring
+    "dense_short_k_weight_reuse": lambda: I.fp8_dense(M=16384, D=256, F=512),
 }
 
 
