@@ -377,12 +377,12 @@ def region_figures(flush, peaks):
                 "hbm_frac_of_measured": kcr.bytes / tk / 1e9 / peaks["hbm_gbs"]}
             out[name + "_region_kernel"].update(stream(kreg, g, kcr))
             kcr.release()
-        if name.startswith("resnet50_bottleneck"):
-            # partial quantization (Section 3.2): Q nodes before the three
-            # convolutions, each computed in FP8 (E4M3, kind::f8f6f4): the
-            # quantize launch of the input, then three FP8 GEMM launches
+        if name.startswith(("bert", "resnet50_bottleneck")):
+            # partial quantization (Section 3.2): Q nodes before every dense
+            # layer / convolution, each computed in FP8 (E4M3, kind::f8f6f4):
+            # the quantize launch of the input, then the FP8 GEMM launches
             # (default) or one region kernel
-            qg, _ = I.fp8_bottleneck(seed=3)
+            qg, _ = I.fp8_ffn(seed=1) if name.startswith("bert") else I.fp8_bottleneck(seed=3)
             fp8_peak = 2.0 * peaks["bf16_tflops"]  # measured bf16 x the nominal fp8 / bf16 ratio (4.5 / 2.25)
             for suffix, opts in (("_fp8", 0), ("_fp8_region_kernel", abi.OPT_REGION_KERNEL)):
                 qreg = R.whole_graph_region(qg, options=opts)

@@ -423,6 +423,22 @@ def fp8_dense(M=256, D=768, F=1024, seed=32):
     return _finish(b, [y], seed)
 
 
+# the BERT FFN's hidden activation GELU(x W1^T + b1): pre-activations of
+# standard deviation sqrt(768) x 0.02 = 0.55, quantized over +-4
+FP8_SCALE_FFN_HIDDEN = 4.0 / 448.0
+
+
+def fp8_ffn(M=1024, D=768, F=3072, seed=1):
+    """The BERT FFN of bert_ffn (same seed, same constants) with partial
+    quantization (Section 3.2): Q nodes before both dense layers, each dense
+    in FP8; the hidden activation leaves the first epilogue as E4M3 codes."""
+    b = _Builder("fp8_ffn")
+    x = b.input("x", (M, D))
+    h = b.gelu(b.bias_add(b.dense(b.quantize(x, FP8_SCALE_INPUT), F, std=0.02)))
+    y = b.bias_add(b.dense(b.quantize(h, FP8_SCALE_FFN_HIDDEN), D, std=0.02))
+    return _finish(b, [y], seed)
+
+
 def fp8_bottleneck(N=32, H=14, W=14, C=1024, width=256, seed=3):
     """The ResNet-50 stage-3 bottleneck of resnet_bottleneck (same seed, same
     constants) with partial quantization (Section 3.2): Q nodes before each

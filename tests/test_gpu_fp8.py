@@ -140,6 +140,9 @@ FP8_LAYERS = {
     # two k-blocks per tile, 1024 tiles over a grid that is a multiple of the
     # 8 column tiles: every CTA keeps its weight k-blocks in the ring
     "dense_short_k_weight_reuse": lambda: I.fp8_dense(M=16384, D=256, F=512),
+    # the BERT FFN with Q nodes before both dense layers (config 2 in FP8):
+    # the hidden codes come from the first epilogue, the second dense splits K
+    "ffn": lambda: I.fp8_ffn(),
 }
 
 
@@ -180,10 +183,13 @@ def test_fp8_bottleneck_matches_the_oracle(N, plan):
 
 
 @pytest.mark.gpu
-@pytest.mark.parametrize("name", ["bottleneck"] + sorted(FP8_LAYERS))
+@pytest.mark.parametrize("name", ["bottleneck"] + sorted(n for n in FP8_LAYERS if n != "ffn"))
 def test_fp8_per_composite_equals_the_region_kernel_on_small_integers(name):
     # the two kernels issue different tile shapes (and split-K) over the same
-    # codes; with exact sums and the same epilogue arithmetic the bits agree
+    # codes; with exact sums and the same epilogue arithmetic the bits agree.
+    # (Not the FFN: its second dense reads GELU outputs, whose codes are not
+    # multiples of one power of two, so its fp32 sums are not exact and the
+    # split-K order of the per-composite plan changes their rounding.)
     g, _ = I.fp8_bottleneck(N=2) if name == "bottleneck" else FP8_LAYERS[name]()
     inp = _int_fp8(g, seed=len(name))
     pc, c1 = run_region(R.whole_graph_region(g), inp)
@@ -275,3 +281,18 @@ def test_fp8_more_shapes_per_composite_equals_the_region_kernel_on_small_integer
         assert np.array_equal(pc[o].view(np.uint32), rk[o].view(np.uint32)), o
     c1.release()
     c2.release()
+
+
+@pytest.mark.gpu
+def test_fp8_ffn_quantization_error_against_the_bf16_region():
+    # config 2 with Q nodes before both dense layers, against the unquantized
+    # FFN of the same constants (reported; a loose bound)
+    g, inp = I.fp8_ffn()
+    got, cr = run_region(R.whole_graph_region(g), inp)
+    gb, _ = I.bert_ffn(seed=1)
+    full = ograph.evaluate(gb, inp)[gb.outputs[0]]
+    o = g.outputs[0]
+    rel = np.linalg.norm(got[o] - full) / np.linalg.norm(full)
+    print(f"fp8 FFN: relative L2 error against the unquantized region {rel:.4f}")
+    assert rel < 0.1
+    cr.release()
