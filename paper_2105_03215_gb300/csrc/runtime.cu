@@ -19,6 +19,7 @@
 #include <cudaTypedefs.h>
 
 #include <algorithm>
+#include <type_traits>
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
@@ -665,7 +666,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
             // a tensor with other readers): its own launch
             if ((int)P.launches.size() >= BYOC_PLAN_MAX_LAUNCHES - 1)
                 return fail(BYOC_ERR_UNSUPPORTED, "region needs more than %d launches", BYOC_PLAN_MAX_LAUNCHES - 1);
-            LaunchPlan Q;
+            LaunchPlan Q{};
             Q.kind = BYOC_LAUNCH_QUANT;
             Q.first_op = o;
             Q.n_ops = 1;
@@ -749,7 +750,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
         int cur, res, act;
         const int j = walk_chain(o, af, cur, res, act);
         const TensorInfo Y = P.tensors[cur];
-        LaunchPlan L;
+        LaunchPlan L{};
         L.first_op = o;
         L.n_ops = j - o;
         L.x = op.in[0];
@@ -950,7 +951,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
                 const int64_t Wq = 2 * wpz;
                 if ((int64_t)X.shape[0] * Hq > INT32_MAX)
                     return fail(BYOC_ERR_UNSUPPORTED, "op %d: stem layout too large", o);
-                TensorInfo Z;
+                TensorInfo Z{};
                 Z.ndim = 4;
                 Z.shape[0] = X.shape[0];
                 Z.shape[1] = Hq;
@@ -958,7 +959,7 @@ byoc_status plan_region_impl(const byoc_region_desc *d, int num_sms, Plan &P, in
                 Z.shape[3] = 4;
                 const int zid = (int)P.tensors.size();
                 P.tensors.push_back(Z);
-                LaunchPlan S;
+                LaunchPlan S{};
                 S.kind = BYOC_LAUNCH_S2D;
                 S.x = op.in[0];
                 S.y = zid;
@@ -1289,7 +1290,7 @@ bool make_chain(Plan &P, int bn) {
         if (L.res >= 0 && P.tensors[L.res].dtype != BYOC_BF16) return undo();
         if (L.args.num_tiles != (L.args.M + byoc::kGemmBM - 1) / byoc::kGemmBM * L.args.tiles_n) return undo();
     }
-    LaunchPlan C;
+    LaunchPlan C{};
     C.kind = BYOC_LAUNCH_CHAIN;
     C.chain_bn = bn;
     C.first_op = P.launches[0].first_op;
@@ -1888,14 +1889,16 @@ struct PlanHeader {
 
 // Records are written with their padding zeroed, so that the bytes depend
 // only on the plan (no stray host memory in a serialised region).
+// The objects' bytes as they are: every plan object is value-initialised
+// (T x{}, vector resize), so its padding bytes are zero and copies keep them.
+// (__builtin_clear_padding is not used: GCC 13 cleared array elements of
+// LaunchPlan as if they were padding -- a region kernel's c_npad[1] read
+// back as 0 once the struct's layout changed.)
 template <typename T>
 void put(std::vector<uint8_t> &out, const T *v, size_t n) {
-    for (size_t i = 0; i < n; ++i) {
-        T c = v[i];
-        __builtin_clear_padding(&c);
-        const uint8_t *b = reinterpret_cast<const uint8_t *>(&c);
-        out.insert(out.end(), b, b + sizeof(T));
-    }
+    static_assert(std::is_trivially_copyable<T>::value, "plans are serialised byte for byte");
+    const uint8_t *b = reinterpret_cast<const uint8_t *>(v);
+    out.insert(out.end(), b, b + n * sizeof(T));
 }
 
 void serialize_plan(const Plan &P, std::vector<uint8_t> &out) {
